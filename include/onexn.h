@@ -1,0 +1,202 @@
+/*
+ * onexn.h -- C ABI of the GB300 (sm_103a) 1xN-pruned convolution library.
+ *
+ * 1xN pruning (Lin et al., "1xN Pattern for Pruning Convolutional Neural
+ * Networks") groups the weights of a layer W in R^{n x m x h x w}
+ * (n = C_out, m = C_in, h x w = KH x KW, Sec. 3.1) into blocks of N
+ * consecutive output channels that share one input index, keeps the blocks
+ * with the largest l1 norms (Sec. 3.2, Eq. 4-5), optionally re-orders the
+ * filters by l1 norm first (Sec. 3.3), stores the kept blocks in a BSR
+ * layout (D, I, P) (Sec. 3.4) and computes the layer output block by block
+ * (Eq. 7).  This header is the whole public surface: plain C types, host or
+ * device pointers, and sizes.
+ *
+ * Conventions used by every call
+ * ------------------------------
+ *  - Weights W are host fp32 in OIHW order: W[o][c][kh][kw].
+ *  - Index space.  A block is one (col-group g, input index k), where
+ *    g in [0, G), G = C_out / N, and k = (kh*KW + kw)*C_in + c in [0, K),
+ *    K = KH*KW*C_in ("tap-major": it matches the NHWC activation layout).
+ *    This is the per-(c, kh, kw) block granularity (ONEXN_GRAN_TAP).
+ *    ONEXN_GRAN_KERNEL is the paper's own block of Sec. 3.2, one block per
+ *    (g, c) holding N whole KH x KW kernels; a kept (g, c) keeps all KH*KW
+ *    indices k of channel c.  The two coincide for 1x1 layers.
+ *  - mask is uint8 [G][K] (1 = kept), the transpose of the paper's
+ *    T in {0,1}^{m x n/N} expanded to the index space.
+ *  - BSR (Sec. 3.4), 0-based: P int32 [G+1] with P[0] = 0 and P[G] = t,
+ *    I int32 [t] (strictly increasing inside each col-group), D [t][N]
+ *    (the N weights of a kept block stored contiguously), fp32 or bf16.
+ *  - Activations are NHWC: x[b][h][w][c]; outputs y[b][ho][wo][o].
+ *  - Every call returns an onexn_status; nothing else crosses the ABI.
+ *    On failure onexn_last_error() returns a message (thread-local, valid
+ *    until the next call on the same thread).  Calls allocate nothing that
+ *    outlives them and take no ownership of caller buffers.
+ */
+#ifndef ONEXN_H
+#define ONEXN_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+    ONEXN_OK = 0,
+    ONEXN_EINVAL = 1,        /* bad argument: shape, null pointer, range, alignment */
+    ONEXN_EUNSUPPORTED = 2,  /* valid request that no kernel here implements */
+    ONEXN_ENOMEM = 3,        /* a host allocation failed */
+    ONEXN_ECUDA = 4,         /* a CUDA runtime call or kernel launch failed */
+    ONEXN_EDEVICE = 5,       /* a kernel reported a bad input through its status word */
+    ONEXN_ETIMEOUT = 6       /* a bounded device-side wait ran out */
+} onexn_status;
+
+typedef enum { ONEXN_F32 = 0, ONEXN_BF16 = 1 } onexn_dtype;
+
+typedef enum { ONEXN_GRAN_TAP = 0, ONEXN_GRAN_KERNEL = 1 } onexn_granularity;
+
+/* onexn_conv_fwd flags */
+#define ONEXN_RELU 0x1u               /* y = max(y, 0) after the bias */
+/* Kernel selection (bits 8..11).  AUTO picks by dtype, N and density. */
+#define ONEXN_ALGO_SHIFT 8
+#define ONEXN_ALGO_MASK (0xFu << ONEXN_ALGO_SHIFT)
+#define ONEXN_ALGO_AUTO (0u << ONEXN_ALGO_SHIFT)
+#define ONEXN_ALGO_FMA (1u << ONEXN_ALGO_SHIFT)   /* CUDA-core FFMA, any N, fp32/bf16 */
+#define ONEXN_ALGO_MMA (2u << ONEXN_ALGO_SHIFT)   /* bf16 tensor cores, N % 8 == 0 */
+
+/* Message for the last failed call on this thread ("" if none). */
+const char *onexn_last_error(void);
+
+/* Library ABI version, (major << 16) | minor. */
+int onexn_version(void);
+
+/*
+ * onexn_keep_count -- number of blocks the mask keeps (Eq. 1 constraint
+ * ||T||_0 / K = 1 - p).  The rate is taken at a resolution of 1e-6 and
+ * keep = round-half-up(total * (1 - p)) in exact int64 arithmetic.
+ * EINVAL if rate is outside [0, 1], total < 0 or keep is NULL.
+ */
+onexn_status onexn_keep_count(int64_t total_blocks, double rate, int64_t *keep);
+
+/*
+ * onexn_prune -- the 1xN mask of Eq. 4 / Eq. 5: score every block by its l1
+ * norm, keep the top (1 - rate) fraction of blocks (onexn_keep_count).
+ *   W      host fp32 OIHW [C_out][C_in][KH][KW], read only.
+ *   N      block width; must divide C_out.
+ *   rate   pruning rate p in [0, 1].
+ *   gran   ONEXN_GRAN_TAP or ONEXN_GRAN_KERNEL.
+ *   mask   host uint8 [G][K], written in full (caller-owned).
+ *   kept   number of kept blocks at the chosen granularity (so the number
+ *          of kept indices is kept, or kept*KH*KW for GRAN_KERNEL).
+ * A block's score is the sum of |w| over its weights in fp64, in the order
+ * n, then kh, then kw.  Ties go to the lower block index g*nb + b (nb = K
+ * for TAP, C_in for KERNEL).  The result is deterministic.
+ * EINVAL: NULL pointer, N < 1, N not dividing C_out, non-positive dims,
+ * rate outside [0, 1].  ENOMEM: scratch allocation failed.
+ */
+onexn_status onexn_prune(const float *W, int C_out, int C_in, int KH, int KW, int N,
+                         double rate, int gran, uint8_t *mask, int64_t *kept);
+
+/*
+ * onexn_rearrange -- filter rearrangement of Sec. 3.3, in place.
+ *   W_l    host fp32 OIHW [C_out][C_in][KH][KW]; its filters (output
+ *          channels) are re-ordered by l1 norm, largest first; equal norms
+ *          keep their original order.
+ *   W_next nullable host fp32 OIHW [C_out_next][C_out][KH_next][KW_next];
+ *          its input channels get the same permutation, so the composition
+ *          of the two layers is unchanged.
+ *   perm   host int32 [C_out]: perm[o'] = original index now at o'.  Apply
+ *          it to anything else indexed by layer l's outputs (bias, BN,
+ *          depthwise channels in between).
+ * The norm of filter o is the fp64 sum of |w| in (c, kh, kw) order.
+ * EINVAL: NULL W_l/perm, non-positive dims.  ENOMEM: scratch failed.
+ */
+onexn_status onexn_rearrange(float *W_l, int C_out, int C_in, int KH, int KW,
+                             float *W_next, int C_out_next, int KH_next, int KW_next,
+                             int32_t *perm);
+
+/*
+ * onexn_pack -- BSR encoding of Sec. 3.4 (Fig. 3).
+ *   W, mask   as in onexn_prune (host).
+ *   wdtype    ONEXN_F32 (D is float) or ONEXN_BF16 (D is bfloat16 bits,
+ *             round-to-nearest-even of the fp32 weight).
+ *   P         host int32 [G+1]; I host int32 [t_cap]; D host [t_cap][N].
+ *   t         out: number of kept blocks t (= sum of mask).
+ * Col-group g's kept indices are written in increasing k order into
+ * I[P[g] .. P[g+1]), with their N weights in the same rows of D.
+ * EINVAL: NULL pointer, bad dims, t_cap smaller than the kept count (t is
+ * still written), a mask byte other than 0/1.
+ */
+onexn_status onexn_pack(const float *W, const uint8_t *mask, int C_out, int C_in, int KH,
+                        int KW, int N, int wdtype, int32_t *P, int32_t *I, void *D,
+                        int64_t t_cap, int64_t *t);
+
+/*
+ * onexn_packed_validate -- host check of a BSR index structure before it is
+ * copied to the device: P[0] = 0, P non-decreasing, P[G] = t, each
+ * col-group's I strictly increasing and inside [0, K).  EINVAL on the first
+ * violation (the message names it).
+ */
+onexn_status onexn_packed_validate(const int32_t *P, const int32_t *I, int G, int64_t t,
+                                   int K);
+
+/* Geometry of one convolution.  Output size per dimension:
+ * Ho = (H + 2*pad_h - dil_h*(KH-1) - 1) / stride_h + 1 (same for W). */
+typedef struct {
+    int B, H, W, C_in;                 /* input  x: [B][H][W][C_in]   */
+    int C_out, KH, KW;                 /* weights: [C_out][C_in][KH][KW] */
+    int stride_h, stride_w;
+    int pad_h, pad_w;                  /* zero padding */
+    int dil_h, dil_w;
+} onexn_conv_desc;
+
+/* Output spatial size of desc; EINVAL if it is empty or desc is invalid. */
+onexn_status onexn_conv_out_shape(const onexn_conv_desc *desc, int *Ho, int *Wo);
+
+/*
+ * onexn_conv_fwd -- forward convolution of a 1xN-pruned layer, computed
+ * block by block from the BSR weights (Eq. 7):
+ *   y[p, gN:(g+1)N] = bias[gN:(g+1)N] + sum_{z=P[g]}^{P[g+1]-1} X[p, I[z]] * D[z, :]
+ * where X[p, k] is the input value under output pixel p at tap
+ * (kh, kw) = ((k / C_in) / KW, (k / C_in) % KW) and channel c = k % C_in
+ * (zero in the padding), followed by max(., 0) if flags has ONEXN_RELU.
+ *
+ *   desc    host pointer to the geometry.
+ *   P, I, D DEVICE pointers to the BSR weights of onexn_pack (N, t as
+ *           packed; D's element type must equal dtype).  P and I must pass
+ *           onexn_packed_validate; the kernels never read outside
+ *           I[0..t) and D[0..t*N) even if they do not.
+ *   x       DEVICE NHWC activations, fp32 (dtype ONEXN_F32) or bf16
+ *           (ONEXN_BF16), 16-byte aligned; C_in % 4 == 0 (fp32) or
+ *           C_in % 8 == 0 (bf16).
+ *   y       DEVICE NHWC output [B][Ho][Wo][C_out], same element type as x,
+ *           16-byte aligned, must not overlap x.  bf16 outputs are the
+ *           round-to-nearest-even of the fp32 result.
+ *   bias    nullable DEVICE fp32 [C_out].
+ *   dtype   ONEXN_F32: fp32 inputs and weights, fp32 accumulation.
+ *           ONEXN_BF16: bf16 inputs and weights, fp32 accumulation.
+ *   flags   ONEXN_RELU | one ONEXN_ALGO_* value.
+ *   stream  cudaStream_t to launch on (NULL = legacy default stream).
+ * Asynchronous: returns after the launch; errors of the launch itself are
+ * returned as ECUDA.  No allocation, no synchronisation, no host read of
+ * device memory.  EINVAL: bad geometry, N not dividing C_out, alignment,
+ * NULL pointers.  EUNSUPPORTED: the forced ALGO cannot run this case.
+ */
+onexn_status onexn_conv_fwd(const onexn_conv_desc *desc, const int32_t *P, const int32_t *I,
+                            const void *D, int N, int64_t t, const void *x, void *y,
+                            const float *bias, int dtype, unsigned flags, void *stream);
+
+/*
+ * onexn_conv_algo -- which kernel family onexn_conv_fwd would run for these
+ * arguments (an ONEXN_ALGO_* value other than AUTO), without launching.
+ * EINVAL / EUNSUPPORTED as onexn_conv_fwd.
+ */
+onexn_status onexn_conv_algo(const onexn_conv_desc *desc, int N, int64_t t, int dtype,
+                             unsigned flags, unsigned *algo);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* ONEXN_H */

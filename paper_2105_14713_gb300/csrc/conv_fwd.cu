@@ -1,0 +1,129 @@
+// onexn_conv_fwd: argument checks and kernel selection for the forward
+// convolution of a 1xN-pruned layer (Eq. 7).  Launches only; never
+// allocates, synchronises or reads device memory from the host.
+#include "conv_common.cuh"
+#include "onexn_internal.h"
+
+namespace onexn {
+cudaError_t launch_fma(const ConvArgs &a, int dtype, cudaStream_t st);
+cudaError_t launch_mma(const ConvArgs &a, cudaStream_t st);
+bool mma_supports(const ConvArgs &a);
+}  // namespace onexn
+
+using onexn::fail;
+
+namespace {
+
+bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+// Shape, dtype and flag checks; fills the geometry part of *a.
+onexn_status check_shape(const onexn_conv_desc *d, int N, int64_t t, int dtype, unsigned flags,
+                         onexn::ConvArgs *a)
+{
+    if (!d) return fail(ONEXN_EINVAL, "conv: desc is NULL");
+    int Ho = 0, Wo = 0;
+    onexn_status st = onexn_conv_out_shape(d, &Ho, &Wo);
+    if (st != ONEXN_OK) return st;
+    if (dtype != ONEXN_F32 && dtype != ONEXN_BF16)
+        return fail(ONEXN_EINVAL, "conv: unknown dtype %d", dtype);
+    if (N < 1 || d->C_out % N) return fail(ONEXN_EINVAL, "conv: N=%d must divide C_out=%d", N, d->C_out);
+    const int64_t K = static_cast<int64_t>(d->KH) * d->KW * d->C_in;
+    const int64_t G = d->C_out / N;
+    if (K >= (int64_t(1) << 30)) return fail(ONEXN_EINVAL, "conv: index space too large");
+    if (t < 0 || t > G * K || t >= (int64_t(1) << 31))
+        return fail(ONEXN_EINVAL, "conv: t=%lld outside [0, G*K]", (long long)t);
+    const int64_t npix = static_cast<int64_t>(d->B) * Ho * Wo;
+    if (npix >= (int64_t(1) << 31) || static_cast<int64_t>(d->B) * d->H * d->W >= (int64_t(1) << 31))
+        return fail(ONEXN_EINVAL, "conv: too many pixels for one launch");
+    const int cv = dtype == ONEXN_F32 ? 4 : 8;
+    if (d->C_in % cv)
+        return fail(ONEXN_EINVAL, "conv: C_in=%d must be a multiple of %d for %s", d->C_in, cv,
+                    dtype == ONEXN_F32 ? "fp32" : "bf16");
+    if (flags & ~(ONEXN_RELU | ONEXN_ALGO_MASK)) return fail(ONEXN_EINVAL, "conv: unknown flags");
+    a->B = d->B; a->H = d->H; a->W = d->W; a->C = d->C_in;
+    a->C_out = d->C_out; a->KH = d->KH; a->KW = d->KW;
+    a->sh = d->stride_h; a->sw = d->stride_w; a->ph = d->pad_h; a->pw = d->pad_w;
+    a->dh = d->dil_h; a->dw = d->dil_w; a->Ho = Ho; a->Wo = Wo;
+    a->N = N; a->t = static_cast<int>(t); a->P_pix = static_cast<int>(npix);
+    a->relu = (flags & ONEXN_RELU) ? 1 : 0;
+    return ONEXN_OK;
+}
+
+// Pointer checks; fills the pointer part of *a.
+onexn_status check_pointers(const int32_t *P, const int32_t *I, const void *D, const void *x,
+                            void *y, const float *bias, int dtype, onexn::ConvArgs *a)
+{
+    if (!P) return fail(ONEXN_EINVAL, "conv: P is NULL");
+    if (a->t > 0 && (!I || !D)) return fail(ONEXN_EINVAL, "conv: I or D is NULL");
+    if (a->P_pix > 0 && (!x || !y)) return fail(ONEXN_EINVAL, "conv: x or y is NULL");
+    if (!aligned16(x) || !aligned16(y) || !aligned16(D))
+        return fail(ONEXN_EINVAL, "conv: x, y and D must be 16-byte aligned");
+    if ((reinterpret_cast<uintptr_t>(bias) & 3u) || (reinterpret_cast<uintptr_t>(P) & 3u) ||
+        (reinterpret_cast<uintptr_t>(I) & 3u))
+        return fail(ONEXN_EINVAL, "conv: bias, P and I must be 4-byte aligned");
+    if (a->P_pix > 0) {
+        const size_t es = dtype == ONEXN_F32 ? 4 : 2;
+        const uintptr_t x0 = reinterpret_cast<uintptr_t>(x),
+                        x1 = x0 + static_cast<size_t>(a->B) * a->H * a->W * a->C * es;
+        const uintptr_t y0 = reinterpret_cast<uintptr_t>(y),
+                        y1 = y0 + static_cast<size_t>(a->P_pix) * a->C_out * es;
+        if (x0 < y1 && y0 < x1) return fail(ONEXN_EINVAL, "conv: x and y overlap");
+    }
+    a->x = x; a->y = y; a->bias = bias; a->P = P; a->I = I; a->D = D;
+    return ONEXN_OK;
+}
+
+// Kernel family for AUTO: bf16 with N a multiple of 8 runs on tensor cores;
+// everything else (fp32, and bf16 with N < 8) on the FFMA kernel.
+unsigned pick_algo(const onexn::ConvArgs &a, int dtype, unsigned flags)
+{
+    const unsigned forced = flags & ONEXN_ALGO_MASK;
+    if (forced != ONEXN_ALGO_AUTO) return forced;
+    if (dtype == ONEXN_BF16 && onexn::mma_supports(a)) return ONEXN_ALGO_MMA;
+    return ONEXN_ALGO_FMA;
+}
+
+}  // namespace
+
+extern "C" onexn_status onexn_conv_algo(const onexn_conv_desc *desc, int N, int64_t t, int dtype,
+                                        unsigned flags, unsigned *algo)
+{
+    onexn::clear_error();
+    if (!algo) return fail(ONEXN_EINVAL, "conv_algo: algo is NULL");
+    onexn::ConvArgs a{};
+    onexn_status st = check_shape(desc, N, t, dtype, flags, &a);
+    if (st != ONEXN_OK) return st;
+    const unsigned al = pick_algo(a, dtype, flags);
+    if (al == ONEXN_ALGO_MMA && (dtype != ONEXN_BF16 || !onexn::mma_supports(a)))
+        return fail(ONEXN_EUNSUPPORTED, "conv: the MMA kernel needs bf16 and N %% 8 == 0");
+    if (al != ONEXN_ALGO_FMA && al != ONEXN_ALGO_MMA) return fail(ONEXN_EINVAL, "conv: unknown algo");
+    *algo = al;
+    return ONEXN_OK;
+}
+
+extern "C" onexn_status onexn_conv_fwd(const onexn_conv_desc *desc, const int32_t *P,
+                                       const int32_t *I, const void *D, int N, int64_t t,
+                                       const void *x, void *y, const float *bias, int dtype,
+                                       unsigned flags, void *stream)
+{
+    onexn::clear_error();
+    onexn::ConvArgs a{};
+    onexn_status st = check_shape(desc, N, t, dtype, flags, &a);
+    if (st != ONEXN_OK) return st;
+    st = check_pointers(P, I, D, x, y, bias, dtype, &a);
+    if (st != ONEXN_OK) return st;
+    const unsigned algo = pick_algo(a, dtype, flags);
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    cudaError_t e;
+    if (algo == ONEXN_ALGO_FMA) {
+        e = onexn::launch_fma(a, dtype, s);
+    } else if (algo == ONEXN_ALGO_MMA) {
+        if (dtype != ONEXN_BF16 || !onexn::mma_supports(a))
+            return fail(ONEXN_EUNSUPPORTED, "conv: the MMA kernel needs bf16 and N %% 8 == 0");
+        e = onexn::launch_mma(a, s);
+    } else {
+        return fail(ONEXN_EINVAL, "conv: unknown algo %u", algo >> ONEXN_ALGO_SHIFT);
+    }
+    if (e != cudaSuccess) return fail(ONEXN_ECUDA, "conv: launch failed: %s", cudaGetErrorString(e));
+    return ONEXN_OK;
+}

@@ -1,0 +1,96 @@
+"""A 1xN-pruned convolution layer on the onexn C ABI.
+
+``PrunedConv2d`` runs the offline steps once on the host -- block scoring
+and selection (``onexn_prune``), BSR encoding (``onexn_pack``), the index
+check (``onexn_packed_validate``) -- copies (P, I, D) and the bias to the
+GPU, and then calls ``onexn_conv_fwd`` per forward pass.  Filter
+rearrangement (``onexn_rearrange``) is applied by the caller across a pair
+of layers before pruning, as in the paper's workflow (Sec. 3.3).
+"""
+from __future__ import annotations
+
+import numpy as np
+import torch
+
+from . import onexn as _c
+
+
+class PrunedConv2d:
+    def __init__(self, weight, N: int, rate: float, *, bias=None, stride=1, padding=0,
+                 dilation=1, dtype: str = "f32", gran: int = _c.ONEXN_GRAN_TAP,
+                 device="cuda", mask=None):
+        W = np.ascontiguousarray(np.asarray(weight, np.float32))
+        self.C_out, self.C_in, self.KH, self.KW = W.shape
+        self.N = int(N)
+        self.rate = float(rate)
+        self.dtype = dtype
+        self.cdtype = _c.ONEXN_F32 if dtype == "f32" else _c.ONEXN_BF16
+        self.stride = stride if isinstance(stride, (tuple, list)) else (stride, stride)
+        self.padding = padding if isinstance(padding, (tuple, list)) else (padding, padding)
+        self.dilation = dilation if isinstance(dilation, (tuple, list)) else (dilation, dilation)
+        if mask is None:
+            mask, self.kept = _c.onexn_prune(W, self.N, self.rate, gran)
+        else:
+            self.kept = None
+        self.mask = mask
+        P, I, D = _c.onexn_pack(W, mask, self.N, self.cdtype)
+        self.t = len(I)
+        _c.onexn_packed_validate(P, I, self.C_out // self.N, self.t, self.KH * self.KW * self.C_in)
+        self.P_host, self.I_host, self.D_host = P, I, D
+        dev = torch.device(device)
+        self.device = dev
+        self.P = torch.from_numpy(P).to(dev)
+        self.I = torch.from_numpy(np.ascontiguousarray(I) if self.t else np.zeros(1, np.int32)).to(dev)
+        if self.cdtype == _c.ONEXN_F32:
+            Dt = torch.from_numpy(D if self.t else np.zeros((1, self.N), np.float32))
+        else:
+            Dt = torch.from_numpy((D if self.t else np.zeros((1, self.N), np.uint16)).view(np.int16))
+            Dt = Dt.view(torch.bfloat16)
+        self.D = Dt.to(dev).contiguous()
+        self.bias = None if bias is None else torch.as_tensor(
+            np.asarray(bias, np.float32)).to(dev).contiguous()
+
+    @property
+    def torch_dtype(self):
+        return torch.float32 if self.cdtype == _c.ONEXN_F32 else torch.bfloat16
+
+    def desc(self, B: int, H: int, W: int) -> _c.ConvDesc:
+        return _c.make_desc(B, H, W, self.C_in, self.C_out, self.KH, self.KW, self.stride,
+                            self.padding, self.dilation)
+
+    def out_shape(self, x_shape):
+        B, H, W, _ = x_shape
+        Ho, Wo = _c.onexn_conv_out_shape(self.desc(B, H, W))
+        return (B, Ho, Wo, self.C_out)
+
+    def algo(self, x_shape, flags: int = 0) -> str:
+        B, H, W, _ = x_shape
+        a = _c.onexn_conv_algo(self.desc(B, H, W), self.N, self.t, self.cdtype, flags)
+        return _c.ALGO_NAMES[a]
+
+    def forward(self, x: torch.Tensor, y: torch.Tensor = None, relu: bool = False,
+                algo: int = _c.ONEXN_ALGO_AUTO, stream=None) -> torch.Tensor:
+        """x: NHWC CUDA tensor of this layer's dtype.  Returns y (NHWC)."""
+        if x.dtype != self.torch_dtype or not x.is_cuda or not x.is_contiguous():
+            raise ValueError(f"x must be a contiguous CUDA {self.torch_dtype} NHWC tensor")
+        B, H, W, C = x.shape
+        if C != self.C_in:
+            raise ValueError(f"x has {C} channels, layer expects {self.C_in}")
+        if y is None:
+            y = torch.empty(self.out_shape(x.shape), dtype=x.dtype, device=x.device)
+        flags = (_c.ONEXN_RELU if relu else 0) | algo
+        _c.onexn_conv_fwd(self.desc(B, H, W), self.P, self.I, self.D, self.N, self.t, x, y,
+                          self.bias, self.cdtype, flags, stream)
+        return y
+
+    __call__ = forward
+
+    def forward_host(self, x_host: torch.Tensor, relu: bool = False,
+                     algo: int = _c.ONEXN_ALGO_AUTO) -> torch.Tensor:
+        """End-to-end call from host memory: copy x in, convolve, copy y out."""
+        x = x_host.to(self.device, non_blocking=True)
+        y = self.forward(x, relu=relu, algo=algo)
+        out = torch.empty(y.shape, dtype=y.dtype, pin_memory=True)
+        out.copy_(y, non_blocking=True)
+        torch.cuda.current_stream(self.device).synchronize()
+        return out

@@ -1,0 +1,184 @@
+"""Thin ctypes binding of libonexn.so (include/onexn.h), same call names.
+
+Argument marshalling only: numpy arrays for the host calls, torch device
+tensors (pointers and the current CUDA stream) for ``onexn_conv_fwd``.  All
+arithmetic happens in the library.  Importing this module loads the shared
+library and fails loudly if it has not been built; there is no fallback.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+
+import numpy as np
+
+ONEXN_OK, ONEXN_EINVAL, ONEXN_EUNSUPPORTED, ONEXN_ENOMEM = 0, 1, 2, 3
+ONEXN_ECUDA, ONEXN_EDEVICE, ONEXN_ETIMEOUT = 4, 5, 6
+ONEXN_F32, ONEXN_BF16 = 0, 1
+ONEXN_GRAN_TAP, ONEXN_GRAN_KERNEL = 0, 1
+ONEXN_RELU = 0x1
+ONEXN_ALGO_SHIFT = 8
+ONEXN_ALGO_AUTO = 0 << ONEXN_ALGO_SHIFT
+ONEXN_ALGO_FMA = 1 << ONEXN_ALGO_SHIFT
+ONEXN_ALGO_MMA = 2 << ONEXN_ALGO_SHIFT
+ALGO_NAMES = {ONEXN_ALGO_FMA: "fma", ONEXN_ALGO_MMA: "mma"}
+
+_STATUS = {0: "OK", 1: "EINVAL", 2: "EUNSUPPORTED", 3: "ENOMEM", 4: "ECUDA", 5: "EDEVICE",
+           6: "ETIMEOUT"}
+
+_SO = os.path.join(os.path.dirname(os.path.abspath(__file__)), "_lib", "libonexn.so")
+
+# Every function the header declares, with its ctypes signature.
+_P = ctypes.c_void_p
+_I32, _I64, _DBL, _U32 = ctypes.c_int, ctypes.c_int64, ctypes.c_double, ctypes.c_uint
+
+
+class ConvDesc(ctypes.Structure):
+    """Mirror of onexn_conv_desc."""
+    _fields_ = [(n, ctypes.c_int) for n in (
+        "B", "H", "W", "C_in", "C_out", "KH", "KW",
+        "stride_h", "stride_w", "pad_h", "pad_w", "dil_h", "dil_w")]
+
+
+SIGNATURES = {
+    "onexn_last_error": ([], ctypes.c_char_p),
+    "onexn_version": ([], _I32),
+    "onexn_keep_count": ([_I64, _DBL, _P], _I32),
+    "onexn_prune": ([_P, _I32, _I32, _I32, _I32, _I32, _DBL, _I32, _P, _P], _I32),
+    "onexn_rearrange": ([_P, _I32, _I32, _I32, _I32, _P, _I32, _I32, _I32, _P], _I32),
+    "onexn_pack": ([_P, _P, _I32, _I32, _I32, _I32, _I32, _I32, _P, _P, _P, _I64, _P], _I32),
+    "onexn_packed_validate": ([_P, _P, _I32, _I64, _I32], _I32),
+    "onexn_conv_out_shape": ([ctypes.POINTER(ConvDesc), _P, _P], _I32),
+    "onexn_conv_fwd": ([ctypes.POINTER(ConvDesc), _P, _P, _P, _I32, _I64, _P, _P, _P, _I32,
+                        _U32, _P], _I32),
+    "onexn_conv_algo": ([ctypes.POINTER(ConvDesc), _I32, _I64, _I32, _U32, _P], _I32),
+}
+
+
+class OnexnError(RuntimeError):
+    def __init__(self, status: int, msg: str):
+        super().__init__(f"{_STATUS.get(status, status)}: {msg}")
+        self.status = status
+
+
+def _load():
+    if not os.path.exists(_SO):
+        raise ImportError(f"libonexn.so is not built ({_SO}); run __graft_entry__.build()")
+    lib = ctypes.CDLL(_SO)
+    for name, (args, res) in SIGNATURES.items():
+        fn = getattr(lib, name)
+        fn.argtypes = args
+        fn.restype = res
+    return lib
+
+
+lib = _load()
+LIB_PATH = _SO
+
+
+def _check(status: int):
+    if status != ONEXN_OK:
+        raise OnexnError(status, lib.onexn_last_error().decode())
+
+
+def _np_ptr(a):
+    return None if a is None else a.ctypes.data_as(ctypes.c_void_p)
+
+
+def _f32(a):
+    return np.ascontiguousarray(a, dtype=np.float32)
+
+
+def onexn_version() -> int:
+    return lib.onexn_version()
+
+
+def onexn_keep_count(total_blocks: int, rate: float) -> int:
+    out = ctypes.c_int64(0)
+    _check(lib.onexn_keep_count(int(total_blocks), float(rate), ctypes.byref(out)))
+    return out.value
+
+
+def onexn_prune(W, N: int, rate: float, gran: int = ONEXN_GRAN_TAP):
+    """Host W [C_out, C_in, KH, KW] fp32 -> (mask uint8 [G, KH*KW*C_in], kept)."""
+    W = _f32(W)
+    C_out, C_in, KH, KW = W.shape
+    G = C_out // N if N > 0 else 0
+    mask = np.empty((max(G, 1), KH * KW * C_in), np.uint8)
+    kept = ctypes.c_int64(0)
+    _check(lib.onexn_prune(_np_ptr(W), C_out, C_in, KH, KW, int(N), float(rate), int(gran),
+                           _np_ptr(mask), ctypes.byref(kept)))
+    return mask, kept.value
+
+
+def onexn_rearrange(W_l, W_next=None):
+    """Returns (W_l', W_next' or None, perm); inputs are copied, not modified."""
+    W_l = np.array(W_l, dtype=np.float32, order="C", copy=True)
+    C_out, C_in, KH, KW = W_l.shape
+    perm = np.empty(C_out, np.int32)
+    if W_next is not None:
+        W_next = np.array(W_next, dtype=np.float32, order="C", copy=True)
+        Cn, Cin_n, KHn, KWn = W_next.shape
+        if Cin_n != C_out:
+            raise OnexnError(ONEXN_EINVAL, "next layer's C_in differs from C_out")
+    else:
+        Cn = KHn = KWn = 0
+    _check(lib.onexn_rearrange(_np_ptr(W_l), C_out, C_in, KH, KW, _np_ptr(W_next), Cn, KHn, KWn,
+                               _np_ptr(perm)))
+    return W_l, W_next, perm
+
+
+def onexn_pack(W, mask, N: int, wdtype: int = ONEXN_F32):
+    """BSR encoding -> (P int32 [G+1], I int32 [t], D [t, N] float32 or uint16 bf16 bits)."""
+    W = _f32(W)
+    mask = np.ascontiguousarray(mask, dtype=np.uint8)
+    C_out, C_in, KH, KW = W.shape
+    G = C_out // N
+    t_cap = int(mask.sum())
+    P = np.empty(G + 1, np.int32)
+    I = np.empty(max(t_cap, 1), np.int32)
+    D = np.empty((max(t_cap, 1), N), np.float32 if wdtype == ONEXN_F32 else np.uint16)
+    t = ctypes.c_int64(0)
+    _check(lib.onexn_pack(_np_ptr(W), _np_ptr(mask), C_out, C_in, KH, KW, int(N), int(wdtype),
+                          _np_ptr(P), _np_ptr(I), _np_ptr(D), t_cap, ctypes.byref(t)))
+    return P, I[:t.value].copy(), D[:t.value].copy()
+
+
+def onexn_packed_validate(P, I, G: int, t: int, K: int) -> None:
+    P = np.ascontiguousarray(P, np.int32)
+    I = np.ascontiguousarray(I, np.int32)
+    _check(lib.onexn_packed_validate(_np_ptr(P), _np_ptr(I) if I.size else None, int(G), int(t),
+                                     int(K)))
+
+
+def make_desc(B, H, W, C_in, C_out, KH=1, KW=1, stride=(1, 1), pad=(0, 0), dil=(1, 1)):
+    s = stride if isinstance(stride, (tuple, list)) else (stride, stride)
+    p = pad if isinstance(pad, (tuple, list)) else (pad, pad)
+    d = dil if isinstance(dil, (tuple, list)) else (dil, dil)
+    return ConvDesc(B, H, W, C_in, C_out, KH, KW, s[0], s[1], p[0], p[1], d[0], d[1])
+
+
+def onexn_conv_out_shape(desc: ConvDesc):
+    ho, wo = ctypes.c_int(0), ctypes.c_int(0)
+    _check(lib.onexn_conv_out_shape(ctypes.byref(desc), ctypes.byref(ho), ctypes.byref(wo)))
+    return ho.value, wo.value
+
+
+def onexn_conv_algo(desc: ConvDesc, N: int, t: int, dtype: int, flags: int = 0) -> int:
+    out = ctypes.c_uint(0)
+    _check(lib.onexn_conv_algo(ctypes.byref(desc), int(N), int(t), int(dtype), int(flags),
+                               ctypes.byref(out)))
+    return out.value
+
+
+def onexn_conv_fwd(desc: ConvDesc, P, I, D, N: int, t: int, x, y, bias, dtype: int,
+                   flags: int = 0, stream=None) -> None:
+    """Launch the convolution.  P, I, D, x, y, bias are torch CUDA tensors
+    (bias may be None); stream is a torch.cuda.Stream or None (current)."""
+    import torch
+    if stream is None:
+        stream = torch.cuda.current_stream(x.device)
+    ptr = (lambda tns: None if tns is None else ctypes.c_void_p(tns.data_ptr()))
+    _check(lib.onexn_conv_fwd(ctypes.byref(desc), ptr(P), ptr(I), ptr(D), int(N), int(t), ptr(x),
+                              ptr(y), ptr(bias), int(dtype), int(flags),
+                              ctypes.c_void_p(stream.cuda_stream)))

@@ -1,0 +1,130 @@
+"""GPU parity of onexn_conv_fwd against the fp64 oracle (Eq. 6 / Eq. 7).
+
+Small cases span several 128-pixel tiles, several column tiles and a ragged
+tail; every geometry feature (stride, padding, dilation, non-square
+kernels, partial channel chunks) and every block width class is covered, for
+each kernel family that can run the case.  Tolerances: fp32 1e-5 and bf16
+1e-2 (fp32 master inputs) / 2.5e-3 (bf16-rounded inputs), normalised by
+sum |w x| + |b|."""
+import numpy as np
+import pytest
+import torch
+
+from paper_2105_14713_gb300 import onexn as ox
+from paper_2105_14713_gb300 import workloads as wl
+from tests.gpu_util import norm_err, run_layer, tol
+
+pytestmark = pytest.mark.gpu
+
+L = wl.ConvLayer
+
+GEOMS = [
+    # name, B, H, W, C_in, C_out, KH, KW, stride, pad, dil
+    ("1x1", 3, 13, 11, 64, 64, 1, 1, 1, 0, 1),
+    ("1x1_c24", 2, 17, 9, 24, 48, 1, 1, 1, 0, 1),
+    ("1x1_s2", 2, 15, 15, 40, 32, 1, 1, 2, 0, 1),
+    ("3x3_p1", 2, 14, 14, 64, 64, 3, 3, 1, 1, 1),
+    ("3x3_s2", 3, 15, 13, 32, 64, 3, 3, 2, 1, 1),
+    ("3x3_d2", 2, 16, 16, 48, 32, 3, 3, 1, 2, 2),
+    ("1x3", 2, 9, 20, 16, 32, 1, 3, 1, 1, 1),
+    ("5x5_p0", 1, 20, 20, 8, 32, 5, 5, 1, 0, 1),
+]
+
+ALGOS = {"fma": ox.ONEXN_ALGO_FMA, "mma": ox.ONEXN_ALGO_MMA, "auto": ox.ONEXN_ALGO_AUTO}
+
+
+def _algos_for(dtype, N):
+    out = ["auto", "fma"]
+    if dtype == "bf16" and N % 8 == 0:
+        probe = ox.make_desc(1, 8, 8, 8, N, 1, 1)
+        try:
+            ox.onexn_conv_algo(probe, N, 1, ox.ONEXN_BF16, ox.ONEXN_ALGO_MMA)
+            out.append("mma")
+        except ox.OnexnError:
+            pass
+    return out
+
+
+@pytest.mark.parametrize("geom", GEOMS, ids=[g[0] for g in GEOMS])
+@pytest.mark.parametrize("N", [1, 2, 4, 8, 16, 32])
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+def test_geometry_and_block_width(geom, N, dtype):
+    name, B, H, W, Ci, Co, KH, KW, s, p, d = geom
+    if Co % N:
+        pytest.skip("N must divide C_out")
+    layer = L(name, B, H, W, Ci, Co, KH, KW, s, p, d, N=N, rate=0.5, dtype=dtype, seed=N)
+    for algo in _algos_for(dtype, N):
+        y, yr, a, conv = run_layer(layer, relu=(N % 2 == 0), algo=ALGOS[algo])
+        e = norm_err(y, yr, a)
+        assert e <= tol(layer), f"{algo}: err {e:.3e}"
+
+
+@pytest.mark.parametrize("rate", [0.0, 0.3, 0.7, 0.9, 1.0])
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+def test_rates(rate, dtype):
+    layer = L("rates", 2, 12, 12, 64, 128, 3, 3, 1, 1, 1, N=8, rate=rate, dtype=dtype, seed=3)
+    for algo in _algos_for(dtype, 8):
+        y, yr, a, _ = run_layer(layer, relu=True, algo=ALGOS[algo])
+        assert norm_err(y, yr, a) <= tol(layer)
+
+
+@pytest.mark.parametrize("N", [3, 5, 6, 12, 24, 64, 128])
+def test_odd_and_wide_blocks(N):
+    Co = 120 if N in (3, 5, 6, 12, 24) else N * 2
+    layer = L("oddN", 2, 10, 10, 32, Co, 3, 3, 1, 1, 1, N=N, rate=0.4, dtype="f32", seed=N)
+    y, yr, a, _ = run_layer(layer, algo=ox.ONEXN_ALGO_FMA)
+    assert norm_err(y, yr, a) <= 1e-5
+
+
+def test_odd_output_channels_scalar_stores():
+    layer = L("co6", 2, 9, 9, 16, 6, 1, 1, N=2, rate=0.5, dtype="f32", seed=1)
+    y, yr, a, _ = run_layer(layer)
+    assert norm_err(y, yr, a) <= 1e-5
+
+
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+def test_dense_path_rate0_N_equals_cout(dtype):
+    layer = L("dense", 2, 14, 14, 64, 128, 3, 3, 1, 1, 1, N=128, rate=0.0, dtype=dtype, seed=5)
+    y, yr, a, conv = run_layer(layer)
+    assert conv.t == 576
+    assert norm_err(y, yr, a) <= tol(layer)
+
+
+def test_bf16_against_fp32_master_inputs():
+    layer = L("master", 2, 14, 14, 64, 64, 3, 3, 1, 1, 1, N=8, rate=0.5, dtype="bf16", seed=6)
+    y, yr, a, _ = run_layer(layer, relu=True, master=True)
+    assert norm_err(y, yr, a) <= 1e-2
+
+
+def test_kernel_granularity_mode():
+    """The paper's own block (N whole KH x KW kernels of one channel)."""
+    layer = L("gran", 2, 12, 12, 32, 64, 3, 3, 1, 1, 1, N=4, rate=0.5, dtype="f32", seed=7)
+    y, yr, a, conv = run_layer(layer, gran=ox.ONEXN_GRAN_KERNEL)
+    assert conv.t == conv.kept * 9
+    assert norm_err(y, yr, a) <= 1e-5
+
+
+def test_empty_batch_and_no_bias():
+    layer = L("empty", 0, 8, 8, 16, 16, 3, 3, 1, 1, 1, N=4, rate=0.5, dtype="f32")
+    W = wl.weights(layer).numpy()
+    from paper_2105_14713_gb300.layer import PrunedConv2d
+    conv = PrunedConv2d(W, 4, 0.5, padding=1)
+    x = torch.zeros((0, 8, 8, 16), device="cuda")
+    y = conv(x)
+    assert tuple(y.shape) == (0, 8, 8, 16)
+    layer2 = layer.with_(B=1)
+    y, yr, a, _ = run_layer(layer2, with_bias=False)
+    assert norm_err(y, yr, a) <= 1e-5
+
+
+def test_streams_and_repeat_calls_are_deterministic():
+    layer = L("det", 4, 16, 16, 64, 64, 3, 3, 1, 1, 1, N=8, rate=0.5, dtype="f32", seed=8)
+    from paper_2105_14713_gb300.layer import PrunedConv2d
+    conv = PrunedConv2d(wl.weights(layer).numpy(), 8, 0.5, padding=1, bias=wl.bias(layer).numpy())
+    x = wl.activations(layer).cuda()
+    s = torch.cuda.Stream()
+    with torch.cuda.stream(s):
+        y1 = conv(x)
+        y2 = conv(x)
+    s.synchronize()
+    assert torch.equal(y1, y2)

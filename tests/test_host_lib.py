@@ -1,0 +1,177 @@
+"""Host side of the C ABI (no GPU): prune / rearrange / pack / validate are
+bit-exact against the oracle, argument errors are reported as status codes,
+and the shared library exports every symbol include/onexn.h declares."""
+import ctypes
+import os
+import re
+
+import numpy as np
+import pytest
+
+import oracle
+from paper_2105_14713_gb300 import onexn as ox
+from paper_2105_14713_gb300 import workloads as wl
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+def _declared_functions():
+    src = open(os.path.join(ROOT, "include", "onexn.h")).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"\b(onexn_\w+)\s*\(", src)))
+
+
+def test_library_exports_every_declared_symbol():
+    names = _declared_functions()
+    assert "onexn_conv_fwd" in names and "onexn_prune" in names
+    lib = ctypes.CDLL(ox.LIB_PATH)
+    for n in names:
+        assert hasattr(lib, n), f"{n} declared in onexn.h but not exported"
+    assert set(names) == set(ox.SIGNATURES), "binding and header disagree"
+
+
+SHAPES = [((8, 6, 3, 3), 4), ((8, 6, 3, 3), 2), ((64, 64, 1, 1), 4), ((128, 128, 3, 3), 8),
+          ((32, 24, 1, 3), 16), ((12, 5, 2, 2), 3), ((16, 16, 3, 3), 16), ((24, 40, 1, 1), 1)]
+
+
+@pytest.mark.parametrize("shape,N", SHAPES)
+@pytest.mark.parametrize("rate", [0.0, 0.3, 0.5, 0.7, 0.9, 1.0])
+@pytest.mark.parametrize("gran", [ox.ONEXN_GRAN_TAP, ox.ONEXN_GRAN_KERNEL])
+def test_prune_and_pack_bitexact_vs_oracle(shape, N, rate, gran):
+    rng = np.random.default_rng(hash((shape, N)) % 2**32)
+    W = rng.standard_normal(shape).astype(np.float32)
+    m_lib, k_lib = ox.onexn_prune(W, N, rate, gran)
+    m_or, k_or = oracle.prune(W, N, rate, gran)
+    assert k_lib == k_or
+    np.testing.assert_array_equal(m_lib, m_or)
+    for wdt, odt in ((ox.ONEXN_F32, "f32"), (ox.ONEXN_BF16, "bf16")):
+        P, I, D = ox.onexn_pack(W, m_lib, N, wdt)
+        Po, Io, Do = oracle.pack(W, m_or, N, odt)
+        np.testing.assert_array_equal(P, Po)
+        np.testing.assert_array_equal(I, Io)
+        np.testing.assert_array_equal(D, Do)
+        ox.onexn_packed_validate(P, I, shape[0] // N, len(I), shape[1] * shape[2] * shape[3])
+
+
+def test_prune_ties_integer_weights_bitexact():
+    rng = np.random.default_rng(9)
+    for N in (1, 2, 4):
+        W = rng.integers(-2, 3, size=(16, 12, 3, 3)).astype(np.float32)
+        for rate in (0.25, 0.5, 0.75):
+            for gran in (0, 1):
+                a, ka = ox.onexn_prune(W, N, rate, gran)
+                b, kb = oracle.prune(W, N, rate, gran)
+                assert ka == kb
+                np.testing.assert_array_equal(a, b)
+
+
+@pytest.mark.parametrize("total", [1, 5, 9216, 147456, 4718592])
+@pytest.mark.parametrize("rate", [0.0, 0.3, 0.5, 0.7, 0.9, 1.0, 0.123456789])
+def test_keep_count_matches_oracle(total, rate):
+    assert ox.onexn_keep_count(total, rate) == oracle.keep_count(total, rate)
+
+
+@pytest.mark.parametrize("with_next", [False, True])
+def test_rearrange_bitexact_vs_oracle(with_next):
+    rng = np.random.default_rng(4)
+    W = rng.standard_normal((48, 16, 3, 3)).astype(np.float32)
+    W[5] = W[9]                        # a tie: stable order must keep 5 before 9
+    Wn = rng.standard_normal((20, 48, 1, 1)).astype(np.float32) if with_next else None
+    a, an, pa = ox.onexn_rearrange(W, Wn)
+    b, bn, pb = oracle.rearrange(W, Wn)
+    np.testing.assert_array_equal(pa, pb)
+    np.testing.assert_array_equal(a, b)
+    if with_next:
+        np.testing.assert_array_equal(an, bn)
+    assert list(pa).index(5) < list(pa).index(9)
+
+
+def test_workload_config_shapes():
+    c3 = wl.config3()
+    assert len(c3) == 34 and c3[-1].C_out == 1280 and c3[0].H == 112
+    c4 = wl.config4()
+    assert len(c4) == 52 and sum(1 for l in c4 if l.KH == 3) == 16
+    assert all(l.C_out % l.N == 0 for l in c3 + c4)
+    assert wl.config2()[0].pixels == 64 * 28 * 28
+
+
+def test_mbv2_keep_counts_closed_form():
+    """kept = round((1 - rate) * C_out/N * C_in*KH*KW) on every MBv2 1x1 layer."""
+    for layer in wl.config3()[:6]:
+        W = wl.weights(layer.with_(B=1)).numpy()
+        _, kept = ox.onexn_prune(W, layer.N, layer.rate)
+        total = layer.C_out // layer.N * layer.K
+        assert kept == int(np.floor((1 - layer.rate) * total + 0.5))
+
+
+# ---------------------------------------------------------------- errors
+
+def _status(fn, *a):
+    with pytest.raises(ox.OnexnError) as e:
+        fn(*a)
+    return e.value.status
+
+
+def test_prune_argument_errors():
+    W = np.ones((6, 4, 1, 1), np.float32)
+    assert _status(ox.onexn_prune, W, 4, 0.5) == ox.ONEXN_EINVAL         # N does not divide
+    assert _status(ox.onexn_prune, W, 3, -0.1) == ox.ONEXN_EINVAL
+    assert _status(ox.onexn_prune, W, 3, 1.1) == ox.ONEXN_EINVAL
+    assert _status(ox.onexn_prune, W, 0, 0.5) == ox.ONEXN_EINVAL
+    assert _status(ox.onexn_prune, W, 3, 0.5, 7) == ox.ONEXN_EINVAL      # granularity
+    assert ox.lib.onexn_prune(None, 6, 4, 1, 1, 3, 0.5, 0, None, None) == ox.ONEXN_EINVAL
+    assert b"NULL" in ox.lib.onexn_last_error()
+
+
+def test_pack_errors():
+    W = np.ones((4, 2, 1, 1), np.float32)
+    mask = np.ones((2, 2), np.uint8)
+    P = np.zeros(3, np.int32)
+    I = np.zeros(4, np.int32)
+    D = np.zeros((4, 2), np.float32)
+    t = ctypes.c_int64(0)
+    p = lambda a: a.ctypes.data_as(ctypes.c_void_p)
+    st = ox.lib.onexn_pack(p(W), p(mask), 4, 2, 1, 1, 2, 0, p(P), p(I), p(D), 3, ctypes.byref(t))
+    assert st == ox.ONEXN_EINVAL and t.value == 4                       # t_cap too small
+    mask[0, 0] = 2
+    st = ox.lib.onexn_pack(p(W), p(mask), 4, 2, 1, 1, 2, 0, p(P), p(I), p(D), 4, ctypes.byref(t))
+    assert st == ox.ONEXN_EINVAL
+    st = ox.lib.onexn_pack(p(W), p(mask), 4, 2, 1, 1, 2, 5, p(P), p(I), p(D), 4, ctypes.byref(t))
+    assert st == ox.ONEXN_EINVAL                                         # dtype
+
+
+@pytest.mark.parametrize("P,I,G,t,K,frag", [
+    ([1, 2], [0, 1], 1, 2, 4, "P[0]"),
+    ([0, 3], [0, 1, 2], 1, 2, 4, "P[G]"),
+    ([0, 2, 1], [0, 1], 2, 1, 4, "decreases"),
+    ([0, 2], [1, 1], 1, 2, 4, "increasing"),
+    ([0, 2], [0, 4], 1, 2, 4, "outside"),
+    ([0, 1], [-1], 1, 1, 4, "outside"),
+])
+def test_validate_catches_corrupted_bsr(P, I, G, t, K, frag):
+    with pytest.raises(ox.OnexnError) as e:
+        ox.onexn_packed_validate(np.array(P), np.array(I), G, t, K)
+    assert frag in str(e.value)
+
+
+def test_conv_shape_and_argument_errors_need_no_gpu():
+    d = ox.make_desc(2, 7, 7, 8, 16, 3, 3, 2, 1, 1)
+    assert ox.onexn_conv_out_shape(d) == (4, 4)
+    assert ox.onexn_conv_algo(d, 8, 100, ox.ONEXN_F32) == ox.ONEXN_ALGO_FMA
+    bad = ox.make_desc(1, 2, 2, 8, 16, 5, 5)
+    assert _status(ox.onexn_conv_out_shape, bad) == ox.ONEXN_EINVAL
+    assert _status(ox.onexn_conv_algo, d, 3, 10, ox.ONEXN_F32) == ox.ONEXN_EINVAL    # N | C_out
+    d6 = ox.make_desc(1, 4, 4, 6, 16)
+    assert _status(ox.onexn_conv_algo, d6, 8, 10, ox.ONEXN_F32) == ox.ONEXN_EINVAL   # C_in % 4
+    assert _status(ox.onexn_conv_algo, d, 8, 10**9, ox.ONEXN_F32) == ox.ONEXN_EINVAL  # t > G*K
+    assert _status(ox.onexn_conv_algo, d, 8, 10, 7) == ox.ONEXN_EINVAL               # dtype
+    assert _status(ox.onexn_conv_algo, d, 8, 10, 0, 1 << 20) == ox.ONEXN_EINVAL      # flags
+    # conv_fwd rejects bad pointers before touching the GPU
+    st = ox.lib.onexn_conv_fwd(ctypes.byref(d), None, None, None, 8, 0, None, None, None, 0, 0,
+                               None)
+    assert st == ox.ONEXN_EINVAL
+    buf = (ctypes.c_char * 64)()
+    base = ctypes.addressof(buf)
+    mis = ctypes.c_void_p(base + (16 - base % 16) % 16 + 4)
+    st = ox.lib.onexn_conv_fwd(ctypes.byref(d), mis, mis, mis, 8, 1, mis, mis, None, 0, 0, None)
+    assert st == ox.ONEXN_EINVAL and b"aligned" in ox.lib.onexn_last_error()
