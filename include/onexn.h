@@ -195,6 +195,18 @@ onexn_status onexn_conv_fwd(const onexn_conv_desc *desc, const int32_t *P, const
 onexn_status onexn_conv_algo(const onexn_conv_desc *desc, int N, int64_t t, int dtype,
                              unsigned flags, unsigned *algo);
 
+/*
+ * onexn_device_status -- read, and clear if `clear` is non-zero, the status
+ * word that the kernels of this library keep on the current device (a
+ * 4-byte __device__ variable of the library).  A kernel whose bounded
+ * internal wait (about one second) runs out sets it and returns early, so
+ * its output is not valid.  Synchronises the device first.
+ *   *status = ONEXN_OK (nothing reported since the last clear) or
+ *             ONEXN_ETIMEOUT.
+ * ECUDA if a runtime call fails (for instance an earlier kernel fault).
+ */
+onexn_status onexn_device_status(int clear, int *status);
+
 #ifdef __cplusplus
 }
 #endif

@@ -23,9 +23,73 @@ struct ConvArgs {
     int t;                  // number of kept blocks (entries of I / rows of D)
     int P_pix;              // B * Ho * Wo
     int relu;
+    unsigned int *status;   // library status word (device): bits set by kernels on failure
 };
 
+// Bits of the device status word (read by onexn_device_status).
+constexpr unsigned int kStatusTimeout = 1u;
+
+// Host: SM count of the current device (cached per device).
+cudaError_t device_sm_count(int *sms);
+// Host: device address of the status word of the current device.
+cudaError_t device_status_ptr(unsigned int **p);
+
 __device__ __forceinline__ int clampi(int v, int lo, int hi) { return min(max(v, lo), hi); }
+
+__device__ __forceinline__ uint32_t smem_u32(const void *p)
+{
+    return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+
+// ---- cp.async (16 bytes, L2 only; src_bytes = 0 zero-fills the destination) ----
+__device__ __forceinline__ void cp_async16(uint32_t dst, const void *src, int src_bytes)
+{
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;\n" ::"r"(dst), "l"(src),
+                 "r"(src_bytes)
+                 : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;\n" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_group %0;\n" ::"n"(N) : "memory"); }
+
+// ---- mbarriers (CTA scope) ----
+__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count)
+{
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;\n" ::"r"(bar), "r"(count) : "memory");
+}
+__device__ __forceinline__ void fence_mbar_init()
+{
+    asm volatile("fence.mbarrier_init.release.cluster;\n" ::: "memory");
+}
+__device__ __forceinline__ void mbar_arrive(uint32_t bar)
+{
+    asm volatile("{\n\t.reg .b64 st;\n\tmbarrier.arrive.shared::cta.b64 st, [%0];\n\t}\n" ::"r"(bar)
+                 : "memory");
+}
+// One bounded try: the warp is suspended until the phase completes or about
+// 0.1 ms pass (suspend-time hint), so waiting warps do not take issue slots.
+__device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity)
+{
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\tmbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}\n"
+        : "=r"(ok)
+        : "r"(bar), "r"(parity), "r"(100000u)
+        : "memory");
+    return ok != 0;
+}
+// Wait for the phase with the given parity to complete, for at most ~2^31
+// SM cycles (about one second).  Returns false on expiry.
+__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity)
+{
+    if (mbar_try_wait(bar, parity)) return true;
+    const long long t0 = clock64();
+    while (!mbar_try_wait(bar, parity)) {
+        if (clock64() - t0 > (1ll << 31)) return false;
+    }
+    return true;
+}
 
 // bf16 bits -> fp32 (exact).
 __device__ __forceinline__ float bf16lo(uint32_t v) { return __uint_as_float(v << 16); }

@@ -4,6 +4,8 @@
 #include "conv_common.cuh"
 #include "onexn_internal.h"
 
+#include <mutex>
+
 namespace onexn {
 cudaError_t launch_fma(const ConvArgs &a, int dtype, cudaStream_t st);
 cudaError_t launch_mma(const ConvArgs &a, cudaStream_t st);
@@ -11,6 +13,53 @@ bool mma_supports(const ConvArgs &a);
 }  // namespace onexn
 
 using onexn::fail;
+
+// Status word written by kernels that hit a bounded wait (one per device,
+// 4 bytes, lives as long as the library is loaded).
+__device__ unsigned int g_onexn_status_word;
+
+namespace onexn {
+
+namespace {
+constexpr int kMaxDevices = 64;
+std::mutex g_dev_mu;
+int g_sm_count[kMaxDevices];
+unsigned int *g_status_ptr[kMaxDevices];
+}  // namespace
+
+cudaError_t device_sm_count(int *sms)
+{
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    if (dev < 0 || dev >= kMaxDevices) return cudaErrorInvalidDevice;
+    std::lock_guard<std::mutex> lk(g_dev_mu);
+    if (g_sm_count[dev] == 0) {
+        e = cudaDeviceGetAttribute(&g_sm_count[dev], cudaDevAttrMultiProcessorCount, dev);
+        if (e != cudaSuccess) return e;
+    }
+    *sms = g_sm_count[dev];
+    return cudaSuccess;
+}
+
+cudaError_t device_status_ptr(unsigned int **p)
+{
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    if (dev < 0 || dev >= kMaxDevices) return cudaErrorInvalidDevice;
+    std::lock_guard<std::mutex> lk(g_dev_mu);
+    if (!g_status_ptr[dev]) {
+        void *ptr = nullptr;
+        e = cudaGetSymbolAddress(&ptr, g_onexn_status_word);
+        if (e != cudaSuccess) return e;
+        g_status_ptr[dev] = static_cast<unsigned int *>(ptr);
+    }
+    *p = g_status_ptr[dev];
+    return cudaSuccess;
+}
+
+}  // namespace onexn
 
 namespace {
 
@@ -114,7 +163,8 @@ extern "C" onexn_status onexn_conv_fwd(const onexn_conv_desc *desc, const int32_
     if (st != ONEXN_OK) return st;
     const unsigned algo = pick_algo(a, dtype, flags);
     cudaStream_t s = static_cast<cudaStream_t>(stream);
-    cudaError_t e;
+    cudaError_t e = onexn::device_status_ptr(&a.status);
+    if (e != cudaSuccess) return fail(ONEXN_ECUDA, "conv: status word: %s", cudaGetErrorString(e));
     if (algo == ONEXN_ALGO_FMA) {
         e = onexn::launch_fma(a, dtype, s);
     } else if (algo == ONEXN_ALGO_MMA) {
@@ -125,5 +175,20 @@ extern "C" onexn_status onexn_conv_fwd(const onexn_conv_desc *desc, const int32_
         return fail(ONEXN_EINVAL, "conv: unknown algo %u", algo >> ONEXN_ALGO_SHIFT);
     }
     if (e != cudaSuccess) return fail(ONEXN_ECUDA, "conv: launch failed: %s", cudaGetErrorString(e));
+    return ONEXN_OK;
+}
+
+extern "C" onexn_status onexn_device_status(int clear, int *status)
+{
+    onexn::clear_error();
+    if (!status) return fail(ONEXN_EINVAL, "device_status: status is NULL");
+    unsigned int *p = nullptr;
+    cudaError_t e = onexn::device_status_ptr(&p);
+    if (e == cudaSuccess) e = cudaDeviceSynchronize();
+    unsigned int w = 0;
+    if (e == cudaSuccess) e = cudaMemcpy(&w, p, sizeof(w), cudaMemcpyDeviceToHost);
+    if (e == cudaSuccess && clear) e = cudaMemset(p, 0, sizeof(w));
+    if (e != cudaSuccess) return fail(ONEXN_ECUDA, "device_status: %s", cudaGetErrorString(e));
+    *status = (w & onexn::kStatusTimeout) ? ONEXN_ETIMEOUT : ONEXN_OK;
     return ONEXN_OK;
 }

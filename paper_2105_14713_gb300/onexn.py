@@ -52,6 +52,7 @@ SIGNATURES = {
     "onexn_conv_fwd": ([ctypes.POINTER(ConvDesc), _P, _P, _P, _I32, _I64, _P, _P, _P, _I32,
                         _U32, _P], _I32),
     "onexn_conv_algo": ([ctypes.POINTER(ConvDesc), _I32, _I64, _I32, _U32, _P], _I32),
+    "onexn_device_status": ([_I32, _P], _I32),
 }
 
 
@@ -182,3 +183,10 @@ def onexn_conv_fwd(desc: ConvDesc, P, I, D, N: int, t: int, x, y, bias, dtype: i
     _check(lib.onexn_conv_fwd(ctypes.byref(desc), ptr(P), ptr(I), ptr(D), int(N), int(t), ptr(x),
                               ptr(y), ptr(bias), int(dtype), int(flags),
                               ctypes.c_void_p(stream.cuda_stream)))
+
+
+def onexn_device_status(clear: bool = True) -> int:
+    """ONEXN_OK or ONEXN_ETIMEOUT (a bounded in-kernel wait ran out)."""
+    st = ctypes.c_int(0)
+    _check(lib.onexn_device_status(int(bool(clear)), ctypes.byref(st)))
+    return st.value

@@ -28,7 +28,7 @@ def oracle_input(x_cpu: torch.Tensor, dtype: str) -> np.ndarray:
     return x if dtype == "f32" else oracle.round_bf16(x)
 
 
-TOL_BF16_ROUNDED = 2.5e-3   # bf16 output rounding (2^-9 relative) + fp32 accumulation
+TOL_BF16_ROUNDED = 4e-3     # bf16 output rounding (2^-8 relative, 8 significant bits) + fp32 accumulation
 
 
 def oracle_ref(layer, W, x_cpu, b, *, relu=False, pixels=None, gran=ox.ONEXN_GRAN_TAP,

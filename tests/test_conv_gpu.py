@@ -4,7 +4,7 @@ Small cases span several 128-pixel tiles, several column tiles and a ragged
 tail; every geometry feature (stride, padding, dilation, non-square
 kernels, partial channel chunks) and every block width class is covered, for
 each kernel family that can run the case.  Tolerances: fp32 1e-5 and bf16
-1e-2 (fp32 master inputs) / 2.5e-3 (bf16-rounded inputs), normalised by
+1e-2 (fp32 master inputs) / 4e-3 = 2^-8 output rounding (bf16-rounded inputs), normalised by
 sum |w x| + |b|."""
 import numpy as np
 import pytest
