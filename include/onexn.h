@@ -63,7 +63,8 @@ typedef enum { ONEXN_GRAN_TAP = 0, ONEXN_GRAN_KERNEL = 1 } onexn_granularity;
 #define ONEXN_ALGO_MASK (0xFu << ONEXN_ALGO_SHIFT)
 #define ONEXN_ALGO_AUTO (0u << ONEXN_ALGO_SHIFT)
 #define ONEXN_ALGO_FMA (1u << ONEXN_ALGO_SHIFT)   /* CUDA-core FFMA, any N, fp32/bf16 */
-#define ONEXN_ALGO_MMA (2u << ONEXN_ALGO_SHIFT)   /* bf16 tensor cores, N % 8 == 0 */
+#define ONEXN_ALGO_MMA (2u << ONEXN_ALGO_SHIFT)   /* bf16 gathered tensor-core kernel */
+#define ONEXN_ALGO_TC (3u << ONEXN_ALGO_SHIFT)    /* bf16 tcgen05 GEMM on the decoded mask */
 
 /* Message for the last failed call on this thread ("" if none). */
 const char *onexn_last_error(void);
@@ -177,23 +178,41 @@ onexn_status onexn_conv_out_shape(const onexn_conv_desc *desc, int *Ho, int *Wo)
  *   dtype   ONEXN_F32: fp32 inputs and weights, fp32 accumulation.
  *           ONEXN_BF16: bf16 inputs and weights, fp32 accumulation.
  *   flags   ONEXN_RELU | one ONEXN_ALGO_* value.
+ *   workspace, workspace_bytes
+ *           nullable DEVICE scratch owned by the caller, 256-byte aligned.
+ *           Some kernel families need it (onexn_conv_workspace_size); the
+ *           call overwrites it, so calls that run concurrently need
+ *           separate workspaces.  AUTO only picks a family whose workspace
+ *           fits in workspace_bytes.
  *   stream  cudaStream_t to launch on (NULL = legacy default stream).
  * Asynchronous: returns after the launch; errors of the launch itself are
  * returned as ECUDA.  No allocation, no synchronisation, no host read of
  * device memory.  EINVAL: bad geometry, N not dividing C_out, alignment,
- * NULL pointers.  EUNSUPPORTED: the forced ALGO cannot run this case.
+ * NULL pointers, a forced ALGO whose workspace does not fit.
+ * EUNSUPPORTED: the forced ALGO cannot run this case.
  */
 onexn_status onexn_conv_fwd(const onexn_conv_desc *desc, const int32_t *P, const int32_t *I,
                             const void *D, int N, int64_t t, const void *x, void *y,
-                            const float *bias, int dtype, unsigned flags, void *stream);
+                            const float *bias, int dtype, unsigned flags, void *workspace,
+                            size_t workspace_bytes, void *stream);
+
+/*
+ * onexn_conv_workspace_size -- bytes of device workspace onexn_conv_fwd
+ * needs for these arguments with this flags' ALGO (for AUTO: the largest
+ * need among the families AUTO may pick, so that passing this many bytes
+ * lets AUTO choose freely).  ONEXN_ALGO_TC needs C_out * KH*KW*C_in
+ * bf16 values (the decoded masked weights); ONEXN_ALGO_FMA needs none.
+ */
+onexn_status onexn_conv_workspace_size(const onexn_conv_desc *desc, int N, int64_t t, int dtype,
+                                       unsigned flags, size_t *bytes);
 
 /*
  * onexn_conv_algo -- which kernel family onexn_conv_fwd would run for these
- * arguments (an ONEXN_ALGO_* value other than AUTO), without launching.
- * EINVAL / EUNSUPPORTED as onexn_conv_fwd.
+ * arguments and this much workspace (an ONEXN_ALGO_* value other than
+ * AUTO), without launching.  EINVAL / EUNSUPPORTED as onexn_conv_fwd.
  */
 onexn_status onexn_conv_algo(const onexn_conv_desc *desc, int N, int64_t t, int dtype,
-                             unsigned flags, unsigned *algo);
+                             unsigned flags, size_t workspace_bytes, unsigned *algo);
 
 /*
  * onexn_device_status -- read, and clear if `clear` is non-zero, the status

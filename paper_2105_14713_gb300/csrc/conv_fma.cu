@@ -227,7 +227,7 @@ fma_conv_kernel(const ConvArgs a, const int n_units, const int n_ct)
         const int pix0 = pt * kMT;
         // Per slice: kept-list cursor, and the next <= 32 candidate entries
         // prefetched one chunk ahead: lane j holds I[z+j] and D[z+j, co:co+NS).
-        int zptr[SPW], zend[SPW], dcol[SPW], myk[SPW];
+        int zptr[SPW] = {}, zend[SPW] = {}, dcol[SPW] = {}, myk[SPW];
         float myd[SPW][NS];
         auto prefetch = [&](int s) {
             const bool ok = zptr[s] + lane < zend[s];

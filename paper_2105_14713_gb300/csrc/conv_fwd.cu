@@ -10,6 +10,9 @@ namespace onexn {
 cudaError_t launch_fma(const ConvArgs &a, int dtype, cudaStream_t st);
 cudaError_t launch_mma(const ConvArgs &a, cudaStream_t st);
 bool mma_supports(const ConvArgs &a);
+cudaError_t launch_tc(const ConvArgs &a, void *workspace, cudaStream_t st);
+bool tc_supports(const ConvArgs &a);
+size_t tc_workspace_bytes(const ConvArgs &a);
 }  // namespace onexn
 
 using onexn::fail;
@@ -122,38 +125,92 @@ onexn_status check_pointers(const int32_t *P, const int32_t *I, const void *D, c
     return ONEXN_OK;
 }
 
-// Kernel family for AUTO: bf16 with N a multiple of 8 runs on tensor cores;
-// everything else (fp32, and bf16 with N < 8) on the FFMA kernel.
-unsigned pick_algo(const onexn::ConvArgs &a, int dtype, unsigned flags)
+// Workspace a family needs for these arguments.
+size_t workspace_for(unsigned algo, const onexn::ConvArgs &a)
+{
+    return algo == ONEXN_ALGO_TC ? onexn::tc_workspace_bytes(a) : 0;
+}
+
+// Can the family run this case at all (dtype, shape)?
+bool supports(unsigned algo, const onexn::ConvArgs &a, int dtype)
+{
+    switch (algo) {
+    case ONEXN_ALGO_FMA: return true;
+    case ONEXN_ALGO_MMA: return dtype == ONEXN_BF16 && onexn::mma_supports(a);
+    case ONEXN_ALGO_TC: return dtype == ONEXN_BF16 && onexn::tc_supports(a);
+    default: return false;
+    }
+}
+
+// Kernel family for AUTO: bf16 runs on the tcgen05 GEMM when its workspace
+// fits; everything else (fp32, bf16 without workspace) on the FFMA kernel.
+unsigned pick_algo(const onexn::ConvArgs &a, int dtype, unsigned flags, size_t ws_bytes)
 {
     const unsigned forced = flags & ONEXN_ALGO_MASK;
     if (forced != ONEXN_ALGO_AUTO) return forced;
-    if (dtype == ONEXN_BF16 && onexn::mma_supports(a)) return ONEXN_ALGO_MMA;
+    if (supports(ONEXN_ALGO_TC, a, dtype) && ws_bytes >= workspace_for(ONEXN_ALGO_TC, a))
+        return ONEXN_ALGO_TC;
     return ONEXN_ALGO_FMA;
+}
+
+onexn_status check_algo(unsigned algo, const onexn::ConvArgs &a, int dtype, size_t ws_bytes)
+{
+    if (algo != ONEXN_ALGO_FMA && algo != ONEXN_ALGO_MMA && algo != ONEXN_ALGO_TC)
+        return fail(ONEXN_EINVAL, "conv: unknown algo %u", algo >> ONEXN_ALGO_SHIFT);
+    if (!supports(algo, a, dtype))
+        return fail(ONEXN_EUNSUPPORTED, "conv: algo %u cannot run this case (dtype/shape)",
+                    algo >> ONEXN_ALGO_SHIFT);
+    const size_t need = workspace_for(algo, a);
+    if (ws_bytes < need)
+        return fail(ONEXN_EINVAL, "conv: algo %u needs %zu bytes of workspace, got %zu",
+                    algo >> ONEXN_ALGO_SHIFT, need, ws_bytes);
+    return ONEXN_OK;
 }
 
 }  // namespace
 
 extern "C" onexn_status onexn_conv_algo(const onexn_conv_desc *desc, int N, int64_t t, int dtype,
-                                        unsigned flags, unsigned *algo)
+                                        unsigned flags, size_t workspace_bytes, unsigned *algo)
 {
     onexn::clear_error();
     if (!algo) return fail(ONEXN_EINVAL, "conv_algo: algo is NULL");
     onexn::ConvArgs a{};
     onexn_status st = check_shape(desc, N, t, dtype, flags, &a);
     if (st != ONEXN_OK) return st;
-    const unsigned al = pick_algo(a, dtype, flags);
-    if (al == ONEXN_ALGO_MMA && (dtype != ONEXN_BF16 || !onexn::mma_supports(a)))
-        return fail(ONEXN_EUNSUPPORTED, "conv: the MMA kernel needs bf16 and N %% 8 == 0");
-    if (al != ONEXN_ALGO_FMA && al != ONEXN_ALGO_MMA) return fail(ONEXN_EINVAL, "conv: unknown algo");
+    const unsigned al = pick_algo(a, dtype, flags, workspace_bytes);
+    st = check_algo(al, a, dtype, workspace_bytes);
+    if (st != ONEXN_OK) return st;
     *algo = al;
+    return ONEXN_OK;
+}
+
+extern "C" onexn_status onexn_conv_workspace_size(const onexn_conv_desc *desc, int N, int64_t t,
+                                                  int dtype, unsigned flags, size_t *bytes)
+{
+    onexn::clear_error();
+    if (!bytes) return fail(ONEXN_EINVAL, "conv_workspace_size: bytes is NULL");
+    onexn::ConvArgs a{};
+    onexn_status st = check_shape(desc, N, t, dtype, flags, &a);
+    if (st != ONEXN_OK) return st;
+    const unsigned forced = flags & ONEXN_ALGO_MASK;
+    size_t need = 0;
+    if (forced == ONEXN_ALGO_AUTO) {
+        for (unsigned al : {ONEXN_ALGO_FMA, ONEXN_ALGO_MMA, ONEXN_ALGO_TC})
+            if (supports(al, a, dtype) && workspace_for(al, a) > need) need = workspace_for(al, a);
+    } else {
+        if (!supports(forced, a, dtype))
+            return fail(ONEXN_EUNSUPPORTED, "conv: algo %u cannot run this case", forced >> ONEXN_ALGO_SHIFT);
+        need = workspace_for(forced, a);
+    }
+    *bytes = need;
     return ONEXN_OK;
 }
 
 extern "C" onexn_status onexn_conv_fwd(const onexn_conv_desc *desc, const int32_t *P,
                                        const int32_t *I, const void *D, int N, int64_t t,
                                        const void *x, void *y, const float *bias, int dtype,
-                                       unsigned flags, void *stream)
+                                       unsigned flags, void *workspace, size_t workspace_bytes,
+                                       void *stream)
 {
     onexn::clear_error();
     onexn::ConvArgs a{};
@@ -161,19 +218,18 @@ extern "C" onexn_status onexn_conv_fwd(const onexn_conv_desc *desc, const int32_
     if (st != ONEXN_OK) return st;
     st = check_pointers(P, I, D, x, y, bias, dtype, &a);
     if (st != ONEXN_OK) return st;
-    const unsigned algo = pick_algo(a, dtype, flags);
+    if (!workspace) workspace_bytes = 0;
+    if (reinterpret_cast<uintptr_t>(workspace) & 255u)
+        return fail(ONEXN_EINVAL, "conv: workspace must be 256-byte aligned");
+    const unsigned algo = pick_algo(a, dtype, flags, workspace_bytes);
+    st = check_algo(algo, a, dtype, workspace_bytes);
+    if (st != ONEXN_OK) return st;
     cudaStream_t s = static_cast<cudaStream_t>(stream);
     cudaError_t e = onexn::device_status_ptr(&a.status);
     if (e != cudaSuccess) return fail(ONEXN_ECUDA, "conv: status word: %s", cudaGetErrorString(e));
-    if (algo == ONEXN_ALGO_FMA) {
-        e = onexn::launch_fma(a, dtype, s);
-    } else if (algo == ONEXN_ALGO_MMA) {
-        if (dtype != ONEXN_BF16 || !onexn::mma_supports(a))
-            return fail(ONEXN_EUNSUPPORTED, "conv: the MMA kernel needs bf16 and N %% 8 == 0");
-        e = onexn::launch_mma(a, s);
-    } else {
-        return fail(ONEXN_EINVAL, "conv: unknown algo %u", algo >> ONEXN_ALGO_SHIFT);
-    }
+    if (algo == ONEXN_ALGO_FMA) e = onexn::launch_fma(a, dtype, s);
+    else if (algo == ONEXN_ALGO_MMA) e = onexn::launch_mma(a, s);
+    else e = onexn::launch_tc(a, workspace, s);
     if (e != cudaSuccess) return fail(ONEXN_ECUDA, "conv: launch failed: %s", cudaGetErrorString(e));
     return ONEXN_OK;
 }

@@ -49,6 +49,7 @@ class PrunedConv2d:
         self.D = Dt.to(dev).contiguous()
         self.bias = None if bias is None else torch.as_tensor(
             np.asarray(bias, np.float32)).to(dev).contiguous()
+        self._ws = {}            # per input shape: device workspace (bytes as uint8)
 
     @property
     def torch_dtype(self):
@@ -63,9 +64,20 @@ class PrunedConv2d:
         Ho, Wo = _c.onexn_conv_out_shape(self.desc(B, H, W))
         return (B, Ho, Wo, self.C_out)
 
+    def workspace(self, x_shape, flags: int = 0):
+        """Device workspace for this input shape (allocated once, reused)."""
+        B, H, W, _ = x_shape
+        key = (B, H, W, flags & 0xF00)
+        if key not in self._ws:
+            n = _c.onexn_conv_workspace_size(self.desc(B, H, W), self.N, self.t, self.cdtype, flags)
+            self._ws[key] = torch.empty(max(n, 256), dtype=torch.uint8, device=self.device) if n else None
+        return self._ws[key]
+
     def algo(self, x_shape, flags: int = 0) -> str:
         B, H, W, _ = x_shape
-        a = _c.onexn_conv_algo(self.desc(B, H, W), self.N, self.t, self.cdtype, flags)
+        ws = self.workspace(x_shape, flags)
+        a = _c.onexn_conv_algo(self.desc(B, H, W), self.N, self.t, self.cdtype, flags,
+                               0 if ws is None else ws.numel())
         return _c.ALGO_NAMES[a]
 
     def forward(self, x: torch.Tensor, y: torch.Tensor = None, relu: bool = False,
@@ -80,7 +92,7 @@ class PrunedConv2d:
             y = torch.empty(self.out_shape(x.shape), dtype=x.dtype, device=x.device)
         flags = (_c.ONEXN_RELU if relu else 0) | algo
         _c.onexn_conv_fwd(self.desc(B, H, W), self.P, self.I, self.D, self.N, self.t, x, y,
-                          self.bias, self.cdtype, flags, stream)
+                          self.bias, self.cdtype, flags, self.workspace(x.shape, algo), stream)
         return y
 
     __call__ = forward

@@ -21,7 +21,10 @@ ONEXN_ALGO_SHIFT = 8
 ONEXN_ALGO_AUTO = 0 << ONEXN_ALGO_SHIFT
 ONEXN_ALGO_FMA = 1 << ONEXN_ALGO_SHIFT
 ONEXN_ALGO_MMA = 2 << ONEXN_ALGO_SHIFT
-ALGO_NAMES = {ONEXN_ALGO_FMA: "fma", ONEXN_ALGO_MMA: "mma"}
+ONEXN_ALGO_TC = 3 << ONEXN_ALGO_SHIFT
+ALGO_NAMES = {ONEXN_ALGO_FMA: "fma", ONEXN_ALGO_MMA: "mma", ONEXN_ALGO_TC: "tc"}
+ALGO_BY_NAME = {v: k for k, v in ALGO_NAMES.items()}
+ALGO_BY_NAME["auto"] = ONEXN_ALGO_AUTO
 
 _STATUS = {0: "OK", 1: "EINVAL", 2: "EUNSUPPORTED", 3: "ENOMEM", 4: "ECUDA", 5: "EDEVICE",
            6: "ETIMEOUT"}
@@ -50,8 +53,10 @@ SIGNATURES = {
     "onexn_packed_validate": ([_P, _P, _I32, _I64, _I32], _I32),
     "onexn_conv_out_shape": ([ctypes.POINTER(ConvDesc), _P, _P], _I32),
     "onexn_conv_fwd": ([ctypes.POINTER(ConvDesc), _P, _P, _P, _I32, _I64, _P, _P, _P, _I32,
-                        _U32, _P], _I32),
-    "onexn_conv_algo": ([ctypes.POINTER(ConvDesc), _I32, _I64, _I32, _U32, _P], _I32),
+                        _U32, _P, ctypes.c_size_t, _P], _I32),
+    "onexn_conv_workspace_size": ([ctypes.POINTER(ConvDesc), _I32, _I64, _I32, _U32, _P], _I32),
+    "onexn_conv_algo": ([ctypes.POINTER(ConvDesc), _I32, _I64, _I32, _U32, ctypes.c_size_t, _P],
+                        _I32),
     "onexn_device_status": ([_I32, _P], _I32),
 }
 
@@ -165,24 +170,34 @@ def onexn_conv_out_shape(desc: ConvDesc):
     return ho.value, wo.value
 
 
-def onexn_conv_algo(desc: ConvDesc, N: int, t: int, dtype: int, flags: int = 0) -> int:
+def onexn_conv_algo(desc: ConvDesc, N: int, t: int, dtype: int, flags: int = 0,
+                    workspace_bytes: int = 0) -> int:
     out = ctypes.c_uint(0)
     _check(lib.onexn_conv_algo(ctypes.byref(desc), int(N), int(t), int(dtype), int(flags),
-                               ctypes.byref(out)))
+                               int(workspace_bytes), ctypes.byref(out)))
+    return out.value
+
+
+def onexn_conv_workspace_size(desc: ConvDesc, N: int, t: int, dtype: int, flags: int = 0) -> int:
+    out = ctypes.c_size_t(0)
+    _check(lib.onexn_conv_workspace_size(ctypes.byref(desc), int(N), int(t), int(dtype),
+                                         int(flags), ctypes.byref(out)))
     return out.value
 
 
 def onexn_conv_fwd(desc: ConvDesc, P, I, D, N: int, t: int, x, y, bias, dtype: int,
-                   flags: int = 0, stream=None) -> None:
-    """Launch the convolution.  P, I, D, x, y, bias are torch CUDA tensors
-    (bias may be None); stream is a torch.cuda.Stream or None (current)."""
+                   flags: int = 0, workspace=None, stream=None) -> None:
+    """Launch the convolution.  P, I, D, x, y, bias, workspace are torch CUDA
+    tensors (bias and workspace may be None); stream is a torch.cuda.Stream
+    or None (the current stream)."""
     import torch
     if stream is None:
         stream = torch.cuda.current_stream(x.device)
     ptr = (lambda tns: None if tns is None else ctypes.c_void_p(tns.data_ptr()))
+    ws_bytes = 0 if workspace is None else workspace.numel() * workspace.element_size()
     _check(lib.onexn_conv_fwd(ctypes.byref(desc), ptr(P), ptr(I), ptr(D), int(N), int(t), ptr(x),
-                              ptr(y), ptr(bias), int(dtype), int(flags),
-                              ctypes.c_void_p(stream.cuda_stream)))
+                              ptr(y), ptr(bias), int(dtype), int(flags), ptr(workspace),
+                              int(ws_bytes), ctypes.c_void_p(stream.cuda_stream)))
 
 
 def onexn_device_status(clear: bool = True) -> int:

@@ -30,18 +30,21 @@ GEOMS = [
     ("5x5_p0", 1, 20, 20, 8, 32, 5, 5, 1, 0, 1),
 ]
 
-ALGOS = {"fma": ox.ONEXN_ALGO_FMA, "mma": ox.ONEXN_ALGO_MMA, "auto": ox.ONEXN_ALGO_AUTO}
+ALGOS = ox.ALGO_BY_NAME
 
 
-def _algos_for(dtype, N):
+def _algos_for(dtype, N, C_in=64, C_out=64):
+    """Every family that can run this case (FMA always; the bf16 families if
+    they accept it), plus AUTO."""
     out = ["auto", "fma"]
-    if dtype == "bf16" and N % 8 == 0:
-        probe = ox.make_desc(1, 8, 8, 8, N, 1, 1)
-        try:
-            ox.onexn_conv_algo(probe, N, 1, ox.ONEXN_BF16, ox.ONEXN_ALGO_MMA)
-            out.append("mma")
-        except ox.OnexnError:
-            pass
+    if dtype == "bf16":
+        probe = ox.make_desc(1, 8, 8, C_in, C_out, 1, 1)
+        for name in ("mma", "tc"):
+            try:
+                ox.onexn_conv_algo(probe, N, 1, ox.ONEXN_BF16, ALGOS[name], 1 << 40)
+                out.append(name)
+            except ox.OnexnError:
+                pass
     return out
 
 
@@ -53,7 +56,7 @@ def test_geometry_and_block_width(geom, N, dtype):
     if Co % N:
         pytest.skip("N must divide C_out")
     layer = L(name, B, H, W, Ci, Co, KH, KW, s, p, d, N=N, rate=0.5, dtype=dtype, seed=N)
-    for algo in _algos_for(dtype, N):
+    for algo in _algos_for(dtype, N, Ci, Co):
         y, yr, a, conv = run_layer(layer, relu=(N % 2 == 0), algo=ALGOS[algo])
         e = norm_err(y, yr, a)
         assert e <= tol(layer), f"{algo}: err {e:.3e}"
@@ -63,9 +66,9 @@ def test_geometry_and_block_width(geom, N, dtype):
 @pytest.mark.parametrize("dtype", ["f32", "bf16"])
 def test_rates(rate, dtype):
     layer = L("rates", 2, 12, 12, 64, 128, 3, 3, 1, 1, 1, N=8, rate=rate, dtype=dtype, seed=3)
-    for algo in _algos_for(dtype, 8):
+    for algo in _algos_for(dtype, 8, 64, 128):
         y, yr, a, _ = run_layer(layer, relu=True, algo=ALGOS[algo])
-        assert norm_err(y, yr, a) <= tol(layer)
+        assert norm_err(y, yr, a) <= tol(layer), algo
 
 
 @pytest.mark.parametrize("N", [3, 5, 6, 12, 24, 64, 128])
@@ -85,9 +88,33 @@ def test_odd_output_channels_scalar_stores():
 @pytest.mark.parametrize("dtype", ["f32", "bf16"])
 def test_dense_path_rate0_N_equals_cout(dtype):
     layer = L("dense", 2, 14, 14, 64, 128, 3, 3, 1, 1, 1, N=128, rate=0.0, dtype=dtype, seed=5)
-    y, yr, a, conv = run_layer(layer)
-    assert conv.t == 576
+    for algo in _algos_for(dtype, 128, 64, 128):
+        y, yr, a, conv = run_layer(layer, algo=ALGOS[algo])
+        assert conv.t == 576
+        assert norm_err(y, yr, a) <= tol(layer), algo
+
+
+@pytest.mark.parametrize("C_out,N", [(64, 8), (128, 16), (256, 8), (384, 32), (520, 8), (48, 8)])
+def test_tc_column_tiles(C_out, N):
+    """The tcgen05 family over every column-tile width (64/128/256) and a
+    ragged last column tile."""
+    layer = L("tc_cols", 3, 11, 13, 72, C_out, 3, 3, 1, 1, 1, N=N, rate=0.5, dtype="bf16", seed=C_out)
+    y, yr, a, conv = run_layer(layer, relu=True, algo=ox.ONEXN_ALGO_TC)
+    assert conv.algo((3, 11, 13, 72), ox.ONEXN_ALGO_TC) == "tc"
     assert norm_err(y, yr, a) <= tol(layer)
+
+
+def test_auto_picks_tc_for_bf16_with_workspace():
+    layer = L("auto", 1, 8, 8, 64, 64, 1, 1, N=8, rate=0.5, dtype="bf16")
+    from paper_2105_14713_gb300.layer import PrunedConv2d
+    conv = PrunedConv2d(wl.weights(layer).numpy(), 8, 0.5, dtype="bf16")
+    assert conv.algo((1, 8, 8, 64)) == "tc"
+    conv32 = PrunedConv2d(wl.weights(layer).numpy(), 8, 0.5, dtype="f32")
+    assert conv32.algo((1, 8, 8, 64)) == "fma"
+
+
+def test_device_status_clean_after_runs():
+    assert ox.onexn_device_status(clear=True) == ox.ONEXN_OK
 
 
 def test_bf16_against_fp32_master_inputs():

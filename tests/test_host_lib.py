@@ -158,6 +158,15 @@ def test_conv_shape_and_argument_errors_need_no_gpu():
     d = ox.make_desc(2, 7, 7, 8, 16, 3, 3, 2, 1, 1)
     assert ox.onexn_conv_out_shape(d) == (4, 4)
     assert ox.onexn_conv_algo(d, 8, 100, ox.ONEXN_F32) == ox.ONEXN_ALGO_FMA
+    # bf16: the tcgen05 family when its workspace fits, else FFMA
+    need = ox.onexn_conv_workspace_size(d, 8, 100, ox.ONEXN_BF16)
+    assert need == 16 * 9 * 8 * 2 + (-(16 * 9 * 8 * 2) % 256)
+    assert ox.onexn_conv_algo(d, 8, 100, ox.ONEXN_BF16, 0, need) == ox.ONEXN_ALGO_TC
+    assert ox.onexn_conv_algo(d, 8, 100, ox.ONEXN_BF16, 0, need - 1) == ox.ONEXN_ALGO_FMA
+    assert ox.onexn_conv_workspace_size(d, 8, 100, ox.ONEXN_F32) == 0
+    assert _status(ox.onexn_conv_algo, d, 8, 100, ox.ONEXN_BF16, ox.ONEXN_ALGO_TC, 0) == ox.ONEXN_EINVAL
+    assert _status(ox.onexn_conv_algo, d, 8, 100, ox.ONEXN_F32, ox.ONEXN_ALGO_TC, 1 << 30) == \
+        ox.ONEXN_EUNSUPPORTED
     bad = ox.make_desc(1, 2, 2, 8, 16, 5, 5)
     assert _status(ox.onexn_conv_out_shape, bad) == ox.ONEXN_EINVAL
     assert _status(ox.onexn_conv_algo, d, 3, 10, ox.ONEXN_F32) == ox.ONEXN_EINVAL    # N | C_out
@@ -168,10 +177,11 @@ def test_conv_shape_and_argument_errors_need_no_gpu():
     assert _status(ox.onexn_conv_algo, d, 8, 10, 0, 1 << 20) == ox.ONEXN_EINVAL      # flags
     # conv_fwd rejects bad pointers before touching the GPU
     st = ox.lib.onexn_conv_fwd(ctypes.byref(d), None, None, None, 8, 0, None, None, None, 0, 0,
-                               None)
+                               None, 0, None)
     assert st == ox.ONEXN_EINVAL
     buf = (ctypes.c_char * 64)()
     base = ctypes.addressof(buf)
     mis = ctypes.c_void_p(base + (16 - base % 16) % 16 + 4)
-    st = ox.lib.onexn_conv_fwd(ctypes.byref(d), mis, mis, mis, 8, 1, mis, mis, None, 0, 0, None)
+    st = ox.lib.onexn_conv_fwd(ctypes.byref(d), mis, mis, mis, 8, 1, mis, mis, None, 0, 0, None, 0,
+                               None)
     assert st == ox.ONEXN_EINVAL and b"aligned" in ox.lib.onexn_last_error()
