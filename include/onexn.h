@@ -215,6 +215,36 @@ onexn_status onexn_conv_algo(const onexn_conv_desc *desc, int N, int64_t t, int 
                              unsigned flags, size_t workspace_bytes, unsigned *algo);
 
 /*
+ * onexn_conv_fwd_noalloc -- onexn_conv_fwd for callers that cannot allocate
+ * device memory.  The paper has no counterpart; it is a deployment aid.
+ *
+ * It runs the bf16 tensor-core family (ONEXN_ALGO_TC; flags may carry
+ * ONEXN_RELU and AUTO or TC) with its scratch -- the decoded weight matrix,
+ * C_out * KH*KW*C_in bf16 values -- in a fixed 8 MiB array that is part of
+ * the library's device image, instead of a caller workspace.  It never
+ * calls cudaMalloc, cudaFree or any other allocating routine.  Who needs it:
+ * code running while a stream is captured into a CUDA graph (allocating
+ * there breaks the capture), hosts that forbid allocation after start-up to
+ * keep latency predictable, and plug-ins that only receive raw pointers
+ * from a framework that owns all device memory.
+ *   Arguments as onexn_conv_fwd (x, y, P, I, D, bias are caller-owned).
+ *   EINVAL: the decoded weights would exceed 8 MiB (use onexn_conv_fwd with
+ *   a workspace), or another ALGO was forced.  EUNSUPPORTED: the
+ *   tensor-core family cannot run the case (for instance fp32).
+ * Every GPU that loads the library keeps the 8 MiB until the process exits.
+ * All calls share the array, so calls that overlap on the GPU (different
+ * streams or host threads) race and may return wrong results.  Each call
+ * rewrites the part it uses before reading it; nothing needs clearing.  The
+ * first call on a device looks up the array's device address
+ * (cudaGetSymbolAddress) with that device current; make that first call
+ * before any stream capture starts.
+ */
+onexn_status onexn_conv_fwd_noalloc(const onexn_conv_desc *desc, const int32_t *P,
+                                    const int32_t *I, const void *D, int N, int64_t t,
+                                    const void *x, void *y, const float *bias, int dtype,
+                                    unsigned flags, void *stream);
+
+/*
  * onexn_device_status -- read, and clear if `clear` is non-zero, the status
  * word that the kernels of this library keep on the current device (a
  * 4-byte __device__ variable of the library).  A kernel whose bounded

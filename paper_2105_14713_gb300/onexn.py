@@ -58,6 +58,8 @@ SIGNATURES = {
     "onexn_conv_algo": ([ctypes.POINTER(ConvDesc), _I32, _I64, _I32, _U32, ctypes.c_size_t, _P],
                         _I32),
     "onexn_device_status": ([_I32, _P], _I32),
+    "onexn_conv_fwd_noalloc": ([ctypes.POINTER(ConvDesc), _P, _P, _P, _I32, _I64, _P, _P, _P, _I32,
+                                _U32, _P], _I32),
 }
 
 
@@ -198,6 +200,21 @@ def onexn_conv_fwd(desc: ConvDesc, P, I, D, N: int, t: int, x, y, bias, dtype: i
     _check(lib.onexn_conv_fwd(ctypes.byref(desc), ptr(P), ptr(I), ptr(D), int(N), int(t), ptr(x),
                               ptr(y), ptr(bias), int(dtype), int(flags), ptr(workspace),
                               int(ws_bytes), ctypes.c_void_p(stream.cuda_stream)))
+
+
+def onexn_conv_fwd_noalloc(desc: ConvDesc, P, I, D, N: int, t: int, x, y, bias, dtype: int,
+                           flags: int = 0, stream=None) -> None:
+    """The tensor-core convolution with the library's fixed 8 MiB scratch:
+    no workspace argument and no allocation, for callers that cannot
+    allocate device memory.  Calls that overlap on the GPU share the scratch
+    and race; see include/onexn.h."""
+    import torch
+    if stream is None:
+        stream = torch.cuda.current_stream(x.device)
+    ptr = (lambda tns: None if tns is None else ctypes.c_void_p(tns.data_ptr()))
+    _check(lib.onexn_conv_fwd_noalloc(ctypes.byref(desc), ptr(P), ptr(I), ptr(D), int(N), int(t),
+                                      ptr(x), ptr(y), ptr(bias), int(dtype), int(flags),
+                                      ctypes.c_void_p(stream.cuda_stream)))
 
 
 def onexn_device_status(clear: bool = True) -> int:
