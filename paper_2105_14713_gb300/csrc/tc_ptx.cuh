@@ -66,6 +66,27 @@ __device__ __forceinline__ void tma_load_im2col_4d(uint32_t dst_smem, const void
         "h"(off_h)
         : "memory");
 }
+// TMA tiled store shared -> global (bulk async group of this thread).
+__device__ __forceinline__ void tma_store_2d(const void *tmap, int c0, int c1, uint32_t src_smem)
+{
+    asm volatile("cp.async.bulk.tensor.2d.global.shared::cta.bulk_group [%0, {%1, %2}], [%3];\n" ::"l"(
+                     reinterpret_cast<uint64_t>(tmap)),
+                 "r"(c0), "r"(c1), "r"(src_smem)
+                 : "memory");
+}
+__device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;\n" ::: "memory"); }
+// Wait until the shared-memory sources of all committed bulk stores of this
+// thread have been read (the buffer may then be overwritten).
+__device__ __forceinline__ void bulk_wait_read0() { asm volatile("cp.async.bulk.wait_group.read 0;\n" ::: "memory"); }
+// Wait until all committed bulk stores of this thread have completed.
+__device__ __forceinline__ void bulk_wait0() { asm volatile("cp.async.bulk.wait_group 0;\n" ::: "memory"); }
+
+// Barrier over a subset of the CTA's warps (named barrier `id`, `n` threads).
+__device__ __forceinline__ void named_bar(int id, int n)
+{
+    asm volatile("bar.sync %0, %1;\n" ::"r"(id), "r"(n) : "memory");
+}
+
 // Arrive on an mbarrier and add `bytes` to the transaction count of the phase.
 __device__ __forceinline__ void mbar_arrive_expect_tx(uint32_t mbar, uint32_t bytes)
 {
