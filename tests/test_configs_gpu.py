@@ -1,0 +1,137 @@
+"""Parity of the five synthetic workloads at their full sizes, in the launch
+configuration bench.py times (AUTO kernel selection, caller workspace).
+
+Small layers are compared in full; large ones on seeded sampled output
+pixels (always including the first and last pixel) across all output
+channels, computed one by one by the fp64 oracle.  Tolerances as in
+tests/gpu_util.py: fp32 1e-5, bf16 4e-3 against the oracle on the
+bf16-rounded inputs (and 1e-2 against fp32 master inputs where checked)."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2105_14713_gb300 import onexn as ox
+from paper_2105_14713_gb300 import workloads as wl
+from paper_2105_14713_gb300.layer import PrunedConv2d
+from tests.gpu_util import norm_err, oracle_ref, tol
+
+pytestmark = pytest.mark.gpu
+
+
+def _run(layer, W, x_cpu, b, pixels, relu=False, master=False):
+    conv = PrunedConv2d(W, layer.N, layer.rate, bias=b, stride=layer.stride, padding=layer.pad,
+                        dilation=layer.dil, dtype=layer.dtype)
+    xd = (x_cpu if layer.dtype == "f32" else x_cpu.to(torch.bfloat16)).cuda()
+    y = conv(xd, relu=relu)
+    torch.cuda.synchronize()
+    yf = y.float().reshape(-1, layer.C_out)
+    y_s = (yf if pixels is None else yf[torch.as_tensor(pixels, device="cuda")]).cpu().numpy()
+    y_ref, a = oracle_ref(layer, W, x_cpu, b, relu=relu, pixels=pixels, master=master)
+    return norm_err(y_s.astype(np.float64), y_ref, a), conv
+
+
+def _pixels(layer, count=1024, seed=0):
+    return wl.sample_pixels(layer.pixels, count, seed, must=[0, layer.pixels - 1])
+
+
+# ---------------------------------------------------------------- cfg1
+
+def test_config1_rearranged_pruned_layer():
+    """1x1 64->64, 28x28, N=4, 50%: rearrangement with a random next layer,
+    then pruning; full-output parity, and the two-layer composition at rate 0
+    is unchanged by the rearrangement on the GPU too."""
+    layer = wl.config1()[0]
+    W = wl.weights(layer).numpy()
+    Wn = wl.next_layer_weights(64, 64, seed=0).numpy()
+    b = wl.bias(layer).numpy()
+    Wr, Wnr, perm = ox.onexn_rearrange(W, Wn)
+    x = wl.activations(layer)
+    err, conv = _run(layer, Wr, x, b[perm], None, relu=True)
+    assert err <= 1e-5
+    assert conv.kept == ox.onexn_keep_count(16 * 64, 0.5) == 512
+
+    def two_layers(W1, b1, W2):
+        c1 = PrunedConv2d(W1, 64, 0.0, bias=b1)
+        c2 = PrunedConv2d(W2, 64, 0.0)
+        return c2(c1(x.cuda(), relu=True)).cpu().numpy()
+
+    y0 = two_layers(W, b, Wn)
+    y1 = two_layers(Wr, b[perm], Wnr)
+    assert np.max(np.abs(y0 - y1)) <= 1e-5 * (np.abs(y0).max() + 1e-30)
+
+
+# ---------------------------------------------------------------- cfg2
+
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+def test_config2_full(dtype):
+    layer = wl.config2(dtype)[0]
+    W, x, b = wl.weights(layer).numpy(), wl.activations(layer), wl.bias(layer).numpy()
+    err, conv = _run(layer, W, x, b, None, relu=True)
+    assert conv.t == 9216
+    assert err <= tol(layer)
+    if dtype == "bf16":
+        pix = _pixels(layer, 512)
+        err_m, _ = _run(layer, W, x, b, pix, relu=True, master=True)
+        assert err_m <= 1e-2
+
+
+# ---------------------------------------------------------------- cfg3
+
+def test_config3_mobilenet_v2_stack():
+    """All 34 expand/project 1x1 layers at batch 128, fp32, N=4, 50%, with
+    the expand layer's filters rearranged and the permutation carried through
+    the depthwise channels into the project layer (C10)."""
+    layers = wl.config3()
+    worst = 0.0
+    W_next_perm = {}
+    for i, layer in enumerate(layers):
+        W = wl.weights(layer).numpy()
+        if i in W_next_perm:                     # project layer: permuted input channels
+            W = W[:, W_next_perm.pop(i)]
+        b = wl.bias(layer).numpy()
+        if layer.name.endswith("_expand") and i + 1 < len(layers):
+            nxt = layers[i + 1]
+            Wn = wl.weights(nxt).numpy()
+            W, _, perm = ox.onexn_rearrange(W, Wn)
+            b = b[perm]
+            W_next_perm[i + 1] = perm
+        x = wl.activations(layer)
+        err, _ = _run(layer, W, x, b, _pixels(layer, 512, seed=i), relu=layer.name.endswith("_expand"))
+        worst = max(worst, err)
+        assert err <= 1e-5, layer.name
+    assert worst <= 1e-5
+
+
+# ---------------------------------------------------------------- cfg4
+
+def test_config4_resnet50_stack():
+    """All 52 bottleneck and downsample convs at batch 256, bf16, N=16, 70%."""
+    for i, layer in enumerate(wl.config4()):
+        W, x, b = wl.weights(layer).numpy(), wl.activations(layer), wl.bias(layer).numpy()
+        err, conv = _run(layer, W, x, b, _pixels(layer, 384, seed=i), relu=True)
+        assert err <= tol(layer), layer.name
+
+
+# ---------------------------------------------------------------- cfg5
+
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+@pytest.mark.parametrize("N", wl.SWEEP_N)
+def test_config5_sweep(dtype, N):
+    """3x3 512->512 on 128x14x14, every block width and rate (seed 0)."""
+    base = wl.config5(N=N, rate=0.0, dtype=dtype, seed=0)[0]
+    x = wl.activations(base)
+    for rate in wl.SWEEP_RATE:
+        layer = base.with_(rate=rate)
+        W, b = wl.weights(layer).numpy(), wl.bias(layer).numpy()
+        err, conv = _run(layer, W, x, b, _pixels(layer, 128, seed=N), relu=True)
+        assert err <= tol(layer), (N, rate, dtype)
+
+
+@pytest.mark.parametrize("seed", [1, 2])
+def test_config5_other_seeds(seed):
+    for dtype, N, rate in (("f32", 4, 0.5), ("bf16", 16, 0.7), ("f32", 32, 0.9), ("bf16", 1, 0.3)):
+        layer = wl.config5(N=N, rate=rate, dtype=dtype, seed=seed)[0]
+        W, x, b = wl.weights(layer).numpy(), wl.activations(layer), wl.bias(layer).numpy()
+        err, _ = _run(layer, W, x, b, _pixels(layer, 128, seed=seed), relu=True)
+        assert err <= tol(layer), (seed, dtype, N, rate)
