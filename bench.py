@@ -1,15 +1,20 @@
 """Benchmark of the 1xN-pruned convolution forward pass on GB300.
 
-Workload (one "step"): the ResNet-50 stage-2 3x3 convolution, batch 64,
-28x28, 128 -> 128 channels, stride 1, pad 1, 1xN blocks with N = 8 at a 50%
-block pruning rate, run once with fp32 inputs ("f32" leg) and once with bf16
-inputs / fp32 accumulation ("bf16" leg).  Inputs are seeded synthetic
-tensors resident in HBM; L2 is flushed (256 MB write) before every step.
+Workloads (--config, default 2; seeded synthetic inputs resident in HBM; L2
+flushed with a 256 MB write before every step, outside the timed events):
+  1  1x1 conv 64 -> 64, 1x28x28, fp32, N=4, 50%
+  2  ResNet-50 stage-2 3x3 conv, 64x28x28, 128 -> 128, N=8, 50%: one fp32 leg
+     and one bf16-input / fp32-accumulate leg per step           (default)
+  3  MobileNet-V2 expand/project 1x1 stack (34 layers), 128x224x224 input, fp32, N=4, 50%
+  4  ResNet-50 bottleneck stack (52 convs), 256x224x224 input, bf16, N=16, 70%
+  5  3x3 512 -> 512 on 128x14x14: sweep N in {1..32} x rate in {0..0.9} x {fp32, bf16}
 
-Prints one JSON line.  Metric: effective TFLOP/s = 2 * pixels * t * N / time
-(t = kept blocks), summed over both legs.
+A "step" is one pass over every layer (leg) of the workload.  Prints one JSON
+line.  Metric: effective TFLOP/s = 2 * pixels * t * N / time summed over the
+legs (t = kept blocks), plus the roofline fraction of the dominant kernel and
+the speedup over the library's own dense path (rate 0, N = C_out).
 
-  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+  python bench.py [--config C] [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
 
 --impl reference times the CPU oracle (fp64, plain C) on the host cores on a
 bounded pixel sample of the same workload.
@@ -36,10 +41,30 @@ L2_FLUSH_BYTES = 256 << 20
 SM_COUNT_GB300 = 152
 FP32_LANES_PER_SM = 128
 
+DESCRIPTIONS = {
+    1: "1x1 conv, 1x28x28x64 -> 64, fp32, NHWC; 1xN N=4, 50% block rate",
+    2: "ResNet-50 stage-2 3x3 conv, 64x28x28x128 -> 128, s1 p1, NHWC; 1xN N=8, 50% block rate; "
+       "fp32 leg + bf16-in/fp32-acc leg",
+    3: "MobileNet-V2 (width 1.0) expand/project 1x1 stack + conv_last, 34 layers, batch 128, "
+       "224x224 input, fp32; 1xN N=4, 50% block rate",
+    4: "ResNet-50 bottleneck 1x1/3x3 + downsample convs, 52 layers, batch 256, 224x224 input, "
+       "bf16-in/fp32-acc; 1xN N=16, 70% block rate",
+    5: "3x3 conv 128x14x14x512 -> 512, s1 p1; sweep N in {1,2,4,8,16,32} x rate in "
+       "{0,.3,.5,.7,.9} x {fp32, bf16}, seed 0",
+}
 
-def workload():
+
+def workload(cfg: int):
     from paper_2105_14713_gb300 import workloads as wl
-    return [wl.config2("f32")[0], wl.config2("bf16")[0]]
+    if cfg == 1:
+        return wl.config1()
+    if cfg == 2:
+        return [wl.config2("f32")[0], wl.config2("bf16")[0]]
+    if cfg == 3:
+        return wl.config3()
+    if cfg == 4:
+        return wl.config4()
+    raise ValueError(cfg)
 
 
 def kept_flops(layer, t):
@@ -69,6 +94,23 @@ def peaks():
     fp32 = SM_COUNT_GB300 * FP32_LANES_PER_SM * 2 * sm_max * 1e6 / 1e12
     return {"hbm_gbs": hbm, "bf16_tflops": bf16, "bf16_tflops_sustained": bf16_s,
             "fp32_ffma_tflops": fp32, "sm_max_mhz": sm_max, "source": src}
+
+
+def leg_roofline(layer, t, algo, ms, pk):
+    fl, by = kept_flops(layer, t), alg_bytes(layer, t)
+    if algo == "fma":
+        pipe, pipe_name, pipe_src = pk["fp32_ffma_tflops"], "alu", \
+            "FFMA: 152 SMs x 128 lanes x 2 x %.0f MHz (derived)" % pk["sm_max_mhz"]
+    else:
+        pipe, pipe_name, pipe_src = pk["bf16_tflops"], "tensor", f"{pk['source']} bf16 tensor (burst)"
+    t_pipe = fl / (pipe * 1e12)
+    t_mem = by / (pk["hbm_gbs"] * 1e9)
+    sec = ms * 1e-3
+    if t_pipe >= t_mem:
+        return {"bound": pipe_name, "achieved": fl / sec / 1e12, "peak": pipe, "unit": "TFLOP/s",
+                "frac": t_pipe / sec, "peak_source": pipe_src}
+    return {"bound": "hbm", "achieved": by / sec / 1e9, "peak": pk["hbm_gbs"], "unit": "GB/s",
+            "frac": t_mem / sec, "peak_source": f"{pk['source']} HBM copy"}
 
 
 class ClockSampler:
@@ -154,7 +196,7 @@ def traffic_for(kernel_key: str):
 # distributed plumbing (replicas: no data-path collective)
 # --------------------------------------------------------------------------
 
-def dist_setup(n_gpus: int):
+def dist_setup():
     ws = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
     local = int(os.environ.get("LOCAL_RANK", "0"))
@@ -188,24 +230,13 @@ def max_over_ranks(v: float, ws: int) -> float:
 # oracle (CPU baseline and the reference arm)
 # --------------------------------------------------------------------------
 
-def oracle_step(layers, packs, pixels):
-    import oracle
-    t0 = time.perf_counter()
-    flops = 0.0
-    for layer, (x, P, I, D, b) in zip(layers, packs):
-        oracle.conv_bsr(x, P, I, D, layer.C_out, layer.KH, layer.KW, layer.N, b,
-                        (layer.stride,) * 2, (layer.pad,) * 2, (layer.dil,) * 2, pixels=pixels)
-        flops += 2.0 * len(pixels) * len(I) * layer.N
-    return time.perf_counter() - t0, flops
-
-
 def oracle_setup(layers):
     import oracle
     from paper_2105_14713_gb300 import workloads as wl
     packs = []
     for layer in layers:
         W = wl.weights(layer).numpy()
-        x = wl.activations(layer).numpy()
+        x = wl.activations(layer.with_(B=1)).numpy()           # image 0 of the batch
         if layer.dtype == "bf16":
             x = oracle.round_bf16(x)
         mask, _ = oracle.prune(W, layer.N, layer.rate)
@@ -214,92 +245,87 @@ def oracle_setup(layers):
     return packs
 
 
+def oracle_pass(layers, packs, max_pix, rng):
+    """Oracle over up to max_pix output pixels of image 0 of every layer."""
+    import oracle
+    t0 = time.perf_counter()
+    flops = 0.0
+    for layer, (x, P, I, D, b) in zip(layers, packs):
+        n_img = layer.Ho * layer.Wo
+        pix = np.sort(rng.choice(n_img, size=min(max_pix, n_img), replace=False)).astype(np.int64)
+        oracle.conv_bsr(x, P, I, D, layer.C_out, layer.KH, layer.KW, layer.N, b,
+                        (layer.stride,) * 2, (layer.pad,) * 2, (layer.dil,) * 2, pixels=pix)
+        flops += 2.0 * len(pix) * len(I) * layer.N
+    return time.perf_counter() - t0, flops
+
+
 def cpu_baseline(layers, budget_s: float = 10.0):
     """The oracle as it stands, on this host's cores, on a bounded sample:
-    whole images (784 output pixels each), as many as fit in ~budget_s."""
+    output pixels of image 0 of every layer, repeated until ~budget_s."""
     import oracle
     packs = oracle_setup(layers)
-    npix_img = layers[0].Ho * layers[0].Wo
-    n_img, spent, flops = 0, 0.0, 0.0
-    while spent < budget_s and n_img < layers[0].B:
-        pix = np.arange(n_img * npix_img, (n_img + 1) * npix_img, dtype=np.int64)
-        dt, fl = oracle_step(layers, packs, pix)
+    rng = np.random.default_rng(0)
+    max_pix = 784 if len(layers) <= 2 else 64
+    spent, flops, passes = 0.0, 0.0, 0
+    while spent < budget_s and passes < 64:
+        dt, fl = oracle_pass(layers, packs, max_pix, rng)
         spent += dt
         flops += fl
-        n_img += 1
+        passes += 1
     return {"value": flops / spent / 1e12, "unit": "TFLOP/s", "cores": oracle.num_threads(),
             "kind": "oracle",
-            "sample": f"{n_img} of {layers[0].B} images ({n_img * npix_img} output pixels x all "
-                      f"{layers[0].C_out} channels), both legs, fp64 plain-C oracle, "
-                      f"{spent:.1f} s"}
+            "sample": f"{passes} passes x up to {max_pix} output pixels (all channels) of image 0 of "
+                      f"each of {len(layers)} layer(s); fp64 plain-C oracle; {spent:.1f} s"}
 
 
 def run_reference(args, rank, ws):
     if rank != 0:
         return
     import oracle
-    layers = workload()
+    cfg = args.config if args.config != 5 else 2
+    layers = workload(cfg)
     packs = oracle_setup(layers)
-    npix_img = layers[0].Ho * layers[0].Wo
     rng = np.random.default_rng(0)
+    max_pix = 784 if len(layers) <= 2 else 32
     times, flops = [], []
     for i in range(args.warmup + args.steps):
-        img = int(rng.integers(0, layers[0].B))
-        pix = np.arange(img * npix_img, (img + 1) * npix_img, dtype=np.int64)
-        dt, fl = oracle_step(layers, packs, pix)
+        dt, fl = oracle_pass(layers, packs, max_pix, rng)
         if i >= args.warmup:
             times.append(dt)
             flops.append(fl)
     v = sum(flops) / sum(times) / 1e12
     ms = 1e3 * sum(times) / len(times)
-    sample = (f"one random image per step (784 output pixels x 128 channels), both legs; "
-              f"fp64 plain-C oracle, {oracle.num_threads()} threads")
+    sample = (f"per step up to {max_pix} random output pixels (all channels) of image 0 of each of "
+              f"{len(layers)} layer(s); fp64 plain-C oracle, {oracle.num_threads()} threads")
     print(json.dumps({
         "impl": "reference", "metric": METRIC, "value": v, "unit": "TFLOP/s", "n_gpus": args.gpus,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-        "config": config_json(layers, "cpu oracle sample"),
+        "config": config_json(cfg, layers, "cpu oracle sample"),
         "cpu_baseline": {"value": v, "unit": "TFLOP/s", "cores": oracle.num_threads(),
                          "kind": "oracle", "sample": sample},
         "e2e": {"value": v, "unit": "TFLOP/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }), flush=True)
 
 
-def config_json(layers, l2="flushed before every step (256 MB write)"):
+def config_json(cfg, layers, l2="flushed before every step (256 MB write)"):
     l0 = layers[0]
-    return {"workload": "ResNet-50 stage-2 3x3 conv, 64x28x28x128 -> 128, s1 p1, NHWC; "
-                        "1xN N=8, 50% block rate; fp32 leg + bf16-in/fp32-acc leg",
-            "batch": l0.B, "H": l0.H, "W": l0.W, "C_in": l0.C_in, "C_out": l0.C_out,
-            "kernel": [l0.KH, l0.KW], "N": l0.N, "rate": l0.rate,
-            "legs": [l.dtype for l in layers], "parallelism": "replicas", "l2": l2}
+    out = {"workload": DESCRIPTIONS[cfg], "config_id": cfg, "layers": len(layers),
+           "batch": l0.B, "N": l0.N, "rate": l0.rate,
+           "dtypes": sorted({l.dtype for l in layers}), "parallelism": "replicas", "l2": l2}
+    if len(layers) <= 2:
+        out.update({"H": l0.H, "W": l0.W, "C_in": l0.C_in, "C_out": l0.C_out,
+                    "kernel": [l0.KH, l0.KW]})
+    return out
 
 
 # --------------------------------------------------------------------------
 # GPU arm
 # --------------------------------------------------------------------------
 
-def main():
-    ap = argparse.ArgumentParser()
-    ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=20)
-    ap.add_argument("--warmup", type=int, default=5)
-    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
-    ap.add_argument("--no-cpu-baseline", action="store_true")
-    args = ap.parse_args()
-    args.warmup = max(args.warmup, 3)
-    rank, local, ws = dist_setup(args.gpus)
-    if args.impl == "reference":
-        run_reference(args, rank, ws)
-        return
-
-    from paper_2105_14713_gb300 import onexn as ox
+def build_legs(layers, dev):
     from paper_2105_14713_gb300 import workloads as wl
     from paper_2105_14713_gb300.layer import PrunedConv2d
-
-    torch.cuda.set_device(local)
-    dev = torch.device("cuda", local)
-    stream = torch.cuda.current_stream(dev)
-    layers = workload()
     legs = []
     for layer in layers:
         W = wl.weights(layer).numpy()
@@ -310,116 +336,172 @@ def main():
         x_cpu = x_cpu if layer.dtype == "f32" else x_cpu.to(torch.bfloat16)
         x = x_cpu.to(dev)
         y = torch.empty(conv.out_shape(x.shape), dtype=x.dtype, device=dev)
-        legs.append({"layer": layer, "conv": conv, "x": x, "y": y,
-                     "x_host": x_cpu.pin_memory(), "algo": conv.algo(x.shape)})
-    flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=dev)
+        conv.workspace(x.shape)
+        legs.append({"layer": layer, "conv": conv, "x": x, "y": y, "x_cpu": x_cpu,
+                     "algo": conv.algo(x.shape)})
+    return legs
 
-    def step(evs=None):
-        for i, lg in enumerate(legs):
-            if evs is not None:
-                evs[i][0].record(stream)
-            lg["conv"](lg["x"], lg["y"])
-            if evs is not None:
-                evs[i][1].record(stream)
 
-    for _ in range(args.warmup):
+def time_legs(legs, steps, warmup, flush, stream, sampler=None):
+    """Per-leg CUDA-event times (ms) of `steps` steps, L2 flushed before each."""
+    for _ in range(warmup):
         flush.fill_(1)
-        step()
+        for lg in legs:
+            lg["conv"](lg["x"], lg["y"])
     torch.cuda.synchronize()
-
-    # ---- timed region: K steps, L2 flushed before each (outside the events) ----
     evs = [[[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in legs]
-           for _ in range(args.steps)]
-    sampler = ClockSampler(local)
-    barrier(ws)
-    torch.cuda.synchronize()
-    with sampler:
+           for _ in range(steps)]
+    ctx = sampler if sampler is not None else _Null()
+    with ctx:
         wall0 = time.perf_counter()
-        for k in range(args.steps):
+        for k in range(steps):
             flush.fill_(k & 0xff)
-            step(evs[k])
+            for i, lg in enumerate(legs):
+                evs[k][i][0].record(stream)
+                lg["conv"](lg["x"], lg["y"])
+                evs[k][i][1].record(stream)
         torch.cuda.synchronize()
         wall = time.perf_counter() - wall0
-    barrier(ws)
-    leg_ms = [[evs[k][i][0].elapsed_time(evs[k][i][1]) for k in range(args.steps)]
-              for i in range(len(legs))]
-    step_ms = sum(sum(m) for m in leg_ms) / args.steps
-    step_ms_max = max_over_ranks(step_ms, ws)
-    flops_step = sum(kept_flops(lg["layer"], lg["conv"].t) for lg in legs)
-    value = ws * flops_step / (step_ms_max * 1e-3) / 1e12
-    clocks = sampler.summary()
+    return [[evs[k][i][0].elapsed_time(evs[k][i][1]) for k in range(steps)]
+            for i in range(len(legs))], wall
 
-    # ---- per-leg roofline (live CUDA-event durations of each kernel) ----
-    pk = peaks()
-    leg_info = []
-    for i, lg in enumerate(legs):
-        layer, t = lg["layer"], lg["conv"].t
-        ms = sum(leg_ms[i]) / len(leg_ms[i])
-        fl, by = kept_flops(layer, t), alg_bytes(layer, t)
-        if lg["algo"] == "fma":
-            bound_peak, unit_peak, bound = pk["fp32_ffma_tflops"], "TFLOP/s", "alu"
-        else:
-            bound_peak, unit_peak, bound = pk["bf16_tflops"], "TFLOP/s", "tensor"
-        t_roof = max(fl / (bound_peak * 1e12), by / (pk["hbm_gbs"] * 1e9))
-        leg_info.append({
-            "dtype": layer.dtype, "algo": lg["algo"], "ms": ms, "t_kept_blocks": t,
-            "tflops": fl / (ms * 1e-3) / 1e12, "gbs": by / (ms * 1e-3) / 1e9,
-            "roofline_frac": t_roof / (ms * 1e-3), "bound": bound,
-            "pipe_peak_tflops": bound_peak})
 
-    dom = max(range(len(legs)), key=lambda i: leg_info[i]["ms"])
-    dl = leg_info[dom]
-    dlay = legs[dom]["layer"]
-    roof = {"bound": dl["bound"], "achieved": dl["tflops"], "peak": dl["pipe_peak_tflops"],
-            "unit": "TFLOP/s", "frac": dl["tflops"] / dl["pipe_peak_tflops"],
-            "traffic": traffic_for(f"{dl['algo']}_{dlay.dtype}_cfg2"),
-            "kernel": f"{dl['algo']} ({dlay.dtype} leg)",
-            "peak_source": ("FFMA: 152 SMs x 128 lanes x 2 x %.0f MHz (derived)" % pk["sm_max_mhz"]
-                            if dl["bound"] == "alu" else f"{pk['source']} bf16 tensor")}
+class _Null:
+    def __enter__(self):
+        return self
 
-    # ---- dense path (rate 0, N = C_out) at the same shape, same timing method ----
-    speedup = {}
+    def __exit__(self, *a):
+        return False
+
+
+def dense_times(legs, dev, flush, stream, reps=5):
+    """The library's own dense path (rate 0, N = C_out) at each leg's shape."""
+    from paper_2105_14713_gb300 import workloads as wl
+    from paper_2105_14713_gb300.layer import PrunedConv2d
+    out = []
     for lg in legs:
         layer = lg["layer"]
-        dl_layer = wl.dense_counterpart(layer)
-        dconv = PrunedConv2d(wl.weights(layer).numpy(), dl_layer.N, 0.0,
-                             bias=wl.bias(layer).numpy(), stride=layer.stride,
-                             padding=layer.pad, dilation=layer.dil, dtype=layer.dtype,
-                             device=dev)
-        dts = []
-        for r in range(args.warmup + 10):
+        d = wl.dense_counterpart(layer)
+        dconv = PrunedConv2d(wl.weights(layer).numpy(), d.N, 0.0, bias=wl.bias(layer).numpy(),
+                             stride=layer.stride, padding=layer.pad, dilation=layer.dil,
+                             dtype=layer.dtype, device=dev)
+        ts = []
+        for r in range(2 + reps):
             flush.fill_(r & 0xff)
             e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
             e0.record(stream)
             dconv(lg["x"], lg["y"])
             e1.record(stream)
             torch.cuda.synchronize()
-            if r >= args.warmup:
-                dts.append(e0.elapsed_time(e1))
-        dense_ms = sum(dts) / len(dts)
-        sparse_ms = [li for li in leg_info if li["dtype"] == layer.dtype][0]["ms"]
-        speedup[layer.dtype] = {"dense_ms": dense_ms, "sparse_ms": sparse_ms,
-                                "speedup": dense_ms / sparse_ms,
-                                "dense_algo": dconv.algo(lg["x"].shape)}
+            if r >= 2:
+                ts.append(e0.elapsed_time(e1))
+        out.append((sum(ts) / len(ts), dconv.algo(lg["x"].shape)))
+        del dconv
+    return out
 
-    # ---- end to end through the public API, host buffers, copies timed ----
-    e2e_ms = []
-    h2d = sum(lg["x_host"].numel() * lg["x_host"].element_size() for lg in legs)
-    d2h = sum(lg["y"].numel() * lg["y"].element_size() for lg in legs)
+
+def e2e_time(legs, dev, steps, warmup, flush, stream):
+    """Public API end to end: pinned host input -> device, conv, device -> pinned host."""
+    x_pin = [lg["x_cpu"].pin_memory() for lg in legs]
     y_host = [torch.empty(lg["y"].shape, dtype=lg["y"].dtype, pin_memory=True) for lg in legs]
-    for r in range(args.warmup + args.steps):
+    ts = []
+    for r in range(warmup + steps):
         flush.fill_(r & 0xff)
         e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         e0.record(stream)
         for i, lg in enumerate(legs):
-            xd = lg["x_host"].to(dev, non_blocking=True)
+            xd = x_pin[i].to(dev, non_blocking=True)
             yd = lg["conv"](xd)
             y_host[i].copy_(yd, non_blocking=True)
         e1.record(stream)
         torch.cuda.synchronize()
-        if r >= args.warmup:
-            e2e_ms.append(e0.elapsed_time(e1))
-    e2e_step = max_over_ranks(sum(e2e_ms) / len(e2e_ms), ws)
+        if r >= warmup:
+            ts.append(e0.elapsed_time(e1))
+    h2d = sum(t.numel() * t.element_size() for t in x_pin)
+    d2h = sum(t.numel() * t.element_size() for t in y_host)
+    return sum(ts) / len(ts), h2d, d2h
+
+
+def launches_per_step(legs):
+    # fma: one kernel; tc: the weight scatter + the GEMM (the memset is a runtime call)
+    return sum(1 if lg["algo"] == "fma" else 2 for lg in legs)
+
+
+def measure(layers, args, dev, stream, flush, ws, pk, sampler=None):
+    legs = build_legs(layers, dev)
+    leg_ms, wall = time_legs(legs, args.steps, args.warmup, flush, stream, sampler)
+    step_ms = sum(sum(m) for m in leg_ms) / args.steps
+    step_ms_max = max_over_ranks(step_ms, ws)
+    flops_step = sum(kept_flops(lg["layer"], lg["conv"].t) for lg in legs)
+    info = []
+    for i, lg in enumerate(legs):
+        layer, t = lg["layer"], lg["conv"].t
+        ms = sum(leg_ms[i]) / len(leg_ms[i])
+        rf = leg_roofline(layer, t, lg["algo"], ms, pk)
+        info.append({"name": layer.name, "dtype": layer.dtype, "algo": lg["algo"], "N": layer.N,
+                     "rate": layer.rate, "ms": ms, "t_kept_blocks": t,
+                     "tflops": kept_flops(layer, t) / (ms * 1e-3) / 1e12,
+                     "gbs": alg_bytes(layer, t) / (ms * 1e-3) / 1e9,
+                     "roofline_frac": rf["frac"], "bound": rf["bound"]})
+    return legs, leg_ms, step_ms_max, flops_step, info, wall
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--config", type=int, default=2, choices=[1, 2, 3, 4, 5])
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    args.warmup = max(args.warmup, 3)
+    rank, local, ws = dist_setup()
+    if args.impl == "reference":
+        run_reference(args, rank, ws)
+        if ws > 1:
+            import torch.distributed as dist
+            dist.destroy_process_group()
+        return
+
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    stream = torch.cuda.current_stream(dev)
+    flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=dev)
+    pk = peaks()
+
+    if args.config == 5:
+        run_sweep(args, dev, stream, flush, ws, rank, pk)
+        return
+
+    layers = workload(args.config)
+    sampler = ClockSampler(local)
+    barrier(ws)
+    torch.cuda.synchronize()
+    legs, leg_ms, step_ms_max, flops_step, info, wall = measure(
+        layers, args, dev, stream, flush, ws, pk, sampler)
+    barrier(ws)
+    value = ws * flops_step / (step_ms_max * 1e-3) / 1e12
+    clocks = sampler.summary()
+
+    # dominant kernel: the leg with the largest time
+    dom = max(range(len(legs)), key=lambda i: info[i]["ms"])
+    dl, dlay = info[dom], legs[dom]["layer"]
+    rf = leg_roofline(dlay, legs[dom]["conv"].t, dl["algo"], dl["ms"], pk)
+    roof = dict(rf)
+    roof["traffic"] = traffic_for(f"{dl['algo']}_{dlay.name}")
+    roof["kernel"] = f"{dl['algo']} ({dlay.name})"
+
+    dts = dense_times(legs, dev, flush, stream)
+    sparse_ms = [i["ms"] for i in info]
+    speedup = {"dense_ms": sum(d for d, _ in dts), "sparse_ms": sum(sparse_ms),
+               "speedup": sum(d for d, _ in dts) / sum(sparse_ms),
+               "per_leg": [{"name": info[i]["name"], "dense_ms": dts[i][0], "dense_algo": dts[i][1],
+                            "sparse_ms": sparse_ms[i], "speedup": dts[i][0] / sparse_ms[i]}
+                           for i in range(len(legs))]}
+
+    e2e_ms, h2d, d2h = e2e_time(legs, dev, max(3, args.steps // 4), 2, flush, stream)
+    e2e_ms = max_over_ranks(e2e_ms, ws)
 
     cpu = None
     if rank == 0 and ws == 1 and not args.no_cpu_baseline:
@@ -430,16 +512,15 @@ def main():
             "metric": METRIC, "value": value, "unit": "TFLOP/s", "n_gpus": ws,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": step_ms_max,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
-            "dtype": "f32+bf16", "data": "synthetic (seeded Kaiming-normal weights, ReLU(N(0,1)) "
-                                         "activations)",
-            "config": config_json(layers),
+            "dtype": "+".join(sorted({l.dtype for l in layers})),
+            "data": "synthetic (seeded Kaiming-normal or N(0,0.05) weights, ReLU(N(0,1)) activations)",
+            "config": config_json(args.config, layers),
             "roofline": roof,
-            "legs": leg_info,
+            "legs": info,
             "speedup_vs_dense": speedup,
-            "e2e": {"value": ws * flops_step / (e2e_step * 1e-3) / 1e12, "unit": "TFLOP/s",
-                    "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
-                    "ms_per_step": e2e_step},
-            "gpu_launches": len(legs) * args.steps,
+            "e2e": {"value": ws * flops_step / (e2e_ms * 1e-3) / 1e12, "unit": "TFLOP/s",
+                    "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "ms_per_step": e2e_ms},
+            "gpu_launches": launches_per_step(legs) * args.steps,
             "clocks": clocks,
             "wall_s_timed_region": wall,
             "peaks": pk,
@@ -449,6 +530,49 @@ def main():
     if ws > 1:
         import torch.distributed as dist
         dist.destroy_process_group()
+
+
+def run_sweep(args, dev, stream, flush, ws, rank, pk):
+    from paper_2105_14713_gb300 import workloads as wl
+    points = []
+    total_flops, total_ms = 0.0, 0.0
+    sampler = ClockSampler(0 if dev.index is None else dev.index)
+    steps = max(3, min(args.steps, 10))
+    with sampler:
+        for dtype in ("f32", "bf16"):
+            for N in wl.SWEEP_N:
+                dense_ms = None
+                for rate in wl.SWEEP_RATE:
+                    layer = wl.config5(N=N, rate=rate, dtype=dtype, seed=0)[0]
+                    a2 = argparse.Namespace(steps=steps, warmup=args.warmup)
+                    legs, leg_ms, step_ms, flops, info, _ = measure([layer], a2, dev, stream, flush,
+                                                                    ws, pk)
+                    if dense_ms is None:
+                        dense_ms = dense_times(legs, dev, flush, stream)[0]
+                    total_flops += flops
+                    total_ms += step_ms
+                    p = dict(info[0])
+                    p["speedup_vs_dense"] = dense_ms[0] / p["ms"]
+                    p["dense_algo"] = dense_ms[1]
+                    points.append(p)
+                    del legs
+    value = ws * total_flops / (total_ms * 1e-3) / 1e12
+    dom = max(points, key=lambda p: p["ms"])
+    layer = wl.config5(N=dom["N"], rate=dom["rate"], dtype=dom["dtype"])[0]
+    rf = leg_roofline(layer, dom["t_kept_blocks"], dom["algo"], dom["ms"], pk)
+    rf["traffic"] = None
+    rf["kernel"] = f"{dom['algo']} ({dom['name']})"
+    if rank == 0:
+        print(json.dumps({
+            "metric": METRIC, "value": value, "unit": "TFLOP/s", "n_gpus": ws,
+            "steps": steps, "warmup": args.warmup, "ms_per_step": total_ms,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32+bf16",
+            "data": "synthetic (seeded Kaiming-normal weights, ReLU(N(0,1)) activations)",
+            "config": {"workload": DESCRIPTIONS[5], "config_id": 5, "points": len(points),
+                       "parallelism": "replicas", "l2": "flushed before every step (256 MB write)"},
+            "roofline": rf, "points": points, "clocks": sampler.summary(),
+            "gpu_launches": sum(1 if p["algo"] == "fma" else 2 for p in points) * steps,
+            "peaks": pk, "cpu_baseline": None}), flush=True)
 
 
 if __name__ == "__main__":
