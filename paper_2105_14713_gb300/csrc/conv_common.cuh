@@ -91,6 +91,31 @@ __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity)
     return true;
 }
 
+// Single test of a phase, without suspending.
+__device__ __forceinline__ bool mbar_test(uint32_t bar, uint32_t parity)
+{
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\tmbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}\n"
+        : "=r"(ok)
+        : "r"(bar), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+// Bounded wait (~2^31 SM cycles) that sleeps `ns` nanoseconds between tests,
+// for warps that are not on the critical path: they stay off the issue slots.
+__device__ __forceinline__ bool mbar_wait_backoff(uint32_t bar, uint32_t parity, unsigned ns)
+{
+    if (mbar_test(bar, parity)) return true;
+    const long long t0 = clock64();
+    do {
+        __nanosleep(ns);
+        if (mbar_test(bar, parity)) return true;
+    } while (clock64() - t0 <= (1ll << 31));
+    return false;
+}
+
 // bf16 bits -> fp32 (exact).
 __device__ __forceinline__ float bf16lo(uint32_t v) { return __uint_as_float(v << 16); }
 __device__ __forceinline__ float bf16hi(uint32_t v) { return __uint_as_float(v & 0xffff0000u); }

@@ -85,6 +85,22 @@ __device__ __forceinline__ int copy_pixel(int lane, int i)
     else return 16 * i + m;
 }
 
+__device__ __forceinline__ float4 lds128(uint32_t a)
+{
+    float4 v;
+    asm volatile("ld.shared.v4.f32 {%0, %1, %2, %3}, [%4];\n"
+                 : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
+                 : "r"(a)
+                 : "memory");
+    return v;
+}
+__device__ __forceinline__ float lds32(uint32_t a)
+{
+    float v;
+    asm volatile("ld.shared.f32 %0, [%1];\n" : "=f"(v) : "r"(a) : "memory");
+    return v;
+}
+
 template <typename TIN, int NS, int SPW>
 __global__ void __launch_bounds__(kThreads, 1)
 fma_conv_kernel(const ConvArgs a, const int n_units, const int n_ct)
@@ -271,7 +287,7 @@ fma_conv_kernel(const ConvArgs a, const int n_units, const int n_ct)
             const int kend = k0 + min(kKC, a.C - cc0);
             cc0 += kKC;
             if (cc0 >= a.C) { cc0 = 0; tapC += a.C; }
-            const float *xa = xs_all + st * kKC * kXS + 4 * lane;
+            const uint32_t xa = smem_u32(xs_all + st * kKC * kXS + 4 * lane);
             int cnt[SPW], mycl[SPW];
             __syncwarp();                       // previous chunk's reads of ds are done
 #pragma unroll
@@ -294,48 +310,53 @@ fma_conv_kernel(const ConvArgs a, const int n_units, const int n_ct)
             __syncwarp();                       // ds visible to the whole warp
 #pragma unroll
             for (int s = 0; s < SPW; ++s) {
-                const float *dsr = ds + s * 32 * NS;
+                const uint32_t dsr = smem_u32(ds + s * 32 * NS);
                 const int n = cnt[s];
                 if (n == 0) continue;
-                // Software pipeline: the shared loads of entry j+1 are issued
-                // before the 8*NS FFMAs of entry j.
-                float4 xc0, xc1;
-                float dc[NS];
+                // Software pipeline over two register sets (no copies): the
+                // shared loads of entry j+1 are issued before the 8*NS FFMAs
+                // of entry j.
+                float4 xa0, xa1, xb0, xb1;
+                float da[NS], db[NS];
                 auto load_entry = [&](int j, float4 &v0, float4 &v1, float (&dv)[NS]) {
                     const int cl = __shfl_sync(0xffffffffu, mycl[s], j);
-                    v0 = *reinterpret_cast<const float4 *>(xa + cl * kXS);
-                    v1 = *reinterpret_cast<const float4 *>(xa + cl * kXS + 128);
+                    const uint32_t xad = xa + cl * (kXS * 4);
+                    v0 = lds128(xad);
+                    v1 = lds128(xad + 512);
+                    const uint32_t dad = dsr + j * (NS * 4);
                     if constexpr (NS % 4 == 0) {
 #pragma unroll
                         for (int c = 0; c < NS; c += 4) {
-                            const float4 v = *reinterpret_cast<const float4 *>(dsr + j * NS + c);
+                            const float4 v = lds128(dad + 4 * c);
                             dv[c] = v.x; dv[c + 1] = v.y; dv[c + 2] = v.z; dv[c + 3] = v.w;
                         }
                     } else {
 #pragma unroll
-                        for (int c = 0; c < NS; ++c) dv[c] = dsr[j * NS + c];
+                        for (int c = 0; c < NS; ++c) dv[c] = lds32(dad + 4 * c);
                     }
                 };
-                load_entry(0, xc0, xc1, dc);
-                for (int j = 0; j < n; ++j) {
-                    float4 xn0, xn1;
-                    float dn[NS];
-                    load_entry(min(j + 1, n - 1), xn0, xn1, dn);
+                auto fma_entry = [&](const float4 &v0, const float4 &v1, const float (&dv)[NS]) {
 #pragma unroll
                     for (int c = 0; c < NS; ++c) {
-                        acc[s][0][c] = fmaf(xc0.x, dc[c], acc[s][0][c]);
-                        acc[s][1][c] = fmaf(xc0.y, dc[c], acc[s][1][c]);
-                        acc[s][2][c] = fmaf(xc0.z, dc[c], acc[s][2][c]);
-                        acc[s][3][c] = fmaf(xc0.w, dc[c], acc[s][3][c]);
-                        acc[s][4][c] = fmaf(xc1.x, dc[c], acc[s][4][c]);
-                        acc[s][5][c] = fmaf(xc1.y, dc[c], acc[s][5][c]);
-                        acc[s][6][c] = fmaf(xc1.z, dc[c], acc[s][6][c]);
-                        acc[s][7][c] = fmaf(xc1.w, dc[c], acc[s][7][c]);
+                        acc[s][0][c] = fmaf(v0.x, dv[c], acc[s][0][c]);
+                        acc[s][1][c] = fmaf(v0.y, dv[c], acc[s][1][c]);
+                        acc[s][2][c] = fmaf(v0.z, dv[c], acc[s][2][c]);
+                        acc[s][3][c] = fmaf(v0.w, dv[c], acc[s][3][c]);
+                        acc[s][4][c] = fmaf(v1.x, dv[c], acc[s][4][c]);
+                        acc[s][5][c] = fmaf(v1.y, dv[c], acc[s][5][c]);
+                        acc[s][6][c] = fmaf(v1.z, dv[c], acc[s][6][c]);
+                        acc[s][7][c] = fmaf(v1.w, dv[c], acc[s][7][c]);
                     }
-                    xc0 = xn0; xc1 = xn1;
-#pragma unroll
-                    for (int c = 0; c < NS; ++c) dc[c] = dn[c];
+                };
+                load_entry(0, xa0, xa1, da);
+                int j = 0;
+                for (; j + 2 <= n; j += 2) {
+                    load_entry(j + 1, xb0, xb1, db);
+                    fma_entry(xa0, xa1, da);
+                    load_entry(min(j + 2, n - 1), xa0, xa1, da);
+                    fma_entry(xb0, xb1, db);
                 }
+                if (j < n) fma_entry(xa0, xa1, da);
             }
             __syncwarp();
             if (lane == 0) mbar_arrive(bar_empty + 8 * st);
