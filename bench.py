@@ -96,21 +96,42 @@ def peaks():
             "fp32_ffma_tflops": fp32, "sm_max_mhz": sm_max, "source": src}
 
 
+# tf32 / bf16 dense tensor rates, nominal (1.1 / 2.25 PFLOP/s per GB300)
+TF32_PER_BF16 = 1.1 / 2.25
+
+
 def leg_roofline(layer, t, algo, ms, pk):
+    """Roofline of one leg: algorithmic (kept) flops and bytes against the
+    pipe the kernel runs on and HBM.  The tensor-core GEMM multiplies the
+    decoded dense matrix (zeros included), and for fp32 issues three tf32
+    products per term: `issued_frac` is that issued tensor work against the
+    same peak, i.e. how busy the pipe is, not how useful the work is."""
     fl, by = kept_flops(layer, t), alg_bytes(layer, t)
+    issued = None
     if algo == "fma":
         pipe, pipe_name, pipe_src = pk["fp32_ffma_tflops"], "alu", \
             "FFMA: 152 SMs x 128 lanes x 2 x %.0f MHz (derived)" % pk["sm_max_mhz"]
+    elif layer.dtype == "f32":
+        pipe, pipe_name = pk["bf16_tflops"] * TF32_PER_BF16, "tensor"
+        pipe_src = f"tf32 = {pk['source']} bf16 tensor (burst) x nominal tf32/bf16 1.1/2.25"
+        issued = 3 * kept_flops(layer, layer.K * (layer.C_out // layer.N))
     else:
         pipe, pipe_name, pipe_src = pk["bf16_tflops"], "tensor", f"{pk['source']} bf16 tensor (burst)"
+        if algo == "tc":
+            issued = kept_flops(layer, layer.K * (layer.C_out // layer.N))
     t_pipe = fl / (pipe * 1e12)
     t_mem = by / (pk["hbm_gbs"] * 1e9)
     sec = ms * 1e-3
     if t_pipe >= t_mem:
-        return {"bound": pipe_name, "achieved": fl / sec / 1e12, "peak": pipe, "unit": "TFLOP/s",
-                "frac": t_pipe / sec, "peak_source": pipe_src}
-    return {"bound": "hbm", "achieved": by / sec / 1e9, "peak": pk["hbm_gbs"], "unit": "GB/s",
-            "frac": t_mem / sec, "peak_source": f"{pk['source']} HBM copy"}
+        out = {"bound": pipe_name, "achieved": fl / sec / 1e12, "peak": pipe, "unit": "TFLOP/s",
+               "frac": t_pipe / sec, "peak_source": pipe_src}
+    else:
+        out = {"bound": "hbm", "achieved": by / sec / 1e9, "peak": pk["hbm_gbs"], "unit": "GB/s",
+               "frac": t_mem / sec, "peak_source": f"{pk['source']} HBM copy"}
+    if issued is not None:
+        out["issued_tflops"] = issued / sec / 1e12
+        out["issued_frac"] = issued / sec / 1e12 / pipe
+    return out
 
 
 class ClockSampler:
@@ -423,7 +444,7 @@ def e2e_time(legs, dev, steps, warmup, flush, stream):
 
 
 def launches_per_step(legs):
-    # fma: one kernel; tc: the weight scatter + the GEMM (the memset is a runtime call)
+    # fma: one kernel; tc: the weight decode + the GEMM
     return sum(1 if lg["algo"] == "fma" else 2 for lg in legs)
 
 

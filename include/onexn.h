@@ -58,13 +58,16 @@ typedef enum { ONEXN_GRAN_TAP = 0, ONEXN_GRAN_KERNEL = 1 } onexn_granularity;
 
 /* onexn_conv_fwd flags */
 #define ONEXN_RELU 0x1u               /* y = max(y, 0) after the bias */
-/* Kernel selection (bits 8..11).  AUTO picks by dtype, N and density. */
+/* Kernel selection (bits 8..11).  AUTO picks by dtype, N and density:
+ * the tensor-core GEMM when its workspace fits and its dense work is
+ * estimated to take less time than the FFMA kernel's kept work. */
 #define ONEXN_ALGO_SHIFT 8
 #define ONEXN_ALGO_MASK (0xFu << ONEXN_ALGO_SHIFT)
 #define ONEXN_ALGO_AUTO (0u << ONEXN_ALGO_SHIFT)
 #define ONEXN_ALGO_FMA (1u << ONEXN_ALGO_SHIFT)   /* CUDA-core FFMA, any N, fp32/bf16 */
 #define ONEXN_ALGO_MMA (2u << ONEXN_ALGO_SHIFT)   /* bf16 gathered tensor-core kernel */
-#define ONEXN_ALGO_TC (3u << ONEXN_ALGO_SHIFT)    /* bf16 tcgen05 GEMM on the decoded mask */
+#define ONEXN_ALGO_TC (3u << ONEXN_ALGO_SHIFT)    /* tcgen05 GEMM on the decoded mask: bf16,
+                                                     or fp32 as three tf32 products */
 
 /* Message for the last failed call on this thread ("" if none). */
 const char *onexn_last_error(void);
@@ -200,8 +203,10 @@ onexn_status onexn_conv_fwd(const onexn_conv_desc *desc, const int32_t *P, const
  * onexn_conv_workspace_size -- bytes of device workspace onexn_conv_fwd
  * needs for these arguments with this flags' ALGO (for AUTO: the largest
  * need among the families AUTO may pick, so that passing this many bytes
- * lets AUTO choose freely).  ONEXN_ALGO_TC needs C_out * KH*KW*C_in
- * bf16 values (the decoded masked weights); ONEXN_ALGO_FMA needs none.
+ * lets AUTO choose freely).  ONEXN_ALGO_TC needs the decoded masked
+ * weights: C_out * KH*KW*C_in bf16 values (dtype ONEXN_BF16), or twice
+ * C_out * KH*KW*C_in fp32 values, their tf32 high and low parts
+ * (ONEXN_F32); rounded up to 256 bytes.  ONEXN_ALGO_FMA needs none.
  */
 onexn_status onexn_conv_workspace_size(const onexn_conv_desc *desc, int N, int64_t t, int dtype,
                                        unsigned flags, size_t *bytes);
@@ -218,9 +223,9 @@ onexn_status onexn_conv_algo(const onexn_conv_desc *desc, int N, int64_t t, int 
  * onexn_conv_fwd_noalloc -- onexn_conv_fwd for callers that cannot allocate
  * device memory.  The paper has no counterpart; it is a deployment aid.
  *
- * It runs the bf16 tensor-core family (ONEXN_ALGO_TC; flags may carry
+ * It runs the tensor-core family (ONEXN_ALGO_TC; flags may carry
  * ONEXN_RELU and AUTO or TC) with its scratch -- the decoded weight matrix,
- * C_out * KH*KW*C_in bf16 values -- in a fixed 8 MiB array that is part of
+ * as sized by onexn_conv_workspace_size -- in a fixed 8 MiB array that is part of
  * the library's device image, instead of a caller workspace.  It never
  * calls cudaMalloc, cudaFree or any other allocating routine.  Who needs it:
  * code running while a stream is captured into a CUDA graph (allocating
@@ -230,7 +235,7 @@ onexn_status onexn_conv_algo(const onexn_conv_desc *desc, int N, int64_t t, int 
  *   Arguments as onexn_conv_fwd (x, y, P, I, D, bias are caller-owned).
  *   EINVAL: the decoded weights would exceed 8 MiB (use onexn_conv_fwd with
  *   a workspace), or another ALGO was forced.  EUNSUPPORTED: the
- *   tensor-core family cannot run the case (for instance fp32).
+ *   tensor-core family cannot run the case (channel counts, strides).
  * Every GPU that loads the library keeps the 8 MiB until the process exits.
  * All calls share the array, so calls that overlap on the GPU (different
  * streams or host threads) race and may return wrong results.  Each call

@@ -10,9 +10,9 @@ namespace onexn {
 cudaError_t launch_fma(const ConvArgs &a, int dtype, cudaStream_t st);
 cudaError_t launch_mma(const ConvArgs &a, cudaStream_t st);
 bool mma_supports(const ConvArgs &a);
-cudaError_t launch_tc(const ConvArgs &a, void *workspace, cudaStream_t st);
-bool tc_supports(const ConvArgs &a);
-size_t tc_workspace_bytes(const ConvArgs &a);
+cudaError_t launch_tc(const ConvArgs &a, int dtype, void *workspace, cudaStream_t st);
+bool tc_supports(const ConvArgs &a, int dtype);
+size_t tc_workspace_bytes(const ConvArgs &a, int dtype);
 }  // namespace onexn
 
 using onexn::fail;
@@ -126,9 +126,9 @@ onexn_status check_pointers(const int32_t *P, const int32_t *I, const void *D, c
 }
 
 // Workspace a family needs for these arguments.
-size_t workspace_for(unsigned algo, const onexn::ConvArgs &a)
+size_t workspace_for(unsigned algo, const onexn::ConvArgs &a, int dtype)
 {
-    return algo == ONEXN_ALGO_TC ? onexn::tc_workspace_bytes(a) : 0;
+    return algo == ONEXN_ALGO_TC ? onexn::tc_workspace_bytes(a, dtype) : 0;
 }
 
 // Can the family run this case at all (dtype, shape)?
@@ -137,20 +137,40 @@ bool supports(unsigned algo, const onexn::ConvArgs &a, int dtype)
     switch (algo) {
     case ONEXN_ALGO_FMA: return true;
     case ONEXN_ALGO_MMA: return dtype == ONEXN_BF16 && onexn::mma_supports(a);
-    case ONEXN_ALGO_TC: return dtype == ONEXN_BF16 && onexn::tc_supports(a);
+    case ONEXN_ALGO_TC: return onexn::tc_supports(a, dtype);
     default: return false;
     }
 }
 
-// Kernel family for AUTO: bf16 runs on the tcgen05 GEMM when its workspace
-// fits; everything else (fp32, bf16 without workspace) on the FFMA kernel.
+// Cost model of AUTO, in ns per multiply-add, fitted to GB300 timings of a
+// 3x3 512->512 layer on 128x14x14 at 50% and 90% pruned (fp32 and bf16; the
+// affine fit predicts the 70% point within 2%).  The FFMA kernel stages the
+// activations of every 256-pixel x 64-column unit whatever is kept (a floor
+// per dense multiply-add, higher for small N) and then does only the kept
+// work (t*N weights per pixel), faster for wider blocks that share each
+// staged activation.  The tensor-core GEMM decodes the weights into the
+// workspace (about 2000 bytes per ns) and does the dense work (C_out*K per
+// pixel; fp32 issues three tf32 products per term).
+double fma_floor(int N) { return N >= 4 ? 1.33e-5 : N >= 2 ? 1.66e-5 : 2.67e-5; }
+double fma_per_kept(int N) { return N >= 8 ? 3.0e-5 : N >= 4 ? 4.3e-5 : N >= 2 ? 7.2e-5 : 1.44e-4; }
+double tc_per_dense(int dtype) { return dtype == ONEXN_F32 ? 7.9e-6 : 2.3e-6; }
+constexpr double kDecodeNsPerByte = 1.0 / 2000.0;
+
+// Kernel family for AUTO: the tcgen05 GEMM when its workspace fits and the
+// cost model does not expect the FFMA kernel to be faster; otherwise FFMA.
 unsigned pick_algo(const onexn::ConvArgs &a, int dtype, unsigned flags, size_t ws_bytes)
 {
     const unsigned forced = flags & ONEXN_ALGO_MASK;
     if (forced != ONEXN_ALGO_AUTO) return forced;
-    if (supports(ONEXN_ALGO_TC, a, dtype) && ws_bytes >= workspace_for(ONEXN_ALGO_TC, a))
-        return ONEXN_ALGO_TC;
-    return ONEXN_ALGO_FMA;
+    if (!supports(ONEXN_ALGO_TC, a, dtype) || ws_bytes < workspace_for(ONEXN_ALGO_TC, a, dtype))
+        return ONEXN_ALGO_FMA;
+    if (a.t == 0) return ONEXN_ALGO_FMA;                  // bias only
+    const double kept = static_cast<double>(a.t) * a.N * a.P_pix;
+    const double dense = static_cast<double>(a.C_out) * a.KH * a.KW * a.C * a.P_pix;
+    const double fma_ns = dense * fma_floor(a.N) + kept * fma_per_kept(a.N);
+    const double tc_ns = dense * tc_per_dense(dtype) +
+                         static_cast<double>(workspace_for(ONEXN_ALGO_TC, a, dtype)) * kDecodeNsPerByte;
+    return fma_ns < tc_ns ? ONEXN_ALGO_FMA : ONEXN_ALGO_TC;
 }
 
 onexn_status check_algo(unsigned algo, const onexn::ConvArgs &a, int dtype, size_t ws_bytes)
@@ -160,7 +180,7 @@ onexn_status check_algo(unsigned algo, const onexn::ConvArgs &a, int dtype, size
     if (!supports(algo, a, dtype))
         return fail(ONEXN_EUNSUPPORTED, "conv: algo %u cannot run this case (dtype/shape)",
                     algo >> ONEXN_ALGO_SHIFT);
-    const size_t need = workspace_for(algo, a);
+    const size_t need = workspace_for(algo, a, dtype);
     if (ws_bytes < need)
         return fail(ONEXN_EINVAL, "conv: algo %u needs %zu bytes of workspace, got %zu",
                     algo >> ONEXN_ALGO_SHIFT, need, ws_bytes);
@@ -196,11 +216,11 @@ extern "C" onexn_status onexn_conv_workspace_size(const onexn_conv_desc *desc, i
     size_t need = 0;
     if (forced == ONEXN_ALGO_AUTO) {
         for (unsigned al : {ONEXN_ALGO_FMA, ONEXN_ALGO_MMA, ONEXN_ALGO_TC})
-            if (supports(al, a, dtype) && workspace_for(al, a) > need) need = workspace_for(al, a);
+            if (supports(al, a, dtype) && workspace_for(al, a, dtype) > need) need = workspace_for(al, a, dtype);
     } else {
         if (!supports(forced, a, dtype))
             return fail(ONEXN_EUNSUPPORTED, "conv: algo %u cannot run this case", forced >> ONEXN_ALGO_SHIFT);
-        need = workspace_for(forced, a);
+        need = workspace_for(forced, a, dtype);
     }
     *bytes = need;
     return ONEXN_OK;
@@ -229,7 +249,7 @@ extern "C" onexn_status onexn_conv_fwd(const onexn_conv_desc *desc, const int32_
     if (e != cudaSuccess) return fail(ONEXN_ECUDA, "conv: status word: %s", cudaGetErrorString(e));
     if (algo == ONEXN_ALGO_FMA) e = onexn::launch_fma(a, dtype, s);
     else if (algo == ONEXN_ALGO_MMA) e = onexn::launch_mma(a, s);
-    else e = onexn::launch_tc(a, workspace, s);
+    else e = onexn::launch_tc(a, dtype, workspace, s);
     if (e != cudaSuccess) return fail(ONEXN_ECUDA, "conv: launch failed: %s", cudaGetErrorString(e));
     return ONEXN_OK;
 }

@@ -1,8 +1,9 @@
-// onexn_conv_fwd_noalloc: the bf16 tensor-core convolution for callers that
+// onexn_conv_fwd_noalloc: the tensor-core convolution for callers that
 // cannot allocate device memory.
 //
 // The tensor-core family needs scratch space for the decoded weight matrix
-// (C_out x KH*KW*C_in bf16 values).  onexn_conv_fwd expects the caller to
+// (C_out x KH*KW*C_in bf16 values, or twice that many fp32 values for fp32
+// layers).  onexn_conv_fwd expects the caller to
 // provide it.  Some callers cannot: code that runs while a CUDA stream is
 // being captured into a graph (a cudaMalloc there breaks the capture), hosts
 // that forbid allocation after start-up so that latency stays predictable,
@@ -20,9 +21,9 @@
 //    different streams, or from different host threads) race on it and may
 //    produce wrong results; serialise them.
 //  * Nothing in the array has to start at zero: the decode step of each
-//    call rewrites every byte of the region the call uses (zeros, then the
-//    kept weights) before the GEMM reads it; contents left by the previous
-//    call are never read.
+//    call writes every element of the region the call uses (a kept weight
+//    or zero) before the GEMM reads it; contents left by the previous call
+//    are never read.
 //  * The device address of the array is looked up once per device, on the
 //    first call made with that device current (cudaGetSymbolAddress).  Make
 //    that first call before any stream capture begins.

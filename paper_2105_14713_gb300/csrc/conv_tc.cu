@@ -1,32 +1,48 @@
-// bf16 tensor-core (tcgen05) kernel of the 1xN-pruned convolution.
+// Tensor-core (tcgen05) kernels of the 1xN-pruned convolution.
 //
 // The kept blocks of Eq. 7 are first decoded from (P, I, D) into the masked
-// weight matrix W[o][k] (bf16, K-major, zero where a block was pruned),
-// Omega-bar of Eq. 6, in a caller-provided workspace: a memset, then one
-// thread per kept weight D[z][n] writes it to W[gN + n][I[z]].  The layer output
+// weight matrix W[o][k] (K-major, zero where a block was pruned), Omega-bar
+// of Eq. 6, in a caller-provided workspace, by one kernel that writes every
+// element once.  The layer output
 // Y = X (im2col) * W^T is then an implicit GEMM on the 5th-generation tensor
 // cores: per tile M = 128 consecutive output pixels x BN output channels,
-// K walked in chunks of one tap x 64 channels.
+// K walked in chunks of one tap x 128 bytes of channels (64 bf16 / 32 fp32).
 //
-// Warp roles (6 warps, one persistent CTA per SM):
+// Two element types share the kernel:
+//  * bf16 inputs: one tcgen05.mma.kind::f16 per K step of 16, fp32 accumulate.
+//  * fp32 inputs: each product is split into tf32 parts,
+//      x*w ~= x_hi*w_hi + x_lo*w_hi + x_hi*w_lo,
+//    three tcgen05.mma.kind::tf32 per K step of 8 into one fp32 accumulator.
+//    w_hi = w rounded to tf32 and w_lo = w - w_hi are decoded into the
+//    workspace; x_hi = x with its 13 low mantissa bits cleared and
+//    x_lo = x - x_hi are computed per chunk from the A tile in shared memory
+//    and written to tensor memory, from where the MMAs read A (so shared
+//    memory only feeds them B).  Both hi parts are exact tf32 values, so the
+//    products do not depend on how the tensor core reduces an fp32 operand
+//    to tf32.  The dropped x_lo*w_lo term and the tf32 reduction of the lo
+//    parts are ~2^-20 relative to |x*w|.
+//
+// Warp roles (one persistent CTA per SM):
 //  * warp 0, producer: one thread issues, per chunk, a TMA im2col load of the
-//    A tile (128 output pixels x 64 channels of the tap: the hardware walks
-//    the output pixels across rows and images and reads zeros in the
-//    padding) and a TMA tiled load of the B tile (BN rows x 64 of W), both
-//    in the 128-byte-swizzled K-major layout the tensor core reads, counted
-//    in bytes on the stage's "full" mbarrier (ring of S stages).
-//  * warp 1, MMA: allocates 2*BN TMEM columns (a double-buffered 128 x BN
-//    fp32 accumulator); one thread waits "full", issues four
-//    tcgen05.mma (K = 16 each) per chunk and commits them to the stage's
-//    "empty" mbarrier; after the last chunk of a tile it commits to the
-//    accumulator's "tmem_full" mbarrier.
+//    A tile (128 output pixels x 128 bytes of channels of the tap: the
+//    hardware walks the output pixels across rows and images and reads zeros
+//    in the padding; for 1x1, stride-1, unpadded layers a plain tiled 2-D box
+//    of x viewed as [B*H*W][C_in]) and tiled TMA loads of the B tile(s)
+//    (BN rows x 128 bytes of W), all in the 128-byte-swizzled K-major layout
+//    the tensor core reads, counted in bytes on the stage's "full" mbarrier.
+//  * warps 6-9 (fp32 only), split: wait "full" (and for the TMEM A slot to
+//    be free: "empty" of the chunk two back), read one pixel row of the A
+//    tile each, write x_hi | x_lo to the slot's TMEM lanes, arrive "split".
+//  * warp 1, MMA: allocates the TMEM (a double-buffered 128 x BN fp32
+//    accumulator, plus the A ring for fp32); one thread waits for the stage ("full", or "split"
+//    for fp32), issues the MMAs of the chunk and commits them to the
+//    stage's "empty" mbarrier; after the last chunk of a tile it commits to
+//    the accumulator's "tmem_full" mbarrier.
 //  * warps 2-5, epilogue: wait "tmem_full", read the accumulator with
 //    tcgen05.ld (warp w reads TMEM lanes 32*(w%4)..+31 = its 32 pixels),
-//    release it ("tmem_empty") so the MMA warp can reuse the buffer, add the
-//    bias, apply ReLU, round to bf16 into a 128-byte-swizzled staging tile
-//    in shared memory, and write the tile to y[p][o] with TMA bulk stores.
-// For 1x1, stride-1, unpadded layers the A tile is a plain 2-D box of
-// x viewed as [B*H*W][C_in] (tiled TMA) instead of an im2col load.
+//    release it ("tmem_empty"), add the bias, apply ReLU and store NHWC:
+//    bf16 through a 128-byte-swizzled staging tile and TMA bulk stores,
+//    fp32 directly from registers.
 // All waits are bounded (about one second each); on expiry the status word
 // gets ONEXN_ETIMEOUT, every role stops, outstanding MMAs are drained and
 // the TMEM is freed before the kernel returns.
@@ -45,45 +61,108 @@ namespace {
 
 constexpr int kProdWarp = 0;
 constexpr int kMmaWarp = 1;
-constexpr int kEpiWarps = 4;          // warps 2..5
-constexpr int kThreadsTc = 32 * 6;
+constexpr int kEpiWarp0 = 2;          // warps 2..5
+constexpr int kSplitWarp0 = 6;        // warps 6..9 (fp32 only)
 constexpr int kBM = 128;              // pixels per tile (UMMA M)
-constexpr int kBK = 64;               // channels per chunk: one 128-byte swizzle row
+constexpr int kRowBytes = 128;        // bytes of K per tile row: one 128-byte swizzle row
 
-template <int BN>
+struct TcBf16 {
+    using T = __nv_bfloat16;
+    static constexpr bool kSplit = false;
+    static constexpr int kBK = 64;                 // channels per chunk
+    static constexpr int kKStep = 16;              // K per MMA
+    static constexpr CUtensorMapDataType kTmap = CU_TENSOR_MAP_DATA_TYPE_BFLOAT16;
+    static constexpr int kWarps = 6;
+};
+struct TcF32 {
+    using T = float;
+    static constexpr bool kSplit = true;
+    static constexpr int kBK = 32;
+    static constexpr int kKStep = 8;
+    static constexpr CUtensorMapDataType kTmap = CU_TENSOR_MAP_DATA_TYPE_FLOAT32;
+    static constexpr int kWarps = 10;
+};
+
+constexpr int kSmemMax = 232448;      // dynamic shared memory per CTA (opt-in maximum)
+
+constexpr int pow2_at_least(int v, int p = 32) { return p >= v ? p : pow2_at_least(v, 2 * p); }
+
+template <typename Tr, int BN>
 struct TcLayout {
-    static constexpr int kS = BN >= 256 ? 3 : 6;              // stages in the ring
-    static constexpr int kA = kBM * kBK * 2;                  // 16 KB
-    static constexpr int kB = BN * kBK * 2;                   // 8/16/32 KB
-    static constexpr int kStage = kA + kB;                    // multiple of 1024
-    static constexpr int kOut = kS * kStage;                  // output staging: BN/64 atoms
-    static constexpr int kOutBytes = kBM * BN * 2;            //   of [128 rows][64 cols] bf16
-    static constexpr int kBias = kOut + kOutBytes;            // BN fp32
+    static constexpr int kA = kBM * kRowBytes;                       // 16 KB
+    static constexpr int kB = BN * kRowBytes;                        // 8/16/32 KB
+    static constexpr int kStage = kA + (Tr::kSplit ? 2 * kB : kB);   // [A | B_hi | B_lo]
+    static constexpr int kTx = kStage;                               // bytes the TMA brings
+    static constexpr int kOutBytes = Tr::kSplit ? 0 : kBM * BN * 2;  // bf16 staging tile
+    static constexpr int kFixed = 1024 + kOutBytes + BN * 4 + (3 * 6 + 5) * 8 + 16;
+    static constexpr int kS = ((kSmemMax - kFixed) / kStage) > 6 ? 6 : ((kSmemMax - kFixed) / kStage);
+    static constexpr int kOut = kS * kStage;
+    static constexpr int kBias = kOut + kOutBytes;                    // BN fp32
     static constexpr int kBar = kBias + BN * 4;
-    // full[S], empty[S], tmem_full[2], tmem_empty[2], drain, then the TMEM holder
-    static constexpr int kHolder = kBar + (2 * kS + 5) * 8;
+    // full[S], split[S], empty[S], tmem_full[2], tmem_empty[2], drain, TMEM holder
+    static constexpr int kHolder = kBar + (3 * kS + 5) * 8;
     static constexpr int kBytes = kHolder + 16;
-    static constexpr int kAlloc = kBytes + 1024;              // room to align the base to 1024
+    static constexpr int kAlloc = kBytes + 1024;                      // room to align the base to 1024
+    // TMEM columns: the fp32 accumulator buffers (two when they fit next to
+    // the A ring, else one) and, for the split form, a ring of two A slots
+    // of 64 columns (x_hi in the first 32, x_lo in the next 32).
+    static constexpr int kARing = Tr::kSplit ? 128 : 0;
+    static constexpr int kAcc = (2 * BN + kARing <= 512) ? 2 : 1;
+    static constexpr int kTmemCols = pow2_at_least(kAcc * BN + kARing);
+    static_assert(kS >= 2, "ring too small");
+    static_assert(kAlloc <= kSmemMax, "shared memory");
+    static_assert(kTmemCols <= 512, "tensor memory");
 };
 
 // ---------------------------------------------------------------------------
-// Decode of the BSR weights into the masked dense matrix W[o][k] (K-major),
-// after W has been zeroed: CTA (x, g) scatters kept weights e = 256x + tid of
-// col-group g, i.e. D[z][n] with z = P[g] + e / N, n = e % N, to
-// W[g*N + n][I[z]].
+// Decode of the BSR weights into the masked dense matrix W[o][k] (K-major).
+// CTA (x, g, r) writes the 256 columns k0 = 256x .. k0+255 of rows
+// 8r .. 8r+7 (those below N) of col-group g: it marks in shared memory which kept block z of the group
+// (if any) sits at each column, then writes every element of the band once,
+// coalesced: W[g*N + n][k] = D[z][n] for a kept column, 0 otherwise.  For
+// fp32 W gets the tf32 rounding of the value and W_lo the rest.
 // ---------------------------------------------------------------------------
-__global__ void __launch_bounds__(256)
-bsr_scatter_kernel(const int32_t *__restrict__ P, const int32_t *__restrict__ I,
-                   const __nv_bfloat16 *__restrict__ D, int N, int t, int K,
-                   __nv_bfloat16 *__restrict__ W)
+constexpr int kDecodeCols = 256;
+constexpr int kDecodeRows = 8;
+
+__device__ __forceinline__ float tf32_rna(float v)
 {
-    const int g = blockIdx.y;
+    uint32_t r;
+    asm("cvt.rna.tf32.f32 %0, %1;\n" : "=r"(r) : "f"(v));
+    return __uint_as_float(r);
+}
+
+template <typename T>
+__global__ void __launch_bounds__(kDecodeCols)
+bsr_decode_kernel(const int32_t *__restrict__ P, const int32_t *__restrict__ I, const T *__restrict__ D,
+                  int N, int t, int K, T *__restrict__ W, T *__restrict__ W_lo)
+{
+    __shared__ int32_t zmap[kDecodeCols];
+    const int g = blockIdx.y, tid = threadIdx.x;
+    const int k0 = blockIdx.x * kDecodeCols;
+    zmap[tid] = -1;
+    __syncthreads();
     const int z0 = clampi(__ldg(P + g), 0, t), z1 = clampi(__ldg(P + g + 1), z0, t);
-    const int e = blockIdx.x * blockDim.x + threadIdx.x;
-    if (e >= (z1 - z0) * N) return;
-    const int z = z0 + e / N, n = e - (e / N) * N;
-    const int k = __ldg(I + z);
-    if (k >= 0 && k < K) W[static_cast<int64_t>(g * N + n) * K + k] = D[static_cast<int64_t>(z) * N + n];
+    for (int z = z0 + tid; z < z1; z += kDecodeCols) {
+        const int k = __ldg(I + z) - k0;
+        if (k >= 0 && k < kDecodeCols) zmap[k] = z;
+    }
+    __syncthreads();
+    const int k = k0 + tid;
+    if (k >= K) return;
+    const int z = zmap[tid];
+    const int n1 = min(N, static_cast<int>(blockIdx.z + 1) * kDecodeRows);
+    for (int n = blockIdx.z * kDecodeRows; n < n1; ++n) {
+        const int64_t dst = static_cast<int64_t>(g * N + n) * K + k;
+        const T v = z >= 0 ? D[static_cast<int64_t>(z) * N + n] : T(0.f);
+        if constexpr (sizeof(T) == 4) {
+            const float hi = tf32_rna(v);
+            W[dst] = hi;
+            W_lo[dst] = v - hi;
+        } else {
+            W[dst] = v;
+        }
+    }
 }
 
 // barrier over the 4 epilogue warps that also returns the AND of `ok`
@@ -99,39 +178,44 @@ __device__ __forceinline__ bool epi_all(bool ok)
     return r != 0;
 }
 
-template <int BN>
-__global__ void __launch_bounds__(kThreadsTc, 1)
+template <typename Tr, int BN>
+__global__ void __launch_bounds__(Tr::kWarps * 32, 1)
 tc_conv_kernel(const ConvArgs a, const __grid_constant__ CUtensorMap tmap_x,
-               const __grid_constant__ CUtensorMap tmap_w, const __grid_constant__ CUtensorMap tmap_y,
-               const int n_tiles, const int n_tn, const int a_tiled)
+               const __grid_constant__ CUtensorMap tmap_w, const __grid_constant__ CUtensorMap tmap_wlo,
+               const __grid_constant__ CUtensorMap tmap_y, const int n_tiles, const int n_tn,
+               const int a_tiled)
 {
-    using L = TcLayout<BN>;
+    using L = TcLayout<Tr, BN>;
     extern __shared__ unsigned char smem_raw[];
     const uint32_t raw = smem_u32(smem_raw);
     const uint32_t base = (raw + 1023u) & ~1023u;
     unsigned char *smem = smem_raw + (base - raw);
     const uint32_t bar_full = base + L::kBar;
-    const uint32_t bar_empty = bar_full + 8 * L::kS;
+    const uint32_t bar_split = bar_full + 8 * L::kS;
+    const uint32_t bar_empty = bar_split + 8 * L::kS;
     const uint32_t bar_tfull = bar_empty + 8 * L::kS;
     const uint32_t bar_tempty = bar_tfull + 16;
     const uint32_t bar_drain = bar_tempty + 16;
     uint32_t *holder = reinterpret_cast<uint32_t *>(smem + L::kHolder);
+    // the MMA waits on "split" (fp32: x_lo written) or "full" (bf16)
+    const uint32_t bar_ready = Tr::kSplit ? bar_split : bar_full;
 
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     if (tid == 0) {
         for (int s = 0; s < L::kS; ++s) {
             mbar_init(bar_full + 8 * s, 1);
+            mbar_init(bar_split + 8 * s, 128);
             mbar_init(bar_empty + 8 * s, 1);
         }
         for (int b = 0; b < 2; ++b) {
             mbar_init(bar_tfull + 8 * b, 1);
-            mbar_init(bar_tempty + 8 * b, 32 * kEpiWarps);
+            mbar_init(bar_tempty + 8 * b, 128);
         }
         mbar_init(bar_drain, 1);
         fence_mbar_init();
     }
     if (warp == kMmaWarp) {
-        tc::tmem_alloc(smem_u32(holder), 2 * BN);
+        tc::tmem_alloc(smem_u32(holder), L::kTmemCols);
         tc::tmem_relinquish();
     }
     tc::fence_before_sync();
@@ -139,7 +223,7 @@ tc_conv_kernel(const ConvArgs a, const __grid_constant__ CUtensorMap tmap_x,
     tc::fence_after_sync();
     const uint32_t tmem = *holder;
 
-    const int n_cchunk = (a.C + kBK - 1) / kBK;
+    const int n_cchunk = (a.C + Tr::kBK - 1) / Tr::kBK;
     const int n_chunks = a.KH * a.KW * n_cchunk;
     const int my_tiles = blockIdx.x < n_tiles ? (n_tiles - 1 - blockIdx.x) / gridDim.x + 1 : 0;
     auto abort_now = [&]() { atomicOr(a.status, kStatusTimeout); };
@@ -165,8 +249,9 @@ tc_conv_kernel(const ConvArgs a, const __grid_constant__ CUtensorMap tmap_x,
                         !mbar_wait(bar_empty + 8 * st, ((item / L::kS) + 1) & 1)) {
                         abort_now(); failed = true; break;
                     }
-                    const uint32_t sa = base + st * L::kStage, sb = sa + L::kA;
-                    tc::mbar_arrive_expect_tx(bar_full + 8 * st, L::kStage);
+                    const uint32_t sa = base + st * L::kStage;
+                    const uint32_t sb = sa + L::kA;
+                    tc::mbar_arrive_expect_tx(bar_full + 8 * st, L::kTx);
                     if (a_tiled)
                         tc::tma_load_2d(sa, &tmap_x, cc0, p0, bar_full + 8 * st);
                     else
@@ -174,7 +259,9 @@ tc_conv_kernel(const ConvArgs a, const __grid_constant__ CUtensorMap tmap_x,
                                                static_cast<uint16_t>(kw * a.dw), static_cast<uint16_t>(kh * a.dh),
                                                bar_full + 8 * st);
                     tc::tma_load_2d(sb, &tmap_w, k0tap + cc0, tn * BN, bar_full + 8 * st);
-                    cc0 += kBK;
+                    if constexpr (Tr::kSplit)
+                        tc::tma_load_2d(sb + L::kB, &tmap_wlo, k0tap + cc0, tn * BN, bar_full + 8 * st);
+                    cc0 += Tr::kBK;
                     if (cc0 >= a.C) {
                         cc0 = 0; k0tap += a.C;
                         if (++kw == a.KW) { kw = 0; ++kh; }
@@ -186,27 +273,41 @@ tc_conv_kernel(const ConvArgs a, const __grid_constant__ CUtensorMap tmap_x,
     } else if (warp == kMmaWarp) {
         // ============================== MMA ==============================
         if (lane == 0) {
-            constexpr uint32_t idesc = tc::idesc_bf16_f32(kBM, BN);
             int item = 0;
             bool failed = false;
             for (int ti = 0; ti < my_tiles && !failed; ++ti) {
-                const int acc = ti & 1;
-                if (ti >= 2 && !mbar_wait(bar_tempty + 8 * acc, ((ti >> 1) + 1) & 1)) {
+                const int acc = ti % L::kAcc, use = ti / L::kAcc;
+                if (use >= 1 && !mbar_wait(bar_tempty + 8 * acc, (use - 1) & 1)) {
                     abort_now(); failed = true; break;
                 }
                 tc::fence_after_sync();
                 const uint32_t d_tmem = tmem + acc * BN;
                 for (int c = 0; c < n_chunks; ++c, ++item) {
                     const int st = item % L::kS;
-                    if (!mbar_wait(bar_full + 8 * st, (item / L::kS) & 1)) {
+                    if (!mbar_wait(bar_ready + 8 * st, (item / L::kS) & 1)) {
                         abort_now(); failed = true; break;
                     }
                     tc::fence_after_sync();
-                    const uint32_t sa = base + st * L::kStage, sb = sa + L::kA;
-                    const uint64_t ad = tc::desc_kmajor_sw128(sa), bd = tc::desc_kmajor_sw128(sb);
+                    const uint32_t sa = base + st * L::kStage;
+                    const uint64_t bd = tc::desc_kmajor_sw128(sa + L::kA);
+                    if constexpr (Tr::kSplit) {
+                        constexpr uint32_t idesc = tc::idesc_tf32_f32(kBM, BN);
+                        const uint64_t bld = tc::desc_kmajor_sw128(sa + L::kA + L::kB);
+                        // A slot of this chunk: x_hi columns, then x_lo 32 columns on
+                        const uint32_t a_hi = tmem + L::kAcc * BN + (item & 1) * 64;
 #pragma unroll
-                    for (int kk = 0; kk < kBK / 16; ++kk)
-                        tc::mma_bf16(d_tmem, ad + 2 * kk, bd + 2 * kk, idesc, (c | kk) != 0);
+                        for (int kk = 0; kk < Tr::kBK / Tr::kKStep; ++kk) {
+                            tc::mma_tf32_ta(d_tmem, a_hi + 8 * kk, bd + 2 * kk, idesc, (c | kk) != 0);
+                            tc::mma_tf32_ta(d_tmem, a_hi + 32 + 8 * kk, bd + 2 * kk, idesc, 1);
+                            tc::mma_tf32_ta(d_tmem, a_hi + 8 * kk, bld + 2 * kk, idesc, 1);
+                        }
+                    } else {
+                        constexpr uint32_t idesc = tc::idesc_bf16_f32(kBM, BN);
+                        const uint64_t ad = tc::desc_kmajor_sw128(sa);
+#pragma unroll
+                        for (int kk = 0; kk < Tr::kBK / Tr::kKStep; ++kk)
+                            tc::mma_bf16(d_tmem, ad + 2 * kk, bd + 2 * kk, idesc, (c | kk) != 0);
+                    }
                     tc::commit(bar_empty + 8 * st);
                 }
                 if (!failed) tc::commit(bar_tfull + 8 * acc);
@@ -216,23 +317,70 @@ tc_conv_kernel(const ConvArgs a, const __grid_constant__ CUtensorMap tmap_x,
             if (!mbar_wait(bar_drain, 0)) abort_now();
         }
         __syncwarp();
+    } else if (warp >= kSplitWarp0) {
+        // ============================ split (fp32) ========================
+        // Thread i of warp w owns pixel row 32*(w%4) + i of the tile: it reads
+        // the row's 32 fp32 values from the swizzled A tile (logical 16-byte
+        // chunk j of row r sits at physical chunk j ^ (r % 8), so the eight
+        // rows of a quarter-warp hit eight distinct bank groups), splits them
+        // into x_hi = x with the low 13 mantissa bits cleared and
+        // x_lo = x - x_hi, and writes both to its TMEM lane in the chunk's A
+        // slot (item % 2).  Before overwriting a slot it waits until the MMAs
+        // of the chunk two back, which read it, have completed.
+        if constexpr (Tr::kSplit) {
+            const int q = warp & 3;
+            const int row = 32 * q + lane;
+            const uint32_t lane_base = tmem + (static_cast<uint32_t>(32 * q) << 16) + L::kAcc * BN;
+            const int n_items = my_tiles * n_chunks;
+            for (int item = 0; item < n_items; ++item) {
+                const int st = item % L::kS;
+                if (item >= 2 &&
+                    !mbar_wait(bar_empty + 8 * ((item - 2) % L::kS), ((item - 2) / L::kS) & 1)) {
+                    abort_now(); break;
+                }
+                if (!mbar_wait(bar_full + 8 * st, (item / L::kS) & 1)) { abort_now(); break; }
+                tc::fence_after_sync();
+                const uint32_t src = base + st * L::kStage + row * kRowBytes;
+                uint32_t hi[32], lo[32];
+#pragma unroll
+                for (int j = 0; j < 8; ++j) {
+                    uint32_t v[4];
+                    asm volatile("ld.shared.v4.b32 {%0, %1, %2, %3}, [%4];\n"
+                                 : "=r"(v[0]), "=r"(v[1]), "=r"(v[2]), "=r"(v[3])
+                                 : "r"(src + ((j ^ (row & 7)) << 4))
+                                 : "memory");
+#pragma unroll
+                    for (int e = 0; e < 4; ++e) {
+                        hi[4 * j + e] = v[e] & 0xffffe000u;
+                        lo[4 * j + e] = __float_as_uint(__uint_as_float(v[e]) - __uint_as_float(hi[4 * j + e]));
+                    }
+                }
+                const uint32_t slot = lane_base + (item & 1) * 64;
+                tc::st_32x32b_x32(slot, hi);
+                tc::st_32x32b_x32(slot + 32, lo);
+                tc::st_wait();
+                tc::fence_before_sync();
+                mbar_arrive(bar_split + 8 * st);
+            }
+        }
     } else {
         // ============================ epilogue ============================
         const int q = warp & 3;                      // TMEM lanes 32q .. 32q+31
         const int row = 32 * q + lane;               // pixel row of the tile
-        const bool leader = (warp == kMmaWarp + 1) && lane == 0;
+        const bool leader = (warp == kEpiWarp0) && lane == 0;
         float *sbias = reinterpret_cast<float *>(smem + L::kBias);
         const uint32_t sout = base + L::kOut;
         for (int ti = 0; ti < my_tiles; ++ti) {
-            const int acc = ti & 1;
+            const int acc = ti % L::kAcc;
             // all four warps take the same decision (tcgen05.ld and the named
             // barriers below need all of them)
-            if (!epi_all(mbar_wait(bar_tfull + 8 * acc, (ti >> 1) & 1))) { abort_now(); break; }
+            if (!epi_all(mbar_wait(bar_tfull + 8 * acc, (ti / L::kAcc) & 1))) { abort_now(); break; }
             tc::fence_after_sync();
             const int u = blockIdx.x + ti * gridDim.x;
             const int tm = u / n_tn, tn = u - tm * n_tn;
-            // the staging tile is free once the previous tile's stores have read it
-            if (leader) tc::bulk_wait_read0();
+            const int p = tm * kBM + row;
+            // bf16: the staging tile is free once the previous tile's stores have read it
+            if (!Tr::kSplit && leader) tc::bulk_wait_read0();
             for (int c = row; c < BN; c += 128) {
                 const int o = tn * BN + c;
                 sbias[c] = (a.bias && o < a.C_out) ? __ldg(a.bias + o) : 0.f;
@@ -264,33 +412,45 @@ tc_conv_kernel(const ConvArgs a, const __grid_constant__ CUtensorMap tmap_x,
                             if (a.relu) val = fmaxf(val, 0.f);
                             f[e] = val;
                         }
-                        const int atom = c >> 6, jj = (c & 63) >> 3;
-                        const uint32_t dst = sout + atom * (kBM * 128) + row * 128 + ((jj ^ (row & 7)) << 4);
-                        asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};\n" ::"r"(dst),
-                                     "r"(pack_bf16x2(f[0], f[1])), "r"(pack_bf16x2(f[2], f[3])),
-                                     "r"(pack_bf16x2(f[4], f[5])), "r"(pack_bf16x2(f[6], f[7]))
-                                     : "memory");
+                        if constexpr (Tr::kSplit) {
+                            const int col = tn * BN + c;
+                            if (p < a.P_pix && col < a.C_out) {
+                                float4 *dst = reinterpret_cast<float4 *>(static_cast<float *>(a.y) +
+                                                                         static_cast<int64_t>(p) * a.C_out + col);
+                                dst[0] = make_float4(f[0], f[1], f[2], f[3]);
+                                dst[1] = make_float4(f[4], f[5], f[6], f[7]);
+                            }
+                        } else {
+                            const int atom = c >> 6, jj = (c & 63) >> 3;
+                            const uint32_t dst = sout + atom * (kBM * 128) + row * 128 + ((jj ^ (row & 7)) << 4);
+                            asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};\n" ::"r"(dst),
+                                         "r"(pack_bf16x2(f[0], f[1])), "r"(pack_bf16x2(f[2], f[3])),
+                                         "r"(pack_bf16x2(f[4], f[5])), "r"(pack_bf16x2(f[6], f[7]))
+                                         : "memory");
+                        }
                     }
                 }
             }
-            tc::fence_proxy_async_smem();
-            tc::named_bar(1, 128);
-            if (leader) {
+            if constexpr (!Tr::kSplit) {
+                tc::fence_proxy_async_smem();
+                tc::named_bar(1, 128);
+                if (leader) {
 #pragma unroll
-                for (int at = 0; at < BN / 64; ++at)
-                    if (tn * BN + 64 * at < a.C_out)
-                        tc::tma_store_2d(&tmap_y, tn * BN + 64 * at, tm * kBM, sout + at * (kBM * 128));
-                tc::bulk_commit();
+                    for (int at = 0; at < BN / 64; ++at)
+                        if (tn * BN + 64 * at < a.C_out)
+                            tc::tma_store_2d(&tmap_y, tn * BN + 64 * at, tm * kBM, sout + at * (kBM * 128));
+                    tc::bulk_commit();
+                }
             }
         }
-        if (leader) tc::bulk_wait0();
+        if (!Tr::kSplit && leader) tc::bulk_wait0();
     }
 
     tc::fence_before_sync();
     __syncthreads();
     if (warp == kMmaWarp) {
         tc::fence_after_sync();
-        tc::tmem_dealloc(tmem, 2 * BN);
+        tc::tmem_dealloc(tmem, L::kTmemCols);
     }
 }
 
@@ -334,56 +494,65 @@ void im2col_corners(const ConvArgs &a, int lower[2], int upper[2])
     upper[1] = a.ph - a.dh * (a.KH - 1);
 }
 
-// 2-D bf16 tensor map over a row-major [rows][cols] matrix, box 64 x box_rows,
-// 128-byte swizzle, zero fill outside.
-bool tmap_2d(CUtensorMap *m, const void *ptr, uint64_t rows, uint64_t cols, uint32_t box_rows)
+// 2-D tensor map over a row-major [rows][cols] matrix of `elem`-byte values,
+// box 128 bytes x box_rows, 128-byte swizzle, zero fill outside.
+bool tmap_2d(CUtensorMap *m, CUtensorMapDataType type, int elem, const void *ptr, uint64_t rows,
+             uint64_t cols, uint32_t box_rows)
 {
     auto enc_t = encode_tiled_fn();
     if (!enc_t) return false;
     const cuuint64_t dims[2] = {cols, rows};
-    const cuuint64_t strides[1] = {cols * 2};
-    const cuuint32_t box[2] = {static_cast<cuuint32_t>(kBK), box_rows};
+    const cuuint64_t strides[1] = {cols * elem};
+    const cuuint32_t box[2] = {static_cast<cuuint32_t>(kRowBytes / elem), box_rows};
     const cuuint32_t estr[2] = {1, 1};
-    return enc_t(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(ptr), dims, strides, box, estr,
-                 CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+    return enc_t(m, type, 2, const_cast<void *>(ptr), dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                 CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                  CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-template <int BN>
-cudaError_t launch_bn(const ConvArgs &a, const __nv_bfloat16 *W, cudaStream_t st)
+template <typename Tr, int BN>
+cudaError_t launch_bn(const ConvArgs &a, const typename Tr::T *W, const typename Tr::T *W_lo, cudaStream_t st)
 {
-    using L = TcLayout<BN>;
-    auto kern = tc_conv_kernel<BN>;
+    using L = TcLayout<Tr, BN>;
+    constexpr int elem = sizeof(typename Tr::T);
+    auto kern = tc_conv_kernel<Tr, BN>;
     const int K = a.KH * a.KW * a.C;
     auto enc_i = encode_im2col_fn();
     if (!enc_i) return cudaErrorNotSupported;
     // A: a 1x1, stride-1, unpadded layer reads x as a [B*H*W][C] matrix; any
-    // other layer reads x[B][H][W][C] as an im2col view (128 pixels x 64
-    // channels per load).
+    // other layer reads x[B][H][W][C] as an im2col view (128 pixels x 128
+    // bytes of channels per load).
     const int a_tiled = (a.KH == 1 && a.KW == 1 && a.sh == 1 && a.sw == 1 && a.ph == 0 && a.pw == 0);
     CUtensorMap tmap_x;
     if (a_tiled) {
-        if (!tmap_2d(&tmap_x, a.x, static_cast<uint64_t>(a.B) * a.H * a.W, a.C, kBM)) return cudaErrorInvalidValue;
+        if (!tmap_2d(&tmap_x, Tr::kTmap, elem, a.x, static_cast<uint64_t>(a.B) * a.H * a.W, a.C, kBM))
+            return cudaErrorInvalidValue;
     } else {
         const cuuint64_t dims[4] = {static_cast<cuuint64_t>(a.C), static_cast<cuuint64_t>(a.W),
                                     static_cast<cuuint64_t>(a.H), static_cast<cuuint64_t>(a.B)};
-        const cuuint64_t strides[3] = {static_cast<cuuint64_t>(a.C) * 2,
-                                       static_cast<cuuint64_t>(a.C) * 2 * a.W,
-                                       static_cast<cuuint64_t>(a.C) * 2 * a.W * a.H};
+        const cuuint64_t strides[3] = {static_cast<cuuint64_t>(a.C) * elem,
+                                       static_cast<cuuint64_t>(a.C) * elem * a.W,
+                                       static_cast<cuuint64_t>(a.C) * elem * a.W * a.H};
         int lower[2], upper[2];
         im2col_corners(a, lower, upper);
         const cuuint32_t estr[4] = {1, static_cast<cuuint32_t>(a.sw), static_cast<cuuint32_t>(a.sh), 1};
-        if (enc_i(&tmap_x, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void *>(a.x), dims, strides,
-                  lower, upper, kBK, kBM, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+        if (enc_i(&tmap_x, Tr::kTmap, 4, const_cast<void *>(a.x), dims, strides, lower, upper, Tr::kBK, kBM,
+                  estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
                   CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
             return cudaErrorInvalidValue;
     }
-    // B: W[C_out][K] bf16, box 64 (K) x BN rows.  y: [P_pix][C_out] bf16,
-    // stored in boxes of 64 columns x 128 rows (rows/columns outside y are
-    // not written).
-    CUtensorMap tmap_w, tmap_y;
-    if (!tmap_2d(&tmap_w, W, a.C_out, K, BN)) return cudaErrorInvalidValue;
-    if (!tmap_2d(&tmap_y, a.y, a.P_pix, a.C_out, kBM)) return cudaErrorInvalidValue;
+    // B: W[C_out][K] (and W_lo), box 128 bytes of K x BN rows.  y (bf16 only):
+    // [P_pix][C_out], stored in boxes of 64 columns x 128 rows (rows/columns
+    // outside y are not written).
+    CUtensorMap tmap_w, tmap_wlo, tmap_y;
+    if (!tmap_2d(&tmap_w, Tr::kTmap, elem, W, a.C_out, K, BN)) return cudaErrorInvalidValue;
+    if (Tr::kSplit) {
+        if (!tmap_2d(&tmap_wlo, Tr::kTmap, elem, W_lo, a.C_out, K, BN)) return cudaErrorInvalidValue;
+        tmap_y = tmap_w;                                       // unused
+    } else {
+        tmap_wlo = tmap_w;                                     // unused
+        if (!tmap_2d(&tmap_y, Tr::kTmap, elem, a.y, a.P_pix, a.C_out, kBM)) return cudaErrorInvalidValue;
+    }
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, L::kAlloc);
     if (e != cudaSuccess) return e;
     int sms = 0;
@@ -393,24 +562,46 @@ cudaError_t launch_bn(const ConvArgs &a, const __nv_bfloat16 *W, cudaStream_t st
     const int n_tn = (a.C_out + BN - 1) / BN;
     const int n_tiles = n_tm * n_tn;
     const int grid = n_tiles < sms ? n_tiles : sms;
-    kern<<<grid, kThreadsTc, L::kAlloc, st>>>(a, tmap_x, tmap_w, tmap_y, n_tiles, n_tn, a_tiled);
+    kern<<<grid, Tr::kWarps * 32, L::kAlloc, st>>>(a, tmap_x, tmap_w, tmap_wlo, tmap_y, n_tiles, n_tn, a_tiled);
     return cudaGetLastError();
+}
+
+template <typename Tr>
+cudaError_t launch_typed(const ConvArgs &a, void *workspace, cudaStream_t st)
+{
+    using T = typename Tr::T;
+    const int K = a.KH * a.KW * a.C;
+    const size_t n = static_cast<size_t>(a.C_out) * K;
+    T *W = static_cast<T *>(workspace);
+    T *W_lo = Tr::kSplit ? W + n : nullptr;
+    const dim3 grid(static_cast<unsigned>((K + kDecodeCols - 1) / kDecodeCols), a.C_out / a.N,
+                    (a.N + kDecodeRows - 1) / kDecodeRows);
+    bsr_decode_kernel<T><<<grid, kDecodeCols, 0, st>>>(a.P, a.I, static_cast<const T *>(a.D), a.N, a.t, K, W, W_lo);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    if (a.C_out <= 64) return launch_bn<Tr, 64>(a, W, W_lo, st);
+    if (a.C_out <= 128) return launch_bn<Tr, 128>(a, W, W_lo, st);
+    return launch_bn<Tr, 256>(a, W, W_lo, st);
 }
 
 }  // namespace
 
-size_t tc_workspace_bytes(const ConvArgs &a)
+// bf16: C_out * K bf16 values; fp32: C_out * K fp32 values twice (hi, lo).
+size_t tc_workspace_bytes(const ConvArgs &a, int dtype)
 {
-    const size_t bytes = static_cast<size_t>(a.C_out) * a.KH * a.KW * a.C * 2;
+    const size_t n = static_cast<size_t>(a.C_out) * a.KH * a.KW * a.C;
+    const size_t bytes = dtype == ONEXN_F32 ? n * 8 : n * 2;
     return (bytes + 255) & ~static_cast<size_t>(255);
 }
 
-// bf16 inputs; C_in, C_out multiples of 8 (16-byte rows); the im2col box
-// corners within the TMA's [-128, 127] range; strides <= 8; 16-bit offsets.
-bool tc_supports(const ConvArgs &a)
+// C_in, C_out giving 16-byte rows; the im2col box corners within the TMA's
+// [-128, 127] range; strides <= 8; 16-bit tap offsets.
+bool tc_supports(const ConvArgs &a, int dtype)
 {
-    if (a.C % 8 || a.C_out % 8) return false;
+    const int v = dtype == ONEXN_F32 ? 4 : 8;
+    if (a.C % v || a.C_out % 8) return false;
     if (a.sh > 8 || a.sw > 8) return false;
+    if (a.C_out / a.N > 65535) return false;          // decode grid.y
     int lower[2], upper[2];
     im2col_corners(a, lower, upper);
     for (int i = 0; i < 2; ++i)
@@ -419,24 +610,11 @@ bool tc_supports(const ConvArgs &a)
     return true;
 }
 
-cudaError_t launch_tc(const ConvArgs &a, void *workspace, cudaStream_t st)
+cudaError_t launch_tc(const ConvArgs &a, int dtype, void *workspace, cudaStream_t st)
 {
     if (a.P_pix == 0) return cudaSuccess;
-    __nv_bfloat16 *W = static_cast<__nv_bfloat16 *>(workspace);
-    const int K = a.KH * a.KW * a.C;
-    cudaError_t e = cudaMemsetAsync(W, 0, static_cast<size_t>(a.C_out) * K * 2, st);
-    if (e != cudaSuccess) return e;
-    if (a.t > 0) {
-        const int64_t per_group = static_cast<int64_t>(K) * a.N;     // upper bound of t_g * N
-        const dim3 grid(static_cast<unsigned>((per_group + 255) / 256), a.C_out / a.N);
-        bsr_scatter_kernel<<<grid, 256, 0, st>>>(a.P, a.I, static_cast<const __nv_bfloat16 *>(a.D), a.N, a.t,
-                                                 K, W);
-        e = cudaGetLastError();
-    }
-    if (e != cudaSuccess) return e;
-    if (a.C_out <= 64) return launch_bn<64>(a, W, st);
-    if (a.C_out <= 128) return launch_bn<128>(a, W, st);
-    return launch_bn<256>(a, W, st);
+    if (dtype == ONEXN_F32) return launch_typed<TcF32>(a, workspace, st);
+    return launch_typed<TcBf16>(a, workspace, st);
 }
 
 }  // namespace onexn

@@ -34,17 +34,17 @@ ALGOS = ox.ALGO_BY_NAME
 
 
 def _algos_for(dtype, N, C_in=64, C_out=64):
-    """Every family that can run this case (FMA always; the bf16 families if
-    they accept it), plus AUTO."""
+    """Every family that can run this case (FMA always; the tensor-core
+    families if they accept it), plus AUTO."""
     out = ["auto", "fma"]
-    if dtype == "bf16":
-        probe = ox.make_desc(1, 8, 8, C_in, C_out, 1, 1)
-        for name in ("mma", "tc"):
-            try:
-                ox.onexn_conv_algo(probe, N, 1, ox.ONEXN_BF16, ALGOS[name], 1 << 40)
-                out.append(name)
-            except ox.OnexnError:
-                pass
+    probe = ox.make_desc(1, 8, 8, C_in, C_out, 1, 1)
+    dt = ox.ONEXN_BF16 if dtype == "bf16" else ox.ONEXN_F32
+    for name in ("mma", "tc"):
+        try:
+            ox.onexn_conv_algo(probe, N, 1, dt, ALGOS[name], 1 << 40)
+            out.append(name)
+        except ox.OnexnError:
+            pass
     return out
 
 
@@ -104,13 +104,14 @@ def test_tc_column_tiles(C_out, N):
     assert norm_err(y, yr, a) <= tol(layer)
 
 
-def test_auto_picks_tc_for_bf16_with_workspace():
-    layer = L("auto", 1, 8, 8, 64, 64, 1, 1, N=8, rate=0.5, dtype="bf16")
+def test_auto_picks_tc_with_workspace_and_ffma_for_bias_only():
+    layer = L("auto", 4, 32, 32, 64, 64, 1, 1, N=8, rate=0.5, dtype="bf16")
     from paper_2105_14713_gb300.layer import PrunedConv2d
-    conv = PrunedConv2d(wl.weights(layer).numpy(), 8, 0.5, dtype="bf16")
-    assert conv.algo((1, 8, 8, 64)) == "tc"
-    conv32 = PrunedConv2d(wl.weights(layer).numpy(), 8, 0.5, dtype="f32")
-    assert conv32.algo((1, 8, 8, 64)) == "fma"
+    for dt in ("bf16", "f32"):
+        conv = PrunedConv2d(wl.weights(layer).numpy(), 8, 0.5, dtype=dt)
+        assert conv.algo((4, 32, 32, 64)) == "tc"
+        empty = PrunedConv2d(wl.weights(layer).numpy(), 8, 1.0, dtype=dt)
+        assert empty.t == 0 and empty.algo((4, 32, 32, 64)) == "fma"
 
 
 def test_device_status_clean_after_runs():

@@ -154,6 +154,23 @@ def test_validate_catches_corrupted_bsr(P, I, G, t, K, frag):
     assert frag in str(e.value)
 
 
+def test_auto_cost_model():
+    # 3x3 128->128 (K = 1152, 16 groups of N = 8): the tensor-core GEMM does
+    # all 128 * 1152 products per pixel after decoding the weights, the FFMA
+    # kernel only the kept t * N.  On 50176 pixels the GEMM wins even at 99%
+    # pruned; on 4 pixels the decode dominates and FFMA wins when most blocks
+    # are pruned.
+    G, K = 128 // 8, 9 * 128
+    big = ox.make_desc(64, 28, 28, 128, 128, 3, 3, 1, 1, 1)
+    tiny = ox.make_desc(1, 2, 2, 128, 128, 3, 3, 1, 1, 1)
+    for dt in (ox.ONEXN_F32, ox.ONEXN_BF16):
+        ws = ox.onexn_conv_workspace_size(big, 8, G * K, dt)
+        assert ox.onexn_conv_algo(big, 8, G * K // 2, dt, 0, ws) == ox.ONEXN_ALGO_TC      # 50% pruned
+        assert ox.onexn_conv_algo(big, 8, G * K // 100, dt, 0, ws) == ox.ONEXN_ALGO_TC    # 99% pruned
+        assert ox.onexn_conv_algo(big, 8, 0, dt, 0, ws) == ox.ONEXN_ALGO_FMA              # all pruned
+        assert ox.onexn_conv_algo(tiny, 8, G * K // 10, dt, 0, ws) == ox.ONEXN_ALGO_FMA
+
+
 def test_conv_shape_and_argument_errors_need_no_gpu():
     d = ox.make_desc(2, 7, 7, 8, 16, 3, 3, 2, 1, 1)
     assert ox.onexn_conv_out_shape(d) == (4, 4)
@@ -163,10 +180,21 @@ def test_conv_shape_and_argument_errors_need_no_gpu():
     assert need == 16 * 9 * 8 * 2 + (-(16 * 9 * 8 * 2) % 256)
     assert ox.onexn_conv_algo(d, 8, 100, ox.ONEXN_BF16, 0, need) == ox.ONEXN_ALGO_TC
     assert ox.onexn_conv_algo(d, 8, 100, ox.ONEXN_BF16, 0, need - 1) == ox.ONEXN_ALGO_FMA
-    assert ox.onexn_conv_workspace_size(d, 8, 100, ox.ONEXN_F32) == 0
+    # fp32: hi and lo tf32 parts of the decoded weights, 8 bytes per weight
+    need32 = ox.onexn_conv_workspace_size(d, 8, 100, ox.ONEXN_F32)
+    assert need32 == 16 * 9 * 8 * 8 + (-(16 * 9 * 8 * 8) % 256)
+    assert ox.onexn_conv_workspace_size(d, 8, 100, ox.ONEXN_F32, ox.ONEXN_ALGO_FMA) == 0
+    assert ox.onexn_conv_algo(d, 8, 100, ox.ONEXN_F32, 0, need32 - 1) == ox.ONEXN_ALGO_FMA
+    assert ox.onexn_conv_algo(d, 8, 100, ox.ONEXN_F32, ox.ONEXN_ALGO_TC, need32) == ox.ONEXN_ALGO_TC
     assert _status(ox.onexn_conv_algo, d, 8, 100, ox.ONEXN_BF16, ox.ONEXN_ALGO_TC, 0) == ox.ONEXN_EINVAL
-    assert _status(ox.onexn_conv_algo, d, 8, 100, ox.ONEXN_F32, ox.ONEXN_ALGO_TC, 1 << 30) == \
-        ox.ONEXN_EUNSUPPORTED
+    assert _status(ox.onexn_conv_algo, d, 8, 100, ox.ONEXN_F32, ox.ONEXN_ALGO_TC, need32 - 1) == \
+        ox.ONEXN_EINVAL
+    # C_out not a multiple of 8: no tensor-core tiles; AUTO falls back to FFMA
+    d12 = ox.make_desc(1, 4, 4, 8, 12)
+    for dt in (ox.ONEXN_F32, ox.ONEXN_BF16):
+        assert _status(ox.onexn_conv_algo, d12, 4, 1, dt, ox.ONEXN_ALGO_TC, 1 << 30) == ox.ONEXN_EUNSUPPORTED
+        assert ox.onexn_conv_algo(d12, 4, 1, dt, 0, 1 << 30) == ox.ONEXN_ALGO_FMA
+        assert ox.onexn_conv_workspace_size(d12, 4, 1, dt) == 0
     bad = ox.make_desc(1, 2, 2, 8, 16, 5, 5)
     assert _status(ox.onexn_conv_out_shape, bad) == ox.ONEXN_EINVAL
     assert _status(ox.onexn_conv_algo, d, 3, 10, ox.ONEXN_F32) == ox.ONEXN_EINVAL    # N | C_out
