@@ -422,18 +422,23 @@ def dense_times(legs, dev, flush, stream, reps=5):
 
 
 def e2e_time(legs, dev, steps, warmup, flush, stream):
-    """Public API end to end: pinned host input -> device, conv, device -> pinned host."""
+    """Public API end to end: PrunedConv2d.forward_host (onexn_conv_fwd_host)
+    from a pinned host input to a pinned host output, copies included.  Each
+    leg is enqueued on its own stream, so one layer's copies overlap the
+    other's compute, as a caller running a stack of layers would."""
     x_pin = [lg["x_cpu"].pin_memory() for lg in legs]
     y_host = [torch.empty(lg["y"].shape, dtype=lg["y"].dtype, pin_memory=True) for lg in legs]
+    leg_streams = [torch.cuda.Stream(dev) for _ in legs]
     ts = []
     for r in range(warmup + steps):
         flush.fill_(r & 0xff)
         e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         e0.record(stream)
         for i, lg in enumerate(legs):
-            xd = x_pin[i].to(dev, non_blocking=True)
-            yd = lg["conv"](xd)
-            y_host[i].copy_(yd, non_blocking=True)
+            leg_streams[i].wait_event(e0)
+            lg["conv"].forward_host(x_pin[i], y_host[i], stream=leg_streams[i], sync=False)
+        for s in leg_streams:
+            stream.wait_stream(s)
         e1.record(stream)
         torch.cuda.synchronize()
         if r >= warmup:

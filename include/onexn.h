@@ -220,6 +220,46 @@ onexn_status onexn_conv_algo(const onexn_conv_desc *desc, int N, int64_t t, int 
                              unsigned flags, size_t workspace_bytes, unsigned *algo);
 
 /*
+ * onexn_conv_fwd_host -- onexn_conv_fwd on activations in HOST memory:
+ * y_host = conv(x_host), with the copies to and from the GPU inside the
+ * call.  The batch is cut into chunks of whole images; each chunk is copied
+ * in, convolved and copied out on internal streams so that the copy
+ * engines and the SMs overlap (the tensor-core family decodes the weights
+ * once per call).
+ *   desc, P, I, D, N, t, bias, dtype, flags
+ *           as onexn_conv_fwd (P, I, D, bias are DEVICE pointers).
+ *   x_host  HOST NHWC input [B][H][W][C_in] of dtype.  Pinned memory
+ *           (cudaHostAlloc / cudaHostRegister) lets the copies run
+ *           asynchronously; pageable memory works but serialises them.
+ *   y_host  HOST NHWC output [B][Ho][Wo][C_out] of dtype, same rules.
+ *   workspace, workspace_bytes
+ *           DEVICE scratch, 256-byte aligned, at least
+ *           onexn_conv_host_workspace_size bytes: the decoded weights (if
+ *           any) and three device slots each for an input and an output
+ *           chunk.  Overwritten; concurrent calls need separate workspaces.
+ *   stream  the caller's stream: the call's work starts after the work
+ *           enqueued on it before the call, and the stream waits for the
+ *           call's last copy, so synchronising it makes y_host valid.
+ *           Calls on different streams (with different workspaces) overlap.
+ * Asynchronous like onexn_conv_fwd; neither x_host nor y_host may be
+ * touched by the host until the stream has been synchronised.  Errors as
+ * onexn_conv_fwd, plus EINVAL for a NULL host pointer (B > 0) or a
+ * workspace that is too small; an ECUDA in the middle of the enqueueing
+ * leaves the chunks already enqueued running.
+ */
+onexn_status onexn_conv_fwd_host(const onexn_conv_desc *desc, const int32_t *P, const int32_t *I,
+                                 const void *D, int N, int64_t t, const void *x_host, void *y_host,
+                                 const float *bias, int dtype, unsigned flags, void *workspace,
+                                 size_t workspace_bytes, void *stream);
+
+/*
+ * onexn_conv_host_workspace_size -- bytes of device workspace
+ * onexn_conv_fwd_host needs for these arguments (no GPU needed).
+ */
+onexn_status onexn_conv_host_workspace_size(const onexn_conv_desc *desc, int N, int64_t t, int dtype,
+                                            unsigned flags, size_t *bytes);
+
+/*
  * onexn_conv_fwd_noalloc -- onexn_conv_fwd for callers that cannot allocate
  * device memory.  The paper has no counterpart; it is a deployment aid.
  *

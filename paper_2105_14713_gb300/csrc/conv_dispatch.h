@@ -1,0 +1,41 @@
+// Argument checks, kernel-family selection and launches shared by the
+// convolution entry points (conv_fwd.cu, conv_host.cu, conv_noalloc.cu).
+#pragma once
+
+#include <cuda_runtime.h>
+
+#include "conv_common.cuh"
+#include "onexn.h"
+
+namespace onexn {
+
+cudaError_t launch_fma(const ConvArgs &a, int dtype, cudaStream_t st);
+cudaError_t launch_mma(const ConvArgs &a, cudaStream_t st);
+bool mma_supports(const ConvArgs &a);
+// tensor-core family: decode of (P, I, D) into the workspace, then the GEMM
+cudaError_t launch_tc(const ConvArgs &a, int dtype, void *workspace, cudaStream_t st);
+cudaError_t tc_decode(const ConvArgs &a, int dtype, void *workspace, cudaStream_t st);
+cudaError_t tc_gemm(const ConvArgs &a, int dtype, const void *workspace, cudaStream_t st);
+bool tc_supports(const ConvArgs &a, int dtype);
+size_t tc_workspace_bytes(const ConvArgs &a, int dtype);
+
+namespace detail {
+
+// Shape, dtype and flag checks; fills the geometry part of *a.
+onexn_status check_shape(const onexn_conv_desc *d, int N, int64_t t, int dtype, unsigned flags,
+                         ConvArgs *a);
+// Device-pointer checks; fills the pointer part of *a.
+onexn_status check_pointers(const int32_t *P, const int32_t *I, const void *D, const void *x,
+                            void *y, const float *bias, int dtype, ConvArgs *a);
+// Workspace a family needs for these arguments.
+size_t workspace_for(unsigned algo, const ConvArgs &a, int dtype);
+// Can the family run this case at all (dtype, shape)?
+bool supports(unsigned algo, const ConvArgs &a, int dtype);
+// The family onexn_conv_fwd runs (flags' forced ALGO, else the AUTO choice).
+unsigned pick_algo(const ConvArgs &a, int dtype, unsigned flags, size_t ws_bytes);
+onexn_status check_algo(unsigned algo, const ConvArgs &a, int dtype, size_t ws_bytes);
+// Launch one family (decode included for the tensor-core family).
+cudaError_t launch(unsigned algo, const ConvArgs &a, int dtype, void *workspace, cudaStream_t st);
+
+}  // namespace detail
+}  // namespace onexn

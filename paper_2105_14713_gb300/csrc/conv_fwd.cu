@@ -2,18 +2,11 @@
 // convolution of a 1xN-pruned layer (Eq. 7).  Launches only; never
 // allocates, synchronises or reads device memory from the host.
 #include "conv_common.cuh"
+#include "conv_dispatch.h"
 #include "onexn_internal.h"
 
 #include <mutex>
 
-namespace onexn {
-cudaError_t launch_fma(const ConvArgs &a, int dtype, cudaStream_t st);
-cudaError_t launch_mma(const ConvArgs &a, cudaStream_t st);
-bool mma_supports(const ConvArgs &a);
-cudaError_t launch_tc(const ConvArgs &a, int dtype, void *workspace, cudaStream_t st);
-bool tc_supports(const ConvArgs &a, int dtype);
-size_t tc_workspace_bytes(const ConvArgs &a, int dtype);
-}  // namespace onexn
 
 using onexn::fail;
 
@@ -64,9 +57,12 @@ cudaError_t device_status_ptr(unsigned int **p)
 
 }  // namespace onexn
 
-namespace {
+namespace onexn {
+namespace detail {
 
+namespace {
 bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+}  // namespace
 
 // Shape, dtype and flag checks; fills the geometry part of *a.
 onexn_status check_shape(const onexn_conv_desc *d, int N, int64_t t, int dtype, unsigned flags,
@@ -151,10 +147,12 @@ bool supports(unsigned algo, const onexn::ConvArgs &a, int dtype)
 // staged activation.  The tensor-core GEMM decodes the weights into the
 // workspace (about 2000 bytes per ns) and does the dense work (C_out*K per
 // pixel; fp32 issues three tf32 products per term).
+namespace {
 double fma_floor(int N) { return N >= 4 ? 1.33e-5 : N >= 2 ? 1.66e-5 : 2.67e-5; }
 double fma_per_kept(int N) { return N >= 8 ? 3.0e-5 : N >= 4 ? 4.3e-5 : N >= 2 ? 7.2e-5 : 1.44e-4; }
 double tc_per_dense(int dtype) { return dtype == ONEXN_F32 ? 7.9e-6 : 2.3e-6; }
 constexpr double kDecodeNsPerByte = 1.0 / 2000.0;
+}  // namespace
 
 // Kernel family for AUTO: the tcgen05 GEMM when its workspace fits and the
 // cost model does not expect the FFMA kernel to be faster; otherwise FFMA.
@@ -187,7 +185,17 @@ onexn_status check_algo(unsigned algo, const onexn::ConvArgs &a, int dtype, size
     return ONEXN_OK;
 }
 
-}  // namespace
+cudaError_t launch(unsigned algo, const ConvArgs &a, int dtype, void *workspace, cudaStream_t st)
+{
+    if (algo == ONEXN_ALGO_FMA) return launch_fma(a, dtype, st);
+    if (algo == ONEXN_ALGO_MMA) return launch_mma(a, st);
+    return launch_tc(a, dtype, workspace, st);
+}
+
+}  // namespace detail
+}  // namespace onexn
+
+using namespace onexn::detail;
 
 extern "C" onexn_status onexn_conv_algo(const onexn_conv_desc *desc, int N, int64_t t, int dtype,
                                         unsigned flags, size_t workspace_bytes, unsigned *algo)
@@ -247,9 +255,7 @@ extern "C" onexn_status onexn_conv_fwd(const onexn_conv_desc *desc, const int32_
     cudaStream_t s = static_cast<cudaStream_t>(stream);
     cudaError_t e = onexn::device_status_ptr(&a.status);
     if (e != cudaSuccess) return fail(ONEXN_ECUDA, "conv: status word: %s", cudaGetErrorString(e));
-    if (algo == ONEXN_ALGO_FMA) e = onexn::launch_fma(a, dtype, s);
-    else if (algo == ONEXN_ALGO_MMA) e = onexn::launch_mma(a, s);
-    else e = onexn::launch_tc(a, dtype, workspace, s);
+    e = launch(algo, a, dtype, workspace, s);
     if (e != cudaSuccess) return fail(ONEXN_ECUDA, "conv: launch failed: %s", cudaGetErrorString(e));
     return ONEXN_OK;
 }

@@ -47,6 +47,7 @@
 // gets ONEXN_ETIMEOUT, every role stops, outstanding MMAs are drained and
 // the TMEM is freed before the kernel returns.
 #include "conv_common.cuh"
+#include "conv_dispatch.h"
 #include "onexn_internal.h"
 #include "tc_ptx.cuh"
 
@@ -553,8 +554,21 @@ cudaError_t launch_bn(const ConvArgs &a, const typename Tr::T *W, const typename
         tmap_wlo = tmap_w;                                     // unused
         if (!tmap_2d(&tmap_y, Tr::kTmap, elem, a.y, a.P_pix, a.C_out, kBM)) return cudaErrorInvalidValue;
     }
-    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, L::kAlloc);
+    // the shared-memory opt-in, once per device for this kernel
+    static std::mutex attr_mu;
+    static bool attr_done[64];
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
     if (e != cudaSuccess) return e;
+    if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
+    {
+        std::lock_guard<std::mutex> lk(attr_mu);
+        if (!attr_done[dev]) {
+            e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, L::kAlloc);
+            if (e != cudaSuccess) return e;
+            attr_done[dev] = true;
+        }
+    }
     int sms = 0;
     e = device_sm_count(&sms);
     if (e != cudaSuccess) return e;
@@ -567,7 +581,7 @@ cudaError_t launch_bn(const ConvArgs &a, const typename Tr::T *W, const typename
 }
 
 template <typename Tr>
-cudaError_t launch_typed(const ConvArgs &a, void *workspace, cudaStream_t st)
+cudaError_t decode_typed(const ConvArgs &a, void *workspace, cudaStream_t st)
 {
     using T = typename Tr::T;
     const int K = a.KH * a.KW * a.C;
@@ -577,8 +591,16 @@ cudaError_t launch_typed(const ConvArgs &a, void *workspace, cudaStream_t st)
     const dim3 grid(static_cast<unsigned>((K + kDecodeCols - 1) / kDecodeCols), a.C_out / a.N,
                     (a.N + kDecodeRows - 1) / kDecodeRows);
     bsr_decode_kernel<T><<<grid, kDecodeCols, 0, st>>>(a.P, a.I, static_cast<const T *>(a.D), a.N, a.t, K, W, W_lo);
-    cudaError_t e = cudaGetLastError();
-    if (e != cudaSuccess) return e;
+    return cudaGetLastError();
+}
+
+template <typename Tr>
+cudaError_t gemm_typed(const ConvArgs &a, const void *workspace, cudaStream_t st)
+{
+    using T = typename Tr::T;
+    const size_t n = static_cast<size_t>(a.C_out) * a.KH * a.KW * a.C;
+    const T *W = static_cast<const T *>(workspace);
+    const T *W_lo = Tr::kSplit ? W + n : nullptr;
     if (a.C_out <= 64) return launch_bn<Tr, 64>(a, W, W_lo, st);
     if (a.C_out <= 128) return launch_bn<Tr, 128>(a, W, W_lo, st);
     return launch_bn<Tr, 256>(a, W, W_lo, st);
@@ -610,11 +632,22 @@ bool tc_supports(const ConvArgs &a, int dtype)
     return true;
 }
 
+cudaError_t tc_decode(const ConvArgs &a, int dtype, void *workspace, cudaStream_t st)
+{
+    return dtype == ONEXN_F32 ? decode_typed<TcF32>(a, workspace, st) : decode_typed<TcBf16>(a, workspace, st);
+}
+
+cudaError_t tc_gemm(const ConvArgs &a, int dtype, const void *workspace, cudaStream_t st)
+{
+    if (a.P_pix == 0) return cudaSuccess;
+    return dtype == ONEXN_F32 ? gemm_typed<TcF32>(a, workspace, st) : gemm_typed<TcBf16>(a, workspace, st);
+}
+
 cudaError_t launch_tc(const ConvArgs &a, int dtype, void *workspace, cudaStream_t st)
 {
     if (a.P_pix == 0) return cudaSuccess;
-    if (dtype == ONEXN_F32) return launch_typed<TcF32>(a, workspace, st);
-    return launch_typed<TcBf16>(a, workspace, st);
+    const cudaError_t e = tc_decode(a, dtype, workspace, st);
+    return e != cudaSuccess ? e : tc_gemm(a, dtype, workspace, st);
 }
 
 }  // namespace onexn

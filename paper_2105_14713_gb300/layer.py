@@ -97,12 +97,41 @@ class PrunedConv2d:
 
     __call__ = forward
 
-    def forward_host(self, x_host: torch.Tensor, relu: bool = False,
-                     algo: int = _c.ONEXN_ALGO_AUTO) -> torch.Tensor:
-        """End-to-end call from host memory: copy x in, convolve, copy y out."""
-        x = x_host.to(self.device, non_blocking=True)
-        y = self.forward(x, relu=relu, algo=algo)
-        out = torch.empty(y.shape, dtype=y.dtype, pin_memory=True)
-        out.copy_(y, non_blocking=True)
-        torch.cuda.current_stream(self.device).synchronize()
-        return out
+    def host_workspace(self, x_shape, flags: int = 0):
+        """Device workspace of forward_host for this input shape (allocated
+        once, reused)."""
+        B, H, W, _ = x_shape
+        key = ("host", B, H, W, flags & 0xF00)
+        if key not in self._ws:
+            n = _c.onexn_conv_host_workspace_size(self.desc(B, H, W), self.N, self.t, self.cdtype, flags)
+            self._ws[key] = torch.empty(max(n, 256), dtype=torch.uint8, device=self.device)
+        return self._ws[key]
+
+    def forward_host(self, x_host: torch.Tensor, y_host: torch.Tensor = None, relu: bool = False,
+                     algo: int = _c.ONEXN_ALGO_AUTO, stream=None, sync: bool = True) -> torch.Tensor:
+        """End to end from host memory (onexn_conv_fwd_host): the input is
+        copied in and the output copied out chunk by chunk, overlapped with
+        the convolution.  x_host: contiguous CPU NHWC tensor of this layer's
+        dtype (pinned for overlapped copies).  y_host: optional CPU output
+        (allocated pinned if None).  With sync=False the call returns after
+        enqueueing: synchronise `stream` before reading y_host."""
+        if x_host.dtype != self.torch_dtype or x_host.is_cuda or not x_host.is_contiguous():
+            raise ValueError(f"x_host must be a contiguous CPU {self.torch_dtype} NHWC tensor")
+        B, H, W, C = x_host.shape
+        if C != self.C_in:
+            raise ValueError(f"x_host has {C} channels, layer expects {self.C_in}")
+        shape = self.out_shape(x_host.shape)
+        if y_host is None:
+            y_host = torch.empty(shape, dtype=x_host.dtype, pin_memory=True)
+        elif tuple(y_host.shape) != tuple(shape) or y_host.dtype != x_host.dtype or y_host.is_cuda \
+                or not y_host.is_contiguous():
+            raise ValueError(f"y_host must be a contiguous CPU {x_host.dtype} tensor of shape {shape}")
+        if stream is None:
+            stream = torch.cuda.current_stream(self.device)
+        flags = (_c.ONEXN_RELU if relu else 0) | algo
+        _c.onexn_conv_fwd_host(self.desc(B, H, W), self.P, self.I, self.D, self.N, self.t, x_host,
+                               y_host, self.bias, self.cdtype, flags,
+                               self.host_workspace(x_host.shape, algo), stream)
+        if sync:
+            stream.synchronize()
+        return y_host

@@ -60,6 +60,9 @@ SIGNATURES = {
     "onexn_device_status": ([_I32, _P], _I32),
     "onexn_conv_fwd_noalloc": ([ctypes.POINTER(ConvDesc), _P, _P, _P, _I32, _I64, _P, _P, _P, _I32,
                                 _U32, _P], _I32),
+    "onexn_conv_fwd_host": ([ctypes.POINTER(ConvDesc), _P, _P, _P, _I32, _I64, _P, _P, _P, _I32,
+                             _U32, _P, ctypes.c_size_t, _P], _I32),
+    "onexn_conv_host_workspace_size": ([ctypes.POINTER(ConvDesc), _I32, _I64, _I32, _U32, _P], _I32),
 }
 
 
@@ -215,6 +218,29 @@ def onexn_conv_fwd_noalloc(desc: ConvDesc, P, I, D, N: int, t: int, x, y, bias, 
     _check(lib.onexn_conv_fwd_noalloc(ctypes.byref(desc), ptr(P), ptr(I), ptr(D), int(N), int(t),
                                       ptr(x), ptr(y), ptr(bias), int(dtype), int(flags),
                                       ctypes.c_void_p(stream.cuda_stream)))
+
+
+def onexn_conv_host_workspace_size(desc: ConvDesc, N: int, t: int, dtype: int, flags: int = 0) -> int:
+    out = ctypes.c_size_t(0)
+    _check(lib.onexn_conv_host_workspace_size(ctypes.byref(desc), int(N), int(t), int(dtype),
+                                              int(flags), ctypes.byref(out)))
+    return out.value
+
+
+def onexn_conv_fwd_host(desc: ConvDesc, P, I, D, N: int, t: int, x_host, y_host, bias, dtype: int,
+                        flags: int = 0, workspace=None, stream=None) -> None:
+    """The convolution on host-memory activations: x_host and y_host are CPU
+    tensors (pinned for overlapped copies), P, I, D, bias and workspace CUDA
+    tensors; stream a torch.cuda.Stream or None (the current stream).  The
+    call is asynchronous: synchronise the stream before reading y_host."""
+    import torch
+    if stream is None:
+        stream = torch.cuda.current_stream(workspace.device)
+    ptr = (lambda tns: None if tns is None else ctypes.c_void_p(tns.data_ptr()))
+    ws_bytes = 0 if workspace is None else workspace.numel() * workspace.element_size()
+    _check(lib.onexn_conv_fwd_host(ctypes.byref(desc), ptr(P), ptr(I), ptr(D), int(N), int(t),
+                                   ptr(x_host), ptr(y_host), ptr(bias), int(dtype), int(flags),
+                                   ptr(workspace), int(ws_bytes), ctypes.c_void_p(stream.cuda_stream)))
 
 
 def onexn_device_status(clear: bool = True) -> int:

@@ -156,3 +156,66 @@ def test_streams_and_repeat_calls_are_deterministic():
         y2 = conv(x)
     s.synchronize()
     assert torch.equal(y1, y2)
+
+
+# ------------------------------------------------ host-memory entry point
+
+HOST_CASES = [
+    # layer, forced algo
+    (L("h3x3", 13, 14, 14, 64, 64, 3, 3, 1, 1, 1, N=8, rate=0.5, dtype="f32", seed=21), "auto"),
+    (L("h3x3b", 13, 14, 14, 64, 64, 3, 3, 1, 1, 1, N=8, rate=0.5, dtype="bf16", seed=22), "auto"),
+    (L("h1x1s2", 9, 15, 15, 32, 48, 1, 1, 2, 0, 1, N=4, rate=0.7, dtype="f32", seed=23), "fma"),
+    (L("h1x1", 11, 28, 28, 96, 64, 1, 1, 1, 0, 1, N=16, rate=0.5, dtype="bf16", seed=24), "tc"),
+    # 160 images of 200704 bytes: 4 chunks, so the first slot is reused
+    (L("hbig", 160, 28, 28, 64, 64, 3, 3, 1, 1, 1, N=8, rate=0.5, dtype="f32", seed=25), "tc"),
+    (L("hbigb", 330, 28, 28, 64, 64, 3, 3, 1, 1, 1, N=8, rate=0.5, dtype="bf16", seed=26), "auto"),
+]
+
+
+@pytest.mark.parametrize("case", HOST_CASES, ids=[c[0].name for c in HOST_CASES])
+def test_host_entry_matches_device_entry_bitwise(case):
+    """onexn_conv_fwd_host (chunks of images copied in and out on internal
+    streams) gives exactly the device entry's output: every output pixel is
+    computed by the same kernel in the same order, only grouped differently."""
+    layer, algo = case
+    from paper_2105_14713_gb300.layer import PrunedConv2d
+    conv = PrunedConv2d(wl.weights(layer).numpy(), layer.N, layer.rate, bias=wl.bias(layer).numpy(),
+                        stride=layer.stride, padding=layer.pad, dilation=layer.dil, dtype=layer.dtype)
+    x = wl.activations(layer)
+    x = x if layer.dtype == "f32" else x.to(torch.bfloat16)
+    y_dev = conv(x.cuda(), relu=True, algo=ALGOS[algo])
+    for pinned in (True, False):
+        xh = x.pin_memory() if pinned else x.clone()
+        y_host = conv.forward_host(xh, relu=True, algo=ALGOS[algo])
+        assert torch.equal(y_host.view(torch.int16 if layer.dtype == "bf16" else torch.int32),
+                           y_dev.cpu().view(torch.int16 if layer.dtype == "bf16" else torch.int32)), pinned
+
+
+def test_host_entry_overlapping_calls_on_two_streams():
+    """Two layers enqueued back to back on different streams (the second's
+    copies overlap the first's compute) both give the device entry's output."""
+    from paper_2105_14713_gb300.layer import PrunedConv2d
+    layers = [L("ov_a", 24, 28, 28, 64, 128, 3, 3, 1, 1, 1, N=8, rate=0.5, dtype="f32", seed=31),
+              L("ov_b", 24, 28, 28, 64, 64, 3, 3, 1, 1, 1, N=4, rate=0.3, dtype="bf16", seed=32)]
+    convs, xs, refs = [], [], []
+    for layer in layers:
+        conv = PrunedConv2d(wl.weights(layer).numpy(), layer.N, layer.rate, padding=1, dtype=layer.dtype)
+        x = wl.activations(layer)
+        x = (x if layer.dtype == "f32" else x.to(torch.bfloat16)).pin_memory()
+        convs.append(conv)
+        xs.append(x)
+        refs.append(conv(x.cuda()).cpu())
+    streams = [torch.cuda.Stream() for _ in layers]
+    for _ in range(3):
+        outs = [c.forward_host(x, stream=s, sync=False) for c, x, s in zip(convs, xs, streams)]
+        torch.cuda.synchronize()
+        for o, r in zip(outs, refs):
+            assert torch.equal(o.float(), r.float())
+
+
+def test_host_entry_empty_batch():
+    from paper_2105_14713_gb300.layer import PrunedConv2d
+    layer = L("hempty", 0, 8, 8, 16, 16, 3, 3, 1, 1, 1, N=4, rate=0.5, dtype="f32")
+    conv = PrunedConv2d(wl.weights(layer).numpy(), 4, 0.5, padding=1)
+    y = conv.forward_host(torch.zeros(0, 8, 8, 16).pin_memory())
+    assert tuple(y.shape) == (0, 8, 8, 16)

@@ -171,6 +171,27 @@ def test_auto_cost_model():
         assert ox.onexn_conv_algo(tiny, 8, G * K // 10, dt, 0, ws) == ox.ONEXN_ALGO_FMA
 
 
+def test_host_entry_workspace_and_argument_checks_need_no_gpu():
+    # 3x3 128->128 on 64x28x28 fp32: decoded hi/lo weights + 3 input and 3
+    # output slots of one chunk (64 images of 401408 bytes in ~8 MiB chunks:
+    # 3 chunks of 22 images)
+    d = ox.make_desc(64, 28, 28, 128, 128, 3, 3, 1, 1, 1)
+    n = ox.onexn_conv_host_workspace_size(d, 8, 9216, ox.ONEXN_F32)
+    img = 28 * 28 * 128 * 4
+    assert n == 128 * 1152 * 8 + 3 * 2 * 22 * img
+    # FFMA forced: no decoded weights
+    assert ox.onexn_conv_host_workspace_size(d, 8, 9216, ox.ONEXN_F32, ox.ONEXN_ALGO_FMA) == \
+        3 * 2 * 22 * img
+    # bf16: half the bytes per image -> ~8 MiB chunks of 32 images
+    nb = ox.onexn_conv_host_workspace_size(d, 8, 9216, ox.ONEXN_BF16)
+    assert nb == 128 * 1152 * 2 + 3 * 2 * 32 * (img // 2)
+    # argument errors before any device work
+    st = ox.lib.onexn_conv_fwd_host(ctypes.byref(d), None, None, None, 8, 9216, None, None, None,
+                                    ox.ONEXN_F32, 0, None, 0, None)
+    assert st == ox.ONEXN_EINVAL
+    assert _status(ox.onexn_conv_host_workspace_size, d, 3, 10, ox.ONEXN_F32) == ox.ONEXN_EINVAL
+
+
 def test_conv_shape_and_argument_errors_need_no_gpu():
     d = ox.make_desc(2, 7, 7, 8, 16, 3, 3, 2, 1, 1)
     assert ox.onexn_conv_out_shape(d) == (4, 4)
