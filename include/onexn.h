@@ -185,8 +185,8 @@ onexn_status onexn_conv_out_shape(const onexn_conv_desc *desc, int *Ho, int *Wo)
  *           nullable DEVICE scratch owned by the caller, 256-byte aligned.
  *           Some kernel families need it (onexn_conv_workspace_size); the
  *           call overwrites it, so calls that run concurrently need
- *           separate workspaces.  AUTO only picks a family whose workspace
- *           fits in workspace_bytes.
+ *           separate workspaces.  AUTO only picks a family whose minimum
+ *           workspace fits in workspace_bytes.
  *   stream  cudaStream_t to launch on (NULL = legacy default stream).
  * Asynchronous: returns after the launch; errors of the launch itself are
  * returned as ECUDA.  No allocation, no synchronisation, no host read of
@@ -203,10 +203,14 @@ onexn_status onexn_conv_fwd(const onexn_conv_desc *desc, const int32_t *P, const
  * onexn_conv_workspace_size -- bytes of device workspace onexn_conv_fwd
  * needs for these arguments with this flags' ALGO (for AUTO: the largest
  * need among the families AUTO may pick, so that passing this many bytes
- * lets AUTO choose freely).  ONEXN_ALGO_TC needs the decoded masked
- * weights: C_out * KH*KW*C_in bf16 values (dtype ONEXN_BF16), or twice
- * C_out * KH*KW*C_in fp32 values, their tf32 high and low parts
- * (ONEXN_F32); rounded up to 256 bytes.  ONEXN_ALGO_FMA needs none.
+ * lets AUTO choose freely).  ONEXN_ALGO_TC needs at least the decoded
+ * masked weights: C_out * KH*KW*C_in bf16 values (dtype ONEXN_BF16), or
+ * twice C_out * KH*KW*C_in fp32 values, their tf32 high and low parts
+ * (ONEXN_F32), rounded up to 256 bytes; the size reported here adds the
+ * space its GEMM uses to spread the last, partial round of output tiles
+ * over all SMs (one 128 x BN fp32 partial tile for each of 152 CTAs, BN =
+ * 64, 128 or 256 by C_out, and 152 flags).  With only the minimum the GEMM
+ * runs without that balancing.  ONEXN_ALGO_FMA needs none.
  */
 onexn_status onexn_conv_workspace_size(const onexn_conv_desc *desc, int N, int64_t t, int dtype,
                                        unsigned flags, size_t *bytes);

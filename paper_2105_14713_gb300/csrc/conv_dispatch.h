@@ -13,11 +13,14 @@ cudaError_t launch_fma(const ConvArgs &a, int dtype, cudaStream_t st);
 cudaError_t launch_mma(const ConvArgs &a, cudaStream_t st);
 bool mma_supports(const ConvArgs &a);
 // tensor-core family: decode of (P, I, D) into the workspace, then the GEMM
-cudaError_t launch_tc(const ConvArgs &a, int dtype, void *workspace, cudaStream_t st);
-cudaError_t tc_decode(const ConvArgs &a, int dtype, void *workspace, cudaStream_t st);
-cudaError_t tc_gemm(const ConvArgs &a, int dtype, const void *workspace, cudaStream_t st);
+// (which splits its last round of tiles across CTAs when ws_bytes has room
+// for tc_workspace_bytes, else needs tc_workspace_min)
+cudaError_t launch_tc(const ConvArgs &a, int dtype, void *workspace, size_t ws_bytes, cudaStream_t st);
+cudaError_t tc_decode(const ConvArgs &a, int dtype, void *workspace, size_t ws_bytes, cudaStream_t st);
+cudaError_t tc_gemm(const ConvArgs &a, int dtype, const void *workspace, size_t ws_bytes, cudaStream_t st);
 bool tc_supports(const ConvArgs &a, int dtype);
 size_t tc_workspace_bytes(const ConvArgs &a, int dtype);
+size_t tc_workspace_min(const ConvArgs &a, int dtype);
 
 namespace detail {
 
@@ -27,15 +30,17 @@ onexn_status check_shape(const onexn_conv_desc *d, int N, int64_t t, int dtype, 
 // Device-pointer checks; fills the pointer part of *a.
 onexn_status check_pointers(const int32_t *P, const int32_t *I, const void *D, const void *x,
                             void *y, const float *bias, int dtype, ConvArgs *a);
-// Workspace a family needs for these arguments.
+// Workspace a family uses at best / needs at least for these arguments.
 size_t workspace_for(unsigned algo, const ConvArgs &a, int dtype);
+size_t workspace_min_for(unsigned algo, const ConvArgs &a, int dtype);
 // Can the family run this case at all (dtype, shape)?
 bool supports(unsigned algo, const ConvArgs &a, int dtype);
 // The family onexn_conv_fwd runs (flags' forced ALGO, else the AUTO choice).
 unsigned pick_algo(const ConvArgs &a, int dtype, unsigned flags, size_t ws_bytes);
 onexn_status check_algo(unsigned algo, const ConvArgs &a, int dtype, size_t ws_bytes);
 // Launch one family (decode included for the tensor-core family).
-cudaError_t launch(unsigned algo, const ConvArgs &a, int dtype, void *workspace, cudaStream_t st);
+cudaError_t launch(unsigned algo, const ConvArgs &a, int dtype, void *workspace, size_t ws_bytes,
+                   cudaStream_t st);
 
 }  // namespace detail
 }  // namespace onexn

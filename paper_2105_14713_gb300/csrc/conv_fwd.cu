@@ -127,6 +127,11 @@ size_t workspace_for(unsigned algo, const onexn::ConvArgs &a, int dtype)
     return algo == ONEXN_ALGO_TC ? onexn::tc_workspace_bytes(a, dtype) : 0;
 }
 
+size_t workspace_min_for(unsigned algo, const onexn::ConvArgs &a, int dtype)
+{
+    return algo == ONEXN_ALGO_TC ? onexn::tc_workspace_min(a, dtype) : 0;
+}
+
 // Can the family run this case at all (dtype, shape)?
 bool supports(unsigned algo, const onexn::ConvArgs &a, int dtype)
 {
@@ -160,14 +165,14 @@ unsigned pick_algo(const onexn::ConvArgs &a, int dtype, unsigned flags, size_t w
 {
     const unsigned forced = flags & ONEXN_ALGO_MASK;
     if (forced != ONEXN_ALGO_AUTO) return forced;
-    if (!supports(ONEXN_ALGO_TC, a, dtype) || ws_bytes < workspace_for(ONEXN_ALGO_TC, a, dtype))
+    if (!supports(ONEXN_ALGO_TC, a, dtype) || ws_bytes < workspace_min_for(ONEXN_ALGO_TC, a, dtype))
         return ONEXN_ALGO_FMA;
     if (a.t == 0) return ONEXN_ALGO_FMA;                  // bias only
     const double kept = static_cast<double>(a.t) * a.N * a.P_pix;
     const double dense = static_cast<double>(a.C_out) * a.KH * a.KW * a.C * a.P_pix;
     const double fma_ns = dense * fma_floor(a.N) + kept * fma_per_kept(a.N);
     const double tc_ns = dense * tc_per_dense(dtype) +
-                         static_cast<double>(workspace_for(ONEXN_ALGO_TC, a, dtype)) * kDecodeNsPerByte;
+                         static_cast<double>(workspace_min_for(ONEXN_ALGO_TC, a, dtype)) * kDecodeNsPerByte;
     return fma_ns < tc_ns ? ONEXN_ALGO_FMA : ONEXN_ALGO_TC;
 }
 
@@ -178,18 +183,19 @@ onexn_status check_algo(unsigned algo, const onexn::ConvArgs &a, int dtype, size
     if (!supports(algo, a, dtype))
         return fail(ONEXN_EUNSUPPORTED, "conv: algo %u cannot run this case (dtype/shape)",
                     algo >> ONEXN_ALGO_SHIFT);
-    const size_t need = workspace_for(algo, a, dtype);
+    const size_t need = workspace_min_for(algo, a, dtype);
     if (ws_bytes < need)
         return fail(ONEXN_EINVAL, "conv: algo %u needs %zu bytes of workspace, got %zu",
                     algo >> ONEXN_ALGO_SHIFT, need, ws_bytes);
     return ONEXN_OK;
 }
 
-cudaError_t launch(unsigned algo, const ConvArgs &a, int dtype, void *workspace, cudaStream_t st)
+cudaError_t launch(unsigned algo, const ConvArgs &a, int dtype, void *workspace, size_t ws_bytes,
+                   cudaStream_t st)
 {
     if (algo == ONEXN_ALGO_FMA) return launch_fma(a, dtype, st);
     if (algo == ONEXN_ALGO_MMA) return launch_mma(a, st);
-    return launch_tc(a, dtype, workspace, st);
+    return launch_tc(a, dtype, workspace, ws_bytes, st);
 }
 
 }  // namespace detail
@@ -255,7 +261,7 @@ extern "C" onexn_status onexn_conv_fwd(const onexn_conv_desc *desc, const int32_
     cudaStream_t s = static_cast<cudaStream_t>(stream);
     cudaError_t e = onexn::device_status_ptr(&a.status);
     if (e != cudaSuccess) return fail(ONEXN_ECUDA, "conv: status word: %s", cudaGetErrorString(e));
-    e = launch(algo, a, dtype, workspace, s);
+    e = launch(algo, a, dtype, workspace, workspace_bytes, s);
     if (e != cudaSuccess) return fail(ONEXN_ECUDA, "conv: launch failed: %s", cudaGetErrorString(e));
     return ONEXN_OK;
 }

@@ -117,12 +117,14 @@ onexn_status plan(const onexn_conv_desc *desc, int N, int64_t t, int dtype, unsi
     size_t ws = 0;
     for (unsigned al : {ONEXN_ALGO_FMA, ONEXN_ALGO_MMA, ONEXN_ALGO_TC})
         if ((forced == ONEXN_ALGO_AUTO || forced == al) && onexn::detail::supports(al, a, dtype) &&
-            onexn::detail::workspace_for(al, a, dtype) > ws)
-            ws = onexn::detail::workspace_for(al, a, dtype);
+            onexn::detail::workspace_min_for(al, a, dtype) > ws)
+            ws = onexn::detail::workspace_min_for(al, a, dtype);
     hp->algo = onexn::detail::pick_algo(a, dtype, flags, ws);
     st = onexn::detail::check_algo(hp->algo, a, dtype, ws);
     if (st != ONEXN_OK) return st;
-    hp->kernel_ws = onexn::detail::workspace_for(hp->algo, a, dtype);
+    // chunk GEMMs may run concurrently on the two compute streams, so they
+    // get no shared stream-K space: the decoded weights only
+    hp->kernel_ws = onexn::detail::workspace_min_for(hp->algo, a, dtype);
     return ONEXN_OK;
 }
 
@@ -194,7 +196,7 @@ extern "C" onexn_status onexn_conv_fwd_host(const onexn_conv_desc *desc, const i
         ONEXN_TRY(cudaStreamWaitEvent(p.out[k], p.start, 0));
     }
     if (hp.algo == ONEXN_ALGO_TC) {
-        ONEXN_TRY(onexn::tc_decode(a, dtype, ws, p.cmp[0]));
+        ONEXN_TRY(onexn::tc_decode(a, dtype, ws, hp.kernel_ws, p.cmp[0]));
         ONEXN_TRY(cudaEventRecord(p.dec, p.cmp[0]));
         ONEXN_TRY(cudaStreamWaitEvent(p.cmp[1], p.dec, 0));
     }
@@ -222,9 +224,9 @@ extern "C" onexn_status onexn_conv_fwd_host(const onexn_conv_desc *desc, const i
         c.x = xd;
         c.y = yd;
         if (hp.algo == ONEXN_ALGO_TC)
-            ONEXN_TRY(onexn::tc_gemm(c, dtype, ws, cs));
+            ONEXN_TRY(onexn::tc_gemm(c, dtype, ws, hp.kernel_ws, cs));
         else
-            ONEXN_TRY(onexn::detail::launch(hp.algo, c, dtype, ws, cs));
+            ONEXN_TRY(onexn::detail::launch(hp.algo, c, dtype, ws, hp.kernel_ws, cs));
         ONEXN_TRY(cudaEventRecord(p.ev_cmp[slot], cs));
         // out
         ONEXN_TRY(cudaStreamWaitEvent(out, p.ev_cmp[slot], 0));

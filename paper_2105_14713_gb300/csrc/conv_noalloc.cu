@@ -27,6 +27,7 @@
 //  * The device address of the array is looked up once per device, on the
 //    first call made with that device current (cudaGetSymbolAddress).  Make
 //    that first call before any stream capture begins.
+#include "conv_dispatch.h"
 #include "onexn_internal.h"
 
 #include <cuda_runtime.h>
@@ -76,9 +77,14 @@ extern "C" onexn_status onexn_conv_fwd_noalloc(const onexn_conv_desc *desc, cons
     if ((flags & ONEXN_ALGO_MASK) != ONEXN_ALGO_AUTO && (flags & ONEXN_ALGO_MASK) != ONEXN_ALGO_TC)
         return onexn::fail(ONEXN_EINVAL, "conv_noalloc: only the tensor-core family runs here");
     const unsigned f = (flags & ~ONEXN_ALGO_MASK) | ONEXN_ALGO_TC;
-    size_t need = 0;
-    onexn_status st = onexn_conv_workspace_size(desc, N, t, dtype, f, &need);
+    onexn::ConvArgs a{};
+    onexn_status st = onexn::detail::check_shape(desc, N, t, dtype, f, &a);
     if (st != ONEXN_OK) return st;
+    if (!onexn::detail::supports(ONEXN_ALGO_TC, a, dtype))
+        return onexn::fail(ONEXN_EUNSUPPORTED, "conv_noalloc: the tensor-core family cannot run this case");
+    // the decoded weights must fit (the stream-K balancing space is not
+    // needed and does not fit in the fixed scratch)
+    const size_t need = onexn::detail::workspace_min_for(ONEXN_ALGO_TC, a, dtype);
     if (need > kNoAllocScratchBytes)
         return onexn::fail(ONEXN_EINVAL,
                            "conv_noalloc: decoded weights need %zu bytes, more than the fixed %zu-byte "

@@ -40,9 +40,9 @@
 //    the accumulator's "tmem_full" mbarrier.
 //  * warps 2-5, epilogue: wait "tmem_full", read the accumulator with
 //    tcgen05.ld (warp w reads TMEM lanes 32*(w%4)..+31 = its 32 pixels),
-//    release it ("tmem_empty"), add the bias, apply ReLU and store NHWC:
-//    bf16 through a 128-byte-swizzled staging tile and TMA bulk stores,
-//    fp32 directly from registers.
+//    release it ("tmem_empty"), add the bias, apply ReLU and store NHWC one
+//    128-byte column atom at a time through a double-buffered
+//    128-byte-swizzled staging tile and TMA stores.
 // All waits are bounded (about one second each); on expiry the status word
 // gets ONEXN_ETIMEOUT, every role stops, outstanding MMAs are drained and
 // the TMEM is freed before the kernel returns.
@@ -85,6 +85,11 @@ struct TcF32 {
 };
 
 constexpr int kSmemMax = 232448;      // dynamic shared memory per CTA (opt-in maximum)
+constexpr int kPlanCTAs = 152;        // stream-K: at most this many CTAs (GB300's SM count)
+constexpr int kMinSplitIters = 4;     // stream-K: at least this many chunk iterations per CTA
+
+// one partial slot (128 x BN fp32) per CTA
+constexpr size_t sk_partial_bytes(int BN) { return static_cast<size_t>(kPlanCTAs) * kBM * BN * 4; }
 
 constexpr int pow2_at_least(int v, int p = 32) { return p >= v ? p : pow2_at_least(v, 2 * p); }
 
@@ -94,14 +99,15 @@ struct TcLayout {
     static constexpr int kB = BN * kRowBytes;                        // 8/16/32 KB
     static constexpr int kStage = kA + (Tr::kSplit ? 2 * kB : kB);   // [A | B_hi | B_lo]
     static constexpr int kTx = kStage;                               // bytes the TMA brings
-    static constexpr int kOutBytes = Tr::kSplit ? 0 : kBM * BN * 2;  // bf16 staging tile
-    static constexpr int kFixed = 1024 + kOutBytes + BN * 4 + (3 * 6 + 5) * 8 + 16;
+    // output staging: per epilogue warp two buffers of 32 rows x one 128-byte column atom
+    static constexpr int kOutBytes = 4 * 2 * 32 * kRowBytes;
+    static constexpr int kFixed = 1024 + kOutBytes + BN * 4 + (3 * 6 + 6) * 8 + 16;
     static constexpr int kS = ((kSmemMax - kFixed) / kStage) > 6 ? 6 : ((kSmemMax - kFixed) / kStage);
     static constexpr int kOut = kS * kStage;
-    static constexpr int kBias = kOut + kOutBytes;                    // BN fp32
+    static constexpr int kBias = kOut + kOutBytes;                   // BN fp32
     static constexpr int kBar = kBias + BN * 4;
-    // full[S], split[S], empty[S], tmem_full[2], tmem_empty[2], drain, TMEM holder
-    static constexpr int kHolder = kBar + (3 * kS + 5) * 8;
+    // full[S], split[S], empty[S], tmem_full[2], tmem_empty[2], drain, fixup, TMEM holder
+    static constexpr int kHolder = kBar + (3 * kS + 6) * 8;
     static constexpr int kBytes = kHolder + 16;
     static constexpr int kAlloc = kBytes + 1024;                      // room to align the base to 1024
     // TMEM columns: the fp32 accumulator buffers (two when they fit next to
@@ -110,7 +116,11 @@ struct TcLayout {
     static constexpr int kARing = Tr::kSplit ? 128 : 0;
     static constexpr int kAcc = (2 * BN + kARing <= 512) ? 2 : 1;
     static constexpr int kTmemCols = pow2_at_least(kAcc * BN + kARing);
+    // partial tiles (128 x BN fp32) the idle ring holds at a split tile's finish
+    static constexpr int kSlotBytes = kBM * BN * 4;
+    static constexpr int kRingSlots = kS * kStage / kSlotBytes;
     static_assert(kS >= 2, "ring too small");
+    static_assert(kRingSlots >= 1, "ring cannot hold a partial tile");
     static_assert(kAlloc <= kSmemMax, "shared memory");
     static_assert(kTmemCols <= 512, "tensor memory");
 };
@@ -136,10 +146,14 @@ __device__ __forceinline__ float tf32_rna(float v)
 template <typename T>
 __global__ void __launch_bounds__(kDecodeCols)
 bsr_decode_kernel(const int32_t *__restrict__ P, const int32_t *__restrict__ I, const T *__restrict__ D,
-                  int N, int t, int K, T *__restrict__ W, T *__restrict__ W_lo)
+                  int N, int t, int K, T *__restrict__ W, T *__restrict__ W_lo, int *__restrict__ flags,
+                  int n_flags)
 {
     __shared__ int32_t zmap[kDecodeCols];
     const int g = blockIdx.y, tid = threadIdx.x;
+    // the GEMM's stream-K flags start each launch lowered
+    if (flags && (blockIdx.x | blockIdx.y | blockIdx.z) == 0)
+        for (int i = tid; i < n_flags; i += kDecodeCols) flags[i] = 0;
     const int k0 = blockIdx.x * kDecodeCols;
     zmap[tid] = -1;
     __syncthreads();
@@ -179,12 +193,78 @@ __device__ __forceinline__ bool epi_all(bool ok)
     return r != 0;
 }
 
+// Work schedule of one launch, the same in every role of every CTA.  Tiles
+// [0, dp_tiles) are whole tiles taken round-robin (CTA b: b, b+G, ...).  The
+// chunk iterations of the remaining sk_tiles tiles are cut into sk_ctas
+// contiguous ranges, one for each of CTAs 0 .. sk_ctas-1 (stream-K), and a
+// CTA walks its range from the end: first the start of one tile, then whole
+// tiles, last the end of another.  A tile cut between CTAs is finished by
+// the highest of them, which reaches it last: the others (lower CTAs, which
+// reached it first) each write their part to their own partial slot and
+// raise their flag; the finisher waits for those flags, copies the parts
+// into its idle shared-memory ring and adds them to its own accumulator in
+// CTA order, so the result does not depend on timing.  Waiting only on
+// lower CTAs, which were scheduled first, cannot deadlock.
+struct TcSched {
+    int n_tiles, n_tn, n_chunks;
+    int dp_tiles, sk_tiles, sk_ctas;
+    float *partials;     // slot b: CTA b's part of a split tile, [BN/4][128] float4
+    int *flags;          // [kPlanCTAs]: slot b written
+};
+
+struct TcSeg {
+    int tile, c0, c1;    // chunk iterations [c0, c1) of tile
+};
+
+__device__ __forceinline__ int64_t sk_start(int b, int64_t W, int G) { return static_cast<int64_t>(b) * W / G; }
+// the CTA whose stream-K range holds iteration q (largest b with sk_start(b) <= q)
+__device__ __forceinline__ int sk_owner(int64_t q, int64_t W, int G)
+{
+    return static_cast<int>(((q + 1) * G + W - 1) / W) - 1;
+}
+
+struct TcSegIter {
+    int b, G, n_dp, i_dp, C, dp_tiles;
+    int64_t s, e;        // stream-K range still to walk: [s, e), from e down
+    __device__ TcSegIter(const TcSched &sc)
+    {
+        b = blockIdx.x;
+        G = gridDim.x;
+        C = sc.n_chunks;
+        dp_tiles = sc.dp_tiles;
+        n_dp = dp_tiles > b ? (dp_tiles - 1 - b) / G + 1 : 0;
+        i_dp = 0;
+        const int64_t W = static_cast<int64_t>(sc.sk_tiles) * C;
+        s = b < sc.sk_ctas ? sk_start(b, W, sc.sk_ctas) : 0;
+        e = b < sc.sk_ctas ? sk_start(b + 1, W, sc.sk_ctas) : 0;
+    }
+    __device__ bool next(TcSeg &sg)
+    {
+        if (i_dp < n_dp) {
+            sg.tile = b + i_dp * G;
+            sg.c0 = 0;
+            sg.c1 = C;
+            ++i_dp;
+            return true;
+        }
+        if (e <= s) return false;
+        const int t = static_cast<int>((e - 1) / C);
+        const int64_t t0 = static_cast<int64_t>(t) * C;
+        sg.tile = dp_tiles + t;
+        sg.c1 = static_cast<int>(e - t0);
+        sg.c0 = s > t0 ? static_cast<int>(s - t0) : 0;
+        e -= sg.c1 - sg.c0;
+        return true;
+    }
+    // chunk iterations of this CTA
+    __device__ int64_t total() const { return static_cast<int64_t>(n_dp) * C + (e - s); }
+};
+
 template <typename Tr, int BN>
 __global__ void __launch_bounds__(Tr::kWarps * 32, 1)
 tc_conv_kernel(const ConvArgs a, const __grid_constant__ CUtensorMap tmap_x,
                const __grid_constant__ CUtensorMap tmap_w, const __grid_constant__ CUtensorMap tmap_wlo,
-               const __grid_constant__ CUtensorMap tmap_y, const int n_tiles, const int n_tn,
-               const int a_tiled)
+               const __grid_constant__ CUtensorMap tmap_y, const TcSched sched, const int a_tiled)
 {
     using L = TcLayout<Tr, BN>;
     extern __shared__ unsigned char smem_raw[];
@@ -197,8 +277,9 @@ tc_conv_kernel(const ConvArgs a, const __grid_constant__ CUtensorMap tmap_x,
     const uint32_t bar_tfull = bar_empty + 8 * L::kS;
     const uint32_t bar_tempty = bar_tfull + 16;
     const uint32_t bar_drain = bar_tempty + 16;
+    const uint32_t bar_fix = bar_drain + 8;
     uint32_t *holder = reinterpret_cast<uint32_t *>(smem + L::kHolder);
-    // the MMA waits on "split" (fp32: x_lo written) or "full" (bf16)
+    // the MMA waits on "split" (fp32: x_hi / x_lo in TMEM) or "full" (bf16)
     const uint32_t bar_ready = Tr::kSplit ? bar_split : bar_full;
 
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
@@ -213,6 +294,7 @@ tc_conv_kernel(const ConvArgs a, const __grid_constant__ CUtensorMap tmap_x,
             mbar_init(bar_tempty + 8 * b, 128);
         }
         mbar_init(bar_drain, 1);
+        mbar_init(bar_fix, 1);
         fence_mbar_init();
     }
     if (warp == kMmaWarp) {
@@ -225,8 +307,7 @@ tc_conv_kernel(const ConvArgs a, const __grid_constant__ CUtensorMap tmap_x,
     const uint32_t tmem = *holder;
 
     const int n_cchunk = (a.C + Tr::kBK - 1) / Tr::kBK;
-    const int n_chunks = a.KH * a.KW * n_cchunk;
-    const int my_tiles = blockIdx.x < n_tiles ? (n_tiles - 1 - blockIdx.x) / gridDim.x + 1 : 0;
+    const int n_tn = sched.n_tn;
     auto abort_now = [&]() { atomicOr(a.status, kStatusTimeout); };
 
     if (warp == kProdWarp) {
@@ -235,16 +316,20 @@ tc_conv_kernel(const ConvArgs a, const __grid_constant__ CUtensorMap tmap_x,
             const int hw = a.Ho * a.Wo;
             int item = 0;
             bool failed = false;
-            for (int ti = 0; ti < my_tiles && !failed; ++ti) {
-                const int u = blockIdx.x + ti * gridDim.x;
-                const int tm = u / n_tn, tn = u - tm * n_tn;
+            TcSegIter it(sched);
+            TcSeg sg;
+            while (!failed && it.next(sg)) {
+                const int tm = sg.tile / n_tn, tn = sg.tile - tm * n_tn;
                 // first output pixel of the tile -> its traversal start (w, h, n)
                 const int p0 = tm * kBM;
                 const int b0 = p0 / hw, r0 = p0 - b0 * hw;
                 const int oh0 = r0 / a.Wo, ow0 = r0 - oh0 * a.Wo;
                 const int w0 = ow0 * a.sw - a.pw, h0 = oh0 * a.sh - a.ph;
-                int kh = 0, kw = 0, cc0 = 0, k0tap = 0;
-                for (int c = 0; c < n_chunks; ++c, ++item) {
+                // chunk c0 -> tap (kh, kw) and channel offset
+                const int tap = sg.c0 / n_cchunk;
+                int cc0 = (sg.c0 - tap * n_cchunk) * Tr::kBK, k0tap = tap * a.C;
+                int kh = tap / a.KW, kw = tap - (tap / a.KW) * a.KW;
+                for (int c = sg.c0; c < sg.c1; ++c, ++item) {
                     const int st = item % L::kS;
                     if (item >= L::kS &&
                         !mbar_wait(bar_empty + 8 * st, ((item / L::kS) + 1) & 1)) {
@@ -274,16 +359,18 @@ tc_conv_kernel(const ConvArgs a, const __grid_constant__ CUtensorMap tmap_x,
     } else if (warp == kMmaWarp) {
         // ============================== MMA ==============================
         if (lane == 0) {
-            int item = 0;
+            int item = 0, si = 0;
             bool failed = false;
-            for (int ti = 0; ti < my_tiles && !failed; ++ti) {
-                const int acc = ti % L::kAcc, use = ti / L::kAcc;
+            TcSegIter it(sched);
+            TcSeg sg;
+            for (; !failed && it.next(sg); ++si) {
+                const int acc = si % L::kAcc, use = si / L::kAcc;
                 if (use >= 1 && !mbar_wait(bar_tempty + 8 * acc, (use - 1) & 1)) {
                     abort_now(); failed = true; break;
                 }
                 tc::fence_after_sync();
                 const uint32_t d_tmem = tmem + acc * BN;
-                for (int c = 0; c < n_chunks; ++c, ++item) {
+                for (int c = sg.c0; c < sg.c1; ++c, ++item) {
                     const int st = item % L::kS;
                     if (!mbar_wait(bar_ready + 8 * st, (item / L::kS) & 1)) {
                         abort_now(); failed = true; break;
@@ -291,6 +378,7 @@ tc_conv_kernel(const ConvArgs a, const __grid_constant__ CUtensorMap tmap_x,
                     tc::fence_after_sync();
                     const uint32_t sa = base + st * L::kStage;
                     const uint64_t bd = tc::desc_kmajor_sw128(sa + L::kA);
+                    const uint32_t first = (c == sg.c0) ? 1u : 0u;   // the first chunk overwrites D
                     if constexpr (Tr::kSplit) {
                         constexpr uint32_t idesc = tc::idesc_tf32_f32(kBM, BN);
                         const uint64_t bld = tc::desc_kmajor_sw128(sa + L::kA + L::kB);
@@ -298,7 +386,7 @@ tc_conv_kernel(const ConvArgs a, const __grid_constant__ CUtensorMap tmap_x,
                         const uint32_t a_hi = tmem + L::kAcc * BN + (item & 1) * 64;
 #pragma unroll
                         for (int kk = 0; kk < Tr::kBK / Tr::kKStep; ++kk) {
-                            tc::mma_tf32_ta(d_tmem, a_hi + 8 * kk, bd + 2 * kk, idesc, (c | kk) != 0);
+                            tc::mma_tf32_ta(d_tmem, a_hi + 8 * kk, bd + 2 * kk, idesc, !(first && kk == 0));
                             tc::mma_tf32_ta(d_tmem, a_hi + 32 + 8 * kk, bd + 2 * kk, idesc, 1);
                             tc::mma_tf32_ta(d_tmem, a_hi + 8 * kk, bld + 2 * kk, idesc, 1);
                         }
@@ -307,7 +395,7 @@ tc_conv_kernel(const ConvArgs a, const __grid_constant__ CUtensorMap tmap_x,
                         const uint64_t ad = tc::desc_kmajor_sw128(sa);
 #pragma unroll
                         for (int kk = 0; kk < Tr::kBK / Tr::kKStep; ++kk)
-                            tc::mma_bf16(d_tmem, ad + 2 * kk, bd + 2 * kk, idesc, (c | kk) != 0);
+                            tc::mma_bf16(d_tmem, ad + 2 * kk, bd + 2 * kk, idesc, !(first && kk == 0));
                     }
                     tc::commit(bar_empty + 8 * st);
                 }
@@ -332,14 +420,14 @@ tc_conv_kernel(const ConvArgs a, const __grid_constant__ CUtensorMap tmap_x,
             const int q = warp & 3;
             const int row = 32 * q + lane;
             const uint32_t lane_base = tmem + (static_cast<uint32_t>(32 * q) << 16) + L::kAcc * BN;
-            const int n_items = my_tiles * n_chunks;
-            for (int item = 0; item < n_items; ++item) {
-                const int st = item % L::kS;
-                if (item >= 2 &&
-                    !mbar_wait(bar_empty + 8 * ((item - 2) % L::kS), ((item - 2) / L::kS) & 1)) {
+            const int64_t n_items = TcSegIter(sched).total();
+            for (int64_t item = 0; item < n_items; ++item) {
+                const int st = static_cast<int>(item % L::kS);
+                if (item >= 2 && !mbar_wait(bar_empty + 8 * static_cast<int>((item - 2) % L::kS),
+                                            static_cast<int>((item - 2) / L::kS) & 1)) {
                     abort_now(); break;
                 }
-                if (!mbar_wait(bar_full + 8 * st, (item / L::kS) & 1)) { abort_now(); break; }
+                if (!mbar_wait(bar_full + 8 * st, static_cast<int>(item / L::kS) & 1)) { abort_now(); break; }
                 tc::fence_after_sync();
                 const uint32_t src = base + st * L::kStage + row * kRowBytes;
                 uint32_t hi[32], lo[32];
@@ -356,7 +444,7 @@ tc_conv_kernel(const ConvArgs a, const __grid_constant__ CUtensorMap tmap_x,
                         lo[4 * j + e] = __float_as_uint(__uint_as_float(v[e]) - __uint_as_float(hi[4 * j + e]));
                     }
                 }
-                const uint32_t slot = lane_base + (item & 1) * 64;
+                const uint32_t slot = lane_base + static_cast<uint32_t>(item & 1) * 64;
                 tc::st_32x32b_x32(slot, hi);
                 tc::st_32x32b_x32(slot + 32, lo);
                 tc::st_wait();
@@ -366,85 +454,188 @@ tc_conv_kernel(const ConvArgs a, const __grid_constant__ CUtensorMap tmap_x,
         }
     } else {
         // ============================ epilogue ============================
+        // Per tile, column atom by column atom (128 bytes of output columns:
+        // 64 bf16 / 32 fp32): read the atom's accumulator columns from TMEM
+        // (warp w owns TMEM lanes = pixel rows 32*(w%4)..+31), add the bias,
+        // apply ReLU, convert, write the row into the warp's 128-byte-swizzled
+        // staging buffer (two, alternating) and store the warp's 32 x atom box
+        // with TMA.
+        using T = typename Tr::T;
+        constexpr int kAtomCols = kRowBytes / static_cast<int>(sizeof(T));
+        constexpr int kAtoms = BN / kAtomCols;
+        constexpr int kLd = kAtomCols / 32;               // tcgen05.ld x32 per atom
+        constexpr int kSlotF4 = BN / 4 * kBM;            // float4 per partial slot
         const int q = warp & 3;                      // TMEM lanes 32q .. 32q+31
         const int row = 32 * q + lane;               // pixel row of the tile
         const bool leader = (warp == kEpiWarp0) && lane == 0;
-        float *sbias = reinterpret_cast<float *>(smem + L::kBias);
         const uint32_t sout = base + L::kOut;
-        for (int ti = 0; ti < my_tiles; ++ti) {
-            const int acc = ti % L::kAcc;
+        float *sbias = reinterpret_cast<float *>(smem + L::kBias);
+        const int64_t W_sk = static_cast<int64_t>(sched.sk_tiles) * sched.n_chunks;
+        int n_emit = 0;                              // atoms stored so far (staging buffer parity)
+        TcSegIter it(sched);
+        TcSeg sg;
+        for (int si = 0; it.next(sg); ++si) {
+            const int acc = si % L::kAcc;
             // all four warps take the same decision (tcgen05.ld and the named
             // barriers below need all of them)
-            if (!epi_all(mbar_wait(bar_tfull + 8 * acc, (ti / L::kAcc) & 1))) { abort_now(); break; }
+            if (!epi_all(mbar_wait(bar_tfull + 8 * acc, (si / L::kAcc) & 1))) { abort_now(); break; }
             tc::fence_after_sync();
-            const int u = blockIdx.x + ti * gridDim.x;
-            const int tm = u / n_tn, tn = u - tm * n_tn;
-            const int p = tm * kBM + row;
-            // bf16: the staging tile is free once the previous tile's stores have read it
-            if (!Tr::kSplit && leader) tc::bulk_wait_read0();
-            for (int c = row; c < BN; c += 128) {
-                const int o = tn * BN + c;
-                sbias[c] = (a.bias && o < a.C_out) ? __ldg(a.bias + o) : 0.f;
-            }
-            tc::named_bar(1, 128);
-            // read the accumulator in batches of up to 128 columns (registers)
-            constexpr int kGrp = BN < 128 ? BN : 128;
+            const int tm = sg.tile / n_tn, tn = sg.tile - tm * n_tn;
+            const uint32_t t_acc = tmem + (static_cast<uint32_t>(32 * q) << 16) + acc * BN;
+            // read the accumulator columns of atom `at`; release the TMEM after the last
+            auto load_atom = [&](int at, uint32_t (&r)[kLd][32]) {
 #pragma unroll
-            for (int g0 = 0; g0 < BN; g0 += kGrp) {
-                uint32_t r[kGrp / 32][32];
-#pragma unroll
-                for (int cb = 0; cb < kGrp / 32; ++cb)
-                    tc::ld_32x32b_x32(tmem + (static_cast<uint32_t>(32 * q) << 16) + acc * BN + g0 + 32 * cb,
-                                      r[cb]);
+                for (int l = 0; l < kLd; ++l) tc::ld_32x32b_x32(t_acc + at * kAtomCols + 32 * l, r[l]);
                 tc::ld_wait();
-                if (g0 + kGrp >= BN) {
+                if (at == kAtoms - 1) {
                     tc::fence_before_sync();
-                    mbar_arrive(bar_tempty + 8 * acc);   // accumulator free for tile ti + 2
+                    mbar_arrive(bar_tempty + 8 * acc);   // accumulator free for segment si + kAcc
                 }
+            };
+            // bias / ReLU / convert the row's atom values f and store the
+            // warp's 32 rows of the atom: each warp has its own two staging
+            // buffers (32 rows x 128 bytes) and TMA stores, so no warp waits
+            // for another
+            // the tile's bias in shared memory, read as broadcast float4
+            const float4 *sb4 = reinterpret_cast<const float4 *>(sbias);
+            auto stage_bias = [&]() {
+                tc::named_bar(1, 128);               // the previous tile's reads are done
+                for (int c = row; c < BN; c += 128) {
+                    const int o = tn * BN + c;
+                    sbias[c] = (a.bias && o < a.C_out) ? __ldg(a.bias + o) : 0.f;
+                }
+                tc::named_bar(1, 128);
+            };
+            auto emit_atom = [&](int at, float (&f)[kAtomCols]) {
+                const int buf = n_emit++ & 1;        // alternate across atoms and tiles
+                if (lane == 0) tc::bulk_wait_read1();   // this warp's store two atoms back has read buf
+                __syncwarp();
+                const uint32_t wbuf = sout + (q * 2 + buf) * (32 * kRowBytes);
+                const int col0 = tn * BN + at * kAtomCols;
 #pragma unroll
-                for (int cb = 0; cb < kGrp / 32; ++cb) {
+                for (int j = 0; j < 8; ++j) {        // 16-byte chunk j of the row
+                    uint32_t w[4];
+                    if constexpr (sizeof(T) == 4) {
+                        const float4 bv = sb4[at * (kAtomCols / 4) + j];
+                        const float bb[4] = {bv.x, bv.y, bv.z, bv.w};
 #pragma unroll
-                    for (int v8 = 0; v8 < 4; ++v8) {
-                        const int c = g0 + 32 * cb + 8 * v8;  // first of 8 columns
-                        float f[8];
-#pragma unroll
-                        for (int e = 0; e < 8; ++e) {
-                            float val = __uint_as_float(r[cb][8 * v8 + e]) + sbias[c + e];
-                            if (a.relu) val = fmaxf(val, 0.f);
-                            f[e] = val;
+                        for (int e = 0; e < 4; ++e) {
+                            const float v = f[4 * j + e] + bb[e];
+                            w[e] = __float_as_uint(a.relu ? fmaxf(v, 0.f) : v);
                         }
-                        if constexpr (Tr::kSplit) {
-                            const int col = tn * BN + c;
-                            if (p < a.P_pix && col < a.C_out) {
-                                float4 *dst = reinterpret_cast<float4 *>(static_cast<float *>(a.y) +
-                                                                         static_cast<int64_t>(p) * a.C_out + col);
-                                dst[0] = make_float4(f[0], f[1], f[2], f[3]);
-                                dst[1] = make_float4(f[4], f[5], f[6], f[7]);
-                            }
-                        } else {
-                            const int atom = c >> 6, jj = (c & 63) >> 3;
-                            const uint32_t dst = sout + atom * (kBM * 128) + row * 128 + ((jj ^ (row & 7)) << 4);
-                            asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};\n" ::"r"(dst),
-                                         "r"(pack_bf16x2(f[0], f[1])), "r"(pack_bf16x2(f[2], f[3])),
-                                         "r"(pack_bf16x2(f[4], f[5])), "r"(pack_bf16x2(f[6], f[7]))
-                                         : "memory");
+                    } else {
+                        const float4 b0 = sb4[at * (kAtomCols / 4) + 2 * j], b1 = sb4[at * (kAtomCols / 4) + 2 * j + 1];
+                        const float bb[8] = {b0.x, b0.y, b0.z, b0.w, b1.x, b1.y, b1.z, b1.w};
+#pragma unroll
+                        for (int e = 0; e < 4; ++e) {
+                            float v0 = f[8 * j + 2 * e] + bb[2 * e];
+                            float v1 = f[8 * j + 2 * e + 1] + bb[2 * e + 1];
+                            if (a.relu) { v0 = fmaxf(v0, 0.f); v1 = fmaxf(v1, 0.f); }
+                            w[e] = pack_bf16x2(v0, v1);
                         }
+                    }
+                    asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};\n" ::"r"(
+                                     wbuf + lane * kRowBytes + ((j ^ (lane & 7)) << 4)),
+                                 "r"(w[0]), "r"(w[1]), "r"(w[2]), "r"(w[3])
+                                 : "memory");
+                }
+                tc::fence_proxy_async_smem();
+                __syncwarp();
+                // one commit group per atom, empty for an atom past C_out, so
+                // that "at most one group pending" always means buf is free
+                if (lane == 0) {
+                    if (col0 < a.C_out) tc::tma_store_2d(&tmap_y, col0, tm * kBM + 32 * q, wbuf);
+                    tc::bulk_commit();
+                }
+            };
+
+            if (sg.c0 == 0 && sg.c1 == sched.n_chunks) {
+                // ---- whole tile: accumulator -> bias / ReLU -> y ----
+                stage_bias();
+#pragma unroll 1
+                for (int at = 0; at < kAtoms; ++at) {
+                    uint32_t r[kLd][32];
+                    load_atom(at, r);
+                    float f[kAtomCols];
+#pragma unroll
+                    for (int e = 0; e < kAtomCols; ++e) f[e] = __uint_as_float(r[e / 32][e % 32]);
+                    emit_atom(at, f);
+                }
+                continue;
+            }
+
+            // ---- part of a split tile ----
+            const int t_sk = sg.tile - sched.dp_tiles;
+            const int64_t q0 = static_cast<int64_t>(t_sk) * sched.n_chunks;
+            const int b_first = sk_owner(q0, W_sk, sched.sk_ctas);
+            const int b_last = sk_owner(q0 + sched.n_chunks - 1, W_sk, sched.sk_ctas);
+            if (static_cast<int>(blockIdx.x) != b_last) {
+                // a lower CTA: accumulator -> own partial slot, then the flag
+                float4 *mine = reinterpret_cast<float4 *>(sched.partials) + static_cast<int64_t>(blockIdx.x) * kSlotF4;
+#pragma unroll 1
+                for (int at = 0; at < kAtoms; ++at) {
+                    uint32_t r[kLd][32];
+                    load_atom(at, r);
+#pragma unroll
+                    for (int v4 = 0; v4 < kAtomCols / 4; ++v4) {
+                        const int e = 4 * v4;
+                        __stcg(mine + (at * kAtomCols / 4 + v4) * kBM + row,
+                               make_float4(__uint_as_float(r[e / 32][e % 32]), __uint_as_float(r[e / 32][e % 32 + 1]),
+                                           __uint_as_float(r[e / 32][e % 32 + 2]),
+                                           __uint_as_float(r[e / 32][e % 32 + 3])));
+                    }
+                }
+                __threadfence();
+                tc::fence_proxy_async_global();      // the finisher reads the slot with TMA
+                tc::named_bar(1, 128);
+                if (leader) tc::st_release_gpu(sched.flags + blockIdx.x, 1);
+                continue;
+            }
+            // The finisher (this split tile is this CTA's last segment, so the
+            // ring is idle): wait for the lower CTAs' flags, bring their parts
+            // into the ring, add them to the accumulator in CTA order.
+            const int n_contrib = b_last - b_first;
+            bool ok = true;
+            if (leader) {
+                for (int k = b_first; k < b_last && ok; ++k) {
+                    const long long t0 = clock64();
+                    while (tc::ld_acquire_gpu(sched.flags + k) == 0)
+                        if (clock64() - t0 > (1ll << 31)) { ok = false; break; }
+                }
+                if (ok) {
+                    tc::fence_proxy_async_global();
+                    tc::mbar_arrive_expect_tx(bar_fix, static_cast<uint32_t>(n_contrib) * L::kSlotBytes);
+                    for (int k = 0; k < n_contrib; ++k) {
+                        const unsigned char *src = reinterpret_cast<const unsigned char *>(
+                            sched.partials + static_cast<int64_t>(b_first + k) * kSlotF4 * 4);
+                        for (int off = 0; off < L::kSlotBytes; off += 16384)
+                            tc::bulk_load(base + k * L::kSlotBytes + off, src + off, 16384, bar_fix);
+                        sched.flags[b_first + k] = 0;   // ready for the next launch
                     }
                 }
             }
-            if constexpr (!Tr::kSplit) {
-                tc::fence_proxy_async_smem();
-                tc::named_bar(1, 128);
-                if (leader) {
+            if (!epi_all(ok)) { abort_now(); break; }
+            if (!epi_all(mbar_wait(bar_fix, 0))) { abort_now(); break; }
+            stage_bias();
+#pragma unroll 1
+            for (int at = 0; at < kAtoms; ++at) {
+                uint32_t r[kLd][32];
+                load_atom(at, r);
+                float f[kAtomCols];
 #pragma unroll
-                    for (int at = 0; at < BN / 64; ++at)
-                        if (tn * BN + 64 * at < a.C_out)
-                            tc::tma_store_2d(&tmap_y, tn * BN + 64 * at, tm * kBM, sout + at * (kBM * 128));
-                    tc::bulk_commit();
+                for (int e = 0; e < kAtomCols; ++e) f[e] = __uint_as_float(r[e / 32][e % 32]);
+                for (int k = 0; k < n_contrib; ++k) {
+                    const float4 *part = reinterpret_cast<const float4 *>(smem + k * L::kSlotBytes);
+#pragma unroll
+                    for (int v4 = 0; v4 < kAtomCols / 4; ++v4) {
+                        const float4 v = part[(at * kAtomCols / 4 + v4) * kBM + row];
+                        f[4 * v4] += v.x; f[4 * v4 + 1] += v.y; f[4 * v4 + 2] += v.z; f[4 * v4 + 3] += v.w;
+                    }
                 }
+                emit_atom(at, f);
             }
         }
-        if (!Tr::kSplit && leader) tc::bulk_wait0();
+        if (lane == 0) tc::bulk_wait0();
     }
 
     tc::fence_before_sync();
@@ -512,7 +703,8 @@ bool tmap_2d(CUtensorMap *m, CUtensorMapDataType type, int elem, const void *ptr
 }
 
 template <typename Tr, int BN>
-cudaError_t launch_bn(const ConvArgs &a, const typename Tr::T *W, const typename Tr::T *W_lo, cudaStream_t st)
+cudaError_t launch_bn(const ConvArgs &a, const typename Tr::T *W, const typename Tr::T *W_lo, void *sk_space,
+                      cudaStream_t st)
 {
     using L = TcLayout<Tr, BN>;
     constexpr int elem = sizeof(typename Tr::T);
@@ -542,18 +734,17 @@ cudaError_t launch_bn(const ConvArgs &a, const typename Tr::T *W, const typename
                   CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
             return cudaErrorInvalidValue;
     }
-    // B: W[C_out][K] (and W_lo), box 128 bytes of K x BN rows.  y (bf16 only):
-    // [P_pix][C_out], stored in boxes of 64 columns x 128 rows (rows/columns
-    // outside y are not written).
+    // B: W[C_out][K] (and W_lo), box 128 bytes of K x BN rows.  y:
+    // [P_pix][C_out], stored in boxes of 128 bytes of columns x 32 rows, one
+    // per epilogue warp (rows / columns outside y are not written).
     CUtensorMap tmap_w, tmap_wlo, tmap_y;
     if (!tmap_2d(&tmap_w, Tr::kTmap, elem, W, a.C_out, K, BN)) return cudaErrorInvalidValue;
     if (Tr::kSplit) {
         if (!tmap_2d(&tmap_wlo, Tr::kTmap, elem, W_lo, a.C_out, K, BN)) return cudaErrorInvalidValue;
-        tmap_y = tmap_w;                                       // unused
     } else {
         tmap_wlo = tmap_w;                                     // unused
-        if (!tmap_2d(&tmap_y, Tr::kTmap, elem, a.y, a.P_pix, a.C_out, kBM)) return cudaErrorInvalidValue;
     }
+    if (!tmap_2d(&tmap_y, Tr::kTmap, elem, a.y, a.P_pix, a.C_out, 32)) return cudaErrorInvalidValue;
     // the shared-memory opt-in, once per device for this kernel
     static std::mutex attr_mu;
     static bool attr_done[64];
@@ -572,49 +763,95 @@ cudaError_t launch_bn(const ConvArgs &a, const typename Tr::T *W, const typename
     int sms = 0;
     e = device_sm_count(&sms);
     if (e != cudaSuccess) return e;
-    const int n_tm = (a.P_pix + kBM - 1) / kBM;
-    const int n_tn = (a.C_out + BN - 1) / BN;
-    const int n_tiles = n_tm * n_tn;
-    const int grid = n_tiles < sms ? n_tiles : sms;
-    kern<<<grid, Tr::kWarps * 32, L::kAlloc, st>>>(a, tmap_x, tmap_w, tmap_wlo, tmap_y, n_tiles, n_tn, a_tiled);
+    TcSched sc{};
+    sc.n_tn = (a.C_out + BN - 1) / BN;
+    sc.n_tiles = ((a.P_pix + kBM - 1) / kBM) * sc.n_tn;
+    sc.n_chunks = a.KH * a.KW * ((a.C + Tr::kBK - 1) / Tr::kBK);
+    int grid = sc.n_tiles < sms ? sc.n_tiles : sms;
+    sc.dp_tiles = sc.n_tiles;
+    // Stream-K when there are fewer tiles than SMs, with room for the
+    // partial slots.  Each CTA gets at least kMinSplitIters chunk iterations
+    // and at least C / R of them, R = the partial tiles the finisher's ring
+    // holds, so that a split tile has at most R parts besides the
+    // finisher's.  (The schedule also supports balancing the last, partial
+    // round after whole rounds, but on GB300 that measured slower than
+    // leaving the round ragged: the fixup and the shorter segments cost more
+    // than the idle SMs.)
+    const int G = sms < kPlanCTAs ? sms : kPlanCTAs;
+    if (sk_space && sc.n_tiles < G) {
+        const int dp = (sc.n_tiles / G) * G, skt = sc.n_tiles - dp;
+        const int64_t iters = static_cast<int64_t>(skt) * sc.n_chunks;
+        int need = (sc.n_chunks + L::kRingSlots - 1) / L::kRingSlots;
+        if (need < kMinSplitIters) need = kMinSplitIters;
+        const int gs = static_cast<int>(iters / need < G ? iters / need : G);
+        if (gs > skt) {
+            grid = dp ? G : gs;
+            sc.dp_tiles = dp;
+            sc.sk_tiles = skt;
+            sc.sk_ctas = gs;
+            sc.partials = static_cast<float *>(sk_space);
+            sc.flags = reinterpret_cast<int *>(static_cast<unsigned char *>(sk_space) + sk_partial_bytes(BN));
+        }
+    }
+    kern<<<grid, Tr::kWarps * 32, L::kAlloc, st>>>(a, tmap_x, tmap_w, tmap_wlo, tmap_y, sc, a_tiled);
     return cudaGetLastError();
 }
 
+int tc_bn(const ConvArgs &a) { return a.C_out <= 64 ? 64 : a.C_out <= 128 ? 128 : 256; }
+
+size_t round256(size_t v) { return (v + 255) & ~static_cast<size_t>(255); }
+
+// decoded weights: bf16 C_out * K values; fp32 C_out * K values twice (hi, lo)
+size_t weights_bytes(const ConvArgs &a, int dtype)
+{
+    const size_t n = static_cast<size_t>(a.C_out) * a.KH * a.KW * a.C;
+    return round256(dtype == ONEXN_F32 ? n * 8 : n * 2);
+}
+
+// stream-K space after the weights: the partial slots, then the flags
+size_t sk_bytes(const ConvArgs &a) { return sk_partial_bytes(tc_bn(a)) + round256(kPlanCTAs * sizeof(int)); }
+
 template <typename Tr>
-cudaError_t decode_typed(const ConvArgs &a, void *workspace, cudaStream_t st)
+cudaError_t decode_typed(const ConvArgs &a, void *workspace, size_t ws_bytes, cudaStream_t st)
 {
     using T = typename Tr::T;
     const int K = a.KH * a.KW * a.C;
     const size_t n = static_cast<size_t>(a.C_out) * K;
     T *W = static_cast<T *>(workspace);
     T *W_lo = Tr::kSplit ? W + n : nullptr;
+    const size_t wb = weights_bytes(a, Tr::kSplit ? ONEXN_F32 : ONEXN_BF16);
+    int *flags = nullptr;
+    if (ws_bytes >= wb + sk_bytes(a))
+        flags = reinterpret_cast<int *>(static_cast<unsigned char *>(workspace) + wb + sk_partial_bytes(tc_bn(a)));
     const dim3 grid(static_cast<unsigned>((K + kDecodeCols - 1) / kDecodeCols), a.C_out / a.N,
                     (a.N + kDecodeRows - 1) / kDecodeRows);
-    bsr_decode_kernel<T><<<grid, kDecodeCols, 0, st>>>(a.P, a.I, static_cast<const T *>(a.D), a.N, a.t, K, W, W_lo);
+    bsr_decode_kernel<T><<<grid, kDecodeCols, 0, st>>>(a.P, a.I, static_cast<const T *>(a.D), a.N, a.t, K, W, W_lo,
+                                                        flags, kPlanCTAs);
     return cudaGetLastError();
 }
 
 template <typename Tr>
-cudaError_t gemm_typed(const ConvArgs &a, const void *workspace, cudaStream_t st)
+cudaError_t gemm_typed(const ConvArgs &a, const void *workspace, size_t ws_bytes, cudaStream_t st)
 {
     using T = typename Tr::T;
     const size_t n = static_cast<size_t>(a.C_out) * a.KH * a.KW * a.C;
     const T *W = static_cast<const T *>(workspace);
     const T *W_lo = Tr::kSplit ? W + n : nullptr;
-    if (a.C_out <= 64) return launch_bn<Tr, 64>(a, W, W_lo, st);
-    if (a.C_out <= 128) return launch_bn<Tr, 128>(a, W, W_lo, st);
-    return launch_bn<Tr, 256>(a, W, W_lo, st);
+    const size_t wb = weights_bytes(a, Tr::kSplit ? ONEXN_F32 : ONEXN_BF16);
+    void *sk = ws_bytes >= wb + sk_bytes(a)
+                   ? static_cast<void *>(static_cast<unsigned char *>(const_cast<void *>(workspace)) + wb)
+                   : nullptr;
+    if (a.C_out <= 64) return launch_bn<Tr, 64>(a, W, W_lo, sk, st);
+    if (a.C_out <= 128) return launch_bn<Tr, 128>(a, W, W_lo, sk, st);
+    return launch_bn<Tr, 256>(a, W, W_lo, sk, st);
 }
 
 }  // namespace
 
-// bf16: C_out * K bf16 values; fp32: C_out * K fp32 values twice (hi, lo).
-size_t tc_workspace_bytes(const ConvArgs &a, int dtype)
-{
-    const size_t n = static_cast<size_t>(a.C_out) * a.KH * a.KW * a.C;
-    const size_t bytes = dtype == ONEXN_F32 ? n * 8 : n * 2;
-    return (bytes + 255) & ~static_cast<size_t>(255);
-}
+// The decoded weights; with room for the stream-K partial slots and
+// flags after them the GEMM also balances its last round of tiles.
+size_t tc_workspace_min(const ConvArgs &a, int dtype) { return weights_bytes(a, dtype); }
+size_t tc_workspace_bytes(const ConvArgs &a, int dtype) { return weights_bytes(a, dtype) + sk_bytes(a); }
 
 // C_in, C_out giving 16-byte rows; the im2col box corners within the TMA's
 // [-128, 127] range; strides <= 8; 16-bit tap offsets.
@@ -632,22 +869,24 @@ bool tc_supports(const ConvArgs &a, int dtype)
     return true;
 }
 
-cudaError_t tc_decode(const ConvArgs &a, int dtype, void *workspace, cudaStream_t st)
+cudaError_t tc_decode(const ConvArgs &a, int dtype, void *workspace, size_t ws_bytes, cudaStream_t st)
 {
-    return dtype == ONEXN_F32 ? decode_typed<TcF32>(a, workspace, st) : decode_typed<TcBf16>(a, workspace, st);
+    return dtype == ONEXN_F32 ? decode_typed<TcF32>(a, workspace, ws_bytes, st)
+                              : decode_typed<TcBf16>(a, workspace, ws_bytes, st);
 }
 
-cudaError_t tc_gemm(const ConvArgs &a, int dtype, const void *workspace, cudaStream_t st)
+cudaError_t tc_gemm(const ConvArgs &a, int dtype, const void *workspace, size_t ws_bytes, cudaStream_t st)
 {
     if (a.P_pix == 0) return cudaSuccess;
-    return dtype == ONEXN_F32 ? gemm_typed<TcF32>(a, workspace, st) : gemm_typed<TcBf16>(a, workspace, st);
+    return dtype == ONEXN_F32 ? gemm_typed<TcF32>(a, workspace, ws_bytes, st)
+                              : gemm_typed<TcBf16>(a, workspace, ws_bytes, st);
 }
 
-cudaError_t launch_tc(const ConvArgs &a, int dtype, void *workspace, cudaStream_t st)
+cudaError_t launch_tc(const ConvArgs &a, int dtype, void *workspace, size_t ws_bytes, cudaStream_t st)
 {
     if (a.P_pix == 0) return cudaSuccess;
-    const cudaError_t e = tc_decode(a, dtype, workspace, st);
-    return e != cudaSuccess ? e : tc_gemm(a, dtype, workspace, st);
+    const cudaError_t e = tc_decode(a, dtype, workspace, ws_bytes, st);
+    return e != cudaSuccess ? e : tc_gemm(a, dtype, workspace, ws_bytes, st);
 }
 
 }  // namespace onexn

@@ -172,28 +172,52 @@ HOST_CASES = [
 ]
 
 
+def _device_out_min_workspace(conv, x, flags):
+    """onexn_conv_fwd with only the minimum workspace (the decoded weights
+    for the tensor-core family: its GEMM then takes whole tiles only)."""
+    B, H, W, _ = x.shape
+    K = conv.KH * conv.KW * conv.C_in
+    wmin = conv.C_out * K * (8 if conv.cdtype == ox.ONEXN_F32 else 2)
+    wmin = -(-wmin // 256) * 256
+    ws = torch.empty(wmin, dtype=torch.uint8, device="cuda")
+    y = torch.empty(conv.out_shape(x.shape), dtype=x.dtype, device="cuda")
+    ox.onexn_conv_fwd(conv.desc(B, H, W), conv.P, conv.I, conv.D, conv.N, conv.t, x, y, conv.bias,
+                      conv.cdtype, flags, ws)
+    return y
+
+
 @pytest.mark.parametrize("case", HOST_CASES, ids=[c[0].name for c in HOST_CASES])
-def test_host_entry_matches_device_entry_bitwise(case):
+def test_host_entry_matches_device_entry(case):
     """onexn_conv_fwd_host (chunks of images copied in and out on internal
-    streams) gives exactly the device entry's output: every output pixel is
-    computed by the same kernel in the same order, only grouped differently."""
+    streams) gives bit for bit the device entry's output when that runs whole
+    tiles too (minimum workspace): every output pixel is computed by the same
+    kernel in the same order, only grouped differently.  Against the device
+    entry with its full workspace (split tiles summed from partial parts) the
+    outputs agree to fp32 rounding."""
     layer, algo = case
     from paper_2105_14713_gb300.layer import PrunedConv2d
     conv = PrunedConv2d(wl.weights(layer).numpy(), layer.N, layer.rate, bias=wl.bias(layer).numpy(),
                         stride=layer.stride, padding=layer.pad, dilation=layer.dil, dtype=layer.dtype)
     x = wl.activations(layer)
     x = x if layer.dtype == "f32" else x.to(torch.bfloat16)
-    y_dev = conv(x.cuda(), relu=True, algo=ALGOS[algo])
+    flags = ox.ONEXN_RELU | ALGOS[algo]
+    y_min = _device_out_min_workspace(conv, x.cuda(), flags).cpu()
+    y_full = conv(x.cuda(), relu=True, algo=ALGOS[algo]).cpu()
+    iv = torch.int16 if layer.dtype == "bf16" else torch.int32
     for pinned in (True, False):
         xh = x.pin_memory() if pinned else x.clone()
         y_host = conv.forward_host(xh, relu=True, algo=ALGOS[algo])
-        assert torch.equal(y_host.view(torch.int16 if layer.dtype == "bf16" else torch.int32),
-                           y_dev.cpu().view(torch.int16 if layer.dtype == "bf16" else torch.int32)), pinned
+        assert torch.equal(y_host.view(iv), y_min.view(iv)), pinned
+    # the fp32 parity tolerance on the output scale; bf16: a rounding flip
+    scale = y_min.float().abs().max().item() + 1e-30
+    tol_rel = 2.0 ** -7 if layer.dtype == "bf16" else 1e-5
+    assert (y_full.float() - y_min.float()).abs().max().item() <= tol_rel * scale
 
 
 def test_host_entry_overlapping_calls_on_two_streams():
     """Two layers enqueued back to back on different streams (the second's
-    copies overlap the first's compute) both give the device entry's output."""
+    copies overlap the first's compute) both give the device entry's output
+    (whole-tile form, as the host entry runs)."""
     from paper_2105_14713_gb300.layer import PrunedConv2d
     layers = [L("ov_a", 24, 28, 28, 64, 128, 3, 3, 1, 1, 1, N=8, rate=0.5, dtype="f32", seed=31),
               L("ov_b", 24, 28, 28, 64, 64, 3, 3, 1, 1, 1, N=4, rate=0.3, dtype="bf16", seed=32)]
@@ -204,7 +228,7 @@ def test_host_entry_overlapping_calls_on_two_streams():
         x = (x if layer.dtype == "f32" else x.to(torch.bfloat16)).pin_memory()
         convs.append(conv)
         xs.append(x)
-        refs.append(conv(x.cuda()).cpu())
+        refs.append(_device_out_min_workspace(conv, x.cuda(), 0).cpu())
     streams = [torch.cuda.Stream() for _ in layers]
     for _ in range(3):
         outs = [c.forward_host(x, stream=s, sync=False) for c, x, s in zip(convs, xs, streams)]

@@ -172,9 +172,10 @@ def test_auto_cost_model():
 
 
 def test_host_entry_workspace_and_argument_checks_need_no_gpu():
-    # 3x3 128->128 on 64x28x28 fp32: decoded hi/lo weights + 3 input and 3
-    # output slots of one chunk (64 images of 401408 bytes in ~8 MiB chunks:
-    # 3 chunks of 22 images)
+    # 3x3 128->128 on 64x28x28 fp32: decoded hi/lo weights (no stream-K
+    # space: chunk GEMMs may run concurrently) + 3 input and 3 output slots
+    # of one chunk (64 images of 401408 bytes in ~8 MiB chunks: 3 chunks of
+    # 22 images)
     d = ox.make_desc(64, 28, 28, 128, 128, 3, 3, 1, 1, 1)
     n = ox.onexn_conv_host_workspace_size(d, 8, 9216, ox.ONEXN_F32)
     img = 28 * 28 * 128 * 4
@@ -196,19 +197,23 @@ def test_conv_shape_and_argument_errors_need_no_gpu():
     d = ox.make_desc(2, 7, 7, 8, 16, 3, 3, 2, 1, 1)
     assert ox.onexn_conv_out_shape(d) == (4, 4)
     assert ox.onexn_conv_algo(d, 8, 100, ox.ONEXN_F32) == ox.ONEXN_ALGO_FMA
-    # bf16: the tcgen05 family when its workspace fits, else FFMA
-    need = ox.onexn_conv_workspace_size(d, 8, 100, ox.ONEXN_BF16)
-    assert need == 16 * 9 * 8 * 2 + (-(16 * 9 * 8 * 2) % 256)
-    assert ox.onexn_conv_algo(d, 8, 100, ox.ONEXN_BF16, 0, need) == ox.ONEXN_ALGO_TC
-    assert ox.onexn_conv_algo(d, 8, 100, ox.ONEXN_BF16, 0, need - 1) == ox.ONEXN_ALGO_FMA
-    # fp32: hi and lo tf32 parts of the decoded weights, 8 bytes per weight
-    need32 = ox.onexn_conv_workspace_size(d, 8, 100, ox.ONEXN_F32)
-    assert need32 == 16 * 9 * 8 * 8 + (-(16 * 9 * 8 * 8) % 256)
+    # tcgen05 family: the decoded weights (bf16: 2 bytes per weight; fp32:
+    # hi and lo tf32 parts, 8 bytes), plus the stream-K space (one
+    # 128 x BN fp32 partial slot per CTA for 152 CTAs, and 152 flags) that
+    # the reported size includes; the weights alone are the minimum.
+    sk = 152 * 128 * 64 * 4 + 768
+    w16, w32 = 16 * 9 * 8 * 2, 16 * 9 * 8 * 8
+    assert w16 % 256 == 0 and w32 % 256 == 0
+    assert ox.onexn_conv_workspace_size(d, 8, 100, ox.ONEXN_BF16) == w16 + sk
+    assert ox.onexn_conv_workspace_size(d, 8, 100, ox.ONEXN_F32) == w32 + sk
+    # bf16: the tcgen05 family when the weights fit, else FFMA
+    assert ox.onexn_conv_algo(d, 8, 100, ox.ONEXN_BF16, 0, w16) == ox.ONEXN_ALGO_TC
+    assert ox.onexn_conv_algo(d, 8, 100, ox.ONEXN_BF16, 0, w16 - 1) == ox.ONEXN_ALGO_FMA
     assert ox.onexn_conv_workspace_size(d, 8, 100, ox.ONEXN_F32, ox.ONEXN_ALGO_FMA) == 0
-    assert ox.onexn_conv_algo(d, 8, 100, ox.ONEXN_F32, 0, need32 - 1) == ox.ONEXN_ALGO_FMA
-    assert ox.onexn_conv_algo(d, 8, 100, ox.ONEXN_F32, ox.ONEXN_ALGO_TC, need32) == ox.ONEXN_ALGO_TC
+    assert ox.onexn_conv_algo(d, 8, 100, ox.ONEXN_F32, 0, w32 - 1) == ox.ONEXN_ALGO_FMA
+    assert ox.onexn_conv_algo(d, 8, 100, ox.ONEXN_F32, ox.ONEXN_ALGO_TC, w32) == ox.ONEXN_ALGO_TC
     assert _status(ox.onexn_conv_algo, d, 8, 100, ox.ONEXN_BF16, ox.ONEXN_ALGO_TC, 0) == ox.ONEXN_EINVAL
-    assert _status(ox.onexn_conv_algo, d, 8, 100, ox.ONEXN_F32, ox.ONEXN_ALGO_TC, need32 - 1) == \
+    assert _status(ox.onexn_conv_algo, d, 8, 100, ox.ONEXN_F32, ox.ONEXN_ALGO_TC, w32 - 1) == \
         ox.ONEXN_EINVAL
     # C_out not a multiple of 8: no tensor-core tiles; AUTO falls back to FFMA
     d12 = ox.make_desc(1, 4, 4, 8, 12)
