@@ -85,6 +85,7 @@ struct TcF32 {
 };
 
 constexpr int kSmemMax = 232448;      // dynamic shared memory per CTA (opt-in maximum)
+constexpr int kAccMax = 4;            // accumulator buffers in TMEM at most
 constexpr int kPlanCTAs = 152;        // stream-K: at most this many CTAs (GB300's SM count)
 constexpr int kMinSplitIters = 4;     // stream-K: at least this many chunk iterations per CTA
 
@@ -101,20 +102,24 @@ struct TcLayout {
     static constexpr int kTx = kStage;                               // bytes the TMA brings
     // output staging: per epilogue warp two buffers of 32 rows x one 128-byte column atom
     static constexpr int kOutBytes = 4 * 2 * 32 * kRowBytes;
-    static constexpr int kFixed = 1024 + kOutBytes + BN * 4 + (3 * 6 + 6) * 8 + 16;
+    static constexpr int kFixed = 1024 + kOutBytes + BN * 4 + (3 * 6 + 2 * 4 + 2) * 8 + 16;
     static constexpr int kS = ((kSmemMax - kFixed) / kStage) > 6 ? 6 : ((kSmemMax - kFixed) / kStage);
     static constexpr int kOut = kS * kStage;
     static constexpr int kBias = kOut + kOutBytes;                   // BN fp32
     static constexpr int kBar = kBias + BN * 4;
-    // full[S], split[S], empty[S], tmem_full[2], tmem_empty[2], drain, fixup, TMEM holder
-    static constexpr int kHolder = kBar + (3 * kS + 6) * 8;
+    // full[S], split[S], empty[S], tmem_full[4], tmem_empty[4], drain, fixup, TMEM holder
+    static constexpr int kHolder = kBar + (3 * kS + 2 * kAccMax + 2) * 8;
     static constexpr int kBytes = kHolder + 16;
     static constexpr int kAlloc = kBytes + 1024;                      // room to align the base to 1024
     // TMEM columns: the fp32 accumulator buffers (two when they fit next to
     // the A ring, else one) and, for the split form, a ring of two A slots
     // of 64 columns (x_hi in the first 32, x_lo in the next 32).
     static constexpr int kARing = Tr::kSplit ? 128 : 0;
-    static constexpr int kAcc = (2 * BN + kARing <= 512) ? 2 : 1;
+    // as many accumulator buffers as fit next to the A ring (up to 4): the
+    // MMA of tile i + kAcc waits for the epilogue of tile i, so layers with
+    // few chunks per tile need several to keep the tensor core busy
+    static constexpr int kAccFit = (512 - kARing) / BN;
+    static constexpr int kAcc = kAccFit > kAccMax ? kAccMax : kAccFit;
     static constexpr int kTmemCols = pow2_at_least(kAcc * BN + kARing);
     // partial tiles (128 x BN fp32) the idle ring holds at a split tile's finish
     static constexpr int kSlotBytes = kBM * BN * 4;
@@ -151,6 +156,9 @@ bsr_decode_kernel(const int32_t *__restrict__ P, const int32_t *__restrict__ I, 
 {
     __shared__ int32_t zmap[kDecodeCols];
     const int g = blockIdx.y, tid = threadIdx.x;
+    // let the GEMM launch and run its prologue meanwhile; it waits for this
+    // grid's completion before reading anything
+    asm volatile("griddepcontrol.launch_dependents;\n" ::: "memory");
     // the GEMM's stream-K flags start each launch lowered
     if (flags && (blockIdx.x | blockIdx.y | blockIdx.z) == 0)
         for (int i = tid; i < n_flags; i += kDecodeCols) flags[i] = 0;
@@ -275,8 +283,8 @@ tc_conv_kernel(const ConvArgs a, const __grid_constant__ CUtensorMap tmap_x,
     const uint32_t bar_split = bar_full + 8 * L::kS;
     const uint32_t bar_empty = bar_split + 8 * L::kS;
     const uint32_t bar_tfull = bar_empty + 8 * L::kS;
-    const uint32_t bar_tempty = bar_tfull + 16;
-    const uint32_t bar_drain = bar_tempty + 16;
+    const uint32_t bar_tempty = bar_tfull + 8 * kAccMax;
+    const uint32_t bar_drain = bar_tempty + 8 * kAccMax;
     const uint32_t bar_fix = bar_drain + 8;
     uint32_t *holder = reinterpret_cast<uint32_t *>(smem + L::kHolder);
     // the MMA waits on "split" (fp32: x_hi / x_lo in TMEM) or "full" (bf16)
@@ -289,7 +297,7 @@ tc_conv_kernel(const ConvArgs a, const __grid_constant__ CUtensorMap tmap_x,
             mbar_init(bar_split + 8 * s, 128);
             mbar_init(bar_empty + 8 * s, 1);
         }
-        for (int b = 0; b < 2; ++b) {
+        for (int b = 0; b < kAccMax; ++b) {
             mbar_init(bar_tfull + 8 * b, 1);
             mbar_init(bar_tempty + 8 * b, 128);
         }
@@ -305,6 +313,10 @@ tc_conv_kernel(const ConvArgs a, const __grid_constant__ CUtensorMap tmap_x,
     __syncthreads();
     tc::fence_after_sync();
     const uint32_t tmem = *holder;
+    // Launched as a programmatic dependent of the weight decode: everything
+    // above overlapped the decode; global memory is touched only after it
+    // (and everything before it on the stream) has completed.
+    asm volatile("griddepcontrol.wait;\n" ::: "memory");
 
     const int n_cchunk = (a.C + Tr::kBK - 1) / Tr::kBK;
     const int n_tn = sched.n_tn;
@@ -483,14 +495,37 @@ tc_conv_kernel(const ConvArgs a, const __grid_constant__ CUtensorMap tmap_x,
             const int tm = sg.tile / n_tn, tn = sg.tile - tm * n_tn;
             const uint32_t t_acc = tmem + (static_cast<uint32_t>(32 * q) << 16) + acc * BN;
             // read the accumulator columns of atom `at`; release the TMEM after the last
-            auto load_atom = [&](int at, uint32_t (&r)[kLd][32]) {
+            auto issue_atom = [&](int at, uint32_t (&r)[kLd][32]) {
 #pragma unroll
                 for (int l = 0; l < kLd; ++l) tc::ld_32x32b_x32(t_acc + at * kAtomCols + 32 * l, r[l]);
+            };
+            auto release_acc = [&]() {
+                tc::fence_before_sync();
+                mbar_arrive(bar_tempty + 8 * acc);       // accumulator free for segment si + kAcc
+            };
+            // the atoms in order, the TMEM loads of atom at+1 in flight while
+            // atom at is processed; the accumulator is released as soon as
+            // its last columns are in registers
+            auto run_atoms = [&](auto &&body) {
+                uint32_t r[2][kLd][32];
+                issue_atom(0, r[0]);
                 tc::ld_wait();
-                if (at == kAtoms - 1) {
-                    tc::fence_before_sync();
-                    mbar_arrive(bar_tempty + 8 * acc);   // accumulator free for segment si + kAcc
+                if (kAtoms == 1) release_acc();
+#pragma unroll
+                for (int at = 0; at < kAtoms; ++at) {
+                    if (at + 1 < kAtoms) issue_atom(at + 1, r[(at + 1) & 1]);
+                    body(at, r[at & 1]);
+                    if (at + 1 < kAtoms) {
+                        tc::ld_wait();
+                        if (at + 2 == kAtoms) release_acc();
+                    }
                 }
+            };
+            // a lower CTA's part: accumulator atoms -> global slot, no pipelining needed
+            auto load_atom = [&](int at, uint32_t (&r)[kLd][32]) {
+                issue_atom(at, r);
+                tc::ld_wait();
+                if (at == kAtoms - 1) release_acc();
             };
             // bias / ReLU / convert the row's atom values f and store the
             // warp's 32 rows of the atom: each warp has its own two staging
@@ -552,15 +587,12 @@ tc_conv_kernel(const ConvArgs a, const __grid_constant__ CUtensorMap tmap_x,
             if (sg.c0 == 0 && sg.c1 == sched.n_chunks) {
                 // ---- whole tile: accumulator -> bias / ReLU -> y ----
                 stage_bias();
-#pragma unroll 1
-                for (int at = 0; at < kAtoms; ++at) {
-                    uint32_t r[kLd][32];
-                    load_atom(at, r);
+                run_atoms([&](int at, uint32_t (&r)[kLd][32]) {
                     float f[kAtomCols];
 #pragma unroll
                     for (int e = 0; e < kAtomCols; ++e) f[e] = __uint_as_float(r[e / 32][e % 32]);
                     emit_atom(at, f);
-                }
+                });
                 continue;
             }
 
@@ -617,10 +649,7 @@ tc_conv_kernel(const ConvArgs a, const __grid_constant__ CUtensorMap tmap_x,
             if (!epi_all(ok)) { abort_now(); break; }
             if (!epi_all(mbar_wait(bar_fix, 0))) { abort_now(); break; }
             stage_bias();
-#pragma unroll 1
-            for (int at = 0; at < kAtoms; ++at) {
-                uint32_t r[kLd][32];
-                load_atom(at, r);
+            run_atoms([&](int at, uint32_t (&r)[kLd][32]) {
                 float f[kAtomCols];
 #pragma unroll
                 for (int e = 0; e < kAtomCols; ++e) f[e] = __uint_as_float(r[e / 32][e % 32]);
@@ -633,7 +662,7 @@ tc_conv_kernel(const ConvArgs a, const __grid_constant__ CUtensorMap tmap_x,
                     }
                 }
                 emit_atom(at, f);
-            }
+            });
         }
         if (lane == 0) tc::bulk_wait0();
     }
@@ -704,7 +733,7 @@ bool tmap_2d(CUtensorMap *m, CUtensorMapDataType type, int elem, const void *ptr
 
 template <typename Tr, int BN>
 cudaError_t launch_bn(const ConvArgs &a, const typename Tr::T *W, const typename Tr::T *W_lo, void *sk_space,
-                      cudaStream_t st)
+                      bool after_decode, cudaStream_t st)
 {
     using L = TcLayout<Tr, BN>;
     constexpr int elem = sizeof(typename Tr::T);
@@ -793,8 +822,17 @@ cudaError_t launch_bn(const ConvArgs &a, const typename Tr::T *W, const typename
             sc.flags = reinterpret_cast<int *>(static_cast<unsigned char *>(sk_space) + sk_partial_bytes(BN));
         }
     }
-    kern<<<grid, Tr::kWarps * 32, L::kAlloc, st>>>(a, tmap_x, tmap_w, tmap_wlo, tmap_y, sc, a_tiled);
-    return cudaGetLastError();
+    cudaLaunchConfig_t cfg{};
+    cfg.gridDim = dim3(grid);
+    cfg.blockDim = dim3(Tr::kWarps * 32);
+    cfg.dynamicSmemBytes = L::kAlloc;
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = after_decode ? 1 : 0;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kern, a, tmap_x, tmap_w, tmap_wlo, tmap_y, sc, a_tiled);
 }
 
 int tc_bn(const ConvArgs &a) { return a.C_out <= 64 ? 64 : a.C_out <= 128 ? 128 : 256; }
@@ -831,7 +869,8 @@ cudaError_t decode_typed(const ConvArgs &a, void *workspace, size_t ws_bytes, cu
 }
 
 template <typename Tr>
-cudaError_t gemm_typed(const ConvArgs &a, const void *workspace, size_t ws_bytes, cudaStream_t st)
+cudaError_t gemm_typed(const ConvArgs &a, const void *workspace, size_t ws_bytes, bool after_decode,
+                       cudaStream_t st)
 {
     using T = typename Tr::T;
     const size_t n = static_cast<size_t>(a.C_out) * a.KH * a.KW * a.C;
@@ -841,9 +880,9 @@ cudaError_t gemm_typed(const ConvArgs &a, const void *workspace, size_t ws_bytes
     void *sk = ws_bytes >= wb + sk_bytes(a)
                    ? static_cast<void *>(static_cast<unsigned char *>(const_cast<void *>(workspace)) + wb)
                    : nullptr;
-    if (a.C_out <= 64) return launch_bn<Tr, 64>(a, W, W_lo, sk, st);
-    if (a.C_out <= 128) return launch_bn<Tr, 128>(a, W, W_lo, sk, st);
-    return launch_bn<Tr, 256>(a, W, W_lo, sk, st);
+    if (a.C_out <= 64) return launch_bn<Tr, 64>(a, W, W_lo, sk, after_decode, st);
+    if (a.C_out <= 128) return launch_bn<Tr, 128>(a, W, W_lo, sk, after_decode, st);
+    return launch_bn<Tr, 256>(a, W, W_lo, sk, after_decode, st);
 }
 
 }  // namespace
@@ -875,18 +914,28 @@ cudaError_t tc_decode(const ConvArgs &a, int dtype, void *workspace, size_t ws_b
                               : decode_typed<TcBf16>(a, workspace, ws_bytes, st);
 }
 
-cudaError_t tc_gemm(const ConvArgs &a, int dtype, const void *workspace, size_t ws_bytes, cudaStream_t st)
+namespace {
+cudaError_t gemm_any(const ConvArgs &a, int dtype, const void *workspace, size_t ws_bytes, bool after_decode,
+                     cudaStream_t st)
 {
     if (a.P_pix == 0) return cudaSuccess;
-    return dtype == ONEXN_F32 ? gemm_typed<TcF32>(a, workspace, ws_bytes, st)
-                              : gemm_typed<TcBf16>(a, workspace, ws_bytes, st);
+    return dtype == ONEXN_F32 ? gemm_typed<TcF32>(a, workspace, ws_bytes, after_decode, st)
+                              : gemm_typed<TcBf16>(a, workspace, ws_bytes, after_decode, st);
+}
+}  // namespace
+
+cudaError_t tc_gemm(const ConvArgs &a, int dtype, const void *workspace, size_t ws_bytes, cudaStream_t st)
+{
+    return gemm_any(a, dtype, workspace, ws_bytes, false, st);
 }
 
+// decode, then the GEMM as its programmatic dependent (its launch and
+// prologue overlap the decode)
 cudaError_t launch_tc(const ConvArgs &a, int dtype, void *workspace, size_t ws_bytes, cudaStream_t st)
 {
     if (a.P_pix == 0) return cudaSuccess;
     const cudaError_t e = tc_decode(a, dtype, workspace, ws_bytes, st);
-    return e != cudaSuccess ? e : tc_gemm(a, dtype, workspace, ws_bytes, st);
+    return e != cudaSuccess ? e : gemm_any(a, dtype, workspace, ws_bytes, true, st);
 }
 
 }  // namespace onexn
