@@ -36,6 +36,30 @@ cudaError_t device_status_ptr(unsigned int **p);
 
 __device__ __forceinline__ int clampi(int v, int lo, int hi) { return min(max(v, lo), hi); }
 
+// Division of 32-bit unsigned integers by an invariant divisor d >= 1 with
+// one multiply-high, after Granlund and Montgomery, "Division by invariant
+// integers using multiplication" (PLDI 1994), Fig. 4.1:
+//   l = ceil(log2 d), m = floor(2^32 (2^l - d) / d) + 1,
+//   t = mulhi(m, n), q = (t + ((n - t) >> min(l, 1))) >> max(l - 1, 0).
+// The constants are computed on the host; exact for every 32-bit n.
+struct FastDiv {
+    uint32_t d = 1, m = 1, s1 = 0, s2 = 0;
+    FastDiv() = default;
+    __host__ explicit FastDiv(uint32_t dd) : d(dd)
+    {
+        uint32_t l = 0;
+        while (l < 32 && (uint64_t(1) << l) < dd) ++l;
+        m = static_cast<uint32_t>(((uint64_t(1) << 32) * ((uint64_t(1) << l) - dd)) / dd + 1);
+        s1 = l < 1 ? l : 1;
+        s2 = l > 1 ? l - 1 : 0;
+    }
+    __device__ __forceinline__ uint32_t div(uint32_t n) const
+    {
+        const uint32_t t = __umulhi(m, n);
+        return (t + ((n - t) >> s1)) >> s2;
+    }
+};
+
 __device__ __forceinline__ uint32_t smem_u32(const void *p)
 {
     return static_cast<uint32_t>(__cvta_generic_to_shared(p));

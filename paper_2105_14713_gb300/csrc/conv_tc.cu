@@ -54,6 +54,7 @@
 #include <cuda.h>
 #include <cudaTypedefs.h>
 
+#include <cstring>
 #include <mutex>
 
 namespace onexn {
@@ -216,6 +217,8 @@ __device__ __forceinline__ bool epi_all(bool ok)
 struct TcSched {
     int n_tiles, n_tn, n_chunks;
     int dp_tiles, sk_tiles, sk_ctas;
+    // divisors of the per-tile / per-segment index arithmetic
+    FastDiv div_tn, div_hw, div_wo, div_cchunk, div_kw;
     float *partials;     // slot b: CTA b's part of a split tile, [BN/4][128] float4
     int *flags;          // [kPlanCTAs]: slot b written
 };
@@ -331,16 +334,16 @@ tc_conv_kernel(const ConvArgs a, const __grid_constant__ CUtensorMap tmap_x,
             TcSegIter it(sched);
             TcSeg sg;
             while (!failed && it.next(sg)) {
-                const int tm = sg.tile / n_tn, tn = sg.tile - tm * n_tn;
+                const int tm = static_cast<int>(sched.div_tn.div(sg.tile)), tn = sg.tile - tm * n_tn;
                 // first output pixel of the tile -> its traversal start (w, h, n)
                 const int p0 = tm * kBM;
-                const int b0 = p0 / hw, r0 = p0 - b0 * hw;
-                const int oh0 = r0 / a.Wo, ow0 = r0 - oh0 * a.Wo;
+                const int b0 = static_cast<int>(sched.div_hw.div(p0)), r0 = p0 - b0 * hw;
+                const int oh0 = static_cast<int>(sched.div_wo.div(r0)), ow0 = r0 - oh0 * a.Wo;
                 const int w0 = ow0 * a.sw - a.pw, h0 = oh0 * a.sh - a.ph;
                 // chunk c0 -> tap (kh, kw) and channel offset
-                const int tap = sg.c0 / n_cchunk;
+                const int tap = static_cast<int>(sched.div_cchunk.div(sg.c0));
                 int cc0 = (sg.c0 - tap * n_cchunk) * Tr::kBK, k0tap = tap * a.C;
-                int kh = tap / a.KW, kw = tap - (tap / a.KW) * a.KW;
+                int kh = static_cast<int>(sched.div_kw.div(tap)), kw = tap - kh * a.KW;
                 for (int c = sg.c0; c < sg.c1; ++c, ++item) {
                     const int st = item % L::kS;
                     if (item >= L::kS &&
@@ -492,7 +495,7 @@ tc_conv_kernel(const ConvArgs a, const __grid_constant__ CUtensorMap tmap_x,
             // barriers below need all of them)
             if (!epi_all(mbar_wait(bar_tfull + 8 * acc, (si / L::kAcc) & 1))) { abort_now(); break; }
             tc::fence_after_sync();
-            const int tm = sg.tile / n_tn, tn = sg.tile - tm * n_tn;
+            const int tm = static_cast<int>(sched.div_tn.div(sg.tile)), tn = sg.tile - tm * n_tn;
             const uint32_t t_acc = tmem + (static_cast<uint32_t>(32 * q) << 16) + acc * BN;
             // read the accumulator columns of atom `at`; release the TMEM after the last
             auto issue_atom = [&](int at, uint32_t (&r)[kLd][32]) {
@@ -715,6 +718,50 @@ void im2col_corners(const ConvArgs &a, int lower[2], int upper[2])
     upper[1] = a.ph - a.dh * (a.KH - 1);
 }
 
+// Encoded tensor maps are cached by their encoding inputs (a layer called
+// again on the same buffers skips the driver call): a 64-entry direct-mapped
+// table keyed by the device and every argument of the encode.
+struct TmapKey {
+    uint32_t kind, type;
+    int32_t dev, pad0;
+    uint64_t ptr;
+    uint64_t dims[4], strides[3];
+    int32_t lower[2], upper[2];
+    uint32_t box[2], estr[4];
+};
+
+struct TmapEntry {
+    bool valid;
+    TmapKey key;
+    CUtensorMap map;
+};
+
+std::mutex g_tmap_mu;
+TmapEntry g_tmap_cache[64];
+
+template <typename Encode>
+bool tmap_cached(TmapKey &k, CUtensorMap *out, Encode &&encode)
+{
+    if (cudaGetDevice(&k.dev) != cudaSuccess) return false;
+    uint64_t h = 1469598103934665603ull;                      // FNV-1a over the key bytes
+    const unsigned char *kb = reinterpret_cast<const unsigned char *>(&k);
+    for (size_t i = 0; i < sizeof(TmapKey); ++i) h = (h ^ kb[i]) * 1099511628211ull;
+    TmapEntry &e = g_tmap_cache[h & 63];
+    {
+        std::lock_guard<std::mutex> lk(g_tmap_mu);
+        if (e.valid && std::memcmp(&e.key, &k, sizeof(TmapKey)) == 0) {
+            *out = e.map;
+            return true;
+        }
+    }
+    if (!encode(out)) return false;
+    std::lock_guard<std::mutex> lk(g_tmap_mu);
+    e.valid = true;
+    e.key = k;
+    e.map = *out;
+    return true;
+}
+
 // 2-D tensor map over a row-major [rows][cols] matrix of `elem`-byte values,
 // box 128 bytes x box_rows, 128-byte swizzle, zero fill outside.
 bool tmap_2d(CUtensorMap *m, CUtensorMapDataType type, int elem, const void *ptr, uint64_t rows,
@@ -726,9 +773,19 @@ bool tmap_2d(CUtensorMap *m, CUtensorMapDataType type, int elem, const void *ptr
     const cuuint64_t strides[1] = {cols * elem};
     const cuuint32_t box[2] = {static_cast<cuuint32_t>(kRowBytes / elem), box_rows};
     const cuuint32_t estr[2] = {1, 1};
-    return enc_t(m, type, 2, const_cast<void *>(ptr), dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
-                 CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
-                 CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+    TmapKey k;
+    std::memset(&k, 0, sizeof k);
+    k.kind = 0;
+    k.type = static_cast<uint32_t>(type);
+    k.ptr = reinterpret_cast<uint64_t>(ptr);
+    k.dims[0] = cols; k.dims[1] = rows;
+    k.strides[0] = strides[0];
+    k.box[0] = box[0]; k.box[1] = box[1];
+    return tmap_cached(k, m, [&](CUtensorMap *mm) {
+        return enc_t(mm, type, 2, const_cast<void *>(ptr), dims, strides, box, estr,
+                     CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                     CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+    });
 }
 
 template <typename Tr, int BN>
@@ -758,9 +815,21 @@ cudaError_t launch_bn(const ConvArgs &a, const typename Tr::T *W, const typename
         int lower[2], upper[2];
         im2col_corners(a, lower, upper);
         const cuuint32_t estr[4] = {1, static_cast<cuuint32_t>(a.sw), static_cast<cuuint32_t>(a.sh), 1};
-        if (enc_i(&tmap_x, Tr::kTmap, 4, const_cast<void *>(a.x), dims, strides, lower, upper, Tr::kBK, kBM,
-                  estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
-                  CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+        TmapKey k;
+        std::memset(&k, 0, sizeof k);
+        k.kind = 1;
+        k.type = static_cast<uint32_t>(Tr::kTmap);
+        k.ptr = reinterpret_cast<uint64_t>(a.x);
+        for (int i = 0; i < 4; ++i) k.dims[i] = dims[i];
+        for (int i = 0; i < 3; ++i) k.strides[i] = strides[i];
+        for (int i = 0; i < 2; ++i) { k.lower[i] = lower[i]; k.upper[i] = upper[i]; }
+        k.box[0] = Tr::kBK; k.box[1] = kBM;
+        for (int i = 0; i < 4; ++i) k.estr[i] = estr[i];
+        if (!tmap_cached(k, &tmap_x, [&](CUtensorMap *mm) {
+                return enc_i(mm, Tr::kTmap, 4, const_cast<void *>(a.x), dims, strides, lower, upper, Tr::kBK, kBM,
+                             estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+            }))
             return cudaErrorInvalidValue;
     }
     // B: W[C_out][K] (and W_lo), box 128 bytes of K x BN rows.  y:
@@ -795,7 +864,13 @@ cudaError_t launch_bn(const ConvArgs &a, const typename Tr::T *W, const typename
     TcSched sc{};
     sc.n_tn = (a.C_out + BN - 1) / BN;
     sc.n_tiles = ((a.P_pix + kBM - 1) / kBM) * sc.n_tn;
-    sc.n_chunks = a.KH * a.KW * ((a.C + Tr::kBK - 1) / Tr::kBK);
+    const int n_cchunk = (a.C + Tr::kBK - 1) / Tr::kBK;
+    sc.n_chunks = a.KH * a.KW * n_cchunk;
+    sc.div_tn = FastDiv(static_cast<uint32_t>(sc.n_tn));
+    sc.div_hw = FastDiv(static_cast<uint32_t>(a.Ho * a.Wo));
+    sc.div_wo = FastDiv(static_cast<uint32_t>(a.Wo));
+    sc.div_cchunk = FastDiv(static_cast<uint32_t>(n_cchunk));
+    sc.div_kw = FastDiv(static_cast<uint32_t>(a.KW));
     int grid = sc.n_tiles < sms ? sc.n_tiles : sms;
     sc.dp_tiles = sc.n_tiles;
     // Stream-K when there are fewer tiles than SMs, with room for the

@@ -9,6 +9,8 @@ of layers before pruning, as in the paper's workflow (Sec. 3.3).
 """
 from __future__ import annotations
 
+import ctypes
+
 import numpy as np
 import torch
 
@@ -50,6 +52,8 @@ class PrunedConv2d:
         self.bias = None if bias is None else torch.as_tensor(
             np.asarray(bias, np.float32)).to(dev).contiguous()
         self._ws = {}            # per input shape: device workspace (bytes as uint8)
+        self._args = {}          # per buffers / layout / flags / stream: marshalled C arguments
+        self._descs = []
 
     @property
     def torch_dtype(self):
@@ -82,18 +86,45 @@ class PrunedConv2d:
 
     def forward(self, x: torch.Tensor, y: torch.Tensor = None, relu: bool = False,
                 algo: int = _c.ONEXN_ALGO_AUTO, stream=None) -> torch.Tensor:
-        """x: NHWC CUDA tensor of this layer's dtype.  Returns y (NHWC)."""
+        """x: NHWC CUDA tensor of this layer's dtype.  Returns y (NHWC).
+
+        The checked and marshalled C arguments are cached per (x, y, stream,
+        flags) buffers and layout, so a layer called again on the same
+        buffers costs one C call."""
+        if y is None:
+            y = torch.empty(self.out_shape(x.shape), dtype=x.dtype, device=x.device)
+        s = torch.cuda.current_stream(x.device) if stream is None else stream
+        flags = (_c.ONEXN_RELU if relu else 0) | algo
+        key = (x.data_ptr(), y.data_ptr(), x.shape, x.stride(), x.dtype, y.shape, y.stride(), y.dtype,
+               flags, s.cuda_stream)
+        args = self._args.get(key)
+        if args is None:
+            if len(self._args) >= 64:
+                self._args.clear()
+                self._descs.clear()
+            args = self._marshal(x, y, flags, s)
+            self._args[key] = args
+        st = _c.lib.onexn_conv_fwd(*args)
+        if st != _c.ONEXN_OK:
+            raise _c.OnexnError(st, _c.lib.onexn_last_error().decode(errors="replace"))
+        return y
+
+    def _marshal(self, x, y, flags, s):
         if x.dtype != self.torch_dtype or not x.is_cuda or not x.is_contiguous():
             raise ValueError(f"x must be a contiguous CUDA {self.torch_dtype} NHWC tensor")
         B, H, W, C = x.shape
         if C != self.C_in:
             raise ValueError(f"x has {C} channels, layer expects {self.C_in}")
-        if y is None:
-            y = torch.empty(self.out_shape(x.shape), dtype=x.dtype, device=x.device)
-        flags = (_c.ONEXN_RELU if relu else 0) | algo
-        _c.onexn_conv_fwd(self.desc(B, H, W), self.P, self.I, self.D, self.N, self.t, x, y,
-                          self.bias, self.cdtype, flags, self.workspace(x.shape, algo), stream)
-        return y
+        if tuple(y.shape) != tuple(self.out_shape(x.shape)) or y.dtype != x.dtype or not y.is_contiguous() \
+                or y.device != x.device:
+            raise ValueError(f"y must be a contiguous {x.dtype} tensor of shape {self.out_shape(x.shape)}")
+        desc = self.desc(B, H, W)
+        ws = self.workspace(x.shape, flags & _c.ONEXN_ALGO_MASK)
+        ptr = (lambda t: None if t is None else ctypes.c_void_p(t.data_ptr()))
+        ws_bytes = 0 if ws is None else ws.numel()
+        self._descs.append(desc)                 # kept alive for the cached byref
+        return (ctypes.byref(desc), ptr(self.P), ptr(self.I), ptr(self.D), self.N, self.t, ptr(x), ptr(y),
+                ptr(self.bias), self.cdtype, flags, ptr(ws), ws_bytes, ctypes.c_void_p(s.cuda_stream))
 
     __call__ = forward
 

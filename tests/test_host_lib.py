@@ -30,6 +30,39 @@ def test_library_exports_every_declared_symbol():
     assert set(names) == set(ox.SIGNATURES), "binding and header disagree"
 
 
+def test_binding_constants_match_the_header():
+    # every #define ONEXN_* and enum ONEXN_* value of include/onexn.h, evaluated
+    # in C by the preprocessor's arithmetic (shifts and ors of integer literals)
+    src = open(os.path.join(ROOT, "include", "onexn.h")).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    vals = {}
+    for name, expr in re.findall(r"#define[ \t]+(ONEXN_\w+)[ \t]+(.+)", src):
+        expr = re.sub(r"\b(0x[0-9A-Fa-f]+|\d+)u\b", r"\1", expr.strip())
+        vals[name] = eval(expr, {}, dict(vals))   # only literals and earlier ONEXN_ names
+    for body in re.findall(r"typedef enum\s*\{(.*?)\}", src, flags=re.S):
+        nxt = 0
+        for item in body.split(","):
+            item = item.strip()
+            if not item:
+                continue
+            if "=" in item:
+                n, v = (t.strip() for t in item.split("="))
+                nxt = int(v, 0)
+            else:
+                n = item
+            vals[n] = nxt
+            nxt += 1
+    checked = 0
+    for name, v in vals.items():
+        if hasattr(ox, name):
+            assert getattr(ox, name) == v, name
+            checked += 1
+    for name in ("ONEXN_RELU", "ONEXN_ALGO_MASK", "ONEXN_ALGO_TC", "ONEXN_F32", "ONEXN_BF16", "ONEXN_ETIMEOUT",
+                 "ONEXN_GRAN_KERNEL"):
+        assert name in vals and hasattr(ox, name), name
+    assert checked >= 15
+
+
 SHAPES = [((8, 6, 3, 3), 4), ((8, 6, 3, 3), 2), ((64, 64, 1, 1), 4), ((128, 128, 3, 3), 8),
           ((32, 24, 1, 3), 16), ((12, 5, 2, 2), 3), ((16, 16, 3, 3), 16), ((24, 40, 1, 1), 1)]
 
