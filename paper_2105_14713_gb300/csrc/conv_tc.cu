@@ -910,7 +910,27 @@ cudaError_t launch_bn(const ConvArgs &a, const typename Tr::T *W, const typename
     return cudaLaunchKernelEx(&cfg, kern, a, tmap_x, tmap_w, tmap_wlo, tmap_y, sc, a_tiled);
 }
 
-int tc_bn(const ConvArgs &a) { return a.C_out <= 64 ? 64 : a.C_out <= 128 ? 128 : 256; }
+// Column-tile width: the BN in {64, 128, 256} with the least estimated time,
+// rounds of kPlanCTAs tiles x a per-tile cost linear in BN (the MMA's N)
+// plus a BN-independent share (A loads, epilogue start), 64 columns' worth.
+// Narrow tiles win when there are few pixel tiles (more CTAs busy); wide
+// tiles re-read the A operand fewer times.  Ties go to the wider tile.
+int tc_bn(const ConvArgs &a)
+{
+    const int64_t n_m = (static_cast<int64_t>(a.P_pix) + kBM - 1) / kBM;
+    int best = 256;
+    int64_t best_cost = -1;
+    for (int bn : {256, 128, 64}) {
+        if (bn > 64 && a.C_out <= bn / 2) continue;      // half the tile or more would be empty
+        const int64_t tiles = n_m * ((a.C_out + bn - 1) / bn);
+        const int64_t cost = ((tiles + kPlanCTAs - 1) / kPlanCTAs) * (bn + 64);
+        if (best_cost < 0 || cost < best_cost) {
+            best = bn;
+            best_cost = cost;
+        }
+    }
+    return best;
+}
 
 size_t round256(size_t v) { return (v + 255) & ~static_cast<size_t>(255); }
 
@@ -955,8 +975,9 @@ cudaError_t gemm_typed(const ConvArgs &a, const void *workspace, size_t ws_bytes
     void *sk = ws_bytes >= wb + sk_bytes(a)
                    ? static_cast<void *>(static_cast<unsigned char *>(const_cast<void *>(workspace)) + wb)
                    : nullptr;
-    if (a.C_out <= 64) return launch_bn<Tr, 64>(a, W, W_lo, sk, after_decode, st);
-    if (a.C_out <= 128) return launch_bn<Tr, 128>(a, W, W_lo, sk, after_decode, st);
+    const int bn = tc_bn(a);
+    if (bn == 64) return launch_bn<Tr, 64>(a, W, W_lo, sk, after_decode, st);
+    if (bn == 128) return launch_bn<Tr, 128>(a, W, W_lo, sk, after_decode, st);
     return launch_bn<Tr, 256>(a, W, W_lo, sk, after_decode, st);
 }
 
