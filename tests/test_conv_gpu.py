@@ -243,3 +243,18 @@ def test_host_entry_empty_batch():
     conv = PrunedConv2d(wl.weights(layer).numpy(), 4, 0.5, padding=1)
     y = conv.forward_host(torch.zeros(0, 8, 8, 16).pin_memory())
     assert tuple(y.shape) == (0, 8, 8, 16)
+
+
+# ------------------------------------------- fully connected layers as 1x1
+
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+@pytest.mark.parametrize("B", [1, 7, 256])
+def test_fully_connected_layer_as_1x1_conv(dtype, B):
+    """A fully connected layer (here MobileNet-V2's 1280 -> 1000 classifier)
+    is a 1x1 convolution on a 1x1 image: x [B, 1, 1, 1280] -> y [B, 1, 1,
+    1000].  Few pixel tiles, so the tensor-core GEMM splits the K loop of
+    each output tile across CTAs (stream-K)."""
+    layer = L("fc", B, 1, 1, 1280, 1000, 1, 1, 1, 0, 1, N=4, rate=0.5, dtype=dtype, seed=B)
+    for algo in _algos_for(dtype, 4, 1280, 1000):
+        y, yr, a, conv = run_layer(layer, relu=False, algo=ALGOS[algo])
+        assert norm_err(y, yr, a) <= tol(layer), (algo, B)
