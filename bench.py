@@ -71,10 +71,19 @@ def kept_flops(layer, t):
     return 2.0 * layer.pixels * t * layer.N
 
 
+def _touched(n_in, n_out, k, s, p, d):
+    """Input rows (or columns) that some output position reads: the union of
+    o*s - p + i*d over o < n_out, i < k, inside [0, n_in)."""
+    return len({o * s - p + i * d for o in range(n_out) for i in range(k)} & set(range(n_in)))
+
+
 def alg_bytes(layer, t):
-    """X + Y + D + I + P, each once (halo re-reads and skipped work not counted)."""
+    """X + Y + D + I + P, each once (halo re-reads and skipped work not counted;
+    X only where some output reads it, e.g. a quarter of it for a stride-2 1x1)."""
     es = 4 if layer.dtype == "f32" else 2
-    x = layer.B * layer.H * layer.W * layer.C_in * es
+    rows = _touched(layer.H, layer.Ho, layer.KH, layer.stride, layer.pad, layer.dil)
+    cols = _touched(layer.W, layer.Wo, layer.KW, layer.stride, layer.pad, layer.dil)
+    x = layer.B * rows * cols * layer.C_in * es
     y = layer.pixels * layer.C_out * es
     return x + y + t * layer.N * es + t * 4 + (layer.C_out // layer.N + 1) * 4
 
