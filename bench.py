@@ -8,6 +8,7 @@ flushed with a 256 MB write before every step, outside the timed events):
   3  MobileNet-V2 expand/project 1x1 stack (34 layers), 128x224x224 input, fp32, N=4, 50%
   4  ResNet-50 bottleneck stack (52 convs), 256x224x224 input, bf16, N=16, 70%
   5  3x3 512 -> 512 on 128x14x14: sweep N in {1..32} x rate in {0..0.9} x {fp32, bf16}
+  6  fully connected 1280 -> 1000 as a 1x1 conv on 256 1x1 inputs, fp32 + bf16, N=4, 50%
 
 A "step" is one pass over every layer (leg) of the workload.  Prints one JSON
 line.  Metric: effective TFLOP/s = 2 * pixels * t * N / time summed over the
@@ -51,6 +52,8 @@ DESCRIPTIONS = {
        "bf16-in/fp32-acc; 1xN N=16, 70% block rate",
     5: "3x3 conv 128x14x14x512 -> 512, s1 p1; sweep N in {1,2,4,8,16,32} x rate in "
        "{0,.3,.5,.7,.9} x {fp32, bf16}, seed 0",
+    6: "fully connected 1280 -> 1000 (MobileNet-V2 classifier) as a 1x1 conv on 256x1x1 inputs; "
+       "1xN N=4, 50% block rate; fp32 leg + bf16-in/fp32-acc leg",
 }
 
 
@@ -64,6 +67,8 @@ def workload(cfg: int):
         return wl.config3()
     if cfg == 4:
         return wl.config4()
+    if cfg == 6:
+        return wl.config6()
     raise ValueError(cfg)
 
 
@@ -483,7 +488,7 @@ def measure(layers, args, dev, stream, flush, ws, pk, sampler=None):
 
 def main():
     ap = argparse.ArgumentParser()
-    ap.add_argument("--config", type=int, default=2, choices=[1, 2, 3, 4, 5])
+    ap.add_argument("--config", type=int, default=2, choices=[1, 2, 3, 4, 5, 6])
     ap.add_argument("--gpus", type=int, default=1)
     ap.add_argument("--steps", type=int, default=20)
     ap.add_argument("--warmup", type=int, default=5)

@@ -192,6 +192,14 @@ def config4() -> List[ConvLayer]:
     return resnet50_bottlenecks(B=256, N=16, rate=0.7, dtype="bf16")
 
 
+def config6(B: int = 256) -> List[ConvLayer]:
+    """MobileNet-V2's 1280 -> 1000 classifier as a 1x1 convolution on a 1x1
+    image (the fully connected layer of Sec. 3.1's Omega when h = w = 1),
+    N=4, 50%, an fp32 and a bf16 leg."""
+    return [ConvLayer(f"fc_1280_1000_b{B}_{dt}", B, 1, 1, 1280, 1000, 1, 1, 1, 0, 1, N=4, rate=0.5,
+                      dtype=dt, seed=0) for dt in ("f32", "bf16")]
+
+
 SWEEP_N = (1, 2, 4, 8, 16, 32)
 SWEEP_RATE = (0.0, 0.3, 0.5, 0.7, 0.9)
 
