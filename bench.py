@@ -164,9 +164,9 @@ class ClockSampler:
             self.fh = open(self.path, "w")
             self.proc = subprocess.Popen(
                 ["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.Q}",
-                 "--format=csv,noheader,nounits", "-lms", "100"], stdout=self.fh,
+                 "--format=csv,noheader,nounits", "-lms", "50"], stdout=self.fh,
                 stderr=subprocess.DEVNULL)
-            time.sleep(0.3)
+            time.sleep(0.2)
         except (OSError, FileNotFoundError):
             self.proc = None
         return self
@@ -490,7 +490,9 @@ def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--config", type=int, default=2, choices=[1, 2, 3, 4, 5, 6])
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=20)
+    # default: a timed region of ~1 s on the default workload, so that the
+    # clock samples (every 50 ms) fall inside it
+    ap.add_argument("--steps", type=int, default=5000)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
@@ -540,7 +542,7 @@ def main():
                             "sparse_ms": sparse_ms[i], "speedup": dts[i][0] / sparse_ms[i]}
                            for i in range(len(legs))]}
 
-    e2e_ms, h2d, d2h = e2e_time(legs, dev, max(3, args.steps // 4), 2, flush, stream)
+    e2e_ms, h2d, d2h = e2e_time(legs, dev, max(3, min(args.steps // 4, 200)), 2, flush, stream)
     e2e_ms = max_over_ranks(e2e_ms, ws)
 
     cpu = None
