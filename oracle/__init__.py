@@ -81,6 +81,7 @@ def _load():
                                            P, i64, P, P]
         lib.oracle_conv_bsr.argtypes = [P, P, P, P, i32, P, ctypes.POINTER(_Geom),
                                         i32, P, i64, P]
+        lib.oracle_dwconv.argtypes = [P, P, P, ctypes.POINTER(_Geom), P]
         lib.oracle_num_threads.restype = i32
         _lib = lib
         return lib
@@ -183,21 +184,49 @@ def out_hw(H, W, KH, KW, stride=(1, 1), pad=(0, 0), dil=(1, 1)):
     return Ho, Wo
 
 
+def _act_code(relu):
+    """False / True / "relu6" (or 0 / 1 / 2): none, ReLU, ReLU6."""
+    if relu == "relu6" or (not isinstance(relu, bool) and relu == 2):
+        return 2
+    return int(bool(relu))
+
+
 def _geom(x_shape, C_out, KH, KW, stride, pad, dil, relu):
     B, H, W, C_in = x_shape
     return _Geom(B, H, W, C_in, C_out, KH, KW, stride[0], stride[1], pad[0], pad[1],
-                 dil[0], dil[1], int(bool(relu)))
+                 dil[0], dil[1], _act_code(relu))
+
+
+def activation(y, relu):
+    """The activation applied after bias (and residual): none, ReLU, ReLU6."""
+    code = _act_code(relu)
+    if code >= 1:
+        y = np.maximum(y, 0.0)
+    if code == 2:
+        y = np.minimum(y, 6.0)
+    return y
 
 
 def conv_masked(x, W, mask=None, bias=None, N: int = 1, stride=(1, 1), pad=(0, 0),
-                dil=(1, 1), relu=False, pixels=None, want_abs=False):
-    """Eq. 6: y = (W (+) T) * x (+bias, ReLU), NHWC, fp64 accumulation.
+                dil=(1, 1), relu=False, pixels=None, want_abs=False, residual=None):
+    """Eq. 6: y = (W (+) T) * x (+bias, activation), NHWC, fp64 accumulation.
+
+    relu: False / True / "relu6".  residual (optional, the output's shape or
+    [len(pixels), C_out]): y = act(conv + bias + residual), the residual add
+    of MobileNet-V2's inverted-residual block, applied here in numpy.
 
     x: [B, H, W, C_in] float32 (already rounded if the path is bf16);
     W: [C_out, C_in, KH, KW] float32; mask: [C_out/N, KH*KW*C_in] or None.
     pixels: optional int64 list of flattened output pixels (b*Ho*Wo+oh*Wo+ow);
     then y is [len(pixels), C_out], else [B, Ho, Wo, C_out].
     want_abs also returns sum |w x| + |b| per output (reading C12)."""
+    if residual is not None:
+        out = conv_masked(x, W, mask, bias, N, stride, pad, dil, False, pixels, want_abs)
+        y, a = out if want_abs else (out, None)
+        y = activation(y + np.asarray(residual, np.float64).reshape(y.shape), relu)
+        if a is not None:
+            a = a + np.abs(np.asarray(residual, np.float64)).reshape(a.shape)
+        return (y, a) if want_abs else y
     x, W = _c(x, np.float32), _c(W, np.float32)
     C_out, C_in, KH, KW = W.shape
     B, H, Wd, Cx = x.shape
@@ -216,6 +245,22 @@ def conv_masked(x, W, mask=None, bias=None, N: int = 1, stride=(1, 1), pad=(0, 0
         y = y.reshape(B, Ho, Wo, C_out)
         a = a.reshape(B, Ho, Wo, C_out) if a is not None else None
     return (y, a) if want_abs else y
+
+
+def dwconv(x, W, bias=None, stride=(1, 1), pad=(0, 0), dil=(1, 1), relu=False):
+    """Dense depthwise convolution: y[b,oh,ow,c] = act(bias[c] + sum_{kh,kw}
+    W[c,kh,kw] * x[b, oh*s-p+kh*d, ow*s-p+kw*d, c]), NHWC, fp64.
+    x: [B, H, W, C] float32; W: [C, KH, KW] float32."""
+    x, W = _c(x, np.float32), _c(W, np.float32)
+    C, KH, KW = W.shape
+    B, H, Wd, Cx = x.shape
+    assert Cx == C
+    g = _geom(x.shape, C, KH, KW, stride, pad, dil, relu)
+    Ho, Wo = out_hw(H, Wd, KH, KW, stride, pad, dil)
+    bias = _c(bias, np.float32)
+    y = np.empty((B, Ho, Wo, C), np.float64)
+    _load().oracle_dwconv(_ptr(x), _ptr(W), _ptr(bias), ctypes.byref(g), _ptr(y))
+    return y
 
 
 def conv_bsr(x, P, I, D, C_out, KH, KW, N, bias=None, stride=(1, 1), pad=(0, 0),

@@ -278,6 +278,15 @@ typedef struct {
     int relu;
 } oracle_geom;
 
+/* Activation after the bias: 0 none, 1 ReLU max(s, 0), 2 ReLU6            */
+/* min(max(s, 0), 6) (MobileNet-V2's activation).                           */
+static double act(double s, int kind)
+{
+    if (kind >= 1 && s < 0.0) s = 0.0;
+    if (kind == 2 && s > 6.0) s = 6.0;
+    return s;
+}
+
 /* x value at NHWC input position, zero outside the image (zero padding). */
 static double x_at(const float *x, const oracle_geom *g, int b, int ih, int iw, int c)
 {
@@ -289,7 +298,8 @@ static double x_at(const float *x, const oracle_geom *g, int b, int ih, int iw, 
 /* Eq. 6: masked direct convolution, y[b,oh,ow,o] =                    */
 /*   bias[o] + sum_{kh,kw,c} mask[o/N][(kh*KW+kw)*C_in+c] * W[o,c,kh,kw] */
 /*                        * x[b, oh*sh - ph + kh*dh, ow*sw - pw + kw*dw, c] */
-/* then ReLU if requested.  absacc[...] = sum |mask*W*x| + |bias| (C12). */
+/* then the activation g->relu (1 ReLU, 2 ReLU6).                          */
+/* absacc[...] = sum |mask*W*x| + |bias| (C12).                            */
 /* pix (nullable): list of npix flattened output pixels b*Ho*Wo+oh*Wo+ow; */
 /* y/absacc are then [npix][C_out], else [B][Ho][Wo][C_out].             */
 /* mask may be NULL (dense).                                             */
@@ -322,7 +332,7 @@ void oracle_conv_masked(const float *x, const float *W, const uint8_t *mask,
                         s += w * v;
                         a += fabs(w * v);
                     }
-            if (g->relu && s < 0.0) s = 0.0;
+            s = act(s, g->relu);
             y[q * g->C_out + o] = s;
             if (absacc) absacc[q * g->C_out + o] = a;
         }
@@ -369,9 +379,38 @@ void oracle_conv_bsr(const float *x, const int32_t *P, const int32_t *I,
                     }
                     s += v * d;
                 }
-                if (g->relu && s < 0.0) s = 0.0;
+                s = act(s, g->relu);
                 y[q * g->C_out + gi * N + n] = s;
             }
+        }
+    }
+}
+
+/* ------------------------------------------------------------------ */
+/* Depthwise convolution (dense; MobileNet-V2's 3x3 between the expand  */
+/* and project 1x1 convolutions): channel c of the output reads only     */
+/* channel c of the input,                                               */
+/*   y[b,oh,ow,c] = act(bias[c] + sum_{kh,kw} W[c,kh,kw]                 */
+/*                  * x[b, oh*sh - ph + kh*dh, ow*sw - pw + kw*dw, c]).   */
+/* g->C_in == g->C_out == C; W is [C][KH][KW]; y is [B][Ho][Wo][C].      */
+/* ------------------------------------------------------------------ */
+void oracle_dwconv(const float *x, const float *W, const float *bias,
+                   const oracle_geom *g, double *y)
+{
+    int Ho = out_size(g->H, g->KH, g->sh, g->ph, g->dh);
+    int Wo = out_size(g->W, g->KW, g->sw, g->pw, g->dw);
+    int64_t total = (int64_t)g->B * Ho * Wo;
+#pragma omp parallel for schedule(dynamic, 16)
+    for (int64_t p = 0; p < total; p++) {
+        int b = (int)(p / ((int64_t)Ho * Wo));
+        int oh = (int)((p / Wo) % Ho), ow = (int)(p % Wo);
+        for (int c = 0; c < g->C_in; c++) {
+            double s = bias ? (double)bias[c] : 0.0;
+            for (int kh = 0; kh < g->KH; kh++)
+                for (int kw = 0; kw < g->KW; kw++)
+                    s += (double)W[((int64_t)c * g->KH + kh) * g->KW + kw] *
+                         x_at(x, g, b, oh * g->sh - g->ph + kh * g->dh, ow * g->sw - g->pw + kw * g->dw, c);
+            y[p * g->C_in + c] = act(s, g->relu);
         }
     }
 }

@@ -398,3 +398,51 @@ def test_conv_sampled_pixels_match_full():
     P, I, D = oracle.pack(W, mask, 2)
     partb = oracle.conv_bsr(x, P, I, D, 8, 3, 3, 2, None, (2, 2), (1, 1), pixels=pix)
     np.testing.assert_array_equal(partb, part)
+
+
+# ------------------------------------------------ MobileNet-V2 block pieces
+
+@pytest.mark.parametrize("s,p,d", [(1, 1, 1), (2, 1, 1), (1, 2, 2), (2, 0, 1)])
+def test_dwconv_equals_dense_conv_on_block_diagonal_weights(s, p, d):
+    """A depthwise convolution is the dense convolution whose weight is zero
+    off the channel diagonal: the oracle's two routines agree bitwise (the
+    extra terms add exact zeros), and both match torch's grouped conv2d."""
+    rng = np.random.default_rng(s * 7 + p * 3 + d)
+    C = 6
+    x = rng.standard_normal((2, 9, 8, C)).astype(np.float32)
+    Wd = rng.standard_normal((C, 3, 3)).astype(np.float32)
+    b = rng.standard_normal(C).astype(np.float32)
+    Wfull = np.zeros((C, C, 3, 3), np.float32)
+    for c in range(C):
+        Wfull[c, c] = Wd[c]
+    y_dw = oracle.dwconv(x, Wd, b, stride=(s, s), pad=(p, p), dil=(d, d))
+    y_full = oracle.conv_masked(x, Wfull, None, b, 1, stride=(s, s), pad=(p, p), dil=(d, d))
+    assert np.array_equal(y_dw, y_full)
+    xt = torch.from_numpy(x.astype(np.float64)).permute(0, 3, 1, 2)
+    yt = F.conv2d(xt, torch.from_numpy(Wd.astype(np.float64))[:, None], torch.from_numpy(b.astype(np.float64)),
+                  stride=s, padding=p, dilation=d, groups=C).permute(0, 2, 3, 1).numpy()
+    assert np.max(np.abs(y_dw - yt)) <= 1e-12 * (np.abs(yt).max() + 1)
+
+
+def test_relu6_is_the_clamp_of_the_linear_output():
+    rng = np.random.default_rng(11)
+    x = (3 * rng.standard_normal((1, 6, 6, 8))).astype(np.float32)
+    W = rng.standard_normal((8, 8, 3, 3)).astype(np.float32)
+    lin = oracle.conv_masked(x, W, None, None, 1, pad=(1, 1))
+    r6 = oracle.conv_masked(x, W, None, None, 1, pad=(1, 1), relu="relu6")
+    assert np.array_equal(r6, np.clip(lin, 0.0, 6.0))
+    assert (lin > 6).any() and (lin < 0).any()            # both clamps exercised
+    Wd = rng.standard_normal((8, 3, 3)).astype(np.float32)
+    assert np.array_equal(oracle.dwconv(x, Wd, pad=(1, 1), relu="relu6"),
+                          np.clip(oracle.dwconv(x, Wd, pad=(1, 1)), 0.0, 6.0))
+
+
+def test_residual_is_added_before_the_activation():
+    rng = np.random.default_rng(12)
+    x = rng.standard_normal((2, 5, 5, 4)).astype(np.float32)
+    W = rng.standard_normal((4, 4, 1, 1)).astype(np.float32)
+    r = rng.standard_normal((2, 5, 5, 4))
+    lin = oracle.conv_masked(x, W, None, None, 1)
+    assert np.array_equal(oracle.conv_masked(x, W, None, None, 1, residual=r), lin + r)
+    assert np.array_equal(oracle.conv_masked(x, W, None, None, 1, residual=r, relu=True),
+                          np.maximum(lin + r, 0.0))
