@@ -9,6 +9,8 @@ flushed with a 256 MB write before every step, outside the timed events):
   4  ResNet-50 bottleneck stack (52 convs), 256x224x224 input, bf16, N=16, 70%
   5  3x3 512 -> 512 on 128x14x14: sweep N in {1..32} x rate in {0..0.9} x {fp32, bf16}
   6  fully connected 1280 -> 1000 as a 1x1 conv on 256 1x1 inputs, fp32 + bf16, N=4, 50%
+  7  MobileNet-V2's 17 inverted-residual blocks at batch 1 (224x224 input), fp32, N=4, 50%:
+     latency of one image through the blocks, replayed as one CUDA graph
 
 A "step" is one pass over every layer (leg) of the workload.  Prints one JSON
 line.  Metric: effective TFLOP/s = 2 * pixels * t * N / time summed over the
@@ -54,6 +56,9 @@ DESCRIPTIONS = {
        "{0,.3,.5,.7,.9} x {fp32, bf16}, seed 0",
     6: "fully connected 1280 -> 1000 (MobileNet-V2 classifier) as a 1x1 conv on 256x1x1 inputs; "
        "1xN N=4, 50% block rate; fp32 leg + bf16-in/fp32-acc leg",
+    7: "MobileNet-V2 (width 1.0) 17 inverted-residual blocks (expand 1x1 + ReLU6, dense depthwise "
+       "3x3 + ReLU6, project 1x1 + residual), batch 1, 224x224 input, fp32; 1xN N=4, 50% block rate "
+       "on both 1x1 convs; one CUDA graph per image",
 }
 
 
@@ -317,6 +322,9 @@ def run_reference(args, rank, ws):
     if rank != 0:
         return
     import oracle
+    if args.config == 7:
+        run_reference_mbv2(args)
+        return
     cfg = args.config if args.config != 5 else 2
     layers = workload(cfg)
     packs = oracle_setup(layers)
@@ -488,7 +496,7 @@ def measure(layers, args, dev, stream, flush, ws, pk, sampler=None):
 
 def main():
     ap = argparse.ArgumentParser()
-    ap.add_argument("--config", type=int, default=2, choices=[1, 2, 3, 4, 5, 6])
+    ap.add_argument("--config", type=int, default=2, choices=[1, 2, 3, 4, 5, 6, 7])
     ap.add_argument("--gpus", type=int, default=1)
     # default: a timed region of ~1 s on the default workload, so that the
     # clock samples (every 50 ms) fall inside it
@@ -514,6 +522,9 @@ def main():
 
     if args.config == 5:
         run_sweep(args, dev, stream, flush, ws, rank, pk)
+        return
+    if args.config == 7:
+        run_mbv2(args, dev, stream, flush, ws, rank, local, pk)
         return
 
     layers = workload(args.config)
@@ -615,6 +626,244 @@ def run_sweep(args, dev, stream, flush, ws, rank, pk):
             "roofline": rf, "points": points, "clocks": sampler.summary(),
             "gpu_launches": sum(1 if p["algo"] == "fma" else 2 for p in points) * steps,
             "peaks": pk, "cpu_baseline": None}), flush=True)
+
+
+# --------------------------------------------------------------------------
+# config 7: MobileNet-V2 inverted-residual blocks, batch-1 latency
+# --------------------------------------------------------------------------
+
+MBV2_METRIC = "MobileNet-V2 inverted-residual blocks, batch-1 latency (ms per image)"
+
+
+def mbv2_stage_layers(blk):
+    """The block's two pruned 1x1 convs as ConvLayer records (for the roofline)."""
+    from paper_2105_14713_gb300 import workloads as wl
+    out = []
+    if blk.hidden != blk.c_in:
+        out.append(("expand", wl.ConvLayer(blk.name + ".expand", blk.B, blk.hw, blk.hw, blk.c_in, blk.hidden,
+                                           N=blk.N, rate=blk.rate, dtype=blk.dtype)))
+    out.append(("dw", None))
+    out.append(("project", wl.ConvLayer(blk.name + ".project", blk.B, blk.hw_out, blk.hw_out, blk.hidden,
+                                        blk.c_out, N=blk.N, rate=blk.rate, dtype=blk.dtype)))
+    return out
+
+
+def dw_bytes(blk):
+    es = 4 if blk.dtype == "f32" else 2
+    rows = _touched(blk.hw, blk.hw_out, 3, blk.stride, 1, 1)
+    return (blk.B * rows * rows * blk.hidden + blk.B * blk.hw_out ** 2 * blk.hidden) * es + blk.hidden * 40
+
+
+def dw_roofline(blk, ms, pk):
+    by = dw_bytes(blk)
+    return {"bound": "hbm", "achieved": by / (ms * 1e-3) / 1e9, "peak": pk["hbm_gbs"], "unit": "GB/s",
+            "frac": by / (ms * 1e-3) / 1e9 / pk["hbm_gbs"], "peak_source": f"{pk['source']} HBM copy"}
+
+
+def mbv2_net(blocks, dev):
+    from paper_2105_14713_gb300 import workloads as wl
+    from paper_2105_14713_gb300.layer import InvertedResidual
+    net = []
+    for blk in blocks:
+        we, be, wd, bd, wp, bp = wl.block_weights(blk)
+        net.append(InvertedResidual(we, be, wd, bd, wp, bp, stride=blk.stride, N=blk.N, rate=blk.rate,
+                                    dtype=blk.dtype, device=dev))
+    return net
+
+
+def run_mbv2(args, dev, stream, flush, ws, rank, local, pk):
+    from paper_2105_14713_gb300 import workloads as wl
+    blocks = wl.config7()
+    net = mbv2_net(blocks, dev)
+    x0 = wl.block_input(blocks[0]).to(dev)
+
+    def forward(x, s=None):
+        for b in net:
+            x = b(x, stream=s)
+        return x
+
+    for _ in range(args.warmup):
+        y = forward(x0)
+    torch.cuda.synchronize()
+    # eager, per stage: where the time goes (each stage bracketed by events)
+    reps = 20
+    st_ms = [[0.0] * len(mbv2_stage_layers(b)) for b in blocks]
+    for r in range(reps):
+        flush.fill_(r & 0xff)
+        x = x0
+        evs = []
+        for b in net:
+            h, d, o = b.buffers(x.shape, x.dtype, x.device)
+            es = []
+            def ev():
+                e = torch.cuda.Event(enable_timing=True)
+                e.record(stream)
+                es.append(e)
+            ev()
+            if b.expand is not None:
+                b.expand(x, h, relu="relu6")
+                ev()
+            else:
+                h = x
+            b.dw(h, d, relu="relu6")
+            ev()
+            b.project(d, o, residual=x if b.residual else None)
+            ev()
+            evs.append(es)
+            x = o
+        torch.cuda.synchronize()
+        for i, es in enumerate(evs):
+            for j in range(len(es) - 1):
+                st_ms[i][j] += es[j].elapsed_time(es[j + 1]) / reps
+    stages, algos, rfs = [], [], []
+    for blk, b, ms in zip(blocks, net, st_ms):
+        for (kind, layer), m in zip(mbv2_stage_layers(blk), ms):
+            if kind == "dw":
+                rf = dw_roofline(blk, m, pk)
+                algo, t = "dw", None
+            else:
+                conv = b.expand if kind == "expand" else b.project
+                shape = (blk.B, layer.H, layer.W, layer.C_in)
+                algo, t = conv.algo(shape), conv.t
+                rf = leg_roofline(layer, t, algo, m, pk)
+            algos.append(algo)
+            rfs.append(rf)
+            stages.append({"name": f"{blk.name}.{kind}", "algo": algo, "ms": m, "bound": rf["bound"],
+                           "roofline_frac": rf["frac"], "t_kept_blocks": t})
+    eager_ms = sum(sum(m) for m in st_ms)
+
+    # the whole stack as one CUDA graph on a side stream
+    gs = torch.cuda.Stream(dev)
+    gs.wait_stream(stream)
+    with torch.cuda.stream(gs):
+        forward(x0, gs)
+    torch.cuda.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=gs):
+        y_graph = forward(x0, gs)
+    for _ in range(args.warmup):
+        g.replay()
+    torch.cuda.synchronize()
+    steps = args.steps
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in range(steps)]
+    sampler = ClockSampler(local)
+    barrier(ws)
+    torch.cuda.synchronize()
+    with sampler:
+        wall0 = time.perf_counter()
+        for k in range(steps):
+            flush.fill_(k & 0xff)
+            evs[k][0].record(stream)
+            g.replay()
+            evs[k][1].record(stream)
+        torch.cuda.synchronize()
+        wall = time.perf_counter() - wall0
+    ts = sorted(e0.elapsed_time(e1) for e0, e1 in evs)
+    ms = max_over_ranks(sum(ts) / len(ts), ws)
+    barrier(ws)
+
+    # end to end: pinned host image in, pinned host result out, graph in between
+    x_pin = wl.block_input(blocks[0]).pin_memory()
+    y_pin = torch.empty(y_graph.shape, dtype=y_graph.dtype, pin_memory=True)
+    e2e = []
+    for r in range(args.warmup + min(steps, 200)):
+        flush.fill_(r & 0xff)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        x0.copy_(x_pin, non_blocking=True)
+        g.replay()
+        y_pin.copy_(y_graph, non_blocking=True)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        if r >= args.warmup:
+            e2e.append(e0.elapsed_time(e1))
+    e2e_ms = max_over_ranks(sum(e2e) / len(e2e), ws)
+
+    dom = max(range(len(stages)), key=lambda i: stages[i]["ms"])
+    flops = sum(b.kept_flops for b in blocks)
+    cpu = None
+    if rank == 0 and ws == 1 and not args.no_cpu_baseline:
+        cpu = mbv2_cpu_baseline(blocks)
+    launches = sum(2 if a == "tc" else 1 for a in algos)
+    if rank == 0:
+        print(json.dumps({
+            "metric": MBV2_METRIC, "value": ms, "unit": "ms", "n_gpus": ws, "steps": steps,
+            "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": False, "scaling": "weak",
+            "vs_baseline": None, "dtype": "f32",
+            "data": "synthetic (seeded Kaiming-normal weights, N(0,0.1) biases, N(0,1) input)",
+            "config": {"workload": DESCRIPTIONS[7], "config_id": 7, "blocks": len(blocks), "batch": 1,
+                       "N": 4, "rate": 0.5, "parallelism": "replicas",
+                       "l2": "flushed before every replay (256 MB write)"},
+            "latency_ms": {"graph_mean": ms, "graph_median": ts[len(ts) // 2], "graph_min": ts[0],
+                           "eager_sum_of_stages": eager_ms},
+            "effective_tflops": ws * flops / (ms * 1e-3) / 1e12,
+            "roofline": {**rfs[dom], "kernel": f"{stages[dom]['algo']} ({stages[dom]['name']})",
+                         "traffic": None, "note": "batch 1, eager per-stage events: latency-bound stages"},
+            "stages": stages,
+            "e2e": {"value": e2e_ms, "unit": "ms", "h2d_bytes_per_step": x_pin.numel() * 4,
+                    "d2h_bytes_per_step": y_pin.numel() * 4},
+            "gpu_launches": launches * steps,
+            "clocks": sampler.summary(), "wall_s_timed_region": wall, "peaks": pk,
+            "cpu_baseline": cpu}), flush=True)
+
+
+def mbv2_oracle_pass(blocks, packs):
+    import oracle
+    x = None
+    t0 = time.perf_counter()
+    for blk, (we, me, be, wd, bd, wp, mp, bp, x_in) in zip(blocks, packs):
+        x = x_in if x is None else x
+        h = x if we is None else oracle.conv_masked(x, we, me, be, blk.N, relu="relu6").astype(np.float32)
+        d = oracle.dwconv(h, wd, bd, stride=(blk.stride,) * 2, pad=(1, 1), relu="relu6").astype(np.float32)
+        res = x if (blk.stride == 1 and blk.c_in == blk.c_out) else None
+        x = oracle.conv_masked(d, wp, mp, bp, blk.N, residual=res).astype(np.float32)
+    return time.perf_counter() - t0
+
+
+def mbv2_oracle_setup(blocks):
+    import oracle
+    from paper_2105_14713_gb300 import workloads as wl
+    packs = []
+    for i, blk in enumerate(blocks):
+        we, be, wd, bd, wp, bp = wl.block_weights(blk)
+        me = None if we is None else oracle.prune(we, blk.N, blk.rate)[0]
+        mp = oracle.prune(wp, blk.N, blk.rate)[0]
+        packs.append((we, me, be, wd, bd, wp, mp, bp, wl.block_input(blk).numpy() if i == 0 else None))
+    return packs
+
+
+def mbv2_cpu_baseline(blocks, budget_s: float = 10.0):
+    """The oracle composition (no filter rearrangement: it does not change
+    the work) over the 17 blocks for one image, repeated until ~budget_s."""
+    import oracle
+    packs = mbv2_oracle_setup(blocks)
+    spent, n = 0.0, 0
+    while spent < budget_s and n < 50:
+        spent += mbv2_oracle_pass(blocks, packs)
+        n += 1
+    return {"value": 1e3 * spent / n, "unit": "ms", "cores": oracle.num_threads(), "kind": "oracle",
+            "sample": f"{n} full images through the 17 blocks; fp64 plain-C oracle; {spent:.1f} s"}
+
+
+def run_reference_mbv2(args):
+    import oracle
+    from paper_2105_14713_gb300 import workloads as wl
+    blocks = wl.config7()
+    packs = mbv2_oracle_setup(blocks)
+    for _ in range(args.warmup):
+        mbv2_oracle_pass(blocks, packs)
+    ts = [mbv2_oracle_pass(blocks, packs) for _ in range(args.steps)]
+    ms = 1e3 * sum(ts) / len(ts)
+    print(json.dumps({
+        "impl": "reference", "metric": MBV2_METRIC, "value": ms, "unit": "ms", "n_gpus": args.gpus,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": False,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": DESCRIPTIONS[7], "config_id": 7, "blocks": len(blocks), "batch": 1,
+                   "parallelism": "replicas", "l2": "cpu oracle"},
+        "cpu_baseline": {"value": ms, "unit": "ms", "cores": oracle.num_threads(), "kind": "oracle",
+                         "sample": f"{args.steps} full images through the 17 blocks"},
+        "e2e": {"value": ms, "unit": "ms", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }), flush=True)
 
 
 if __name__ == "__main__":

@@ -57,7 +57,8 @@ typedef enum { ONEXN_F32 = 0, ONEXN_BF16 = 1 } onexn_dtype;
 typedef enum { ONEXN_GRAN_TAP = 0, ONEXN_GRAN_KERNEL = 1 } onexn_granularity;
 
 /* onexn_conv_fwd flags */
-#define ONEXN_RELU 0x1u               /* y = max(y, 0) after the bias */
+#define ONEXN_RELU 0x1u               /* y = max(y, 0) after the bias (and residual) */
+#define ONEXN_RELU6 0x2u              /* y = min(max(y, 0), 6) (MobileNet-V2); wins over RELU */
 /* Kernel selection (bits 8..11).  AUTO picks by dtype, N and density:
  * the tensor-core GEMM when its workspace fits and its dense work is
  * estimated to take less time than the FFMA kernel's kept work. */
@@ -180,7 +181,7 @@ onexn_status onexn_conv_out_shape(const onexn_conv_desc *desc, int *Ho, int *Wo)
  *   bias    nullable DEVICE fp32 [C_out].
  *   dtype   ONEXN_F32: fp32 inputs and weights, fp32 accumulation.
  *           ONEXN_BF16: bf16 inputs and weights, fp32 accumulation.
- *   flags   ONEXN_RELU | one ONEXN_ALGO_* value.
+ *   flags   ONEXN_RELU or ONEXN_RELU6, | one ONEXN_ALGO_* value.
  *   workspace, workspace_bytes
  *           nullable DEVICE scratch owned by the caller, 256-byte aligned.
  *           Some kernel families need it (onexn_conv_workspace_size); the
@@ -198,6 +199,40 @@ onexn_status onexn_conv_fwd(const onexn_conv_desc *desc, const int32_t *P, const
                             const void *D, int N, int64_t t, const void *x, void *y,
                             const float *bias, int dtype, unsigned flags, void *workspace,
                             size_t workspace_bytes, void *stream);
+
+/*
+ * onexn_conv_fwd_ex -- onexn_conv_fwd with a residual input:
+ *   y = act(conv(x) + bias + residual)
+ * (the residual add of MobileNet-V2's inverted-residual block, fused into the
+ * convolution's epilogue; the paper's Eq. 7 output plus a skip connection).
+ *   residual  nullable DEVICE NHWC [B][Ho][Wo][C_out] of dtype, 16-byte
+ *             aligned; it may be y itself (y += conv(x) + bias) but must not
+ *             partially overlap y.
+ * Everything else as onexn_conv_fwd, which is onexn_conv_fwd_ex with
+ * residual = NULL.
+ */
+onexn_status onexn_conv_fwd_ex(const onexn_conv_desc *desc, const int32_t *P, const int32_t *I,
+                               const void *D, int N, int64_t t, const void *x, void *y,
+                               const float *bias, const void *residual, int dtype, unsigned flags,
+                               void *workspace, size_t workspace_bytes, void *stream);
+
+/*
+ * onexn_dwconv_fwd -- the dense depthwise convolution between the pruned
+ * expand and project 1x1 convolutions of MobileNet-V2's inverted-residual
+ * block (not pruned; no paper equation of its own):
+ *   y[b,oh,ow,c] = act(bias[c] + sum_{kh,kw} W[c][kh][kw]
+ *                  * x[b, oh*sh - ph + kh*dh, ow*sw - pw + kw*dw, c])
+ *   desc    geometry with C_in == C_out == C; C % 4 == 0 (fp32) or % 8 (bf16).
+ *   W       DEVICE fp32 [C][KH][KW]; bias nullable DEVICE fp32 [C].
+ *   x, y    DEVICE NHWC of dtype (ONEXN_F32 / ONEXN_BF16; bf16 outputs are
+ *           the RNE of the fp32 result), 16-byte aligned, not overlapping.
+ *   flags   0, ONEXN_RELU or ONEXN_RELU6.
+ *   stream  cudaStream_t (NULL = legacy default stream).
+ * Asynchronous; no allocation.  EINVAL on bad geometry, alignment, NULL
+ * pointers or flags; ECUDA on a launch failure.
+ */
+onexn_status onexn_dwconv_fwd(const onexn_conv_desc *desc, const float *W, const float *bias,
+                              const void *x, void *y, int dtype, unsigned flags, void *stream);
 
 /*
  * onexn_conv_workspace_size -- bytes of device workspace onexn_conv_fwd

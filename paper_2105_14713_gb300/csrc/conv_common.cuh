@@ -22,7 +22,8 @@ struct ConvArgs {
     int N;                  // block width
     int t;                  // number of kept blocks (entries of I / rows of D)
     int P_pix;              // B * Ho * Wo
-    int relu;
+    int relu;               // activation after bias (+ residual): 0 none, 1 ReLU, 2 ReLU6
+    const void *residual;   // nullable, NHWC like y: y = act(acc + bias + residual)
     unsigned int *status;   // library status word (device): bits set by kernels on failure
 };
 
@@ -35,6 +36,14 @@ cudaError_t device_sm_count(int *sms);
 cudaError_t device_status_ptr(unsigned int **p);
 
 __device__ __forceinline__ int clampi(int v, int lo, int hi) { return min(max(v, lo), hi); }
+
+// The activation of ConvArgs::relu: 0 none, 1 max(v, 0), 2 min(max(v, 0), 6).
+__device__ __forceinline__ float activate(float v, int kind)
+{
+    if (kind >= 1) v = fmaxf(v, 0.f);
+    if (kind == 2) v = fminf(v, 6.f);
+    return v;
+}
 
 // Division of 32-bit unsigned integers by an invariant divisor d >= 1 with
 // one multiply-high, after Granlund and Montgomery, "Division by invariant

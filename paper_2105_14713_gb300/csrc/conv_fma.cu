@@ -377,10 +377,16 @@ fma_conv_kernel(const ConvArgs a, const int n_units, const int n_ct)
                 if (p >= a.P_pix) continue;
                 float v[NS];
 #pragma unroll
-                for (int n = 0; n < NS; ++n) {
-                    v[n] = acc[s][r][n] + bv[n];
-                    if (a.relu) v[n] = fmaxf(v[n], 0.f);
+                for (int n = 0; n < NS; ++n) v[n] = acc[s][r][n] + bv[n];
+                if (a.residual) {
+                    float rv[NS];
+                    // aligned: NS divides N, which divides C_out, and residual is 16-byte aligned
+                    load_row<NS>(static_cast<const TIN *>(a.residual) + static_cast<int64_t>(p) * a.C_out + col, rv);
+#pragma unroll
+                    for (int n = 0; n < NS; ++n) v[n] += rv[n];
                 }
+#pragma unroll
+                for (int n = 0; n < NS; ++n) v[n] = activate(v[n], a.relu);
                 store_row<NS>(y + static_cast<int64_t>(p) * a.C_out + col, v, vec_ok);
             }
         }

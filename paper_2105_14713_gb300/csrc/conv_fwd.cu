@@ -87,13 +87,13 @@ onexn_status check_shape(const onexn_conv_desc *d, int N, int64_t t, int dtype, 
     if (d->C_in % cv)
         return fail(ONEXN_EINVAL, "conv: C_in=%d must be a multiple of %d for %s", d->C_in, cv,
                     dtype == ONEXN_F32 ? "fp32" : "bf16");
-    if (flags & ~(ONEXN_RELU | ONEXN_ALGO_MASK)) return fail(ONEXN_EINVAL, "conv: unknown flags");
+    if (flags & ~(ONEXN_RELU | ONEXN_RELU6 | ONEXN_ALGO_MASK)) return fail(ONEXN_EINVAL, "conv: unknown flags");
     a->B = d->B; a->H = d->H; a->W = d->W; a->C = d->C_in;
     a->C_out = d->C_out; a->KH = d->KH; a->KW = d->KW;
     a->sh = d->stride_h; a->sw = d->stride_w; a->ph = d->pad_h; a->pw = d->pad_w;
     a->dh = d->dil_h; a->dw = d->dil_w; a->Ho = Ho; a->Wo = Wo;
     a->N = N; a->t = static_cast<int>(t); a->P_pix = static_cast<int>(npix);
-    a->relu = (flags & ONEXN_RELU) ? 1 : 0;
+    a->relu = (flags & ONEXN_RELU6) ? 2 : (flags & ONEXN_RELU) ? 1 : 0;
     return ONEXN_OK;
 }
 
@@ -240,11 +240,11 @@ extern "C" onexn_status onexn_conv_workspace_size(const onexn_conv_desc *desc, i
     return ONEXN_OK;
 }
 
-extern "C" onexn_status onexn_conv_fwd(const onexn_conv_desc *desc, const int32_t *P,
-                                       const int32_t *I, const void *D, int N, int64_t t,
-                                       const void *x, void *y, const float *bias, int dtype,
-                                       unsigned flags, void *workspace, size_t workspace_bytes,
-                                       void *stream)
+extern "C" onexn_status onexn_conv_fwd_ex(const onexn_conv_desc *desc, const int32_t *P,
+                                          const int32_t *I, const void *D, int N, int64_t t,
+                                          const void *x, void *y, const float *bias, const void *residual,
+                                          int dtype, unsigned flags, void *workspace, size_t workspace_bytes,
+                                          void *stream)
 {
     onexn::clear_error();
     onexn::ConvArgs a{};
@@ -252,6 +252,15 @@ extern "C" onexn_status onexn_conv_fwd(const onexn_conv_desc *desc, const int32_
     if (st != ONEXN_OK) return st;
     st = check_pointers(P, I, D, x, y, bias, dtype, &a);
     if (st != ONEXN_OK) return st;
+    if (residual) {
+        if (reinterpret_cast<uintptr_t>(residual) & 15u)
+            return fail(ONEXN_EINVAL, "conv: residual must be 16-byte aligned");
+        const size_t yb = static_cast<size_t>(a.P_pix) * a.C_out * (dtype == ONEXN_F32 ? 4 : 2);
+        const uintptr_t r0 = reinterpret_cast<uintptr_t>(residual), y0 = reinterpret_cast<uintptr_t>(y);
+        if (r0 != y0 && r0 < y0 + yb && y0 < r0 + yb)
+            return fail(ONEXN_EINVAL, "conv: residual overlaps y without being y");
+        a.residual = residual;
+    }
     if (!workspace) workspace_bytes = 0;
     if (reinterpret_cast<uintptr_t>(workspace) & 255u)
         return fail(ONEXN_EINVAL, "conv: workspace must be 256-byte aligned");
@@ -264,6 +273,16 @@ extern "C" onexn_status onexn_conv_fwd(const onexn_conv_desc *desc, const int32_
     e = launch(algo, a, dtype, workspace, workspace_bytes, s);
     if (e != cudaSuccess) return fail(ONEXN_ECUDA, "conv: launch failed: %s", cudaGetErrorString(e));
     return ONEXN_OK;
+}
+
+extern "C" onexn_status onexn_conv_fwd(const onexn_conv_desc *desc, const int32_t *P,
+                                       const int32_t *I, const void *D, int N, int64_t t,
+                                       const void *x, void *y, const float *bias, int dtype,
+                                       unsigned flags, void *workspace, size_t workspace_bytes,
+                                       void *stream)
+{
+    return onexn_conv_fwd_ex(desc, P, I, D, N, t, x, y, bias, nullptr, dtype, flags, workspace, workspace_bytes,
+                             stream);
 }
 
 extern "C" onexn_status onexn_device_status(int clear, int *status)

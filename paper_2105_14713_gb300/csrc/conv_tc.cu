@@ -550,25 +550,31 @@ tc_conv_kernel(const ConvArgs a, const __grid_constant__ CUtensorMap tmap_x,
                 __syncwarp();
                 const uint32_t wbuf = sout + (q * 2 + buf) * (32 * kRowBytes);
                 const int col0 = tn * BN + at * kAtomCols;
+                // the residual row of this atom (16-byte chunks inside y only)
+                const int pix = tm * kBM + row;
+                const uint4 *res = (a.residual && pix < a.P_pix)
+                                       ? reinterpret_cast<const uint4 *>(static_cast<const T *>(a.residual) +
+                                                                         static_cast<int64_t>(pix) * a.C_out + col0)
+                                       : nullptr;
 #pragma unroll
                 for (int j = 0; j < 8; ++j) {        // 16-byte chunk j of the row
                     uint32_t w[4];
+                    uint4 rv = make_uint4(0, 0, 0, 0);
+                    if (res && col0 + j * (16 / static_cast<int>(sizeof(T))) < a.C_out) rv = __ldg(res + j);
+                    const uint32_t rw[4] = {rv.x, rv.y, rv.z, rv.w};
                     if constexpr (sizeof(T) == 4) {
                         const float4 bv = sb4[at * (kAtomCols / 4) + j];
                         const float bb[4] = {bv.x, bv.y, bv.z, bv.w};
 #pragma unroll
-                        for (int e = 0; e < 4; ++e) {
-                            const float v = f[4 * j + e] + bb[e];
-                            w[e] = __float_as_uint(a.relu ? fmaxf(v, 0.f) : v);
-                        }
+                        for (int e = 0; e < 4; ++e)
+                            w[e] = __float_as_uint(activate(f[4 * j + e] + bb[e] + __uint_as_float(rw[e]), a.relu));
                     } else {
                         const float4 b0 = sb4[at * (kAtomCols / 4) + 2 * j], b1 = sb4[at * (kAtomCols / 4) + 2 * j + 1];
                         const float bb[8] = {b0.x, b0.y, b0.z, b0.w, b1.x, b1.y, b1.z, b1.w};
 #pragma unroll
                         for (int e = 0; e < 4; ++e) {
-                            float v0 = f[8 * j + 2 * e] + bb[2 * e];
-                            float v1 = f[8 * j + 2 * e + 1] + bb[2 * e + 1];
-                            if (a.relu) { v0 = fmaxf(v0, 0.f); v1 = fmaxf(v1, 0.f); }
+                            const float v0 = activate(f[8 * j + 2 * e] + bb[2 * e] + bf16lo(rw[e]), a.relu);
+                            const float v1 = activate(f[8 * j + 2 * e + 1] + bb[2 * e + 1] + bf16hi(rw[e]), a.relu);
                             w[e] = pack_bf16x2(v0, v1);
                         }
                     }

@@ -1,4 +1,5 @@
-"""A 1xN-pruned convolution layer on the onexn C ABI.
+"""1xN-pruned convolution layers (and MobileNet-V2's inverted-residual block)
+on the onexn C ABI.
 
 ``PrunedConv2d`` runs the offline steps once on the host -- block scoring
 and selection (``onexn_prune``), BSR encoding (``onexn_pack``), the index
@@ -15,6 +16,13 @@ import numpy as np
 import torch
 
 from . import onexn as _c
+
+
+def act_flags(relu) -> int:
+    """False / True / "relu6" -> 0 / ONEXN_RELU / ONEXN_RELU6."""
+    if relu == "relu6":
+        return _c.ONEXN_RELU6
+    return _c.ONEXN_RELU if relu else 0
 
 
 class PrunedConv2d:
@@ -84,32 +92,36 @@ class PrunedConv2d:
                                0 if ws is None else ws.numel())
         return _c.ALGO_NAMES[a]
 
-    def forward(self, x: torch.Tensor, y: torch.Tensor = None, relu: bool = False,
-                algo: int = _c.ONEXN_ALGO_AUTO, stream=None) -> torch.Tensor:
-        """x: NHWC CUDA tensor of this layer's dtype.  Returns y (NHWC).
+    def forward(self, x: torch.Tensor, y: torch.Tensor = None, relu=False,
+                algo: int = _c.ONEXN_ALGO_AUTO, stream=None, residual: torch.Tensor = None) -> torch.Tensor:
+        """x: NHWC CUDA tensor of this layer's dtype.  Returns y (NHWC):
+        y = act(conv(x) + bias + residual), act = none, ReLU (relu=True) or
+        ReLU6 (relu="relu6"); residual is optional (shape of y; may be y).
 
-        The checked and marshalled C arguments are cached per (x, y, stream,
-        flags) buffers and layout, so a layer called again on the same
-        buffers costs one C call."""
+        The checked and marshalled C arguments are cached per (x, y,
+        residual, stream, flags) buffers and layout, so a layer called again
+        on the same buffers costs one C call."""
         if y is None:
             y = torch.empty(self.out_shape(x.shape), dtype=x.dtype, device=x.device)
         s = torch.cuda.current_stream(x.device) if stream is None else stream
-        flags = (_c.ONEXN_RELU if relu else 0) | algo
+        flags = act_flags(relu) | algo
         key = (x.data_ptr(), y.data_ptr(), x.shape, x.stride(), x.dtype, y.shape, y.stride(), y.dtype,
+               None if residual is None else (residual.data_ptr(), residual.shape, residual.stride(),
+                                              residual.dtype),
                flags, s.cuda_stream)
         args = self._args.get(key)
         if args is None:
             if len(self._args) >= 64:
                 self._args.clear()
                 self._descs.clear()
-            args = self._marshal(x, y, flags, s)
+            args = self._marshal(x, y, flags, s, residual)
             self._args[key] = args
-        st = _c.lib.onexn_conv_fwd(*args)
+        st = _c.lib.onexn_conv_fwd_ex(*args)
         if st != _c.ONEXN_OK:
             raise _c.OnexnError(st, _c.lib.onexn_last_error().decode(errors="replace"))
         return y
 
-    def _marshal(self, x, y, flags, s):
+    def _marshal(self, x, y, flags, s, residual=None):
         if x.dtype != self.torch_dtype or not x.is_cuda or not x.is_contiguous():
             raise ValueError(f"x must be a contiguous CUDA {self.torch_dtype} NHWC tensor")
         B, H, W, C = x.shape
@@ -118,13 +130,17 @@ class PrunedConv2d:
         if tuple(y.shape) != tuple(self.out_shape(x.shape)) or y.dtype != x.dtype or not y.is_contiguous() \
                 or y.device != x.device:
             raise ValueError(f"y must be a contiguous {x.dtype} tensor of shape {self.out_shape(x.shape)}")
+        if residual is not None and (tuple(residual.shape) != tuple(y.shape) or residual.dtype != y.dtype
+                                     or not residual.is_contiguous() or residual.device != y.device):
+            raise ValueError("residual must be a contiguous tensor like y")
         desc = self.desc(B, H, W)
         ws = self.workspace(x.shape, flags & _c.ONEXN_ALGO_MASK)
         ptr = (lambda t: None if t is None else ctypes.c_void_p(t.data_ptr()))
         ws_bytes = 0 if ws is None else ws.numel()
         self._descs.append(desc)                 # kept alive for the cached byref
         return (ctypes.byref(desc), ptr(self.P), ptr(self.I), ptr(self.D), self.N, self.t, ptr(x), ptr(y),
-                ptr(self.bias), self.cdtype, flags, ptr(ws), ws_bytes, ctypes.c_void_p(s.cuda_stream))
+                ptr(self.bias), ptr(residual), self.cdtype, flags, ptr(ws), ws_bytes,
+                ctypes.c_void_p(s.cuda_stream))
 
     __call__ = forward
 
@@ -159,10 +175,132 @@ class PrunedConv2d:
             raise ValueError(f"y_host must be a contiguous CPU {x_host.dtype} tensor of shape {shape}")
         if stream is None:
             stream = torch.cuda.current_stream(self.device)
-        flags = (_c.ONEXN_RELU if relu else 0) | algo
+        flags = act_flags(relu) | algo
         _c.onexn_conv_fwd_host(self.desc(B, H, W), self.P, self.I, self.D, self.N, self.t, x_host,
                                y_host, self.bias, self.cdtype, flags,
                                self.host_workspace(x_host.shape, algo), stream)
         if sync:
             stream.synchronize()
         return y_host
+
+
+class DepthwiseConv2d:
+    """The dense depthwise convolution between the pruned 1x1 convolutions of
+    a MobileNet-V2 block (onexn_dwconv_fwd).  weight: [C, 1, KH, KW] or
+    [C, KH, KW] fp32 (not pruned)."""
+
+    def __init__(self, weight, *, bias=None, stride=1, padding=1, dilation=1, dtype: str = "f32",
+                 device="cuda"):
+        Wd = np.ascontiguousarray(np.asarray(weight, np.float32))
+        if Wd.ndim == 4:
+            Wd = Wd[:, 0]
+        self.C, self.KH, self.KW = Wd.shape
+        self.dtype = dtype
+        self.cdtype = _c.ONEXN_F32 if dtype == "f32" else _c.ONEXN_BF16
+        self.stride = stride if isinstance(stride, (tuple, list)) else (stride, stride)
+        self.padding = padding if isinstance(padding, (tuple, list)) else (padding, padding)
+        self.dilation = dilation if isinstance(dilation, (tuple, list)) else (dilation, dilation)
+        self.device = torch.device(device)
+        self.W = torch.from_numpy(Wd).to(self.device).contiguous()
+        self.bias = None if bias is None else torch.as_tensor(np.asarray(bias, np.float32)).to(self.device)
+        self._args = {}
+        self._descs = []
+
+    def desc(self, B: int, H: int, W: int) -> _c.ConvDesc:
+        return _c.make_desc(B, H, W, self.C, self.C, self.KH, self.KW, self.stride, self.padding,
+                            self.dilation)
+
+    def out_shape(self, x_shape):
+        B, H, W, _ = x_shape
+        Ho, Wo = _c.onexn_conv_out_shape(self.desc(B, H, W))
+        return (B, Ho, Wo, self.C)
+
+    def forward(self, x: torch.Tensor, y: torch.Tensor = None, relu=False, stream=None) -> torch.Tensor:
+        if y is None:
+            y = torch.empty(self.out_shape(x.shape), dtype=x.dtype, device=x.device)
+        s = torch.cuda.current_stream(x.device) if stream is None else stream
+        flags = act_flags(relu)
+        key = (x.data_ptr(), y.data_ptr(), x.shape, x.dtype, y.shape, flags, s.cuda_stream)
+        args = self._args.get(key)
+        if args is None:
+            if not (x.is_cuda and x.is_contiguous() and y.is_contiguous() and x.shape[3] == self.C
+                    and tuple(y.shape) == tuple(self.out_shape(x.shape)) and y.dtype == x.dtype):
+                raise ValueError("x / y do not match the depthwise layer")
+            if len(self._args) >= 64:
+                self._args.clear()
+                self._descs.clear()
+            B, H, W, _ = x.shape
+            desc = self.desc(B, H, W)
+            self._descs.append(desc)
+            ptr = (lambda t: None if t is None else ctypes.c_void_p(t.data_ptr()))
+            args = (ctypes.byref(desc), ptr(self.W), ptr(self.bias), ptr(x), ptr(y), self.cdtype, flags,
+                    ctypes.c_void_p(s.cuda_stream))
+            self._args[key] = args
+        st = _c.lib.onexn_dwconv_fwd(*args)
+        if st != _c.ONEXN_OK:
+            raise _c.OnexnError(st, _c.lib.onexn_last_error().decode(errors="replace"))
+        return y
+
+    __call__ = forward
+
+
+class InvertedResidual:
+    """MobileNet-V2's inverted-residual block on the onexn kernels:
+    expand 1x1 (1xN-pruned, ReLU6; absent for expansion 1) -> depthwise 3x3
+    (dense, ReLU6, stride s) -> project 1x1 (1xN-pruned, linear), plus the
+    block input when s == 1 and C_in == C_out (fused into the project's
+    epilogue).  The filters of the expand layer may be rearranged (Sec. 3.3)
+    before pruning, with the permutation carried through the depthwise
+    channels into the project layer's inputs (reading C10).  Intermediate
+    buffers are allocated per input shape on the first call and reused, so
+    later calls allocate nothing (and can be captured into a CUDA graph)."""
+
+    def __init__(self, w_expand, b_expand, w_dw, b_dw, w_project, b_project, *, stride: int, N: int,
+                 rate: float, dtype: str = "f32", rearrange: bool = True, device="cuda"):
+        w_dw = np.asarray(w_dw, np.float32)
+        w_dw = w_dw[:, 0] if w_dw.ndim == 4 else w_dw
+        b_dw = None if b_dw is None else np.asarray(b_dw, np.float32)
+        w_project = np.asarray(w_project, np.float32)
+        self.expand = None
+        if w_expand is not None:
+            w_expand = np.asarray(w_expand, np.float32)
+            b_expand = None if b_expand is None else np.asarray(b_expand, np.float32)
+            if rearrange:
+                w_expand, w_project, perm = _c.onexn_rearrange(w_expand, w_project)
+                b_expand = None if b_expand is None else b_expand[perm]
+                w_dw = w_dw[perm]
+                b_dw = None if b_dw is None else b_dw[perm]
+            self.expand = PrunedConv2d(w_expand, N, rate, bias=b_expand, dtype=dtype, device=device)
+        # the weights as run (after the rearrangement), for checks
+        self.w_expand, self.b_expand, self.w_dw, self.b_dw = w_expand, b_expand, w_dw, b_dw
+        self.w_project = w_project
+        self.b_project = None if b_project is None else np.asarray(b_project, np.float32)
+        self.dw = DepthwiseConv2d(w_dw, bias=b_dw, stride=stride, padding=1, dtype=dtype, device=device)
+        self.project = PrunedConv2d(w_project, N, rate, bias=b_project, dtype=dtype, device=device)
+        c_in = self.expand.C_in if self.expand is not None else w_dw.shape[0]
+        self.residual = stride == 1 and w_project.shape[0] == c_in
+        self.dtype = dtype
+        self._bufs = {}
+
+    def buffers(self, x_shape, dtype, device):
+        key = tuple(x_shape)
+        if key not in self._bufs:
+            h = self.expand.out_shape(x_shape) if self.expand is not None else tuple(x_shape)
+            d = self.dw.out_shape(h)
+            o = self.project.out_shape(d)
+            self._bufs[key] = (torch.empty(h, dtype=dtype, device=device) if self.expand is not None else None,
+                               torch.empty(d, dtype=dtype, device=device),
+                               torch.empty(o, dtype=dtype, device=device))
+        return self._bufs[key]
+
+    def forward(self, x: torch.Tensor, stream=None) -> torch.Tensor:
+        h, d, o = self.buffers(x.shape, x.dtype, x.device)
+        if self.expand is not None:
+            self.expand(x, h, relu="relu6", stream=stream)
+        else:
+            h = x
+        self.dw(h, d, relu="relu6", stream=stream)
+        self.project(d, o, stream=stream, residual=x if self.residual else None)
+        return o
+
+    __call__ = forward

@@ -17,6 +17,7 @@ ONEXN_ECUDA, ONEXN_EDEVICE, ONEXN_ETIMEOUT = 4, 5, 6
 ONEXN_F32, ONEXN_BF16 = 0, 1
 ONEXN_GRAN_TAP, ONEXN_GRAN_KERNEL = 0, 1
 ONEXN_RELU = 0x1
+ONEXN_RELU6 = 0x2
 ONEXN_ALGO_SHIFT = 8
 ONEXN_ALGO_MASK = 0xF << ONEXN_ALGO_SHIFT
 ONEXN_ALGO_AUTO = 0 << ONEXN_ALGO_SHIFT
@@ -64,6 +65,9 @@ SIGNATURES = {
     "onexn_conv_fwd_host": ([ctypes.POINTER(ConvDesc), _P, _P, _P, _I32, _I64, _P, _P, _P, _I32,
                              _U32, _P, ctypes.c_size_t, _P], _I32),
     "onexn_conv_host_workspace_size": ([ctypes.POINTER(ConvDesc), _I32, _I64, _I32, _U32, _P], _I32),
+    "onexn_conv_fwd_ex": ([ctypes.POINTER(ConvDesc), _P, _P, _P, _I32, _I64, _P, _P, _P, _P, _I32,
+                           _U32, _P, ctypes.c_size_t, _P], _I32),
+    "onexn_dwconv_fwd": ([ctypes.POINTER(ConvDesc), _P, _P, _P, _P, _I32, _U32, _P], _I32),
 }
 
 
@@ -204,6 +208,29 @@ def onexn_conv_fwd(desc: ConvDesc, P, I, D, N: int, t: int, x, y, bias, dtype: i
     _check(lib.onexn_conv_fwd(ctypes.byref(desc), ptr(P), ptr(I), ptr(D), int(N), int(t), ptr(x),
                               ptr(y), ptr(bias), int(dtype), int(flags), ptr(workspace),
                               int(ws_bytes), ctypes.c_void_p(stream.cuda_stream)))
+
+
+def onexn_conv_fwd_ex(desc: ConvDesc, P, I, D, N: int, t: int, x, y, bias, residual, dtype: int,
+                      flags: int = 0, workspace=None, stream=None) -> None:
+    """onexn_conv_fwd with a residual: y = act(conv(x) + bias + residual)."""
+    import torch
+    if stream is None:
+        stream = torch.cuda.current_stream(x.device)
+    ptr = (lambda tns: None if tns is None else ctypes.c_void_p(tns.data_ptr()))
+    ws_bytes = 0 if workspace is None else workspace.numel() * workspace.element_size()
+    _check(lib.onexn_conv_fwd_ex(ctypes.byref(desc), ptr(P), ptr(I), ptr(D), int(N), int(t), ptr(x),
+                                 ptr(y), ptr(bias), ptr(residual), int(dtype), int(flags), ptr(workspace),
+                                 int(ws_bytes), ctypes.c_void_p(stream.cuda_stream)))
+
+
+def onexn_dwconv_fwd(desc: ConvDesc, W, bias, x, y, dtype: int, flags: int = 0, stream=None) -> None:
+    """The dense depthwise convolution (W: CUDA fp32 [C, KH, KW])."""
+    import torch
+    if stream is None:
+        stream = torch.cuda.current_stream(x.device)
+    ptr = (lambda tns: None if tns is None else ctypes.c_void_p(tns.data_ptr()))
+    _check(lib.onexn_dwconv_fwd(ctypes.byref(desc), ptr(W), ptr(bias), ptr(x), ptr(y), int(dtype), int(flags),
+                                ctypes.c_void_p(stream.cuda_stream)))
 
 
 def onexn_conv_fwd_noalloc(desc: ConvDesc, P, I, D, N: int, t: int, x, y, bias, dtype: int,

@@ -158,6 +158,85 @@ def mobilenet_v2_1x1(B: int = 128, res: int = 224, N: int = 4, rate: float = 0.5
     return layers
 
 
+@dataclasses.dataclass(frozen=True)
+class MBv2Block:
+    """One inverted-residual block of MobileNet-V2 (width 1.0): expand 1x1 to
+    `hidden` channels (absent when hidden == c_in, expansion 1), depthwise
+    3x3 with `stride`, project 1x1 to c_out; residual when stride 1 and
+    c_in == c_out.  Input [B, hw, hw, c_in]."""
+    name: str
+    B: int
+    hw: int
+    c_in: int
+    hidden: int
+    c_out: int
+    stride: int
+    N: int = 4
+    rate: float = 0.5
+    dtype: str = "f32"
+    seed: int = 0
+
+    @property
+    def hw_out(self) -> int:
+        return (self.hw + 2 - 3) // self.stride + 1
+
+    @property
+    def kept_flops(self) -> float:
+        """2 x kept multiply-adds of the two pruned 1x1 convs + the dense depthwise."""
+        keep = 1.0 - self.rate
+        e = 0 if self.hidden == self.c_in else self.B * self.hw * self.hw * self.c_in * self.hidden * keep
+        d = self.B * self.hw_out * self.hw_out * self.hidden * 9
+        pr = self.B * self.hw_out * self.hw_out * self.hidden * self.c_out * keep
+        return 2.0 * (e + d + pr)
+
+
+def mobilenet_v2_blocks(B: int = 1, res: int = 224, N: int = 4, rate: float = 0.5,
+                        dtype: str = "f32") -> List[MBv2Block]:
+    """The 17 inverted-residual blocks of MobileNet-V2 (after the 3x3 stem,
+    which leaves res/2 x res/2 x 32)."""
+    settings = [(1, 16, 1, 1), (6, 24, 2, 2), (6, 32, 3, 2), (6, 64, 4, 2),
+                (6, 96, 3, 1), (6, 160, 3, 2), (6, 320, 1, 1)]
+    blocks: List[MBv2Block] = []
+    c_in, hw = 32, res // 2
+    for bi, (t, c, n, s) in enumerate(settings):
+        for r in range(n):
+            stride = s if r == 0 else 1
+            blk = MBv2Block(f"mbv2_block{bi + 1}.{r + 1}", B, hw, c_in, c_in * t, c, stride, N, rate, dtype,
+                            seed=len(blocks))
+            blocks.append(blk)
+            c_in, hw = c, blk.hw_out
+    return blocks
+
+
+def block_weights(blk: MBv2Block):
+    """Seeded Kaiming-normal weights and N(0, 0.1) biases of a block:
+    (w_expand or None, b_expand or None, w_dw [hidden, 3, 3], b_dw,
+    w_project [c_out, hidden, 1, 1], b_project), float32 numpy."""
+    g = _gen(5_000_011 * (blk.seed + 1))
+    def kaiming(shape, fan_in):
+        return (torch.randn(shape, generator=g, dtype=torch.float32) * (2.0 / fan_in) ** 0.5).numpy()
+    def small(n):
+        return (torch.randn((n,), generator=g, dtype=torch.float32) * 0.1).numpy()
+    we = be = None
+    if blk.hidden != blk.c_in:
+        we, be = kaiming((blk.hidden, blk.c_in, 1, 1), blk.c_in), small(blk.hidden)
+    wd, bd = kaiming((blk.hidden, 3, 3), 9), small(blk.hidden)
+    wp, bp = kaiming((blk.c_out, blk.hidden, 1, 1), blk.hidden), small(blk.c_out)
+    return we, be, wd, bd, wp, bp
+
+
+def block_input(blk: MBv2Block) -> torch.Tensor:
+    """NHWC float32 block input, N(0, 1) (a project conv's linear output)."""
+    return torch.randn((blk.B, blk.hw, blk.hw, blk.c_in), generator=_gen(9_000_013 * (blk.seed + 1)),
+                       dtype=torch.float32)
+
+
+def config7(B: int = 1) -> List[MBv2Block]:
+    """MobileNet-V2's 17 inverted-residual blocks at batch 1 (224x224 input),
+    N=4, 50%, fp32: the latency analogue of the paper's Sec. 4.3."""
+    return mobilenet_v2_blocks(B=B, res=224, N=4, rate=0.5, dtype="f32")
+
+
 def config3() -> List[ConvLayer]:
     return mobilenet_v2_1x1(B=128, res=224, N=4, rate=0.5, dtype="f32")
 

@@ -272,3 +272,45 @@ def test_conv_shape_and_argument_errors_need_no_gpu():
     st = ox.lib.onexn_conv_fwd(ctypes.byref(d), mis, mis, mis, 8, 1, mis, mis, None, 0, 0, None, 0,
                                None)
     assert st == ox.ONEXN_EINVAL and b"aligned" in ox.lib.onexn_last_error()
+
+
+def _aligned_host(nbytes, align=256):
+    buf = (ctypes.c_char * (nbytes + align))()
+    base = ctypes.addressof(buf)
+    return buf, base + (align - base % align) % align
+
+
+def test_conv_fwd_ex_residual_errors_need_no_gpu():
+    """The residual operand must be 16-byte aligned and either be y or not
+    overlap it; both are refused before the GPU is touched."""
+    d = ox.make_desc(1, 4, 4, 8, 16)                   # 16 pixels x 16 channels
+    keep, base = _aligned_host(1 << 16)
+    P, I, D = base, base + 256, base + 512
+    x, y = base + 1024, base + 8192                     # y: 16*16*4 = 1 KiB
+    ex = ox.lib.onexn_conv_fwd_ex
+    for r, what in ((y + 4, b"aligned"), (y + 16, b"overlaps"), (y - 512, b"overlaps")):
+        st = ex(ctypes.byref(d), P, I, D, 8, 1, x, y, None, r, ox.ONEXN_F32, 0, None, 0, None)
+        assert st == ox.ONEXN_EINVAL and what in ox.lib.onexn_last_error(), ox.lib.onexn_last_error()
+    st = ex(ctypes.byref(d), P, I, D, 8, 1, x, y, None, y, ox.ONEXN_F32, 1 << 20, None, 0, None)
+    assert st == ox.ONEXN_EINVAL                         # unknown flag bit
+
+
+def test_dwconv_argument_errors_need_no_gpu():
+    keep, base = _aligned_host(1 << 16)
+    W, x, y = base, base + 4096, base + 32768
+    dw = ox.lib.onexn_dwconv_fwd
+    cases = [
+        (ox.make_desc(1, 4, 4, 16, 32, 3, 3, 1, 1, 1), ox.ONEXN_F32, 0, x, y, b"differ"),
+        (ox.make_desc(1, 4, 4, 6, 6, 3, 3, 1, 1, 1), ox.ONEXN_F32, 0, x, y, b"multiple"),
+        (ox.make_desc(1, 4, 4, 12, 12, 3, 3, 1, 1, 1), ox.ONEXN_BF16, 0, x, y, b"multiple"),
+        (ox.make_desc(1, 4, 4, 16, 16, 3, 3, 1, 1, 1), ox.ONEXN_F32, 1 << 20, x, y, b"flags"),
+        (ox.make_desc(1, 4, 4, 16, 16, 3, 3, 1, 1, 1), ox.ONEXN_F32, 0, x, x + 512, b"overlap"),
+        (ox.make_desc(1, 4, 4, 16, 16, 3, 3, 1, 1, 1), ox.ONEXN_F32, 0, x + 8, y, b"aligned"),
+        (ox.make_desc(1, 4, 4, 16, 16, 3, 3, 1, 1, 1), 5, 0, x, y, b"dtype"),
+    ]
+    for d, dt, fl, xp, yp, what in cases:
+        st = dw(ctypes.byref(d), W, None, xp, yp, dt, fl, None)
+        assert st == ox.ONEXN_EINVAL and what in ox.lib.onexn_last_error(), ox.lib.onexn_last_error()
+    # an empty batch is a no-op that needs no device
+    d0 = ox.make_desc(0, 4, 4, 16, 16, 3, 3, 1, 1, 1)
+    assert dw(ctypes.byref(d0), None, None, None, None, ox.ONEXN_F32, 0, None) == ox.ONEXN_OK
