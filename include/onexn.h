@@ -59,6 +59,21 @@ typedef enum { ONEXN_GRAN_TAP = 0, ONEXN_GRAN_KERNEL = 1 } onexn_granularity;
 /* onexn_conv_fwd flags */
 #define ONEXN_RELU 0x1u               /* y = max(y, 0) after the bias (and residual) */
 #define ONEXN_RELU6 0x2u              /* y = min(max(y, 0), 6) (MobileNet-V2); wins over RELU */
+/* ONEXN_DECODED (onexn_conv_fwd / _ex only): the workspace already holds this
+ * layer's decoded weights, written by an earlier ONEXN_ALGO_TC call with the
+ * same P, I, D, N, t, dtype and geometry on the same workspace, which the
+ * caller has ordered before this one (same stream, or an event); the call
+ * skips the decode and runs the GEMM alone.  It implies the tc family (AUTO
+ * resolves to it; another forced ALGO is EINVAL).  Weights that changed since,
+ * a workspace another layer used in between, or a previous call on it that
+ * reported ONEXN_ETIMEOUT through onexn_device_status: run once without the
+ * flag first. */
+#define ONEXN_DECODED 0x10u
+/* ONEXN_REUSE_DECODE (onexn_conv_fwd / _ex / _algo / _workspace_size): a hint
+ * for AUTO that the caller keeps the workspace's decoded weights and passes
+ * ONEXN_DECODED on later calls, so the one-time decode is left out of the
+ * comparison of the families.  It changes nothing else. */
+#define ONEXN_REUSE_DECODE 0x20u
 /* Kernel selection (bits 8..11).  AUTO picks by dtype, N and density:
  * the tensor-core GEMM when its workspace fits and its dense work is
  * estimated to take less time than the FFMA kernel's kept work. */
@@ -181,7 +196,9 @@ onexn_status onexn_conv_out_shape(const onexn_conv_desc *desc, int *Ho, int *Wo)
  *   bias    nullable DEVICE fp32 [C_out].
  *   dtype   ONEXN_F32: fp32 inputs and weights, fp32 accumulation.
  *           ONEXN_BF16: bf16 inputs and weights, fp32 accumulation.
- *   flags   ONEXN_RELU or ONEXN_RELU6, | one ONEXN_ALGO_* value.
+ *   flags   ONEXN_RELU or ONEXN_RELU6, | one ONEXN_ALGO_* value,
+ *           | ONEXN_DECODED (weights already decoded in the workspace),
+ *           | ONEXN_REUSE_DECODE (AUTO hint: the decode will be reused).
  *   workspace, workspace_bytes
  *           nullable DEVICE scratch owned by the caller, 256-byte aligned.
  *           Some kernel families need it (onexn_conv_workspace_size); the
@@ -223,7 +240,7 @@ onexn_status onexn_conv_fwd_ex(const onexn_conv_desc *desc, const int32_t *P, co
  *   y[b,oh,ow,c] = act(bias[c] + sum_{kh,kw} W[c][kh][kw]
  *                  * x[b, oh*sh - ph + kh*dh, ow*sw - pw + kw*dw, c])
  *   desc    geometry with C_in == C_out == C; C % 4 == 0 (fp32) or % 8 (bf16).
- *   W       DEVICE fp32 [C][KH][KW]; bias nullable DEVICE fp32 [C].
+ *   W       DEVICE fp32 [C][KH][KW], 16-byte aligned; bias nullable DEVICE fp32 [C].
  *   x, y    DEVICE NHWC of dtype (ONEXN_F32 / ONEXN_BF16; bf16 outputs are
  *           the RNE of the fp32 result), 16-byte aligned, not overlapping.
  *   flags   0, ONEXN_RELU or ONEXN_RELU6.

@@ -21,6 +21,8 @@ cudaError_t tc_gemm(const ConvArgs &a, int dtype, const void *workspace, size_t 
 bool tc_supports(const ConvArgs &a, int dtype);
 size_t tc_workspace_bytes(const ConvArgs &a, int dtype);
 size_t tc_workspace_min(const ConvArgs &a, int dtype);
+// AUTO's time estimate of the tensor-core family (ns; fixed costs relative to FFMA's)
+double tc_cost_ns(const ConvArgs &a, int dtype, size_t ws_bytes, bool decoded);
 
 namespace detail {
 

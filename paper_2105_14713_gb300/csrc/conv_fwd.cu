@@ -87,7 +87,8 @@ onexn_status check_shape(const onexn_conv_desc *d, int N, int64_t t, int dtype, 
     if (d->C_in % cv)
         return fail(ONEXN_EINVAL, "conv: C_in=%d must be a multiple of %d for %s", d->C_in, cv,
                     dtype == ONEXN_F32 ? "fp32" : "bf16");
-    if (flags & ~(ONEXN_RELU | ONEXN_RELU6 | ONEXN_ALGO_MASK)) return fail(ONEXN_EINVAL, "conv: unknown flags");
+    if (flags & ~(ONEXN_RELU | ONEXN_RELU6 | ONEXN_DECODED | ONEXN_REUSE_DECODE | ONEXN_ALGO_MASK))
+        return fail(ONEXN_EINVAL, "conv: unknown flags");
     a->B = d->B; a->H = d->H; a->W = d->W; a->C = d->C_in;
     a->C_out = d->C_out; a->KH = d->KH; a->KW = d->KW;
     a->sh = d->stride_h; a->sw = d->stride_w; a->ph = d->pad_h; a->pw = d->pad_w;
@@ -143,37 +144,54 @@ bool supports(unsigned algo, const onexn::ConvArgs &a, int dtype)
     }
 }
 
-// Cost model of AUTO, in ns per multiply-add, fitted to GB300 timings of a
-// 3x3 512->512 layer on 128x14x14 at 50% and 90% pruned (fp32 and bf16; the
-// affine fit predicts the 70% point within 2%).  The FFMA kernel stages the
-// activations of every 256-pixel x 64-column unit whatever is kept (a floor
-// per dense multiply-add, higher for small N) and then does only the kept
-// work (t*N weights per pixel), faster for wider blocks that share each
-// staged activation.  The tensor-core GEMM decodes the weights into the
-// workspace (about 2000 bytes per ns) and does the dense work (C_out*K per
-// pixel; fp32 issues three tf32 products per term).
+// Cost model of AUTO.  The machine rates, in ns per multiply-add, are
+// fitted to GB300 timings of a 3x3 512->512 layer on 128x14x14 at 50% and
+// 90% pruned (fp32 and bf16; the affine fit predicts the 70% point within
+// 2%).  The FFMA kernel stages the activations of every 256-pixel x
+// 64-column unit whatever is kept (a floor per dense multiply-add, higher
+// for small N) and then does only the kept work (t*N weights per pixel),
+// faster for wider blocks that share each staged activation.  A unit runs
+// on one SM, so a launch with fewer units than SMs (batch-1 layers: a 7x7
+// output is one unit of pixels) takes 152 / units times the machine-rate
+// time, on pixels and columns padded to whole units.  The tensor-core
+// family's estimate is tc_cost_ns (conv_tc.cu).  Measured on GB300 at batch
+// 1, the FFMA kernel loses to the decoded GEMM on every MobileNet-V2 1x1
+// layer from 14x14 down (e.g. 76 vs 17 us on the 7x7 960->160 projection).
 namespace {
 double fma_floor(int N) { return N >= 4 ? 1.33e-5 : N >= 2 ? 1.66e-5 : 2.67e-5; }
 double fma_per_kept(int N) { return N >= 8 ? 3.0e-5 : N >= 4 ? 4.3e-5 : N >= 2 ? 7.2e-5 : 1.44e-4; }
-double tc_per_dense(int dtype) { return dtype == ONEXN_F32 ? 7.9e-6 : 2.3e-6; }
-constexpr double kDecodeNsPerByte = 1.0 / 2000.0;
+constexpr int kFmaUnitPix = 256, kFmaUnitCols = 64, kSms = 152;
+constexpr double kFmaFixedNs = 700.0;     // pipeline fill beyond a bare launch
+
+double fma_cost_ns(const onexn::ConvArgs &a)
+{
+    const int64_t um = (static_cast<int64_t>(a.P_pix) + kFmaUnitPix - 1) / kFmaUnitPix;
+    const int64_t un = (a.C_out + kFmaUnitCols - 1) / kFmaUnitCols;
+    const int64_t units = um * un;
+    const double pix = static_cast<double>(um * kFmaUnitPix);          // padded pixels
+    const double col_pad = static_cast<double>(un * kFmaUnitCols) / a.C_out;
+    const double K = static_cast<double>(a.KH) * a.KW * a.C;
+    const double floor_ns = pix * a.C_out * col_pad * K * fma_floor(a.N);
+    const double kept_ns = pix * static_cast<double>(a.t) * a.N * fma_per_kept(a.N);
+    const double waves = static_cast<double>((units + kSms - 1) / kSms);
+    return (floor_ns + kept_ns) * kSms * waves / static_cast<double>(units) + kFmaFixedNs;
+}
 }  // namespace
 
 // Kernel family for AUTO: the tcgen05 GEMM when its workspace fits and the
 // cost model does not expect the FFMA kernel to be faster; otherwise FFMA.
+// With ONEXN_DECODED the weights are already decoded: the GEMM.  With
+// ONEXN_REUSE_DECODE the caller will keep the decode, so it is left out.
 unsigned pick_algo(const onexn::ConvArgs &a, int dtype, unsigned flags, size_t ws_bytes)
 {
     const unsigned forced = flags & ONEXN_ALGO_MASK;
     if (forced != ONEXN_ALGO_AUTO) return forced;
+    if (flags & ONEXN_DECODED) return ONEXN_ALGO_TC;
     if (!supports(ONEXN_ALGO_TC, a, dtype) || ws_bytes < workspace_min_for(ONEXN_ALGO_TC, a, dtype))
         return ONEXN_ALGO_FMA;
-    if (a.t == 0) return ONEXN_ALGO_FMA;                  // bias only
-    const double kept = static_cast<double>(a.t) * a.N * a.P_pix;
-    const double dense = static_cast<double>(a.C_out) * a.KH * a.KW * a.C * a.P_pix;
-    const double fma_ns = dense * fma_floor(a.N) + kept * fma_per_kept(a.N);
-    const double tc_ns = dense * tc_per_dense(dtype) +
-                         static_cast<double>(workspace_min_for(ONEXN_ALGO_TC, a, dtype)) * kDecodeNsPerByte;
-    return fma_ns < tc_ns ? ONEXN_ALGO_FMA : ONEXN_ALGO_TC;
+    if (a.t == 0 || a.P_pix == 0) return ONEXN_ALGO_FMA;  // bias only / nothing to do
+    const bool amortised = (flags & ONEXN_REUSE_DECODE) != 0;
+    return fma_cost_ns(a) < onexn::tc_cost_ns(a, dtype, ws_bytes, amortised) ? ONEXN_ALGO_FMA : ONEXN_ALGO_TC;
 }
 
 onexn_status check_algo(unsigned algo, const onexn::ConvArgs &a, int dtype, size_t ws_bytes)
@@ -214,6 +232,8 @@ extern "C" onexn_status onexn_conv_algo(const onexn_conv_desc *desc, int N, int6
     const unsigned al = pick_algo(a, dtype, flags, workspace_bytes);
     st = check_algo(al, a, dtype, workspace_bytes);
     if (st != ONEXN_OK) return st;
+    if ((flags & ONEXN_DECODED) && al != ONEXN_ALGO_TC)
+        return fail(ONEXN_EINVAL, "conv: ONEXN_DECODED needs the tc family");
     *algo = al;
     return ONEXN_OK;
 }
@@ -267,10 +287,12 @@ extern "C" onexn_status onexn_conv_fwd_ex(const onexn_conv_desc *desc, const int
     const unsigned algo = pick_algo(a, dtype, flags, workspace_bytes);
     st = check_algo(algo, a, dtype, workspace_bytes);
     if (st != ONEXN_OK) return st;
+    const bool decoded = (flags & ONEXN_DECODED) != 0;
+    if (decoded && algo != ONEXN_ALGO_TC) return fail(ONEXN_EINVAL, "conv: ONEXN_DECODED needs the tc family");
     cudaStream_t s = static_cast<cudaStream_t>(stream);
     cudaError_t e = onexn::device_status_ptr(&a.status);
     if (e != cudaSuccess) return fail(ONEXN_ECUDA, "conv: status word: %s", cudaGetErrorString(e));
-    e = launch(algo, a, dtype, workspace, workspace_bytes, s);
+    e = decoded ? tc_gemm(a, dtype, workspace, workspace_bytes, s) : launch(algo, a, dtype, workspace, workspace_bytes, s);
     if (e != cudaSuccess) return fail(ONEXN_ECUDA, "conv: launch failed: %s", cudaGetErrorString(e));
     return ONEXN_OK;
 }

@@ -102,6 +102,8 @@ struct HostPlan {
 
 onexn_status plan(const onexn_conv_desc *desc, int N, int64_t t, int dtype, unsigned flags, HostPlan *hp)
 {
+    if (flags & (ONEXN_DECODED | ONEXN_REUSE_DECODE))      // every call decodes into its own workspace
+        return onexn::fail(ONEXN_EINVAL, "conv_host: ONEXN_DECODED / ONEXN_REUSE_DECODE are not accepted here");
     onexn_status st = onexn::detail::check_shape(desc, N, t, dtype, flags, &hp->a);
     if (st != ONEXN_OK) return st;
     const onexn::ConvArgs &a = hp->a;

@@ -76,6 +76,8 @@ extern "C" onexn_status onexn_conv_fwd_noalloc(const onexn_conv_desc *desc, cons
     onexn::clear_error();
     if ((flags & ONEXN_ALGO_MASK) != ONEXN_ALGO_AUTO && (flags & ONEXN_ALGO_MASK) != ONEXN_ALGO_TC)
         return onexn::fail(ONEXN_EINVAL, "conv_noalloc: only the tensor-core family runs here");
+    if (flags & (ONEXN_DECODED | ONEXN_REUSE_DECODE))      // the scratch is shared by every layer
+        return onexn::fail(ONEXN_EINVAL, "conv_noalloc: ONEXN_DECODED / ONEXN_REUSE_DECODE are not accepted here");
     const unsigned f = (flags & ~ONEXN_ALGO_MASK) | ONEXN_ALGO_TC;
     onexn::ConvArgs a{};
     onexn_status st = onexn::detail::check_shape(desc, N, t, dtype, f, &a);

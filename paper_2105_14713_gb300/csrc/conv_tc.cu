@@ -54,6 +54,7 @@
 #include <cuda.h>
 #include <cudaTypedefs.h>
 
+#include <algorithm>
 #include <cstring>
 #include <mutex>
 
@@ -89,6 +90,12 @@ constexpr int kSmemMax = 232448;      // dynamic shared memory per CTA (opt-in m
 constexpr int kAccMax = 4;            // accumulator buffers in TMEM at most
 constexpr int kPlanCTAs = 152;        // stream-K: at most this many CTAs (GB300's SM count)
 constexpr int kMinSplitIters = 4;     // stream-K: at least this many chunk iterations per CTA
+
+// Stream-K moves partial tiles through global memory and makes a finisher
+// wait for them; on GB300 that pays only when a tile's own K loop is long:
+// from 16 chunks per tile for fp32 (three tf32 MMAs per chunk) and 32 for
+// bf16, measured on batch-1 MobileNet-V2 and ResNet-50 layers.
+constexpr int sk_min_chunks(bool split) { return split ? 16 : 32; }
 
 // one partial slot (128 x BN fp32) per CTA
 constexpr size_t sk_partial_bytes(int BN) { return static_cast<size_t>(kPlanCTAs) * kBM * BN * 4; }
@@ -316,10 +323,13 @@ tc_conv_kernel(const ConvArgs a, const __grid_constant__ CUtensorMap tmap_x,
     __syncthreads();
     tc::fence_after_sync();
     const uint32_t tmem = *holder;
-    // Launched as a programmatic dependent of the weight decode: everything
-    // above overlapped the decode; global memory is touched only after it
-    // (and everything before it on the stream) has completed.
+    // Launched as a programmatic dependent of the previous kernel on the
+    // stream (the weight decode, or the layer before): everything above
+    // overlapped it; global memory is touched only after it (and everything
+    // before it on the stream) has completed.  The next kernel may then
+    // start its own prologue (it waits the same way before reading).
     asm volatile("griddepcontrol.wait;\n" ::: "memory");
+    asm volatile("griddepcontrol.launch_dependents;\n" ::: "memory");
 
     const int n_cchunk = (a.C + Tr::kBK - 1) / Tr::kBK;
     const int n_tn = sched.n_tn;
@@ -796,7 +806,7 @@ bool tmap_2d(CUtensorMap *m, CUtensorMapDataType type, int elem, const void *ptr
 
 template <typename Tr, int BN>
 cudaError_t launch_bn(const ConvArgs &a, const typename Tr::T *W, const typename Tr::T *W_lo, void *sk_space,
-                      bool after_decode, cudaStream_t st)
+                      cudaStream_t st)
 {
     using L = TcLayout<Tr, BN>;
     constexpr int elem = sizeof(typename Tr::T);
@@ -888,7 +898,7 @@ cudaError_t launch_bn(const ConvArgs &a, const typename Tr::T *W, const typename
     // leaving the round ragged: the fixup and the shorter segments cost more
     // than the idle SMs.)
     const int G = sms < kPlanCTAs ? sms : kPlanCTAs;
-    if (sk_space && sc.n_tiles < G) {
+    if (sk_space && sc.n_tiles < G && sc.n_chunks >= sk_min_chunks(Tr::kSplit)) {
         const int dp = (sc.n_tiles / G) * G, skt = sc.n_tiles - dp;
         const int64_t iters = static_cast<int64_t>(skt) * sc.n_chunks;
         int need = (sc.n_chunks + L::kRingSlots - 1) / L::kRingSlots;
@@ -910,7 +920,10 @@ cudaError_t launch_bn(const ConvArgs &a, const typename Tr::T *W, const typename
     cfg.stream = st;
     cudaLaunchAttribute attr[1];
     attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-    attr[0].val.programmaticStreamSerializationAllowed = after_decode ? 1 : 0;
+    // always a programmatic dependent of the previous kernel on the stream
+    // (the decode, or the previous layer): the kernel touches global memory
+    // only after griddepcontrol.wait
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
     return cudaLaunchKernelEx(&cfg, kern, a, tmap_x, tmap_w, tmap_wlo, tmap_y, sc, a_tiled);
@@ -970,8 +983,7 @@ cudaError_t decode_typed(const ConvArgs &a, void *workspace, size_t ws_bytes, cu
 }
 
 template <typename Tr>
-cudaError_t gemm_typed(const ConvArgs &a, const void *workspace, size_t ws_bytes, bool after_decode,
-                       cudaStream_t st)
+cudaError_t gemm_typed(const ConvArgs &a, const void *workspace, size_t ws_bytes, cudaStream_t st)
 {
     using T = typename Tr::T;
     const size_t n = static_cast<size_t>(a.C_out) * a.KH * a.KW * a.C;
@@ -982,12 +994,46 @@ cudaError_t gemm_typed(const ConvArgs &a, const void *workspace, size_t ws_bytes
                    ? static_cast<void *>(static_cast<unsigned char *>(const_cast<void *>(workspace)) + wb)
                    : nullptr;
     const int bn = tc_bn(a);
-    if (bn == 64) return launch_bn<Tr, 64>(a, W, W_lo, sk, after_decode, st);
-    if (bn == 128) return launch_bn<Tr, 128>(a, W, W_lo, sk, after_decode, st);
-    return launch_bn<Tr, 256>(a, W, W_lo, sk, after_decode, st);
+    if (bn == 64) return launch_bn<Tr, 64>(a, W, W_lo, sk, st);
+    if (bn == 128) return launch_bn<Tr, 128>(a, W, W_lo, sk, st);
+    return launch_bn<Tr, 256>(a, W, W_lo, sk, st);
 }
 
 }  // namespace
+
+// Estimated time of the family (ns), for AUTO: the dense GEMM on the
+// decoded weights (padded to whole tiles) at the machine rate measured on
+// full-GPU layers (per multiply-add: fp32 as three tf32 products 7.9e-6 ns,
+// bf16 2.3e-6 ns), scaled by 152 / the CTAs busy on average (fewer tiles,
+// or stream-K pieces, than SMs; a ragged last round), plus fixed costs
+// measured on GB300 against batch-1 layers: the GEMM's prologue, the
+// stream-K fixup (partial tiles out, the finisher's wait and reads), and
+// the decode launch unless the weights are already decoded.
+double tc_cost_ns(const ConvArgs &a, int dtype, size_t ws_bytes, bool decoded)
+{
+    constexpr double kGemmFixedNs = 1200.0, kSkFixupNs = 7000.0, kDecodeFixedNs = 2000.0,
+                     kDecodeBytesPerNs = 2000.0;
+    const bool f32 = dtype == ONEXN_F32;
+    const int bn = tc_bn(a);
+    const int bk = f32 ? TcF32::kBK : TcBf16::kBK;
+    const int64_t n_m = (static_cast<int64_t>(a.P_pix) + kBM - 1) / kBM, n_n = (a.C_out + bn - 1) / bn;
+    const int64_t tiles = n_m * n_n, chunks = static_cast<int64_t>(a.KH) * a.KW * ((a.C + bk - 1) / bk);
+    const size_t wb = weights_bytes(a, dtype);
+    const bool sk = ws_bytes >= wb + sk_bytes(a) && tiles < kPlanCTAs && chunks >= sk_min_chunks(f32);
+    double busy;
+    if (tiles >= kPlanCTAs)
+        busy = static_cast<double>(tiles) / static_cast<double>((tiles + kPlanCTAs - 1) / kPlanCTAs);
+    else if (sk)
+        busy = std::min<double>(kPlanCTAs, static_cast<double>(tiles * chunks) / kMinSplitIters);
+    else
+        busy = static_cast<double>(tiles);
+    const double dense = static_cast<double>(n_m * kBM) * static_cast<double>(n_n * bn) *
+                         static_cast<double>(a.KH * a.KW * a.C);
+    double ns = dense * (f32 ? 7.9e-6 : 2.3e-6) * kPlanCTAs / busy + kGemmFixedNs;
+    if (sk) ns += kSkFixupNs;
+    if (!decoded) ns += kDecodeFixedNs + static_cast<double>(wb) / kDecodeBytesPerNs;
+    return ns;
+}
 
 // The decoded weights; with room for the stream-K partial slots and
 // flags after them the GEMM also balances its last round of tiles.
@@ -1017,18 +1063,17 @@ cudaError_t tc_decode(const ConvArgs &a, int dtype, void *workspace, size_t ws_b
 }
 
 namespace {
-cudaError_t gemm_any(const ConvArgs &a, int dtype, const void *workspace, size_t ws_bytes, bool after_decode,
-                     cudaStream_t st)
+cudaError_t gemm_any(const ConvArgs &a, int dtype, const void *workspace, size_t ws_bytes, cudaStream_t st)
 {
     if (a.P_pix == 0) return cudaSuccess;
-    return dtype == ONEXN_F32 ? gemm_typed<TcF32>(a, workspace, ws_bytes, after_decode, st)
-                              : gemm_typed<TcBf16>(a, workspace, ws_bytes, after_decode, st);
+    return dtype == ONEXN_F32 ? gemm_typed<TcF32>(a, workspace, ws_bytes, st)
+                              : gemm_typed<TcBf16>(a, workspace, ws_bytes, st);
 }
 }  // namespace
 
 cudaError_t tc_gemm(const ConvArgs &a, int dtype, const void *workspace, size_t ws_bytes, cudaStream_t st)
 {
-    return gemm_any(a, dtype, workspace, ws_bytes, false, st);
+    return gemm_any(a, dtype, workspace, ws_bytes, st);
 }
 
 // decode, then the GEMM as its programmatic dependent (its launch and
@@ -1037,7 +1082,7 @@ cudaError_t launch_tc(const ConvArgs &a, int dtype, void *workspace, size_t ws_b
 {
     if (a.P_pix == 0) return cudaSuccess;
     const cudaError_t e = tc_decode(a, dtype, workspace, ws_bytes, st);
-    return e != cudaSuccess ? e : gemm_any(a, dtype, workspace, ws_bytes, true, st);
+    return e != cudaSuccess ? e : gemm_any(a, dtype, workspace, ws_bytes, st);
 }
 
 }  // namespace onexn

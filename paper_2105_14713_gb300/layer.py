@@ -28,8 +28,9 @@ def act_flags(relu) -> int:
 class PrunedConv2d:
     def __init__(self, weight, N: int, rate: float, *, bias=None, stride=1, padding=0,
                  dilation=1, dtype: str = "f32", gran: int = _c.ONEXN_GRAN_TAP,
-                 device="cuda", mask=None):
+                 device="cuda", mask=None, reuse_decoded: bool = True):
         W = np.ascontiguousarray(np.asarray(weight, np.float32))
+        self.reuse_decoded = bool(reuse_decoded)
         self.C_out, self.C_in, self.KH, self.KW = W.shape
         self.N = int(N)
         self.rate = float(rate)
@@ -62,6 +63,9 @@ class PrunedConv2d:
         self._ws = {}            # per input shape: device workspace (bytes as uint8)
         self._args = {}          # per buffers / layout / flags / stream: marshalled C arguments
         self._descs = []
+        # workspaces whose decoded weights a completed-in-order tc call has
+        # written: later calls on them pass ONEXN_DECODED and skip the decode
+        self._decoded = set()
 
     @property
     def torch_dtype(self):
@@ -85,10 +89,14 @@ class PrunedConv2d:
             self._ws[key] = torch.empty(max(n, 256), dtype=torch.uint8, device=self.device) if n else None
         return self._ws[key]
 
+    def _reuse_flag(self) -> int:
+        return _c.ONEXN_REUSE_DECODE if self.reuse_decoded else 0
+
     def algo(self, x_shape, flags: int = 0) -> str:
+        """The family forward runs for this input shape (and forced flags)."""
         B, H, W, _ = x_shape
         ws = self.workspace(x_shape, flags)
-        a = _c.onexn_conv_algo(self.desc(B, H, W), self.N, self.t, self.cdtype, flags,
+        a = _c.onexn_conv_algo(self.desc(B, H, W), self.N, self.t, self.cdtype, flags | self._reuse_flag(),
                                0 if ws is None else ws.numel())
         return _c.ALGO_NAMES[a]
 
@@ -104,7 +112,7 @@ class PrunedConv2d:
         if y is None:
             y = torch.empty(self.out_shape(x.shape), dtype=x.dtype, device=x.device)
         s = torch.cuda.current_stream(x.device) if stream is None else stream
-        flags = act_flags(relu) | algo
+        flags = act_flags(relu) | algo | self._reuse_flag()
         key = (x.data_ptr(), y.data_ptr(), x.shape, x.stride(), x.dtype, y.shape, y.stride(), y.dtype,
                None if residual is None else (residual.data_ptr(), residual.shape, residual.stride(),
                                               residual.dtype),
@@ -116,9 +124,15 @@ class PrunedConv2d:
                 self._descs.clear()
             args = self._marshal(x, y, flags, s, residual)
             self._args[key] = args
-        st = _c.lib.onexn_conv_fwd_ex(*args)
+        st = _c.lib.onexn_conv_fwd_ex(*args[0])
         if st != _c.ONEXN_OK:
             raise _c.OnexnError(st, _c.lib.onexn_last_error().decode(errors="replace"))
+        if args[1] is not None and args[1] not in self._decoded:
+            # this call decoded the weights into the workspace: later calls
+            # (ordered after it on the caller's streams, as calls sharing a
+            # workspace must be) run the GEMM alone
+            self._decoded.add(args[1])
+            self._args.pop(key, None)
         return y
 
     def _marshal(self, x, y, flags, s, residual=None):
@@ -137,10 +151,20 @@ class PrunedConv2d:
         ws = self.workspace(x.shape, flags & _c.ONEXN_ALGO_MASK)
         ptr = (lambda t: None if t is None else ctypes.c_void_p(t.data_ptr()))
         ws_bytes = 0 if ws is None else ws.numel()
+        # the tc family decodes the weights into the workspace; once that has
+        # happened on this workspace, skip it (ONEXN_DECODED)
+        ws_key = None
+        if ws is not None and self.reuse_decoded:
+            al = _c.onexn_conv_algo(desc, self.N, self.t, self.cdtype, flags, ws_bytes)
+            if al == _c.ONEXN_ALGO_TC:
+                ws_key = ws.data_ptr()
+                if ws_key in self._decoded:
+                    flags |= _c.ONEXN_DECODED
+                    ws_key = None
         self._descs.append(desc)                 # kept alive for the cached byref
-        return (ctypes.byref(desc), ptr(self.P), ptr(self.I), ptr(self.D), self.N, self.t, ptr(x), ptr(y),
-                ptr(self.bias), ptr(residual), self.cdtype, flags, ptr(ws), ws_bytes,
-                ctypes.c_void_p(s.cuda_stream))
+        return ((ctypes.byref(desc), ptr(self.P), ptr(self.I), ptr(self.D), self.N, self.t, ptr(x), ptr(y),
+                 ptr(self.bias), ptr(residual), self.cdtype, flags, ptr(ws), ws_bytes,
+                 ctypes.c_void_p(s.cuda_stream)), ws_key)
 
     __call__ = forward
 

@@ -18,6 +18,8 @@ ONEXN_F32, ONEXN_BF16 = 0, 1
 ONEXN_GRAN_TAP, ONEXN_GRAN_KERNEL = 0, 1
 ONEXN_RELU = 0x1
 ONEXN_RELU6 = 0x2
+ONEXN_DECODED = 0x10
+ONEXN_REUSE_DECODE = 0x20
 ONEXN_ALGO_SHIFT = 8
 ONEXN_ALGO_MASK = 0xF << ONEXN_ALGO_SHIFT
 ONEXN_ALGO_AUTO = 0 << ONEXN_ALGO_SHIFT

@@ -12,7 +12,7 @@ import torch
 
 from paper_2105_14713_gb300 import onexn as ox
 from paper_2105_14713_gb300 import workloads as wl
-from tests.gpu_util import norm_err, run_layer, tol
+from tests.gpu_util import norm_err, oracle_ref, run_layer, to_device_input, tol
 
 pytestmark = pytest.mark.gpu
 
@@ -156,6 +156,32 @@ def test_streams_and_repeat_calls_are_deterministic():
         y2 = conv(x)
     s.synchronize()
     assert torch.equal(y1, y2)
+
+
+def test_decoded_weights_reused_across_calls():
+    """After one tc call a layer passes ONEXN_DECODED and runs the GEMM
+    alone; results stay bitwise equal, including the stream-K split tiles
+    (8 pixel tiles < 152 SMs), whose flags the finisher resets for the next
+    launch."""
+    from paper_2105_14713_gb300.layer import PrunedConv2d
+    for dt, seed in (("f32", 31), ("bf16", 32)):
+        layer = L("decoded", 4, 16, 16, 64, 64, 3, 3, 1, 1, 1, N=8, rate=0.5, dtype=dt, seed=seed)
+        W, b = wl.weights(layer).numpy(), wl.bias(layer).numpy()
+        conv = PrunedConv2d(W, 8, 0.5, padding=1, bias=b, dtype=dt)
+        fresh = PrunedConv2d(W, 8, 0.5, padding=1, bias=b, dtype=dt, reuse_decoded=False)
+        x = to_device_input(wl.activations(layer), dt)
+        assert conv.algo(x.shape) == "tc"
+        ys = [conv(x).clone() for _ in range(3)]
+        assert len(conv._decoded) == 1
+        flags = [args[0][11] for args in conv._args.values()]
+        assert flags and all(f & ox.ONEXN_DECODED for f in flags)
+        y_ref = fresh(x)
+        assert not fresh._decoded
+        for y in ys:
+            assert torch.equal(y, y_ref)
+        yr, a = oracle_ref(layer, W, wl.activations(layer), b)
+        yo = y_ref.float().cpu().numpy().reshape(-1, 64).astype(np.float64)
+        assert norm_err(yo, yr, a) <= tol(layer)
 
 
 # ------------------------------------------------ host-memory entry point

@@ -191,17 +191,44 @@ def test_auto_cost_model():
     # 3x3 128->128 (K = 1152, 16 groups of N = 8): the tensor-core GEMM does
     # all 128 * 1152 products per pixel after decoding the weights, the FFMA
     # kernel only the kept t * N.  On 50176 pixels the GEMM wins even at 99%
-    # pruned; on 4 pixels the decode dominates and FFMA wins when most blocks
-    # are pruned.
+    # pruned.  On 4 pixels the FFMA kernel has 2 units of 256 pixels x 64
+    # columns for 152 SMs, while the GEMM splits its 2 tiles' 36 K chunks
+    # over 18 CTAs (stream-K): the GEMM wins there too.  With a tiny K
+    # (8 -> 16, 3x3, one kept block) the decode launch is the larger cost.
     G, K = 128 // 8, 9 * 128
     big = ox.make_desc(64, 28, 28, 128, 128, 3, 3, 1, 1, 1)
-    tiny = ox.make_desc(1, 2, 2, 128, 128, 3, 3, 1, 1, 1)
+    four = ox.make_desc(1, 2, 2, 128, 128, 3, 3, 1, 1, 1)
     for dt in (ox.ONEXN_F32, ox.ONEXN_BF16):
         ws = ox.onexn_conv_workspace_size(big, 8, G * K, dt)
         assert ox.onexn_conv_algo(big, 8, G * K // 2, dt, 0, ws) == ox.ONEXN_ALGO_TC      # 50% pruned
         assert ox.onexn_conv_algo(big, 8, G * K // 100, dt, 0, ws) == ox.ONEXN_ALGO_TC    # 99% pruned
         assert ox.onexn_conv_algo(big, 8, 0, dt, 0, ws) == ox.ONEXN_ALGO_FMA              # all pruned
-        assert ox.onexn_conv_algo(tiny, 8, G * K // 10, dt, 0, ws) == ox.ONEXN_ALGO_FMA
+        ws4 = ox.onexn_conv_workspace_size(four, 8, G * K, dt)
+        assert ox.onexn_conv_algo(four, 8, G * K // 10, dt, 0, ws4) == ox.ONEXN_ALGO_TC
+    tiny = ox.make_desc(1, 2, 2, 8, 16, 3, 3, 1, 1, 1)
+    assert ox.onexn_conv_algo(tiny, 8, 1, ox.ONEXN_F32, 0, 1 << 20) == ox.ONEXN_ALGO_FMA
+    # ... unless the caller keeps the decode for later calls
+    assert ox.onexn_conv_algo(tiny, 8, 1, ox.ONEXN_F32, ox.ONEXN_REUSE_DECODE, 1 << 20) == ox.ONEXN_ALGO_TC
+
+
+def test_auto_batch1_mobilenet_v2_layers_pick_the_gemm():
+    """Batch-1 MobileNet-V2 1x1 layers (N=4, 50%): with its workspace and the
+    decode amortised (ONEXN_REUSE_DECODE, as the layer object passes), the
+    tensor-core family on every layer from 28x28 down (measured on GB300:
+    the FFMA kernel is 1.2-4.5x slower there, e.g. 76 vs 17 us on the 7x7
+    960 -> 160 projection), in fp32 and bf16."""
+    for blk in wl.config7():
+        shapes = [(blk.hw, blk.c_in, blk.hidden)] if blk.hidden != blk.c_in else []
+        shapes.append((blk.hw_out, blk.hidden, blk.c_out))
+        for hw, ci, co in shapes:
+            if hw > 28:
+                continue
+            d = ox.make_desc(1, hw, hw, ci, co)
+            t = (co // 4) * ci // 2
+            for dt in (ox.ONEXN_F32, ox.ONEXN_BF16):
+                ws = ox.onexn_conv_workspace_size(d, 4, t, dt)
+                assert ox.onexn_conv_algo(d, 4, t, dt, ox.ONEXN_REUSE_DECODE, ws) == ox.ONEXN_ALGO_TC, \
+                    (blk.name, hw, ci, co, dt)
 
 
 def test_host_entry_workspace_and_argument_checks_need_no_gpu():
@@ -314,3 +341,26 @@ def test_dwconv_argument_errors_need_no_gpu():
     # an empty batch is a no-op that needs no device
     d0 = ox.make_desc(0, 4, 4, 16, 16, 3, 3, 1, 1, 1)
     assert dw(ctypes.byref(d0), None, None, None, None, ox.ONEXN_F32, 0, None) == ox.ONEXN_OK
+
+
+def test_decoded_flag_selects_tc_and_is_checked():
+    """ONEXN_DECODED (weights already decoded in the workspace) implies the
+    tc family: AUTO resolves to it, another forced family is EINVAL, the
+    workspace must still hold the decoded weights, and the host-memory and
+    allocation-free entries refuse it."""
+    d = ox.make_desc(2, 7, 7, 8, 16, 3, 3, 1, 1, 1)
+    w32 = 16 * 9 * 8 * 8
+    D = ox.ONEXN_DECODED
+    assert ox.onexn_conv_algo(d, 8, 100, ox.ONEXN_F32, D, w32) == ox.ONEXN_ALGO_TC
+    assert ox.onexn_conv_algo(d, 8, 100, ox.ONEXN_F32, D | ox.ONEXN_ALGO_TC, w32) == ox.ONEXN_ALGO_TC
+    tiny = ox.make_desc(1, 2, 2, 8, 16, 3, 3, 1, 1, 1)           # AUTO alone would pick FFMA here
+    assert ox.onexn_conv_algo(tiny, 8, 1, ox.ONEXN_F32, 0, w32) == ox.ONEXN_ALGO_FMA
+    assert ox.onexn_conv_algo(tiny, 8, 1, ox.ONEXN_F32, D, w32) == ox.ONEXN_ALGO_TC
+    assert _status(ox.onexn_conv_algo, d, 8, 100, ox.ONEXN_F32, D | ox.ONEXN_ALGO_FMA, w32) == ox.ONEXN_EINVAL
+    assert _status(ox.onexn_conv_algo, d, 8, 100, ox.ONEXN_F32, D, w32 - 1) == ox.ONEXN_EINVAL
+    assert _status(ox.onexn_conv_host_workspace_size, d, 8, 100, ox.ONEXN_F32, D) == ox.ONEXN_EINVAL
+    assert _status(ox.onexn_conv_host_workspace_size, d, 8, 100, ox.ONEXN_F32, ox.ONEXN_REUSE_DECODE) == \
+        ox.ONEXN_EINVAL
+    st = ox.lib.onexn_conv_fwd_noalloc(ctypes.byref(d), None, None, None, 8, 100, None, None, None,
+                                       ox.ONEXN_F32, D, None)
+    assert st == ox.ONEXN_EINVAL and b"DECODED" in ox.lib.onexn_last_error()

@@ -62,6 +62,26 @@ def test_depthwise_conv(dtype, stride, relu):
 
 
 @pytest.mark.parametrize("dtype", ["f32", "bf16"])
+@pytest.mark.parametrize("k,stride,pad,dil", [(5, 1, 4, 2), (1, 2, 0, 1), (5, 2, 2, 1)])
+def test_depthwise_conv_other_kernel_sizes(dtype, k, stride, pad, dil):
+    """The tap-by-tap form (any KH x KW), beside the unrolled 3x3 one."""
+    rng = np.random.default_rng(k * 100 + stride * 10 + dil)
+    C = 24 if dtype == "f32" else 32
+    x = torch.from_numpy(rng.standard_normal((2, 11, 9, C)).astype(np.float32))
+    W = rng.standard_normal((C, k, k)).astype(np.float32)
+    b = rng.standard_normal(C).astype(np.float32)
+    dw = DepthwiseConv2d(W, bias=b, stride=stride, padding=pad, dilation=dil, dtype=dtype)
+    xd = _dev(x, dtype)
+    y = _host32(dw(xd, relu=True))
+    xs = _host32(xd)
+    g = dict(stride=(stride, stride), pad=(pad, pad), dil=(dil, dil))
+    ref = oracle.dwconv(xs, W, b, relu=True, **g)
+    absacc = oracle.dwconv(np.abs(xs), np.abs(W), np.abs(b), **g)
+    assert y.shape == ref.shape
+    assert _err(y, ref, absacc) <= TOL[dtype]
+
+
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
 @pytest.mark.parametrize("algo", ["fma", "tc"])
 @pytest.mark.parametrize("aliased", [False, True])
 def test_conv_with_residual_and_relu6(dtype, algo, aliased):
