@@ -17,6 +17,9 @@ Functions (each follows the passage named in its docstring):
 * ``conv_masked``  -- Eq. 6 masked direct convolution (+bias, ReLU)
 * ``conv_bsr``     -- Eq. 7 block-wise decode from (P, I, D)
 * ``round_bf16``   -- RNE rounding of fp32 to bfloat16 values
+* ``dwconv``       -- dense depthwise convolution of MobileNet-V2's block
+* ``conv_backward_data`` / ``conv_backward_weight`` / ``bsr_gather`` --
+  gradients of Eq. 6 with the mask held fixed (fine-tuning, Sec. 3.2/4.1)
 """
 from __future__ import annotations
 
@@ -82,6 +85,8 @@ def _load():
         lib.oracle_conv_bsr.argtypes = [P, P, P, P, i32, P, ctypes.POINTER(_Geom),
                                         i32, P, i64, P]
         lib.oracle_dwconv.argtypes = [P, P, P, ctypes.POINTER(_Geom), P]
+        lib.oracle_conv_backward_data.argtypes = [P, P, P, ctypes.POINTER(_Geom), i32, P, P]
+        lib.oracle_conv_backward_weight.argtypes = [P, P, P, ctypes.POINTER(_Geom), i32, P, P]
         lib.oracle_num_threads.restype = i32
         _lib = lib
         return lib
@@ -282,3 +287,60 @@ def conv_bsr(x, P, I, D, C_out, KH, KW, N, bias=None, stride=(1, 1), pad=(0, 0),
     _load().oracle_conv_bsr(_ptr(x), _ptr(P), _ptr(I), _ptr(D), dt, _ptr(bias),
                             ctypes.byref(g), N, _ptr(pix), n, _ptr(y))
     return y.reshape(B, Ho, Wo, C_out) if pix is None else y
+
+
+def conv_backward_data(dy, W, mask, N: int, in_hw, stride=(1, 1), pad=(0, 0), dil=(1, 1),
+                       want_abs=False):
+    """Gradient of Eq. 6's pre-activation output with respect to the input,
+    the mask held fixed: dx[b,ih,iw,c] = sum over (o, kh, kw, oh, ow) with
+    oh*s - p + kh*d = ih (and likewise for w) of mask * W[o,c,kh,kw] *
+    dy[b,oh,ow,o].  dy: [B, Ho, Wo, C_out] float32 (the values the GPU
+    sees); W: [C_out, C_in, KH, KW]; in_hw = (H, W) of the input.
+    Returns dx [B, H, W, C_in] fp64 (and sum of |terms| if want_abs)."""
+    dy, W = _c(dy, np.float32), _c(W, np.float32)
+    C_out, C_in, KH, KW = W.shape
+    B, Ho, Wo, Cy = dy.shape
+    H, Wd = in_hw
+    assert Cy == C_out and out_hw(H, Wd, KH, KW, stride, pad, dil) == (Ho, Wo)
+    g = _geom((B, H, Wd, C_in), C_out, KH, KW, stride, pad, dil, False)
+    mask = _c(mask, np.uint8)
+    dx = np.empty((B, H, Wd, C_in), np.float64)
+    a = np.empty_like(dx) if want_abs else None
+    _load().oracle_conv_backward_data(_ptr(dy), _ptr(W), _ptr(mask), ctypes.byref(g), N, _ptr(dx), _ptr(a))
+    return (dx, a) if want_abs else dx
+
+
+def conv_backward_weight(x, dy, kernel, mask, N: int, stride=(1, 1), pad=(0, 0), dil=(1, 1),
+                         want_abs=False):
+    """Gradient of Eq. 6's pre-activation output with respect to the kept
+    weights, the mask held fixed: dW[o,c,kh,kw] = mask * sum_{b,oh,ow}
+    dy[b,oh,ow,o] * x[b, oh*s - p + kh*d, ow*s - p + kw*d, c] (zero where
+    pruned).  x: [B, H, W, C_in], dy: [B, Ho, Wo, C_out] float32; kernel =
+    (KH, KW).  Returns dW [C_out, C_in, KH, KW] fp64 (and sum |terms|)."""
+    x, dy = _c(x, np.float32), _c(dy, np.float32)
+    KH, KW = kernel
+    B, H, Wd, C_in = x.shape
+    C_out = dy.shape[3]
+    assert dy.shape[:3] == (B,) + out_hw(H, Wd, KH, KW, stride, pad, dil)
+    g = _geom(x.shape, C_out, KH, KW, stride, pad, dil, False)
+    mask = _c(mask, np.uint8)
+    dW = np.empty((C_out, C_in, KH, KW), np.float64)
+    a = np.empty_like(dW) if want_abs else None
+    _load().oracle_conv_backward_weight(_ptr(x), _ptr(dy), _ptr(mask), ctypes.byref(g), N, _ptr(dW), _ptr(a))
+    return (dW, a) if want_abs else dW
+
+
+def bsr_gather(dW, P, I, N: int):
+    """The kept blocks of a dense [C_out, C_in, KH, KW] array in BSR order
+    (Sec. 3.4): out[z, n] = dW[g*N + n, c, kh, kw] for P[g] <= z < P[g+1]
+    and I[z] = (kh*KW + kw)*C_in + c.  Returns [t, N] (dW's dtype)."""
+    dW = np.asarray(dW)
+    C_out, C_in, KH, KW = dW.shape
+    P, I = np.asarray(P, np.int64), np.asarray(I, np.int64)
+    out = np.zeros((len(I), N), dW.dtype)
+    for g in range(C_out // N):
+        for z in range(P[g], P[g + 1]):
+            tap, c = divmod(int(I[z]), C_in)
+            kh, kw = divmod(tap, KW)
+            out[z] = dW[g * N:(g + 1) * N, c, kh, kw]
+    return out

@@ -44,6 +44,10 @@
  *   a direct NHWC convolution with zero padding, stride and dilation, with an
  *   optional per-output-channel bias and ReLU.
  *
+ *   Fine-tuning of the pruned network (Sec. 4.1) with the mask held fixed:
+ *   the gradients of that output with respect to the input and to the kept
+ *   weights, written from the definition of the convolution.
+ *
  * Build: gcc -O2 -fopenmp -ffp-contract=off -shared -fPIC oracle.c
  * (the only parallelism is an OpenMP loop over independent output pixels).
  */
@@ -413,6 +417,89 @@ void oracle_dwconv(const float *x, const float *W, const float *bias,
             y[p * g->C_in + c] = act(s, g->relu);
         }
     }
+}
+
+/* ------------------------------------------------------------------ */
+/* Fine-tuning with the mask held fixed (Sec. 3.2 keeps the selected    */
+/* blocks and Sec. 4.1 fine-tunes the pruned network; the pruned blocks  */
+/* stay zero): the gradients of Eq. 6's pre-activation output y with     */
+/* respect to the input and to the kept weights, from dy = dL/dy          */
+/* [B][Ho][Wo][C_out].  Written from the definition of y:                */
+/*   dx[b,ih,iw,c] = sum over (o, kh, kw, oh, ow) with                    */
+/*                   oh*sh - ph + kh*dh = ih and ow*sw - pw + kw*dw = iw   */
+/*                   of mask * W[o,c,kh,kw] * dy[b,oh,ow,o]               */
+/*   dW[o,c,kh,kw] = mask * sum_{b,oh,ow} dy[b,oh,ow,o]                   */
+/*                   * x[b, oh*sh - ph + kh*dh, ow*sw - pw + kw*dw, c]     */
+/* (zero padding: positions outside the image contribute nothing).       */
+/* absacc (nullable) = the same sums over |terms|.                       */
+/* ------------------------------------------------------------------ */
+static double dy_at(const float *dy, const oracle_geom *g, int Ho, int Wo, int b, int oh, int ow, int o)
+{
+    return (double)dy[(((int64_t)b * Ho + oh) * Wo + ow) * g->C_out + o];
+}
+
+void oracle_conv_backward_data(const float *dy, const float *W, const uint8_t *mask,
+                               const oracle_geom *g, int N, double *dx, double *absacc)
+{
+    int Ho = out_size(g->H, g->KH, g->sh, g->ph, g->dh);
+    int Wo = out_size(g->W, g->KW, g->sw, g->pw, g->dw);
+    int K = g->KH * g->KW * g->C_in;
+    int64_t total = (int64_t)g->B * g->H * g->W;
+#pragma omp parallel for schedule(dynamic, 16)
+    for (int64_t q = 0; q < total; q++) {
+        int b = (int)(q / ((int64_t)g->H * g->W));
+        int ih = (int)((q / g->W) % g->H), iw = (int)(q % g->W);
+        for (int c = 0; c < g->C_in; c++) {
+            double s = 0.0, a = 0.0;
+            for (int kh = 0; kh < g->KH; kh++) {
+                int th = ih + g->ph - kh * g->dh;          /* = oh * sh */
+                if (th < 0 || th % g->sh != 0 || th / g->sh >= Ho) continue;
+                for (int kw = 0; kw < g->KW; kw++) {
+                    int tw = iw + g->pw - kw * g->dw;      /* = ow * sw */
+                    if (tw < 0 || tw % g->sw != 0 || tw / g->sw >= Wo) continue;
+                    int k = (kh * g->KW + kw) * g->C_in + c;
+                    for (int o = 0; o < g->C_out; o++) {
+                        if (mask && !mask[(int64_t)(o / N) * K + k]) continue;
+                        double t = w_at(W, g->C_in, g->KH, g->KW, o, c, kh, kw) *
+                                   dy_at(dy, g, Ho, Wo, b, th / g->sh, tw / g->sw, o);
+                        s += t;
+                        a += fabs(t);
+                    }
+                }
+            }
+            dx[q * g->C_in + c] = s;
+            if (absacc) absacc[q * g->C_in + c] = a;
+        }
+    }
+}
+
+void oracle_conv_backward_weight(const float *x, const float *dy, const uint8_t *mask,
+                                 const oracle_geom *g, int N, double *dW, double *absacc)
+{
+    int Ho = out_size(g->H, g->KH, g->sh, g->ph, g->dh);
+    int Wo = out_size(g->W, g->KW, g->sw, g->pw, g->dw);
+    int K = g->KH * g->KW * g->C_in;
+#pragma omp parallel for schedule(dynamic, 1)
+    for (int o = 0; o < g->C_out; o++)
+        for (int c = 0; c < g->C_in; c++)
+            for (int kh = 0; kh < g->KH; kh++)
+                for (int kw = 0; kw < g->KW; kw++) {
+                    int k = (kh * g->KW + kw) * g->C_in + c;
+                    int64_t at = (((int64_t)o * g->C_in + c) * g->KH + kh) * g->KW + kw;
+                    double s = 0.0, a = 0.0;
+                    if (!mask || mask[(int64_t)(o / N) * K + k])
+                        for (int b = 0; b < g->B; b++)
+                            for (int oh = 0; oh < Ho; oh++)
+                                for (int ow = 0; ow < Wo; ow++) {
+                                    double t = dy_at(dy, g, Ho, Wo, b, oh, ow, o) *
+                                               x_at(x, g, b, oh * g->sh - g->ph + kh * g->dh,
+                                                    ow * g->sw - g->pw + kw * g->dw, c);
+                                    s += t;
+                                    a += fabs(t);
+                                }
+                    dW[at] = s;
+                    if (absacc) absacc[at] = a;
+                }
 }
 
 int oracle_num_threads(void)

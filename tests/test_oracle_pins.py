@@ -446,3 +446,118 @@ def test_residual_is_added_before_the_activation():
     assert np.array_equal(oracle.conv_masked(x, W, None, None, 1, residual=r), lin + r)
     assert np.array_equal(oracle.conv_masked(x, W, None, None, 1, residual=r, relu=True),
                           np.maximum(lin + r, 0.0))
+
+
+# --------------------------------------------------------------------------
+# Fine-tuning with the mask held fixed: gradients of Eq. 6
+# --------------------------------------------------------------------------
+
+def _bwd_case(case, rate, N=2, seed=0):
+    B, H, Wd, Ci, Co, KH, KW, s, p, d = case
+    rng = np.random.default_rng(sum(case) + seed)
+    x = rng.standard_normal((B, H, Wd, Ci)).astype(np.float32)
+    W = rng.standard_normal((Co, Ci, KH, KW)).astype(np.float32)
+    mask, _ = oracle.prune(W, N, rate)
+    Ho, Wo = oracle.out_hw(H, Wd, KH, KW, (s, s), (p, p), (d, d))
+    dy = rng.standard_normal((B, Ho, Wo, Co)).astype(np.float32)
+    return x, W, mask, dy, (s, s), (p, p), (d, d), rng
+
+
+def _mask_oihw(mask, N, shape):
+    """The [G][K] tap-major block mask expanded to W's [C_out, C_in, KH, KW]."""
+    Co, Ci, KH, KW = shape
+    m = np.repeat(mask, N, axis=0).reshape(Co, KH, KW, Ci)
+    return m.transpose(0, 3, 1, 2).astype(bool)
+
+
+@pytest.mark.parametrize("case", CONV_CASES)
+@pytest.mark.parametrize("rate", [0.0, 0.5])
+def test_backward_data_is_the_adjoint_of_the_forward(case, rate):
+    """<conv(x), dy> = <x, dx> for the masked convolution: a dropped kernel
+    flip, a transposed W, a stride/dilation slip or an ignored mask breaks
+    it (the forward is the independent Eq. 6 loop)."""
+    x, W, mask, dy, s, p, d, _ = _bwd_case(case, rate)
+    y = oracle.conv_masked(x, W, mask, None, 2, s, p, d)
+    dx = oracle.conv_backward_data(dy, W, mask, 2, x.shape[1:3], s, p, d)
+    lhs, rhs = float(np.sum(y * dy)), float(np.sum(x.astype(np.float64) * dx))
+    scale = float(np.sum(np.abs(y) * np.abs(dy))) + 1.0
+    assert abs(lhs - rhs) <= 1e-12 * scale
+
+
+@pytest.mark.parametrize("case", CONV_CASES)
+def test_backward_weight_is_the_bilinear_partner(case):
+    """<conv(x; W' (+) T), dy> = <W' (+) T, dW> for any W', and dW is zero
+    on every pruned weight."""
+    x, W, mask, dy, s, p, d, rng = _bwd_case(case, 0.5)
+    dW = oracle.conv_backward_weight(x, dy, W.shape[2:], mask, 2, s, p, d)
+    keep = _mask_oihw(mask, 2, W.shape)
+    assert np.all(dW[~keep] == 0.0)
+    W2 = rng.standard_normal(W.shape).astype(np.float32)
+    y2 = oracle.conv_masked(x, W2, mask, None, 2, s, p, d)
+    lhs = float(np.sum(y2 * dy))
+    rhs = float(np.sum(np.where(keep, W2.astype(np.float64), 0.0) * dW))
+    scale = float(np.sum(np.abs(y2) * np.abs(dy))) + 1.0
+    assert abs(lhs - rhs) <= 1e-12 * scale
+
+
+@pytest.mark.parametrize("case", CONV_CASES)
+def test_backward_matches_torch_grad_routines(case):
+    """Against torch.nn.grad.conv2d_input / conv2d_weight (fp64, NCHW) on the
+    masked weights, then the mask applied to the weight gradient."""
+    x, W, mask, dy, s, p, d, _ = _bwd_case(case, 0.5, seed=1)
+    keep = _mask_oihw(mask, 2, W.shape)
+    Wm = torch.from_numpy(np.where(keep, W, 0.0).astype(np.float64))
+    xt = torch.from_numpy(x.astype(np.float64)).permute(0, 3, 1, 2)
+    dyt = torch.from_numpy(dy.astype(np.float64)).permute(0, 3, 1, 2)
+    dx_t = torch.nn.grad.conv2d_input(xt.shape, Wm, dyt, stride=s, padding=p, dilation=d)
+    dW_t = torch.nn.grad.conv2d_weight(xt, Wm.shape, dyt, stride=s, padding=p, dilation=d)
+    dx, ax = oracle.conv_backward_data(dy, W, mask, 2, x.shape[1:3], s, p, d, want_abs=True)
+    dW, aw = oracle.conv_backward_weight(x, dy, W.shape[2:], mask, 2, s, p, d, want_abs=True)
+    assert np.all(np.abs(dx - dx_t.permute(0, 2, 3, 1).numpy()) <= 1e-13 * (ax + 1e-300))
+    assert np.all(np.abs(dW - np.where(keep, dW_t.numpy(), 0.0)) <= 1e-13 * (aw + 1e-300))
+
+
+def test_backward_brute_force_scatter_loops():
+    """The scatter form of both gradients in plain Python loops (every
+    output position sends w * dy to the input it read, and x * dy to the
+    weight it used) equals the oracle's gather form."""
+    case = (2, 5, 4, 3, 4, 3, 2, 2, 1, 1)
+    x, W, mask, dy, s, p, d, _ = _bwd_case(case, 0.5)
+    B, H, Wd, Ci, Co, KH, KW = case[:7]
+    Ho, Wo = dy.shape[1:3]
+    keep = _mask_oihw(mask, 2, W.shape)
+    dx = np.zeros((B, H, Wd, Ci))
+    dW = np.zeros((Co, Ci, KH, KW))
+    for b in range(B):
+        for oh in range(Ho):
+            for ow in range(Wo):
+                for o in range(Co):
+                    for c in range(Ci):
+                        for kh in range(KH):
+                            for kw in range(KW):
+                                ih, iw = oh * s[0] - p[0] + kh * d[0], ow * s[1] - p[1] + kw * d[1]
+                                if not keep[o, c, kh, kw] or not (0 <= ih < H and 0 <= iw < Wd):
+                                    continue
+                                dx[b, ih, iw, c] += float(W[o, c, kh, kw]) * float(dy[b, oh, ow, o])
+                                dW[o, c, kh, kw] += float(x[b, ih, iw, c]) * float(dy[b, oh, ow, o])
+    np.testing.assert_allclose(oracle.conv_backward_data(dy, W, mask, 2, (H, Wd), s, p, d), dx,
+                               rtol=1e-12, atol=1e-12)
+    np.testing.assert_allclose(oracle.conv_backward_weight(x, dy, (KH, KW), mask, 2, s, p, d), dW,
+                               rtol=1e-12, atol=1e-12)
+
+
+@pytest.mark.parametrize("shape,N", [((8, 6, 3, 3), 2), ((16, 8, 1, 1), 4), ((12, 5, 3, 1), 3)])
+def test_bsr_gather_inverts_unpack(shape, N):
+    """The weight gradient in BSR order (Sec. 3.4): unpacking the gathered
+    kept blocks gives back the masked gradient, bit for bit."""
+    rng = np.random.default_rng(shape[0] + N)
+    W = rng.standard_normal(shape).astype(np.float32)
+    mask, _ = oracle.prune(W, N, 0.5)
+    P, I, D = oracle.pack(W, mask, N)
+    g = rng.standard_normal(shape).astype(np.float32)
+    keep = _mask_oihw(mask, N, shape)
+    dD = oracle.bsr_gather(np.where(keep, g, 0.0).astype(np.float32), P, I, N)
+    assert dD.shape == D.shape
+    np.testing.assert_array_equal(oracle.unpack(P, I, dD, shape, N), np.where(keep, g, 0.0))
+    # and on the weights themselves it is the pack's D
+    np.testing.assert_array_equal(oracle.bsr_gather(W, P, I, N), D)
