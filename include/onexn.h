@@ -153,6 +153,53 @@ onexn_status onexn_pack(const float *W, const uint8_t *mask, int C_out, int C_in
                         int64_t t_cap, int64_t *t);
 
 /*
+ * onexn_prune_device -- onexn_prune on the GPU, bit for bit the same mask,
+ * for weights that live in device memory (re-pruning inside a fine-tuning
+ * loop without a host round trip).
+ *   W        DEVICE fp32 OIHW [C_out][C_in][KH][KW].
+ *   mask     DEVICE uint8 [G][K], written in full.
+ *   kept     HOST out: the kept block count (onexn_keep_count; known
+ *            without reading the device).
+ *   workspace, workspace_bytes
+ *            DEVICE scratch, 256-byte aligned, of at least
+ *            onexn_prune_device_workspace_size bytes (the blocks' norms and
+ *            the selection state); calls that run concurrently need their
+ *            own.
+ *   stream   cudaStream_t (NULL = legacy default stream).
+ * Scores, order and tie rule as onexn_prune (fp64 l1 norms summed n, kh, kw;
+ * larger first, then the lower block index).  Asynchronous; no allocation.
+ * EINVAL as onexn_prune, plus a short or misaligned workspace; ECUDA on a
+ * launch failure.
+ */
+onexn_status onexn_prune_device_workspace_size(int C_out, int C_in, int KH, int KW, int N, int gran,
+                                               size_t *bytes);
+onexn_status onexn_prune_device(const float *W, int C_out, int C_in, int KH, int KW, int N, double rate,
+                                int gran, uint8_t *mask, int64_t *kept, void *workspace,
+                                size_t workspace_bytes, void *stream);
+
+/*
+ * onexn_pack_device -- onexn_pack on the GPU, bit for bit the same P, I, D.
+ *   W, mask  DEVICE (as onexn_prune_device); mask bytes are 0 or 1 (any
+ *            non-zero byte counts as kept).
+ *   wdtype   ONEXN_F32 or ONEXN_BF16 (round-to-nearest-even).
+ *   P        DEVICE int32 [G+1], written in full (P[G] = the mask's count).
+ *   I, D     DEVICE int32 [t_cap] and [t_cap][N]: the kept blocks at
+ *            z < t_cap are written; t_cap must be at least the mask's count
+ *            (e.g. onexn_prune_device's kept, times KH*KW for
+ *            ONEXN_GRAN_KERNEL), else the blocks past it are left out while
+ *            P still counts them.
+ *   workspace, workspace_bytes
+ *            DEVICE scratch of onexn_pack_device_workspace_size bytes (the
+ *            per-group counts).
+ * Asynchronous; no allocation.  EINVAL: NULL pointers, bad dims, N not
+ * dividing C_out, unknown wdtype, short workspace.  ECUDA on a launch failure.
+ */
+onexn_status onexn_pack_device_workspace_size(int C_out, int N, size_t *bytes);
+onexn_status onexn_pack_device(const float *W, const uint8_t *mask, int C_out, int C_in, int KH, int KW,
+                               int N, int wdtype, int32_t *P, int32_t *I, void *D, int64_t t_cap,
+                               void *workspace, size_t workspace_bytes, void *stream);
+
+/*
  * onexn_packed_validate -- host check of a BSR index structure before it is
  * copied to the device: P[0] = 0, P non-decreasing, P[G] = t, each
  * col-group's I strictly increasing and inside [0, K).  EINVAL on the first

@@ -70,6 +70,12 @@ SIGNATURES = {
     "onexn_conv_fwd_ex": ([ctypes.POINTER(ConvDesc), _P, _P, _P, _I32, _I64, _P, _P, _P, _P, _I32,
                            _U32, _P, ctypes.c_size_t, _P], _I32),
     "onexn_dwconv_fwd": ([ctypes.POINTER(ConvDesc), _P, _P, _P, _P, _I32, _U32, _P], _I32),
+    "onexn_prune_device_workspace_size": ([_I32, _I32, _I32, _I32, _I32, _I32, _P], _I32),
+    "onexn_prune_device": ([_P, _I32, _I32, _I32, _I32, _I32, _DBL, _I32, _P, _P, _P, ctypes.c_size_t, _P],
+                           _I32),
+    "onexn_pack_device_workspace_size": ([_I32, _I32, _P], _I32),
+    "onexn_pack_device": ([_P, _P, _I32, _I32, _I32, _I32, _I32, _I32, _P, _P, _P, _I64, _P, ctypes.c_size_t,
+                           _P], _I32),
 }
 
 
@@ -278,3 +284,55 @@ def onexn_device_status(clear: bool = True) -> int:
     st = ctypes.c_int(0)
     _check(lib.onexn_device_status(int(bool(clear)), ctypes.byref(st)))
     return st.value
+
+
+def _cuda_stream(t, stream):
+    import torch
+    return torch.cuda.current_stream(t.device) if stream is None else stream
+
+
+def onexn_prune_device(W, N: int, rate: float, gran: int = ONEXN_GRAN_TAP, mask=None, workspace=None,
+                       stream=None):
+    """Device W (CUDA fp32 [C_out, C_in, KH, KW]) -> (mask CUDA uint8 [G, K], kept),
+    the same mask as onexn_prune.  mask / workspace are allocated if None."""
+    import torch
+    C_out, C_in, KH, KW = W.shape
+    if N < 1 or C_out % N:
+        raise OnexnError(ONEXN_EINVAL, f"N={N} must divide C_out={C_out}")
+    G, K = C_out // N, KH * KW * C_in
+    n = ctypes.c_size_t(0)
+    _check(lib.onexn_prune_device_workspace_size(C_out, C_in, KH, KW, int(N), int(gran), ctypes.byref(n)))
+    if mask is None:
+        mask = torch.empty((G, K), dtype=torch.uint8, device=W.device)
+    if workspace is None:
+        workspace = torch.empty(max(n.value, 256), dtype=torch.uint8, device=W.device)
+    kept = ctypes.c_int64(0)
+    s = _cuda_stream(W, stream)
+    _check(lib.onexn_prune_device(ctypes.c_void_p(W.data_ptr()), C_out, C_in, KH, KW, int(N), float(rate),
+                                  int(gran), ctypes.c_void_p(mask.data_ptr()), ctypes.byref(kept),
+                                  ctypes.c_void_p(workspace.data_ptr()), workspace.numel(),
+                                  ctypes.c_void_p(s.cuda_stream)))
+    return mask, kept.value
+
+
+def onexn_pack_device(W, mask, N: int, t: int, wdtype: int = ONEXN_F32, stream=None):
+    """Device BSR encoding -> (P CUDA int32 [G+1], I CUDA int32 [t], D CUDA
+    [t, N] float32 or bfloat16), the same as onexn_pack; t = the mask's
+    count (I and D are sized from it)."""
+    import torch
+    C_out, C_in, KH, KW = W.shape
+    if N < 1 or C_out % N:
+        raise OnexnError(ONEXN_EINVAL, f"N={N} must divide C_out={C_out}")
+    G = C_out // N
+    n = ctypes.c_size_t(0)
+    _check(lib.onexn_pack_device_workspace_size(C_out, int(N), ctypes.byref(n)))
+    ws = torch.empty(max(n.value, 256), dtype=torch.uint8, device=W.device)
+    P = torch.empty(G + 1, dtype=torch.int32, device=W.device)
+    I = torch.empty(max(t, 1), dtype=torch.int32, device=W.device)
+    D = torch.empty((max(t, 1), N), dtype=torch.float32 if wdtype == ONEXN_F32 else torch.bfloat16,
+                    device=W.device)
+    s = _cuda_stream(W, stream)
+    ptr = (lambda x: ctypes.c_void_p(x.data_ptr()))
+    _check(lib.onexn_pack_device(ptr(W), ptr(mask), C_out, C_in, KH, KW, int(N), int(wdtype), ptr(P), ptr(I),
+                                 ptr(D), int(t), ptr(ws), ws.numel(), ctypes.c_void_p(s.cuda_stream)))
+    return P, I[:t], D[:t]

@@ -364,3 +364,25 @@ def test_decoded_flag_selects_tc_and_is_checked():
     st = ox.lib.onexn_conv_fwd_noalloc(ctypes.byref(d), None, None, None, 8, 100, None, None, None,
                                        ox.ONEXN_F32, D, None)
     assert st == ox.ONEXN_EINVAL and b"DECODED" in ox.lib.onexn_last_error()
+
+
+def test_device_prune_and_pack_argument_errors_need_no_gpu():
+    n = ctypes.c_size_t(0)
+    assert ox.lib.onexn_prune_device_workspace_size(64, 32, 3, 3, 8, ox.ONEXN_GRAN_TAP, ctypes.byref(n)) == 0
+    assert n.value >= 8 * 9 * 32 * 8 and n.value % 256 == 0
+    assert ox.lib.onexn_prune_device_workspace_size(64, 32, 3, 3, 7, 0, ctypes.byref(n)) == ox.ONEXN_EINVAL
+    assert ox.lib.onexn_prune_device_workspace_size(64, 32, 3, 3, 8, 5, ctypes.byref(n)) == ox.ONEXN_EINVAL
+    keep, base = _aligned_host(1 << 20)
+    kept = ctypes.c_int64(0)
+    f = ox.lib.onexn_prune_device
+    assert f(base, 64, 32, 3, 3, 8, 1.5, 0, base, ctypes.byref(kept), base, 1 << 20, None) == ox.ONEXN_EINVAL
+    assert f(base, 64, 32, 3, 3, 8, 0.5, 0, base, ctypes.byref(kept), base, 16, None) == ox.ONEXN_EINVAL
+    assert b"workspace" in ox.lib.onexn_last_error()
+    assert f(base, 64, 32, 3, 3, 8, 0.5, 0, None, ctypes.byref(kept), base, 1 << 20, None) == ox.ONEXN_EINVAL
+    assert f(base, 64, 32, 3, 3, 8, 0.5, 0, base, ctypes.byref(kept), base + 8, 1 << 19, None) == \
+        ox.ONEXN_EINVAL
+    assert ox.lib.onexn_pack_device_workspace_size(64, 8, ctypes.byref(n)) == 0 and n.value == 256
+    g = ox.lib.onexn_pack_device
+    assert g(base, base, 64, 32, 3, 3, 8, 7, base, base, base, 10, base, 256, None) == ox.ONEXN_EINVAL
+    assert g(base, base, 64, 32, 3, 3, 8, 0, base, None, None, 10, base, 256, None) == ox.ONEXN_EINVAL
+    assert g(base, base, 64, 32, 3, 3, 8, 0, base, base, base, 10, base, 4, None) == ox.ONEXN_EINVAL
