@@ -74,6 +74,9 @@ typedef enum { ONEXN_GRAN_TAP = 0, ONEXN_GRAN_KERNEL = 1 } onexn_granularity;
  * ONEXN_DECODED on later calls, so the one-time decode is left out of the
  * comparison of the families.  It changes nothing else. */
 #define ONEXN_REUSE_DECODE 0x20u
+/* ONEXN_ACCUMULATE (onexn_conv_bwd_data only): dx += the gradient instead of
+ * dx = the gradient (a layer whose input also feeds another branch). */
+#define ONEXN_ACCUMULATE 0x40u
 /* Kernel selection (bits 8..11).  AUTO picks by dtype, N and density:
  * the tensor-core GEMM when its workspace fits and its dense work is
  * estimated to take less time than the FFMA kernel's kept work. */
@@ -297,6 +300,63 @@ onexn_status onexn_conv_fwd_ex(const onexn_conv_desc *desc, const int32_t *P, co
  */
 onexn_status onexn_dwconv_fwd(const onexn_conv_desc *desc, const float *W, const float *bias,
                               const void *x, void *y, int dtype, unsigned flags, void *stream);
+
+/*
+ * Fine-tuning with the mask held fixed (the pruned network is fine-tuned
+ * after pruning, Sec. 4.1; the pruned blocks stay zero).  desc is the
+ * forward geometry: x [B][H][W][C_in], dy [B][Ho][Wo][C_out] = the
+ * gradient of the loss with respect to the forward's PRE-activation output
+ * (the caller applies the activation's backward, and the residual branch
+ * takes dy as it is).  C_out must be a multiple of 8.
+ *
+ * onexn_conv_bwd_data -- the input gradient
+ *   dx[b,ih,iw,c] = sum over (o, kh, kw, oh, ow) with oh*sh - ph + kh*dh = ih
+ *                   and ow*sw - pw + kw*dw = iw of W[o,c,kh,kw] * dy[b,oh,ow,o]
+ * over the kept blocks (P, I, D as for onexn_conv_fwd).
+ *   dy, dx  DEVICE NHWC of dtype, 16-byte aligned, not overlapping; dx is
+ *           written in full (or added to, with ONEXN_ACCUMULATE).
+ *   flags   0 or ONEXN_ACCUMULATE.
+ *   workspace, workspace_bytes
+ *           DEVICE scratch of onexn_conv_bwd_data_workspace_size bytes,
+ *           256-byte aligned (the decoded weights and their flipped
+ *           transpose); concurrent calls need their own.
+ * Stride-1 layers run on the tensor-core GEMM (dx is a convolution of dy
+ * with the flipped, transposed weights); strided ones on a direct kernel.
+ * fp32: three tf32 products per term as the forward; bf16: bf16 products,
+ * fp32 accumulation, RNE output.  Asynchronous; no allocation.
+ * EINVAL as onexn_conv_fwd plus a short workspace; EUNSUPPORTED: C_out % 8.
+ */
+onexn_status onexn_conv_bwd_data_workspace_size(const onexn_conv_desc *desc, int N, int64_t t, int dtype,
+                                                size_t *bytes);
+onexn_status onexn_conv_bwd_data(const onexn_conv_desc *desc, const int32_t *P, const int32_t *I,
+                                 const void *D, int N, int64_t t, const void *dy, void *dx, int dtype,
+                                 unsigned flags, void *workspace, size_t workspace_bytes, void *stream);
+
+/*
+ * onexn_conv_bwd_weight -- the gradient of the kept weights, in BSR order:
+ *   dD[z][n] = sum_{b,oh,ow} dy[b,oh,ow,gN+n] * x[b, oh*sh - ph + kh*dh,
+ *              ow*sw - pw + kw*dw, c]      for P[g] <= z < P[g+1],
+ *              I[z] = (kh*KW + kw)*C_in + c
+ * (the layout of D, so an optimizer updates D in place), and optionally the
+ * bias gradient db[o] = sum dy[..., o].
+ *   P, I    DEVICE BSR indices (as packed; D itself is not needed).
+ *   x, dy   DEVICE NHWC of dtype, 16-byte aligned.
+ *   dD      DEVICE fp32 [t][N]; db nullable DEVICE fp32 [C_out].
+ *   workspace, workspace_bytes
+ *           DEVICE scratch of onexn_conv_bwd_weight_workspace_size bytes,
+ *           256-byte aligned: dy and the im2col view of x transposed to
+ *           pixel-contiguous rows (fp32: the latter as tf32 high and low
+ *           parts), pixels padded to 64, plus one 128 x BN fp32 partial
+ *           tile per GEMM item.
+ * The products run on the tensor cores (fp32: three tf32 products per
+ * term; bf16: exact bf16 products) with fp32 accumulation over pixel
+ * slices, added in slice order (deterministic).  Asynchronous.
+ * EINVAL: bad geometry or pointers, short workspace; EUNSUPPORTED: C_out % 8.
+ */
+onexn_status onexn_conv_bwd_weight_workspace_size(const onexn_conv_desc *desc, int N, int dtype, size_t *bytes);
+onexn_status onexn_conv_bwd_weight(const onexn_conv_desc *desc, const int32_t *P, const int32_t *I, int N,
+                                   int64_t t, const void *x, const void *dy, float *dD, float *db, int dtype,
+                                   void *workspace, size_t workspace_bytes, void *stream);
 
 /*
  * onexn_conv_workspace_size -- bytes of device workspace onexn_conv_fwd

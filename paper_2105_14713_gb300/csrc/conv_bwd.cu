@@ -1,0 +1,496 @@
+// Backward passes of the 1xN-pruned convolution with the mask held fixed
+// (fine-tuning the pruned network, Sec. 4.1): the input gradient and the
+// gradient of the kept weights, in BSR order.
+//
+// Input gradient dx = the transposed masked convolution of dy.  For a
+// stride-1 layer it is itself a convolution: dy (padded by d(K-1) - p)
+// with the flipped, transposed weights Wt[c][(T-1-tap)*C_out + o] =
+// W[o][tap*C_in + c] (T = KH*KW taps), so it runs on the forward tcgen05
+// GEMM: decode (P, I, D) into W, transpose it per tap with the tap order
+// reversed, and launch the GEMM on (dy, Wt).  Strided layers (and padding
+// beyond d(K-1)) use a direct kernel over the decoded W.
+//
+// Kept-weight gradient dW[o][k] = sum_p dy[p][o] * xcol[p][k] (k = tap*C_in
+// + c, xcol the im2col view of x): a GEMM with M = C_out, N = K and the
+// pixels as its long reduction dimension.  dy and xcol are transposed once
+// into K-major operands (pixels padded to 64 with zeros; fp32: xcol split
+// into its tf32 rounding and the rest, as the decode does for weights), the
+// GEMM runs in split mode (items of pixel slices, one accumulator slot
+// each), and a gather kernel adds each kept block's S slots in slice order
+// into dD[z][n] = dW[g*N + n][I[z]] (fp32), only for the kept blocks.
+#include "conv_common.cuh"
+#include "conv_dispatch.h"
+#include "onexn_internal.h"
+
+#include <cuda_bf16.h>
+
+using onexn::ConvArgs;
+using onexn::fail;
+
+namespace {
+
+constexpr int kTile = 32;           // transpose tiles: 32 x 32 elements, 32 x 8 threads
+constexpr int kPixPad = 64;         // pixels padded to the bf16 K chunk
+
+__device__ __forceinline__ float tf32_rna(float v)
+{
+    uint32_t r;
+    asm("cvt.rna.tf32.f32 %0, %1;\n" : "=r"(r) : "f"(v));
+    return __uint_as_float(r);
+}
+
+template <typename T>
+__device__ __forceinline__ float to_f(T v)
+{
+    if constexpr (sizeof(T) == 4) return v;
+    else return __bfloat162float(v);
+}
+
+// dYt[o][p] = dY[p][o] for p < P, 0 for P <= p < P_pad.
+template <typename T>
+__global__ void __launch_bounds__(kTile * 8)
+dy_transpose_kernel(const T *__restrict__ dy, int64_t P, int64_t P_pad, int C_out, T *__restrict__ dyt)
+{
+    __shared__ T tile[kTile][kTile + 1];
+    const int64_t p0 = static_cast<int64_t>(blockIdx.x) * kTile;
+    const int o0 = blockIdx.y * kTile;
+    const int tx = threadIdx.x, ty = threadIdx.y;
+    for (int i = ty; i < kTile; i += 8) {
+        const int64_t p = p0 + i;
+        const int o = o0 + tx;
+        tile[i][tx] = (p < P && o < C_out) ? dy[p * C_out + o] : T(0.f);
+    }
+    __syncthreads();
+    for (int i = ty; i < kTile; i += 8) {
+        const int o = o0 + i;
+        const int64_t p = p0 + tx;
+        if (o < C_out && p < P_pad) dyt[static_cast<int64_t>(o) * P_pad + p] = tile[tx][i];
+    }
+}
+
+// XcolT[tap*C_in + c][p] = x[b, oh*sh - ph + kh*dh, ow*sw - pw + kw*dw, c]
+// (0 outside the image and for p >= P); fp32 as hi (tf32) and lo parts.
+template <typename T>
+__global__ void __launch_bounds__(kTile * 8)
+xcol_transpose_kernel(const ConvArgs a, int64_t P_pad, T *__restrict__ hi, T *__restrict__ lo)
+{
+    __shared__ T tile[kTile][kTile + 1];
+    const int64_t p0 = static_cast<int64_t>(blockIdx.x) * kTile;
+    const int c0 = blockIdx.y * kTile, tap = blockIdx.z;
+    const int kh = tap / a.KW, kw = tap - (tap / a.KW) * a.KW;
+    const int tx = threadIdx.x, ty = threadIdx.y;
+    const int64_t P = a.P_pix, hw = static_cast<int64_t>(a.Ho) * a.Wo;
+    const T *x = static_cast<const T *>(a.x);
+    for (int i = ty; i < kTile; i += 8) {
+        const int64_t p = p0 + i;
+        const int c = c0 + tx;
+        T v = T(0.f);
+        if (p < P && c < a.C) {
+            const int64_t b = p / hw;
+            const int r = static_cast<int>(p - b * hw);
+            const int oh = r / a.Wo, ow = r - (r / a.Wo) * a.Wo;
+            const int ih = oh * a.sh - a.ph + kh * a.dh, iw = ow * a.sw - a.pw + kw * a.dw;
+            if (ih >= 0 && ih < a.H && iw >= 0 && iw < a.W)
+                v = x[((b * a.H + ih) * a.W + iw) * a.C + c];
+        }
+        tile[i][tx] = v;
+    }
+    __syncthreads();
+    for (int i = ty; i < kTile; i += 8) {
+        const int c = c0 + i;
+        const int64_t p = p0 + tx;
+        if (c >= a.C || p >= P_pad) continue;
+        const int64_t dst = (static_cast<int64_t>(tap) * a.C + c) * P_pad + p;
+        const T v = tile[tx][i];
+        if constexpr (sizeof(T) == 4) {
+            const float h = tf32_rna(v);
+            hi[dst] = h;
+            lo[dst] = v - h;
+        } else {
+            hi[dst] = v;
+        }
+    }
+}
+
+// dD[z][n] = sum over the S slices of the GEMM partial at row g*N + n,
+// column I[z]; one CTA per col-group.  Partial slot i = slice * tiles +
+// tile holds [BN/4][128] float4 (column quad, row).
+__global__ void __launch_bounds__(256)
+wgrad_gather_kernel(const float *__restrict__ partials, const int32_t *__restrict__ P, const int32_t *__restrict__ I,
+                    int N, int64_t t, int bn, int tiles, int n_tn, int S, float *__restrict__ dD)
+{
+    const int g = blockIdx.x;
+    const int64_t z0 = min(static_cast<int64_t>(__ldg(P + g)), t);
+    const int64_t z1 = min(max(static_cast<int64_t>(__ldg(P + g + 1)), z0), t);
+    const int64_t slot_f = static_cast<int64_t>(128) * bn;
+    for (int64_t e = z0 * N + threadIdx.x; e < z1 * N; e += blockDim.x) {
+        const int64_t z = e / N;
+        const int n = static_cast<int>(e - z * N);
+        const int m = g * N + n, k = __ldg(I + z);
+        const int tile = (m / 128) * n_tn + k / bn;
+        const int col = k % bn, row = m % 128;
+        const int64_t off = (static_cast<int64_t>(col / 4) * 128 + row) * 4 + (col & 3);
+        float s = 0.f;
+        for (int sl = 0; sl < S; ++sl) s += __ldg(partials + (static_cast<int64_t>(sl) * tiles + tile) * slot_f + off);
+        dD[e] = s;
+    }
+}
+
+// db[o] = sum_p dYt[o][p], one warp per row, fixed order.
+template <typename T>
+__global__ void __launch_bounds__(256)
+bias_grad_kernel(const T *__restrict__ dyt, int64_t P, int64_t P_pad, int C_out, float *__restrict__ db)
+{
+    const int o = blockIdx.x * 8 + (threadIdx.x >> 5), lane = threadIdx.x & 31;
+    if (o >= C_out) return;
+    const T *row = dyt + static_cast<int64_t>(o) * P_pad;
+    float s = 0.f;
+    for (int64_t p = lane; p < P; p += 32) s += to_f(row[p]);
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) s += __shfl_xor_sync(0xffffffffu, s, off);
+    if (lane == 0) db[o] = s;
+}
+
+__global__ void zero_f32_kernel(float *p, int64_t n)
+{
+    for (int64_t i = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; i < n;
+         i += static_cast<int64_t>(gridDim.x) * blockDim.x)
+        p[i] = 0.f;
+}
+
+// Wt[c][(T-1-tap)*C_out + o] = W[o][tap*C_in + c] (and the lo part for fp32).
+template <typename T>
+__global__ void __launch_bounds__(kTile * 8)
+flip_transpose_kernel(const T *__restrict__ W, const T *__restrict__ W_lo, int C_out, int C_in, int taps,
+                      T *__restrict__ Wt, T *__restrict__ Wt_lo)
+{
+    __shared__ T tile[2][kTile][kTile + 1];
+    const int c0 = blockIdx.x * kTile, o0 = blockIdx.y * kTile, tap = blockIdx.z;
+    const int tx = threadIdx.x, ty = threadIdx.y;
+    const int64_t K = static_cast<int64_t>(taps) * C_in, Kt = static_cast<int64_t>(taps) * C_out;
+    constexpr bool kLo = sizeof(T) == 4;
+    for (int i = ty; i < kTile; i += 8) {
+        const int o = o0 + i, c = c0 + tx;
+        const bool in = o < C_out && c < C_in;
+        const int64_t at = static_cast<int64_t>(o) * K + static_cast<int64_t>(tap) * C_in + c;
+        tile[0][i][tx] = in ? W[at] : T(0.f);
+        if (kLo) tile[1][i][tx] = in ? W_lo[at] : T(0.f);
+    }
+    __syncthreads();
+    const int ftap = taps - 1 - tap;
+    for (int i = ty; i < kTile; i += 8) {
+        const int c = c0 + i, o = o0 + tx;
+        if (c >= C_in || o >= C_out) continue;
+        const int64_t at = static_cast<int64_t>(c) * Kt + static_cast<int64_t>(ftap) * C_out + o;
+        Wt[at] = tile[0][tx][i];
+        if (kLo) Wt_lo[at] = tile[1][tx][i];
+    }
+}
+
+// Direct input gradient (any stride): one thread per 16-byte channel vector
+// of one input pixel; for every tap that maps it onto an output pixel, the
+// dot product over the output channels with the decoded W (fp32: hi + lo,
+// which is the weight exactly).
+template <typename T>
+__global__ void __launch_bounds__(256)
+dgrad_direct_kernel(const ConvArgs a, const T *__restrict__ W, const T *__restrict__ W_lo, const T *__restrict__ dy,
+                    T *__restrict__ dx, int accumulate)
+{
+    constexpr int kV = 16 / sizeof(T);
+    const int n_vec = a.C / kV;
+    const int64_t total = static_cast<int64_t>(a.B) * a.H * a.W * n_vec;
+    const int64_t K = static_cast<int64_t>(a.KH) * a.KW * a.C;
+    for (int64_t i = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; i < total;
+         i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+        const int cv = static_cast<int>(i % n_vec);
+        const int64_t q = i / n_vec;
+        const int iw = static_cast<int>(q % a.W);
+        const int ih = static_cast<int>((q / a.W) % a.H);
+        const int64_t b = q / (static_cast<int64_t>(a.W) * a.H);
+        const int c0 = cv * kV;
+        float acc[kV];
+#pragma unroll
+        for (int j = 0; j < kV; ++j) acc[j] = 0.f;
+        for (int kh = 0; kh < a.KH; ++kh) {
+            const int th = ih + a.ph - kh * a.dh;
+            if (th < 0 || th % a.sh) continue;
+            const int oh = th / a.sh;
+            if (oh >= a.Ho) continue;
+            for (int kw = 0; kw < a.KW; ++kw) {
+                const int tw = iw + a.pw - kw * a.dw;
+                if (tw < 0 || tw % a.sw) continue;
+                const int ow = tw / a.sw;
+                if (ow >= a.Wo) continue;
+                const T *dyr = dy + ((b * a.Ho + oh) * a.Wo + ow) * a.C_out;
+                const int64_t kcol = static_cast<int64_t>(kh * a.KW + kw) * a.C + c0;
+                for (int o = 0; o < a.C_out; ++o) {
+                    const float d = to_f(dyr[o]);
+                    const T *wr = W + o * K + kcol;
+#pragma unroll
+                    for (int j = 0; j < kV; ++j) {
+                        float w = to_f(wr[j]);
+                        if constexpr (sizeof(T) == 4) w += W_lo[o * K + kcol + j];
+                        acc[j] = fmaf(w, d, acc[j]);
+                    }
+                }
+            }
+        }
+        T *out = dx + q * a.C + c0;
+#pragma unroll
+        for (int j = 0; j < kV; ++j) {
+            const float v = accumulate ? acc[j] + to_f(out[j]) : acc[j];
+            if constexpr (sizeof(T) == 4) out[j] = v;
+            else out[j] = __float2bfloat16_rn(v);
+        }
+    }
+}
+
+bool aligned(const void *p, uintptr_t n) { return (reinterpret_cast<uintptr_t>(p) & (n - 1)) == 0; }
+size_t round256(size_t v) { return (v + 255) & ~static_cast<size_t>(255); }
+
+int grid_cap(int64_t work, int per_block, int sms)
+{
+    const int64_t b = (work + per_block - 1) / per_block;
+    const int64_t cap = static_cast<int64_t>(sms) * 16;
+    return static_cast<int>(b < 1 ? 1 : b < cap ? b : cap);
+}
+
+// The transposed convolution that computes dx for a stride-1 layer, or
+// false if the forward kernel cannot run it (then the direct kernel does).
+bool dgrad_as_conv(const ConvArgs &a, int dtype, ConvArgs *t)
+{
+    if (a.sh != 1 || a.sw != 1) return false;
+    const int ph = a.dh * (a.KH - 1) - a.ph, pw = a.dw * (a.KW - 1) - a.pw;
+    if (ph < 0 || pw < 0) return false;
+    ConvArgs c{};
+    c.B = a.B; c.H = a.Ho; c.W = a.Wo; c.C = a.C_out; c.C_out = a.C;
+    c.KH = a.KH; c.KW = a.KW; c.sh = 1; c.sw = 1; c.ph = ph; c.pw = pw; c.dh = a.dh; c.dw = a.dw;
+    c.Ho = a.H; c.Wo = a.W; c.P_pix = a.B * a.H * a.W;
+    c.N = 1; c.t = 0;
+    if (!onexn::tc_supports(c, dtype)) return false;
+    *t = c;
+    return true;
+}
+
+struct DgradWs {
+    size_t w, wt, total;
+};
+
+DgradWs dgrad_ws(const ConvArgs &a, int dtype)
+{
+    DgradWs l{};
+    const size_t wb = onexn::tc_weights_bytes(a, dtype);
+    l.w = 0;
+    l.wt = wb;
+    l.total = 2 * wb;
+    return l;
+}
+
+struct WgradWs {
+    int64_t P_pad;
+    onexn::TcSplitPlan plan;
+    size_t dyt, xhi, xlo, part, total;
+};
+
+WgradWs wgrad_ws(const ConvArgs &a, int dtype)
+{
+    WgradWs l{};
+    const size_t es = dtype == ONEXN_F32 ? 4 : 2;
+    const int64_t K = static_cast<int64_t>(a.KH) * a.KW * a.C;
+    l.P_pad = (static_cast<int64_t>(a.P_pix) + kPixPad - 1) / kPixPad * kPixPad;
+    l.plan = onexn::tc_split_plan(a.C_out, static_cast<int>(K), l.P_pad, dtype);
+    l.dyt = 0;
+    l.xhi = round256(static_cast<size_t>(a.C_out) * l.P_pad * es);
+    l.xlo = l.xhi + round256(static_cast<size_t>(K) * l.P_pad * es);
+    l.part = l.xlo + (dtype == ONEXN_F32 ? round256(static_cast<size_t>(K) * l.P_pad * es) : 0);
+    l.total = l.part + round256(l.plan.partial_bytes);
+    return l;
+}
+
+onexn_status bwd_shape(const onexn_conv_desc *desc, int N, int64_t t, int dtype, ConvArgs *a, const char *who)
+{
+    onexn_status st = onexn::detail::check_shape(desc, N, t, dtype, 0, a);
+    if (st != ONEXN_OK) return st;
+    if (a->C_out % 8) return fail(ONEXN_EUNSUPPORTED, "%s: C_out=%d must be a multiple of 8", who, a->C_out);
+    if (a->C_out / a->N > 65535) return fail(ONEXN_EUNSUPPORTED, "%s: more than 65535 col-groups", who);
+    return ONEXN_OK;
+}
+
+}  // namespace
+
+extern "C" onexn_status onexn_conv_bwd_data_workspace_size(const onexn_conv_desc *desc, int N, int64_t t, int dtype,
+                                                           size_t *bytes)
+{
+    onexn::clear_error();
+    if (!bytes) return fail(ONEXN_EINVAL, "conv_bwd_data: bytes is NULL");
+    ConvArgs a{};
+    onexn_status st = bwd_shape(desc, N, t, dtype, &a, "conv_bwd_data");
+    if (st != ONEXN_OK) return st;
+    *bytes = dgrad_ws(a, dtype).total;
+    return ONEXN_OK;
+}
+
+extern "C" onexn_status onexn_conv_bwd_data(const onexn_conv_desc *desc, const int32_t *P, const int32_t *I,
+                                            const void *D, int N, int64_t t, const void *dy, void *dx, int dtype,
+                                            unsigned flags, void *workspace, size_t workspace_bytes, void *stream)
+{
+    onexn::clear_error();
+    ConvArgs a{};
+    onexn_status st = bwd_shape(desc, N, t, dtype, &a, "conv_bwd_data");
+    if (st != ONEXN_OK) return st;
+    if (flags & ~ONEXN_ACCUMULATE) return fail(ONEXN_EINVAL, "conv_bwd_data: unknown flags");
+    const size_t es = dtype == ONEXN_F32 ? 4 : 2;
+    const size_t x_bytes = static_cast<size_t>(a.B) * a.H * a.W * a.C * es;
+    const size_t y_bytes = static_cast<size_t>(a.P_pix) * a.C_out * es;
+    if (x_bytes == 0) return ONEXN_OK;
+    if (!dy || !dx || !P || (t > 0 && (!I || !D))) return fail(ONEXN_EINVAL, "conv_bwd_data: NULL pointer");
+    if (!aligned(dy, 16) || !aligned(dx, 16)) return fail(ONEXN_EINVAL, "conv_bwd_data: dy and dx must be 16-byte aligned");
+    {
+        const uintptr_t d0 = reinterpret_cast<uintptr_t>(dy), x0 = reinterpret_cast<uintptr_t>(dx);
+        if (d0 < x0 + x_bytes && x0 < d0 + y_bytes) return fail(ONEXN_EINVAL, "conv_bwd_data: dy and dx overlap");
+    }
+    const DgradWs L = dgrad_ws(a, dtype);
+    if (!workspace || workspace_bytes < L.total)
+        return fail(ONEXN_EINVAL, "conv_bwd_data: needs %zu bytes of workspace, got %zu", L.total, workspace_bytes);
+    if (!aligned(workspace, 256)) return fail(ONEXN_EINVAL, "conv_bwd_data: workspace must be 256-byte aligned");
+    a.P = P; a.I = I; a.D = D; a.x = nullptr; a.y = nullptr;
+    cudaError_t e = onexn::device_status_ptr(&a.status);
+    if (e != cudaSuccess) return fail(ONEXN_ECUDA, "conv_bwd_data: status word: %s", cudaGetErrorString(e));
+    int sms = 0;
+    e = onexn::device_sm_count(&sms);
+    if (e != cudaSuccess) return fail(ONEXN_ECUDA, "conv_bwd_data: %s", cudaGetErrorString(e));
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    unsigned char *ws = static_cast<unsigned char *>(workspace);
+    const size_t n_w = static_cast<size_t>(a.C_out) * a.KH * a.KW * a.C;
+    // the masked dense weights (fp32: hi, then lo), as the forward decodes them
+    e = onexn::tc_decode(a, dtype, ws + L.w, onexn::tc_weights_bytes(a, dtype), s);
+    if (e != cudaSuccess) return fail(ONEXN_ECUDA, "conv_bwd_data: decode: %s", cudaGetErrorString(e));
+    const bool acc = (flags & ONEXN_ACCUMULATE) != 0;
+    ConvArgs tr{};
+    if (dgrad_as_conv(a, dtype, &tr)) {
+        const dim3 grid((a.C + kTile - 1) / kTile, (a.C_out + kTile - 1) / kTile, a.KH * a.KW);
+        const dim3 block(kTile, 8);
+        void *wt = ws + L.wt;
+        if (dtype == ONEXN_F32) {
+            const float *w = reinterpret_cast<const float *>(ws + L.w);
+            float *t_hi = static_cast<float *>(wt);
+            flip_transpose_kernel<float><<<grid, block, 0, s>>>(w, w + n_w, a.C_out, a.C, a.KH * a.KW, t_hi,
+                                                                 t_hi + n_w);
+        } else {
+            const __nv_bfloat16 *w = reinterpret_cast<const __nv_bfloat16 *>(ws + L.w);
+            flip_transpose_kernel<__nv_bfloat16><<<grid, block, 0, s>>>(w, nullptr, a.C_out, a.C, a.KH * a.KW,
+                                                                         static_cast<__nv_bfloat16 *>(wt), nullptr);
+        }
+        e = cudaGetLastError();
+        if (e != cudaSuccess) return fail(ONEXN_ECUDA, "conv_bwd_data: transpose: %s", cudaGetErrorString(e));
+        tr.x = dy; tr.y = dx; tr.residual = acc ? dx : nullptr; tr.bias = nullptr; tr.relu = 0;
+        tr.status = a.status;
+        const void *wt_lo = dtype == ONEXN_F32 ? static_cast<const void *>(static_cast<float *>(wt) + n_w) : nullptr;
+        e = onexn::tc_gemm_weights(tr, dtype, wt, wt_lo, nullptr, s);
+        if (e != cudaSuccess) return fail(ONEXN_ECUDA, "conv_bwd_data: GEMM: %s", cudaGetErrorString(e));
+        return ONEXN_OK;
+    }
+    const int kv = dtype == ONEXN_F32 ? 4 : 8;
+    const int grid = grid_cap(static_cast<int64_t>(a.B) * a.H * a.W * (a.C / kv), 256, sms);
+    if (dtype == ONEXN_F32) {
+        const float *w = reinterpret_cast<const float *>(ws + L.w);
+        dgrad_direct_kernel<float><<<grid, 256, 0, s>>>(a, w, w + n_w, static_cast<const float *>(dy),
+                                                         static_cast<float *>(dx), acc ? 1 : 0);
+    } else {
+        const __nv_bfloat16 *w = reinterpret_cast<const __nv_bfloat16 *>(ws + L.w);
+        dgrad_direct_kernel<__nv_bfloat16><<<grid, 256, 0, s>>>(a, w, nullptr, static_cast<const __nv_bfloat16 *>(dy),
+                                                                 static_cast<__nv_bfloat16 *>(dx), acc ? 1 : 0);
+    }
+    e = cudaGetLastError();
+    if (e != cudaSuccess) return fail(ONEXN_ECUDA, "conv_bwd_data: launch failed: %s", cudaGetErrorString(e));
+    return ONEXN_OK;
+}
+
+extern "C" onexn_status onexn_conv_bwd_weight_workspace_size(const onexn_conv_desc *desc, int N, int dtype,
+                                                             size_t *bytes)
+{
+    onexn::clear_error();
+    if (!bytes) return fail(ONEXN_EINVAL, "conv_bwd_weight: bytes is NULL");
+    ConvArgs a{};
+    onexn_status st = bwd_shape(desc, N, 0, dtype, &a, "conv_bwd_weight");
+    if (st != ONEXN_OK) return st;
+    *bytes = wgrad_ws(a, dtype).total;
+    return ONEXN_OK;
+}
+
+extern "C" onexn_status onexn_conv_bwd_weight(const onexn_conv_desc *desc, const int32_t *P, const int32_t *I, int N,
+                                              int64_t t, const void *x, const void *dy, float *dD, float *db,
+                                              int dtype, void *workspace, size_t workspace_bytes, void *stream)
+{
+    onexn::clear_error();
+    ConvArgs a{};
+    onexn_status st = bwd_shape(desc, N, t, dtype, &a, "conv_bwd_weight");
+    if (st != ONEXN_OK) return st;
+    if (!P || (t > 0 && (!I || !dD))) return fail(ONEXN_EINVAL, "conv_bwd_weight: NULL pointer");
+    if (a.P_pix > 0 && (!x || !dy)) return fail(ONEXN_EINVAL, "conv_bwd_weight: x or dy is NULL");
+    if (!aligned(x, 16) || !aligned(dy, 16) || !aligned(dD, 4) || !aligned(db, 4))
+        return fail(ONEXN_EINVAL, "conv_bwd_weight: x and dy must be 16-byte aligned, dD and db 4-byte aligned");
+    const WgradWs L = wgrad_ws(a, dtype);
+    if (!workspace || workspace_bytes < L.total)
+        return fail(ONEXN_EINVAL, "conv_bwd_weight: needs %zu bytes of workspace, got %zu", L.total, workspace_bytes);
+    if (!aligned(workspace, 256)) return fail(ONEXN_EINVAL, "conv_bwd_weight: workspace must be 256-byte aligned");
+    int sms = 0;
+    cudaError_t e = onexn::device_sm_count(&sms);
+    if (e != cudaSuccess) return fail(ONEXN_ECUDA, "conv_bwd_weight: %s", cudaGetErrorString(e));
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    if (a.P_pix == 0) {
+        // no pixels: every gradient is zero
+        if (t > 0) zero_f32_kernel<<<grid_cap(t * N, 256, sms), 256, 0, s>>>(dD, t * N);
+        if (db) zero_f32_kernel<<<grid_cap(a.C_out, 256, sms), 256, 0, s>>>(db, a.C_out);
+        e = cudaGetLastError();
+        return e == cudaSuccess ? ONEXN_OK : fail(ONEXN_ECUDA, "conv_bwd_weight: %s", cudaGetErrorString(e));
+    }
+    a.x = x;
+    unsigned char *ws = static_cast<unsigned char *>(workspace);
+    const dim3 block(kTile, 8);
+    const int K = a.KH * a.KW * a.C;
+    const dim3 g_dy(static_cast<unsigned>((L.P_pad + kTile - 1) / kTile), (a.C_out + kTile - 1) / kTile);
+    const dim3 g_x(static_cast<unsigned>((L.P_pad + kTile - 1) / kTile), (a.C + kTile - 1) / kTile, a.KH * a.KW);
+    if (dtype == ONEXN_F32) {
+        dy_transpose_kernel<float><<<g_dy, block, 0, s>>>(static_cast<const float *>(dy), a.P_pix, L.P_pad, a.C_out,
+                                                           reinterpret_cast<float *>(ws + L.dyt));
+        xcol_transpose_kernel<float><<<g_x, block, 0, s>>>(a, L.P_pad, reinterpret_cast<float *>(ws + L.xhi),
+                                                            reinterpret_cast<float *>(ws + L.xlo));
+    } else {
+        dy_transpose_kernel<__nv_bfloat16><<<g_dy, block, 0, s>>>(static_cast<const __nv_bfloat16 *>(dy), a.P_pix,
+                                                                   L.P_pad, a.C_out,
+                                                                   reinterpret_cast<__nv_bfloat16 *>(ws + L.dyt));
+        xcol_transpose_kernel<__nv_bfloat16><<<g_x, block, 0, s>>>(a, L.P_pad,
+                                                                    reinterpret_cast<__nv_bfloat16 *>(ws + L.xhi),
+                                                                    nullptr);
+    }
+    e = cudaGetLastError();
+    if (e != cudaSuccess) return fail(ONEXN_ECUDA, "conv_bwd_weight: transpose: %s", cudaGetErrorString(e));
+    // the GEMM dW[C_out][K] = dYt[C_out][P_pad] . XcolT[K][P_pad]^T, in pixel slices
+    ConvArgs g{};
+    g.B = 1; g.H = 1; g.W = a.C_out; g.C = static_cast<int>(L.P_pad); g.C_out = K;
+    g.KH = 1; g.KW = 1; g.sh = 1; g.sw = 1; g.ph = 0; g.pw = 0; g.dh = 1; g.dw = 1;
+    g.Ho = 1; g.Wo = a.C_out; g.P_pix = a.C_out; g.N = 1; g.t = 0;
+    g.x = ws + L.dyt; g.y = ws + L.dyt;
+    e = onexn::device_status_ptr(&g.status);
+    if (e != cudaSuccess) return fail(ONEXN_ECUDA, "conv_bwd_weight: status word: %s", cudaGetErrorString(e));
+    if (L.P_pad > INT32_MAX) return fail(ONEXN_EINVAL, "conv_bwd_weight: too many pixels");
+    float *part = reinterpret_cast<float *>(ws + L.part);
+    e = onexn::tc_gemm_split(g, dtype, ws + L.xhi, dtype == ONEXN_F32 ? ws + L.xlo : nullptr, part, L.plan, s);
+    if (e != cudaSuccess) return fail(ONEXN_ECUDA, "conv_bwd_weight: GEMM: %s", cudaGetErrorString(e));
+    if (t > 0)
+        wgrad_gather_kernel<<<a.C_out / a.N, 256, 0, s>>>(part, P, I, a.N, t, L.plan.bn, L.plan.tiles, L.plan.n_tn,
+                                                          L.plan.split_s, dD);
+    if (db) {
+        const int gb = (a.C_out + 7) / 8;
+        if (dtype == ONEXN_F32)
+            bias_grad_kernel<float><<<gb, 256, 0, s>>>(reinterpret_cast<const float *>(ws + L.dyt), a.P_pix, L.P_pad,
+                                                        a.C_out, db);
+        else
+            bias_grad_kernel<__nv_bfloat16><<<gb, 256, 0, s>>>(reinterpret_cast<const __nv_bfloat16 *>(ws + L.dyt),
+                                                                a.P_pix, L.P_pad, a.C_out, db);
+    }
+    e = cudaGetLastError();
+    if (e != cudaSuccess) return fail(ONEXN_ECUDA, "conv_bwd_weight: launch failed: %s", cudaGetErrorString(e));
+    return ONEXN_OK;
+}

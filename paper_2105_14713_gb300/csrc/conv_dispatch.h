@@ -23,6 +23,18 @@ size_t tc_workspace_bytes(const ConvArgs &a, int dtype);
 size_t tc_workspace_min(const ConvArgs &a, int dtype);
 // AUTO's time estimate of the tensor-core family (ns; fixed costs relative to FFMA's)
 double tc_cost_ns(const ConvArgs &a, int dtype, size_t ws_bytes, bool decoded);
+// The tensor-core GEMM on caller-given operands (backward passes).
+cudaError_t tc_gemm_weights(const ConvArgs &a, int dtype, const void *W, const void *W_lo, void *sk_space,
+                            cudaStream_t st);
+struct TcSplitPlan {
+    int bn, tiles, n_tn, split_s;
+    size_t partial_bytes;
+};
+TcSplitPlan tc_split_plan(int M, int Ncols, int64_t K, int dtype);
+cudaError_t tc_gemm_split(const ConvArgs &a, int dtype, const void *W, const void *W_lo, float *partials,
+                          const TcSplitPlan &plan, cudaStream_t st);
+size_t tc_weights_bytes(const ConvArgs &a, int dtype);
+size_t tc_sk_bytes(const ConvArgs &a);
 
 namespace detail {
 

@@ -221,9 +221,16 @@ __device__ __forceinline__ bool epi_all(bool ok)
 // into its idle shared-memory ring and adds them to its own accumulator in
 // CTA order, so the result does not depend on timing.  Waiting only on
 // lower CTAs, which were scheduled first, cannot deadlock.
+//
+// Split mode (split_s > 0; plain GEMMs with a long K, e.g. the weight
+// gradient whose K is the pixels): item i = slice * n_tiles + tile covers
+// chunks [slice * C / S, (slice + 1) * C / S) of its tile; CTA b takes
+// items b, b + G, ...; every item's accumulator goes to partial slot i and
+// a separate kernel adds the S slots of a tile in slice order.
 struct TcSched {
     int n_tiles, n_tn, n_chunks;
     int dp_tiles, sk_tiles, sk_ctas;
+    int split_s;
     // divisors of the per-tile / per-segment index arithmetic
     FastDiv div_tn, div_hw, div_wo, div_cchunk, div_kw;
     float *partials;     // slot b: CTA b's part of a split tile, [BN/4][128] float4
@@ -232,6 +239,7 @@ struct TcSched {
 
 struct TcSeg {
     int tile, c0, c1;    // chunk iterations [c0, c1) of tile
+    int slot;            // split mode: the item's partial slot
 };
 
 __device__ __forceinline__ int64_t sk_start(int b, int64_t W, int G) { return static_cast<int64_t>(b) * W / G; }
@@ -242,7 +250,7 @@ __device__ __forceinline__ int sk_owner(int64_t q, int64_t W, int G)
 }
 
 struct TcSegIter {
-    int b, G, n_dp, i_dp, C, dp_tiles;
+    int b, G, n_dp, i_dp, C, dp_tiles, split_s, n_tiles;
     int64_t s, e;        // stream-K range still to walk: [s, e), from e down
     __device__ TcSegIter(const TcSched &sc)
     {
@@ -250,7 +258,10 @@ struct TcSegIter {
         G = gridDim.x;
         C = sc.n_chunks;
         dp_tiles = sc.dp_tiles;
-        n_dp = dp_tiles > b ? (dp_tiles - 1 - b) / G + 1 : 0;
+        split_s = sc.split_s;
+        n_tiles = sc.n_tiles;
+        const int items = split_s > 0 ? n_tiles * split_s : dp_tiles;
+        n_dp = items > b ? (items - 1 - b) / G + 1 : 0;
         i_dp = 0;
         const int64_t W = static_cast<int64_t>(sc.sk_tiles) * C;
         s = b < sc.sk_ctas ? sk_start(b, W, sc.sk_ctas) : 0;
@@ -258,6 +269,18 @@ struct TcSegIter {
     }
     __device__ bool next(TcSeg &sg)
     {
+        if (split_s > 0) {
+            if (i_dp >= n_dp) return false;
+            const int i = b + i_dp * G;
+            const int slice = i / n_tiles;
+            sg.tile = i - slice * n_tiles;
+            sg.c0 = static_cast<int>(static_cast<int64_t>(slice) * C / split_s);
+            sg.c1 = static_cast<int>(static_cast<int64_t>(slice + 1) * C / split_s);
+            sg.slot = i;
+            ++i_dp;
+            return true;
+        }
+        sg.slot = -1;
         if (i_dp < n_dp) {
             sg.tile = b + i_dp * G;
             sg.c0 = 0;
@@ -275,7 +298,18 @@ struct TcSegIter {
         return true;
     }
     // chunk iterations of this CTA
-    __device__ int64_t total() const { return static_cast<int64_t>(n_dp) * C + (e - s); }
+    __device__ int64_t total() const
+    {
+        if (split_s > 0) {
+            int64_t n = 0;
+            for (int j = 0; j < n_dp; ++j) {
+                const int i = b + j * G, slice = i / n_tiles;
+                n += static_cast<int64_t>(slice + 1) * C / split_s - static_cast<int64_t>(slice) * C / split_s;
+            }
+            return n;
+        }
+        return static_cast<int64_t>(n_dp) * C + (e - s);
+    }
 };
 
 template <typename Tr, int BN>
@@ -603,6 +637,24 @@ tc_conv_kernel(const ConvArgs a, const __grid_constant__ CUtensorMap tmap_x,
                 }
             };
 
+            if (sched.split_s > 0) {
+                // ---- split mode: the item's accumulator -> its partial slot ----
+                float4 *mine = reinterpret_cast<float4 *>(sched.partials) + static_cast<int64_t>(sg.slot) * kSlotF4;
+#pragma unroll 1
+                for (int at = 0; at < kAtoms; ++at) {
+                    uint32_t r[kLd][32];
+                    load_atom(at, r);
+#pragma unroll
+                    for (int v4 = 0; v4 < kAtomCols / 4; ++v4) {
+                        const int e = 4 * v4;
+                        __stcg(mine + (at * kAtomCols / 4 + v4) * kBM + row,
+                               make_float4(__uint_as_float(r[e / 32][e % 32]), __uint_as_float(r[e / 32][e % 32 + 1]),
+                                           __uint_as_float(r[e / 32][e % 32 + 2]),
+                                           __uint_as_float(r[e / 32][e % 32 + 3])));
+                    }
+                }
+                continue;
+            }
             if (sg.c0 == 0 && sg.c1 == sched.n_chunks) {
                 // ---- whole tile: accumulator -> bias / ReLU -> y ----
                 stage_bias();
@@ -806,7 +858,7 @@ bool tmap_2d(CUtensorMap *m, CUtensorMapDataType type, int elem, const void *ptr
 
 template <typename Tr, int BN>
 cudaError_t launch_bn(const ConvArgs &a, const typename Tr::T *W, const typename Tr::T *W_lo, void *sk_space,
-                      cudaStream_t st)
+                      cudaStream_t st, int split_s = 0, float *split_partials = nullptr)
 {
     using L = TcLayout<Tr, BN>;
     constexpr int elem = sizeof(typename Tr::T);
@@ -858,7 +910,10 @@ cudaError_t launch_bn(const ConvArgs &a, const typename Tr::T *W, const typename
     } else {
         tmap_wlo = tmap_w;                                     // unused
     }
-    if (!tmap_2d(&tmap_y, Tr::kTmap, elem, a.y, a.P_pix, a.C_out, 32)) return cudaErrorInvalidValue;
+    if (split_s > 0)
+        tmap_y = tmap_w;                                       // split mode stores no y
+    else if (!tmap_2d(&tmap_y, Tr::kTmap, elem, a.y, a.P_pix, a.C_out, 32))
+        return cudaErrorInvalidValue;
     // the shared-memory opt-in, once per device for this kernel
     static std::mutex attr_mu;
     static bool attr_done[64];
@@ -898,7 +953,13 @@ cudaError_t launch_bn(const ConvArgs &a, const typename Tr::T *W, const typename
     // leaving the round ragged: the fixup and the shorter segments cost more
     // than the idle SMs.)
     const int G = sms < kPlanCTAs ? sms : kPlanCTAs;
-    if (sk_space && sc.n_tiles < G && sc.n_chunks >= sk_min_chunks(Tr::kSplit)) {
+    if (split_s > 0) {
+        if (split_s > sc.n_chunks || !split_partials) return cudaErrorInvalidValue;   // every item non-empty
+        sc.split_s = split_s;
+        sc.partials = split_partials;
+        const int items = sc.n_tiles * split_s;
+        grid = items < sms ? items : sms;
+    } else if (sk_space && sc.n_tiles < G && sc.n_chunks >= sk_min_chunks(Tr::kSplit)) {
         const int dp = (sc.n_tiles / G) * G, skt = sc.n_tiles - dp;
         const int64_t iters = static_cast<int64_t>(skt) * sc.n_chunks;
         int need = (sc.n_chunks + L::kRingSlots - 1) / L::kRingSlots;
@@ -1075,6 +1136,72 @@ cudaError_t tc_gemm(const ConvArgs &a, int dtype, const void *workspace, size_t 
 {
     return gemm_any(a, dtype, workspace, ws_bytes, st);
 }
+
+// ---- the GEMM on caller-given operands (the backward passes) ----
+
+// The conv GEMM of `a` with the weights W (and W_lo for fp32) at explicit
+// addresses instead of the workspace's decode: the input gradient runs the
+// forward kernel on the flipped, transposed weights.
+cudaError_t tc_gemm_weights(const ConvArgs &a, int dtype, const void *W, const void *W_lo, void *sk_space,
+                            cudaStream_t st)
+{
+    if (a.P_pix == 0) return cudaSuccess;
+    const int bn = tc_bn(a);
+    if (dtype == ONEXN_F32) {
+        const float *w = static_cast<const float *>(W), *wl = static_cast<const float *>(W_lo);
+        if (bn == 64) return launch_bn<TcF32, 64>(a, w, wl, sk_space, st);
+        if (bn == 128) return launch_bn<TcF32, 128>(a, w, wl, sk_space, st);
+        return launch_bn<TcF32, 256>(a, w, wl, sk_space, st);
+    }
+    const __nv_bfloat16 *w = static_cast<const __nv_bfloat16 *>(W);
+    if (bn == 64) return launch_bn<TcBf16, 64>(a, w, w, sk_space, st);
+    if (bn == 128) return launch_bn<TcBf16, 128>(a, w, w, sk_space, st);
+    return launch_bn<TcBf16, 256>(a, w, w, sk_space, st);
+}
+
+// Plan of a split-mode GEMM C[M][N] = A[M][K] B[N][K]^T (K-major operands,
+// K a multiple of 64): column tile BN, slices S (about one item per SM,
+// at most one per K chunk) and the partial bytes (items x 128 x BN fp32).
+TcSplitPlan tc_split_plan(int M, int Ncols, int64_t K, int dtype)
+{
+    TcSplitPlan p{};
+    ConvArgs a{};
+    a.P_pix = M;
+    a.C_out = Ncols;
+    p.bn = tc_bn(a);
+    const int64_t tiles = ((static_cast<int64_t>(M) + kBM - 1) / kBM) * ((Ncols + p.bn - 1) / p.bn);
+    const int64_t chunks = (K + (dtype == ONEXN_F32 ? TcF32::kBK : TcBf16::kBK) - 1) /
+                           (dtype == ONEXN_F32 ? TcF32::kBK : TcBf16::kBK);
+    int64_t S = kPlanCTAs / (tiles > 0 ? tiles : 1);
+    if (S < 1) S = 1;
+    if (S > chunks) S = chunks > 0 ? chunks : 1;
+    p.tiles = static_cast<int>(tiles);
+    p.n_tn = (Ncols + p.bn - 1) / p.bn;
+    p.split_s = static_cast<int>(S);
+    p.partial_bytes = static_cast<size_t>(tiles * S) * kBM * p.bn * 4;
+    return p;
+}
+
+// The split-mode GEMM: A = x [M][K] (a.x), B = W [N][K] (and W_lo), the
+// item accumulators into partials (plan.partial_bytes).
+cudaError_t tc_gemm_split(const ConvArgs &a, int dtype, const void *W, const void *W_lo, float *partials,
+                          const TcSplitPlan &plan, cudaStream_t st)
+{
+    if (a.P_pix == 0) return cudaSuccess;
+    if (dtype == ONEXN_F32) {
+        const float *w = static_cast<const float *>(W), *wl = static_cast<const float *>(W_lo);
+        if (plan.bn == 64) return launch_bn<TcF32, 64>(a, w, wl, nullptr, st, plan.split_s, partials);
+        if (plan.bn == 128) return launch_bn<TcF32, 128>(a, w, wl, nullptr, st, plan.split_s, partials);
+        return launch_bn<TcF32, 256>(a, w, wl, nullptr, st, plan.split_s, partials);
+    }
+    const __nv_bfloat16 *w = static_cast<const __nv_bfloat16 *>(W);
+    if (plan.bn == 64) return launch_bn<TcBf16, 64>(a, w, w, nullptr, st, plan.split_s, partials);
+    if (plan.bn == 128) return launch_bn<TcBf16, 128>(a, w, w, nullptr, st, plan.split_s, partials);
+    return launch_bn<TcBf16, 256>(a, w, w, nullptr, st, plan.split_s, partials);
+}
+
+size_t tc_weights_bytes(const ConvArgs &a, int dtype) { return weights_bytes(a, dtype); }
+size_t tc_sk_bytes(const ConvArgs &a) { return sk_bytes(a); }
 
 // decode, then the GEMM as its programmatic dependent (its launch and
 // prologue overlap the decode)

@@ -65,7 +65,9 @@ class PrunedConv2d:
         self._descs = []
         # workspaces whose decoded weights a completed-in-order tc call has
         # written: later calls on them pass ONEXN_DECODED and skip the decode
+        # (until D changes: an optimizer step bumps its version counter)
         self._decoded = set()
+        self._d_version = self.D._version
 
     @property
     def torch_dtype(self):
@@ -112,6 +114,10 @@ class PrunedConv2d:
         if y is None:
             y = torch.empty(self.out_shape(x.shape), dtype=x.dtype, device=x.device)
         s = torch.cuda.current_stream(x.device) if stream is None else stream
+        if self.D._version != self._d_version:          # weights updated in place: decode again
+            self._decoded.clear()
+            self._args.clear()
+            self._d_version = self.D._version
         flags = act_flags(relu) | algo | self._reuse_flag()
         key = (x.data_ptr(), y.data_ptr(), x.shape, x.stride(), x.dtype, y.shape, y.stride(), y.dtype,
                None if residual is None else (residual.data_ptr(), residual.shape, residual.stride(),
@@ -178,6 +184,66 @@ class PrunedConv2d:
             self._ws[key] = torch.empty(max(n, 256), dtype=torch.uint8, device=self.device)
         return self._ws[key]
 
+    # ---------------------------------------------- fine-tuning (mask fixed)
+
+    def backward(self, x: torch.Tensor, dy: torch.Tensor, dx: torch.Tensor = None, *, need_dx: bool = True,
+                 need_dw: bool = True, need_db: bool = True, accumulate: bool = False, stream=None):
+        """Gradients with the mask held fixed (onexn_conv_bwd_data /
+        onexn_conv_bwd_weight): dy is the gradient of the pre-activation
+        output (NHWC like forward's y).  Returns (dx, dD, db): dx like x
+        (added to a given dx with accumulate=True), dD fp32 [t, N] in D's
+        order (only the kept blocks), db fp32 [C_out]; None where not asked."""
+        if dy.dtype != self.torch_dtype or not dy.is_cuda or not dy.is_contiguous():
+            raise ValueError(f"dy must be a contiguous CUDA {self.torch_dtype} NHWC tensor")
+        if x.dtype != self.torch_dtype or not x.is_contiguous():
+            raise ValueError(f"x must be a contiguous CUDA {self.torch_dtype} NHWC tensor")
+        B, H, W, _ = x.shape
+        if tuple(dy.shape) != tuple(self.out_shape(x.shape)):
+            raise ValueError(f"dy must have shape {self.out_shape(x.shape)}")
+        desc = self.desc(B, H, W)
+        s = torch.cuda.current_stream(x.device) if stream is None else stream
+        dD = db = None
+        if need_dx:
+            if dx is None:
+                dx = (torch.zeros_like(x) if accumulate else torch.empty_like(x))
+            key = ("bwd_data", B, H, W)
+            if key not in self._ws:
+                n = _c.onexn_conv_bwd_data_workspace_size(desc, self.N, self.t, self.cdtype)
+                self._ws[key] = torch.empty(max(n, 256), dtype=torch.uint8, device=self.device)
+            _c.onexn_conv_bwd_data(desc, self.P, self.I, self.D, self.N, self.t, dy, dx, self.cdtype,
+                                   _c.ONEXN_ACCUMULATE if accumulate else 0, self._ws[key], s)
+        else:
+            dx = None
+        if need_dw or need_db:
+            key = ("bwd_weight", B, H, W)
+            if key not in self._ws:
+                n = _c.onexn_conv_bwd_weight_workspace_size(desc, self.N, self.cdtype)
+                self._ws[key] = torch.empty(max(n, 256), dtype=torch.uint8, device=self.device)
+            dD = torch.empty((max(self.t, 1), self.N), dtype=torch.float32, device=x.device)[:self.t]
+            db = torch.empty(self.C_out, dtype=torch.float32, device=x.device) if need_db else None
+            _c.onexn_conv_bwd_weight(desc, self.P, self.I, self.N, self.t, x, dy, dD if self.t else None, db,
+                                     self.cdtype, self._ws[key], s)
+            if not need_dw:
+                dD = None
+        return dx, dD, db
+
+    def parameters(self):
+        """The trainable tensors of the pruned layer: D (the kept blocks, Sec.
+        3.4) and the bias, with requires_grad set; the mask (P, I) is fixed."""
+        self.D.requires_grad_(True)
+        out = [self.D]
+        if self.bias is not None:
+            self.bias.requires_grad_(True)
+            out.append(self.bias)
+        return out
+
+    def train_forward(self, x: torch.Tensor) -> torch.Tensor:
+        """Forward as a differentiable op of (x, D, bias) for fine-tuning:
+        the backward runs onexn_conv_bwd_data / onexn_conv_bwd_weight.  The
+        output is the linear (pre-activation) convolution; apply the
+        activation with torch (its backward is elementwise)."""
+        return _PrunedConvFn.apply(x, self.D, self.bias, self)
+
     def forward_host(self, x_host: torch.Tensor, y_host: torch.Tensor = None, relu: bool = False,
                      algo: int = _c.ONEXN_ALGO_AUTO, stream=None, sync: bool = True) -> torch.Tensor:
         """End to end from host memory (onexn_conv_fwd_host): the input is
@@ -206,6 +272,26 @@ class PrunedConv2d:
         if sync:
             stream.synchronize()
         return y_host
+
+
+class _PrunedConvFn(torch.autograd.Function):
+    @staticmethod
+    def forward(ctx, x, D, bias, layer):
+        ctx.layer = layer
+        ctx.save_for_backward(x)
+        with torch.no_grad():
+            return layer.forward(x.contiguous())
+
+    @staticmethod
+    def backward(ctx, gy):
+        (x,) = ctx.saved_tensors
+        layer = ctx.layer
+        need_dx, need_dw, need_db = ctx.needs_input_grad[0], ctx.needs_input_grad[1], ctx.needs_input_grad[2]
+        dx, dD, db = layer.backward(x.contiguous(), gy.contiguous(), need_dx=need_dx, need_dw=need_dw,
+                                    need_db=need_db)
+        if dD is not None:
+            dD = dD.to(layer.D.dtype)
+        return dx, dD, db, None
 
 
 class DepthwiseConv2d:

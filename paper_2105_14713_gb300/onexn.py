@@ -20,6 +20,7 @@ ONEXN_RELU = 0x1
 ONEXN_RELU6 = 0x2
 ONEXN_DECODED = 0x10
 ONEXN_REUSE_DECODE = 0x20
+ONEXN_ACCUMULATE = 0x40
 ONEXN_ALGO_SHIFT = 8
 ONEXN_ALGO_MASK = 0xF << ONEXN_ALGO_SHIFT
 ONEXN_ALGO_AUTO = 0 << ONEXN_ALGO_SHIFT
@@ -74,6 +75,12 @@ SIGNATURES = {
     "onexn_prune_device": ([_P, _I32, _I32, _I32, _I32, _I32, _DBL, _I32, _P, _P, _P, ctypes.c_size_t, _P],
                            _I32),
     "onexn_pack_device_workspace_size": ([_I32, _I32, _P], _I32),
+    "onexn_conv_bwd_data_workspace_size": ([ctypes.POINTER(ConvDesc), _I32, _I64, _I32, _P], _I32),
+    "onexn_conv_bwd_data": ([ctypes.POINTER(ConvDesc), _P, _P, _P, _I32, _I64, _P, _P, _I32, _U32, _P,
+                             ctypes.c_size_t, _P], _I32),
+    "onexn_conv_bwd_weight_workspace_size": ([ctypes.POINTER(ConvDesc), _I32, _I32, _P], _I32),
+    "onexn_conv_bwd_weight": ([ctypes.POINTER(ConvDesc), _P, _P, _I32, _I64, _P, _P, _P, _P, _I32, _P,
+                               ctypes.c_size_t, _P], _I32),
     "onexn_pack_device": ([_P, _P, _I32, _I32, _I32, _I32, _I32, _I32, _P, _P, _P, _I64, _P, ctypes.c_size_t,
                            _P], _I32),
 }
@@ -336,3 +343,38 @@ def onexn_pack_device(W, mask, N: int, t: int, wdtype: int = ONEXN_F32, stream=N
     _check(lib.onexn_pack_device(ptr(W), ptr(mask), C_out, C_in, KH, KW, int(N), int(wdtype), ptr(P), ptr(I),
                                  ptr(D), int(t), ptr(ws), ws.numel(), ctypes.c_void_p(s.cuda_stream)))
     return P, I[:t], D[:t]
+
+
+def onexn_conv_bwd_data_workspace_size(desc: ConvDesc, N: int, t: int, dtype: int) -> int:
+    out = ctypes.c_size_t(0)
+    _check(lib.onexn_conv_bwd_data_workspace_size(ctypes.byref(desc), int(N), int(t), int(dtype),
+                                                  ctypes.byref(out)))
+    return out.value
+
+
+def onexn_conv_bwd_data(desc: ConvDesc, P, I, D, N: int, t: int, dy, dx, dtype: int, flags: int = 0,
+                        workspace=None, stream=None) -> None:
+    """Input gradient of the pruned convolution (CUDA tensors; dy is the
+    gradient of the pre-activation output)."""
+    s = _cuda_stream(dy, stream)
+    ptr = (lambda x: None if x is None else ctypes.c_void_p(x.data_ptr()))
+    _check(lib.onexn_conv_bwd_data(ctypes.byref(desc), ptr(P), ptr(I), ptr(D), int(N), int(t), ptr(dy), ptr(dx),
+                                   int(dtype), int(flags), ptr(workspace),
+                                   0 if workspace is None else workspace.numel(), ctypes.c_void_p(s.cuda_stream)))
+
+
+def onexn_conv_bwd_weight_workspace_size(desc: ConvDesc, N: int, dtype: int) -> int:
+    out = ctypes.c_size_t(0)
+    _check(lib.onexn_conv_bwd_weight_workspace_size(ctypes.byref(desc), int(N), int(dtype), ctypes.byref(out)))
+    return out.value
+
+
+def onexn_conv_bwd_weight(desc: ConvDesc, P, I, N: int, t: int, x, dy, dD, db, dtype: int, workspace=None,
+                          stream=None) -> None:
+    """Kept-weight gradient in BSR order (dD CUDA fp32 [t, N]) and optionally
+    the bias gradient (db CUDA fp32 [C_out])."""
+    s = _cuda_stream(dy, stream)
+    ptr = (lambda x_: None if x_ is None else ctypes.c_void_p(x_.data_ptr()))
+    _check(lib.onexn_conv_bwd_weight(ctypes.byref(desc), ptr(P), ptr(I), int(N), int(t), ptr(x), ptr(dy), ptr(dD),
+                                     ptr(db), int(dtype), ptr(workspace),
+                                     0 if workspace is None else workspace.numel(), ctypes.c_void_p(s.cuda_stream)))
