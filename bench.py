@@ -11,6 +11,8 @@ flushed with a 256 MB write before every step, outside the timed events):
   6  fully connected 1280 -> 1000 as a 1x1 conv on 256 1x1 inputs, fp32 + bf16, N=4, 50%
   7  MobileNet-V2's 17 inverted-residual blocks at batch 1 (224x224 input), fp32, N=4, 50%:
      latency of one image through the blocks, replayed as one CUDA graph
+  8  fine-tuning step of the config-2 layer with the mask fixed: forward, input gradient,
+     kept-weight and bias gradients, SGD update of D; fp32 leg + bf16 leg
 
 A "step" is one pass over every layer (leg) of the workload.  Prints one JSON
 line.  Metric: effective TFLOP/s = 2 * pixels * t * N / time summed over the
@@ -59,6 +61,9 @@ DESCRIPTIONS = {
     7: "MobileNet-V2 (width 1.0) 17 inverted-residual blocks (expand 1x1 + ReLU6, dense depthwise "
        "3x3 + ReLU6, project 1x1 + residual), batch 1, 224x224 input, fp32; 1xN N=4, 50% block rate "
        "on both 1x1 convs; one CUDA graph per image",
+    8: "fine-tuning step (mask fixed) of the ResNet-50 stage-2 3x3 conv, 64x28x28x128 -> 128, s1 p1, "
+       "NHWC; 1xN N=8, 50% block rate: forward (weights decoded every step), input gradient, kept-weight "
+       "(BSR order) and bias gradients, SGD update of D; fp32 leg + bf16-in/fp32-acc leg",
 }
 
 
@@ -325,6 +330,9 @@ def run_reference(args, rank, ws):
     if args.config == 7:
         run_reference_mbv2(args)
         return
+    if args.config == 8:
+        run_reference_train(args)
+        return
     cfg = args.config if args.config != 5 else 2
     layers = workload(cfg)
     packs = oracle_setup(layers)
@@ -497,7 +505,7 @@ def measure(layers, args, dev, stream, flush, ws, pk, sampler=None):
 
 def main():
     ap = argparse.ArgumentParser()
-    ap.add_argument("--config", type=int, default=2, choices=[1, 2, 3, 4, 5, 6, 7])
+    ap.add_argument("--config", type=int, default=2, choices=[1, 2, 3, 4, 5, 6, 7, 8])
     ap.add_argument("--gpus", type=int, default=1)
     # default: a timed region of ~1 s on the default workload, so that the
     # clock samples (every 50 ms) fall inside it
@@ -526,6 +534,9 @@ def main():
         return
     if args.config == 7:
         run_mbv2(args, dev, stream, flush, ws, rank, local, pk)
+        return
+    if args.config == 8:
+        run_train(args, dev, stream, flush, ws, rank, local, pk)
         return
 
     layers = workload(args.config)
@@ -880,6 +891,203 @@ def run_reference_mbv2(args):
         "cpu_baseline": {"value": ms, "unit": "ms", "cores": oracle.num_threads(), "kind": "oracle",
                          "sample": f"{args.steps} full images through the 17 blocks"},
         "e2e": {"value": ms, "unit": "ms", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }), flush=True)
+
+
+# --------------------------------------------------------------------------
+# config 8: fine-tuning step with the mask fixed
+# --------------------------------------------------------------------------
+
+TRAIN_METRIC = "1xN fine-tuning step (fwd + input grad + kept-weight grad) effective TFLOP/s"
+TRAIN_PASSES = ("forward", "input_grad", "weight_grad", "sgd_update")
+
+
+def train_legs(dev):
+    from paper_2105_14713_gb300 import workloads as wl
+    from paper_2105_14713_gb300.layer import PrunedConv2d
+    legs = []
+    for layer in (wl.config2("f32")[0], wl.config2("bf16")[0]):
+        W = wl.weights(layer).numpy()
+        conv = PrunedConv2d(W, layer.N, layer.rate, bias=wl.bias(layer).numpy(), stride=layer.stride,
+                            padding=layer.pad, dilation=layer.dil, dtype=layer.dtype, device=dev,
+                            reuse_decoded=False)
+        tdt = torch.float32 if layer.dtype == "f32" else torch.bfloat16
+        x_cpu = wl.activations(layer).to(tdt)
+        g = torch.Generator().manual_seed(17)
+        dy_cpu = (torch.randn((layer.B, layer.Ho, layer.Wo, layer.C_out), generator=g) * 1e-3).to(tdt)
+        x, dy = x_cpu.to(dev), dy_cpu.to(dev)
+        legs.append({"layer": layer, "conv": conv, "x": x, "dy": dy, "x_cpu": x_cpu, "dy_cpu": dy_cpu,
+                     "y": torch.empty(conv.out_shape(x.shape), dtype=tdt, device=dev),
+                     "dx": torch.empty_like(x)})
+    return legs
+
+
+def train_step(lg, lr=1e-3, evs=None, stream=None):
+    conv = lg["conv"]
+    if evs is not None:
+        evs[0].record(stream)
+    conv(lg["x"], lg["y"])
+    if evs is not None:
+        evs[1].record(stream)
+    _, _, _ = conv.backward(lg["x"], lg["dy"], lg["dx"], need_dw=False, need_db=False)
+    if evs is not None:
+        evs[2].record(stream)
+    _, dD, db = conv.backward(lg["x"], lg["dy"], need_dx=False)
+    if evs is not None:
+        evs[3].record(stream)
+    with torch.no_grad():
+        conv.D.add_(dD.to(conv.D.dtype), alpha=-lr)
+        conv.bias.add_(db, alpha=-lr)
+    if evs is not None:
+        evs[4].record(stream)
+    return db
+
+
+def train_flops(lg):
+    # forward, input gradient and weight gradient each do the kept 2*P*t*N
+    return 3 * kept_flops(lg["layer"], lg["conv"].t)
+
+
+def run_train(args, dev, stream, flush, ws, rank, local, pk):
+    legs = train_legs(dev)
+    for _ in range(args.warmup):
+        for lg in legs:
+            train_step(lg)
+    torch.cuda.synchronize()
+    steps = args.steps
+    evs = [[[torch.cuda.Event(enable_timing=True) for _ in range(5)] for _ in legs] for _ in range(steps)]
+    sampler = ClockSampler(local)
+    barrier(ws)
+    torch.cuda.synchronize()
+    with sampler:
+        wall0 = time.perf_counter()
+        for k in range(steps):
+            flush.fill_(k & 0xff)
+            for i, lg in enumerate(legs):
+                train_step(lg, evs=evs[k][i], stream=stream)
+        torch.cuda.synchronize()
+        wall = time.perf_counter() - wall0
+    per = [[[evs[k][i][j].elapsed_time(evs[k][i][j + 1]) for j in range(4)] for k in range(steps)]
+           for i in range(len(legs))]
+    step_ms = sum(sum(sum(pp) for pp in per[i]) for i in range(len(legs))) / steps
+    step_ms = max_over_ranks(step_ms, ws)
+    flops = sum(train_flops(lg) for lg in legs)
+    info, rfs = [], []
+    for i, lg in enumerate(legs):
+        layer, t = lg["layer"], lg["conv"].t
+        ms = [sum(per[i][k][j] for k in range(steps)) / steps for j in range(4)]
+        entry = {"name": layer.name, "dtype": layer.dtype, "ms": dict(zip(TRAIN_PASSES, ms)),
+                 "tflops": {TRAIN_PASSES[j]: kept_flops(layer, t) / (ms[j] * 1e-3) / 1e12 for j in range(3)}}
+        for j in range(3):
+            rf = leg_roofline(layer, t, "tc", ms[j], pk)
+            rf["kernel"] = f"{TRAIN_PASSES[j]} ({layer.name})"
+            rfs.append((ms[j], rf))
+        info.append(entry)
+    dom = max(rfs, key=lambda r: r[0])[1]
+    dom["traffic"] = None
+    dom["note"] = "the pass with the largest time; its kept flops against the pipe it runs on"
+    # end to end: x and dy from pinned host memory each step, db[0] read back
+    pins = [(lg["x_cpu"].pin_memory(), lg["dy_cpu"].pin_memory()) for lg in legs]
+    out = torch.empty(1, dtype=torch.float32, pin_memory=True)
+    e2e = []
+    for r in range(args.warmup + min(steps, 200)):
+        flush.fill_(r & 0xff)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for lg, (xp, dyp) in zip(legs, pins):
+            lg["x"].copy_(xp, non_blocking=True)
+            lg["dy"].copy_(dyp, non_blocking=True)
+            db = train_step(lg)
+            out.copy_(db[:1], non_blocking=True)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        if r >= args.warmup:
+            e2e.append(e0.elapsed_time(e1))
+    e2e_ms = max_over_ranks(sum(e2e) / len(e2e), ws)
+    h2d = sum(a.numel() * a.element_size() + b.numel() * b.element_size() for a, b in pins)
+    cpu = None
+    if rank == 0 and ws == 1 and not args.no_cpu_baseline:
+        cpu = train_cpu_baseline(legs)
+    # our kernels per leg: forward decode + GEMM; input gradient decode +
+    # transpose + GEMM; weight gradient two transposes + GEMM + gather + bias
+    launches = 10 * len(legs)
+    if rank == 0:
+        print(json.dumps({
+            "metric": TRAIN_METRIC, "value": ws * flops / (step_ms * 1e-3) / 1e12, "unit": "TFLOP/s",
+            "n_gpus": ws, "steps": steps, "warmup": args.warmup, "ms_per_step": step_ms,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16+f32",
+            "data": "synthetic (seeded Kaiming-normal weights, ReLU(N(0,1)) activations, N(0,1e-3) output "
+                    "gradients)",
+            "config": {"workload": DESCRIPTIONS[8], "config_id": 8, "layers": 2, "batch": 64, "N": 8,
+                       "rate": 0.5, "parallelism": "replicas", "l2": "flushed before every step (256 MB write)"},
+            "roofline": dom, "legs": info,
+            "e2e": {"value": ws * flops / (e2e_ms * 1e-3) / 1e12, "unit": "TFLOP/s", "h2d_bytes_per_step": h2d,
+                    "d2h_bytes_per_step": 4 * len(legs), "ms_per_step": e2e_ms},
+            "gpu_launches": launches * steps, "clocks": sampler.summary(), "wall_s_timed_region": wall,
+            "peaks": pk, "cpu_baseline": cpu}), flush=True)
+
+
+def train_oracle_setup(layers):
+    import oracle
+    from paper_2105_14713_gb300 import workloads as wl
+    out = []
+    for layer in layers:
+        W = wl.weights(layer).numpy()
+        mask, _ = oracle.prune(W, layer.N, layer.rate)
+        x = wl.activations(layer.with_(B=1)).numpy()
+        g = torch.Generator().manual_seed(17)
+        dy = (torch.randn((1, layer.Ho, layer.Wo, layer.C_out), generator=g) * 1e-3).numpy()
+        if layer.dtype == "bf16":
+            W, x, dy = oracle.round_bf16(W), oracle.round_bf16(x), oracle.round_bf16(dy)
+        out.append((layer, W, mask, x, dy))
+    return out
+
+
+def train_oracle_pass(packs):
+    """The oracle's forward, input gradient and weight gradient on image 0."""
+    import oracle
+    t0 = time.perf_counter()
+    flops = 0.0
+    for layer, W, mask, x, dy in packs:
+        g = ((layer.stride,) * 2, (layer.pad,) * 2, (layer.dil,) * 2)
+        oracle.conv_masked(x, W, mask, None, layer.N, *g)
+        oracle.conv_backward_data(dy, W, mask, layer.N, (layer.H, layer.W), *g)
+        oracle.conv_backward_weight(x, dy, (layer.KH, layer.KW), mask, layer.N, *g)
+        flops += 3 * 2.0 * layer.Ho * layer.Wo * int(mask.sum()) * layer.N
+    return time.perf_counter() - t0, flops
+
+
+def train_cpu_baseline(legs, budget_s: float = 10.0):
+    import oracle
+    packs = train_oracle_setup([lg["layer"] for lg in legs])
+    spent, flops, n = 0.0, 0.0, 0
+    while spent < budget_s and n < 20:
+        dt, fl = train_oracle_pass(packs)
+        spent += dt
+        flops += fl
+        n += 1
+    return {"value": flops / spent / 1e12, "unit": "TFLOP/s", "cores": oracle.num_threads(), "kind": "oracle",
+            "sample": f"{n} passes of forward + input gradient + weight gradient on image 0 of both legs; "
+                      f"fp64 plain-C oracle; {spent:.1f} s"}
+
+
+def run_reference_train(args):
+    import oracle
+    from paper_2105_14713_gb300 import workloads as wl
+    packs = train_oracle_setup([wl.config2("f32")[0], wl.config2("bf16")[0]])
+    for _ in range(args.warmup):
+        train_oracle_pass(packs)
+    res = [train_oracle_pass(packs) for _ in range(args.steps)]
+    v = sum(f for _, f in res) / sum(t for t, _ in res) / 1e12
+    ms = 1e3 * sum(t for t, _ in res) / len(res)
+    print(json.dumps({
+        "impl": "reference", "metric": TRAIN_METRIC, "value": v, "unit": "TFLOP/s", "n_gpus": args.gpus,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": DESCRIPTIONS[8], "config_id": 8, "parallelism": "replicas", "l2": "cpu oracle"},
+        "cpu_baseline": {"value": v, "unit": "TFLOP/s", "cores": oracle.num_threads(), "kind": "oracle",
+                         "sample": "per step image 0 of both legs: forward + input and weight gradients"},
+        "e2e": {"value": v, "unit": "TFLOP/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }), flush=True)
 
 

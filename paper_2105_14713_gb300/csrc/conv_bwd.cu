@@ -11,13 +11,16 @@
 // beyond d(K-1)) use a direct kernel over the decoded W.
 //
 // Kept-weight gradient dW[o][k] = sum_p dy[p][o] * xcol[p][k] (k = tap*C_in
-// + c, xcol the im2col view of x): a GEMM with M = C_out, N = K and the
-// pixels as its long reduction dimension.  dy and xcol are transposed once
-// into K-major operands (pixels padded to 64 with zeros; fp32: xcol split
-// into its tf32 rounding and the rest, as the decode does for weights), the
-// GEMM runs in split mode (items of pixel slices, one accumulator slot
-// each), and a gather kernel adds each kept block's S slots in slice order
-// into dD[z][n] = dW[g*N + n][I[z]] (fp32), only for the kept blocks.
+// + c, xcol the im2col view of x): a GEMM with the pixels as its long
+// reduction dimension, run as dW^T[k][o] (M = K rows, N = C_out columns) so
+// that the large operand, xcol, is the A operand: it is transposed once into
+// pixel-contiguous rows (pixels padded to 64 with zeros) and, for fp32, split
+// into tf32 high and low parts on the fly by the GEMM's split warps; dy is
+// the small B operand, transposed with its tf32 split (fp32) and per-32-pixel
+// column sums for the bias gradient.  The GEMM runs in split mode (items of
+// pixel slices, one accumulator slot each) and a gather kernel adds each kept
+// block's S slots in slice order into dD[z][n] = dW[g*N + n][I[z]] (fp32),
+// only for the kept blocks.
 #include "conv_common.cuh"
 #include "conv_dispatch.h"
 #include "onexn_internal.h"
@@ -46,10 +49,14 @@ __device__ __forceinline__ float to_f(T v)
     else return __bfloat162float(v);
 }
 
-// dYt[o][p] = dY[p][o] for p < P, 0 for P <= p < P_pad.
+// dYt[o][p] = dY[p][o] for p < P, 0 for P <= p < P_pad (fp32: as its tf32
+// rounding `hi` and the rest `lo`, the B operand of the weight-gradient
+// GEMM), and the column sums of each 32-pixel block, colsum[o][blockIdx.x]
+// (the bias gradient's first stage).
 template <typename T>
 __global__ void __launch_bounds__(kTile * 8)
-dy_transpose_kernel(const T *__restrict__ dy, int64_t P, int64_t P_pad, int C_out, T *__restrict__ dyt)
+dy_transpose_kernel(const T *__restrict__ dy, int64_t P, int64_t P_pad, int C_out, T *__restrict__ hi,
+                    T *__restrict__ lo, float *__restrict__ colsum, int n_pb)
 {
     __shared__ T tile[kTile][kTile + 1];
     const int64_t p0 = static_cast<int64_t>(blockIdx.x) * kTile;
@@ -61,46 +68,16 @@ dy_transpose_kernel(const T *__restrict__ dy, int64_t P, int64_t P_pad, int C_ou
         tile[i][tx] = (p < P && o < C_out) ? dy[p * C_out + o] : T(0.f);
     }
     __syncthreads();
+    if (ty == 0 && o0 + tx < C_out) {
+        float c = 0.f;
+        for (int i = 0; i < kTile; ++i) c += to_f(tile[i][tx]);
+        colsum[static_cast<int64_t>(o0 + tx) * n_pb + blockIdx.x] = c;
+    }
     for (int i = ty; i < kTile; i += 8) {
         const int o = o0 + i;
         const int64_t p = p0 + tx;
-        if (o < C_out && p < P_pad) dyt[static_cast<int64_t>(o) * P_pad + p] = tile[tx][i];
-    }
-}
-
-// XcolT[tap*C_in + c][p] = x[b, oh*sh - ph + kh*dh, ow*sw - pw + kw*dw, c]
-// (0 outside the image and for p >= P); fp32 as hi (tf32) and lo parts.
-template <typename T>
-__global__ void __launch_bounds__(kTile * 8)
-xcol_transpose_kernel(const ConvArgs a, int64_t P_pad, T *__restrict__ hi, T *__restrict__ lo)
-{
-    __shared__ T tile[kTile][kTile + 1];
-    const int64_t p0 = static_cast<int64_t>(blockIdx.x) * kTile;
-    const int c0 = blockIdx.y * kTile, tap = blockIdx.z;
-    const int kh = tap / a.KW, kw = tap - (tap / a.KW) * a.KW;
-    const int tx = threadIdx.x, ty = threadIdx.y;
-    const int64_t P = a.P_pix, hw = static_cast<int64_t>(a.Ho) * a.Wo;
-    const T *x = static_cast<const T *>(a.x);
-    for (int i = ty; i < kTile; i += 8) {
-        const int64_t p = p0 + i;
-        const int c = c0 + tx;
-        T v = T(0.f);
-        if (p < P && c < a.C) {
-            const int64_t b = p / hw;
-            const int r = static_cast<int>(p - b * hw);
-            const int oh = r / a.Wo, ow = r - (r / a.Wo) * a.Wo;
-            const int ih = oh * a.sh - a.ph + kh * a.dh, iw = ow * a.sw - a.pw + kw * a.dw;
-            if (ih >= 0 && ih < a.H && iw >= 0 && iw < a.W)
-                v = x[((b * a.H + ih) * a.W + iw) * a.C + c];
-        }
-        tile[i][tx] = v;
-    }
-    __syncthreads();
-    for (int i = ty; i < kTile; i += 8) {
-        const int c = c0 + i;
-        const int64_t p = p0 + tx;
-        if (c >= a.C || p >= P_pad) continue;
-        const int64_t dst = (static_cast<int64_t>(tap) * a.C + c) * P_pad + p;
+        if (o >= C_out || p >= P_pad) continue;
+        const int64_t dst = static_cast<int64_t>(o) * P_pad + p;
         const T v = tile[tx][i];
         if constexpr (sizeof(T) == 4) {
             const float h = tf32_rna(v);
@@ -112,43 +89,140 @@ xcol_transpose_kernel(const ConvArgs a, int64_t P_pad, T *__restrict__ hi, T *__
     }
 }
 
-// dD[z][n] = sum over the S slices of the GEMM partial at row g*N + n,
-// column I[z]; one CTA per col-group.  Partial slot i = slice * tiles +
-// tile holds [BN/4][128] float4 (column quad, row).
+// XcolT[tap*C_in + c][p] = x[b, oh*sh - ph + kh*dh, ow*sw - pw + kw*dw, c]
+// (0 outside the image and for p >= P).  A CTA takes 64 channels of one tap
+// and kXcolTiles tiles of 64 pixels: it first finds, once per pixel, the
+// input pixel the tap reads (or none), then moves each tile through shared
+// memory with 4-channel vector reads and 4-pixel vector writes.
+constexpr int kXcolTiles = 4;
+constexpr int kXT = 64;                          // pixels and channels per tile
+
+template <typename T> struct Vec4;
+template <> struct Vec4<float> { using type = float4; };
+template <> struct Vec4<__nv_bfloat16> { using type = uint2; };
+
+template <typename T>
+__device__ __forceinline__ void unpack4(const typename Vec4<T>::type &v, T (&e)[4])
+{
+    if constexpr (sizeof(T) == 4) {
+        e[0] = v.x; e[1] = v.y; e[2] = v.z; e[3] = v.w;
+    } else {
+        const __nv_bfloat162 a = *reinterpret_cast<const __nv_bfloat162 *>(&v.x);
+        const __nv_bfloat162 b = *reinterpret_cast<const __nv_bfloat162 *>(&v.y);
+        e[0] = a.x; e[1] = a.y; e[2] = b.x; e[3] = b.y;
+    }
+}
+
+template <typename T>
+__device__ __forceinline__ typename Vec4<T>::type pack4(const T (&e)[4])
+{
+    typename Vec4<T>::type v;
+    if constexpr (sizeof(T) == 4) {
+        v = make_float4(e[0], e[1], e[2], e[3]);
+    } else {
+        __nv_bfloat162 a, b;
+        a.x = e[0]; a.y = e[1]; b.x = e[2]; b.y = e[3];
+        v.x = *reinterpret_cast<uint32_t *>(&a);
+        v.y = *reinterpret_cast<uint32_t *>(&b);
+    }
+    return v;
+}
+
+template <typename T>
+__global__ void __launch_bounds__(256)
+xcol_transpose_kernel(const ConvArgs a, int P_pad, const onexn::FastDiv div_hw, const onexn::FastDiv div_wo,
+                      T *__restrict__ out)
+{
+    using V = typename Vec4<T>::type;
+    __shared__ T tile[kXT][kXT + 1];             // [channel][pixel]
+    __shared__ int src[kXcolTiles * kXT];        // input pixel (b*H + ih)*W + iw, or -1
+    const int c0 = blockIdx.y * kXT, tap = blockIdx.z;
+    const int kh = tap / a.KW, kw = tap - (tap / a.KW) * a.KW;
+    const int tid = threadIdx.x;
+    const int hw = a.Ho * a.Wo;
+    const int pb = blockIdx.x * kXcolTiles * kXT;
+    for (int i = tid; i < kXcolTiles * kXT; i += 256) {
+        const int p = pb + i;
+        int sp = -1;
+        if (p < a.P_pix) {
+            const uint32_t b = div_hw.div(static_cast<uint32_t>(p));
+            const uint32_t r = static_cast<uint32_t>(p) - b * hw;
+            const int oh = static_cast<int>(div_wo.div(r)), ow = static_cast<int>(r) - oh * a.Wo;
+            const int ih = oh * a.sh - a.ph + kh * a.dh, iw = ow * a.sw - a.pw + kw * a.dw;
+            if (ih >= 0 && ih < a.H && iw >= 0 && iw < a.W) sp = (static_cast<int>(b) * a.H + ih) * a.W + iw;
+        }
+        src[i] = sp;
+    }
+    __syncthreads();
+    // read role: 16 threads per pixel row, each 4 channels; write role: 16
+    // threads per channel row, each 4 pixels
+    const int q = tid & 15, r16 = tid >> 4;
+    const int cq = c0 + 4 * q;                   // this thread's channel quad
+    const bool c_ok = cq < a.C;
+    const T *x = static_cast<const T *>(a.x);
+    T *obase = out + (static_cast<int64_t>(tap) * a.C + c0) * P_pad;
+    for (int tt = 0; tt < kXcolTiles; ++tt) {
+        const int p0 = pb + tt * kXT;
+        if (p0 >= P_pad) break;
+#pragma unroll
+        for (int i = r16; i < kXT; i += 16) {
+            const int sp = src[tt * kXT + i];
+            T e[4] = {T(0.f), T(0.f), T(0.f), T(0.f)};
+            if (sp >= 0 && c_ok) unpack4<T>(__ldg(reinterpret_cast<const V *>(x + static_cast<int64_t>(sp) * a.C + cq)), e);
+#pragma unroll
+            for (int j = 0; j < 4; ++j) tile[4 * q + j][i] = e[j];
+        }
+        __syncthreads();
+#pragma unroll
+        for (int i = r16; i < kXT; i += 16) {
+            if (c0 + i >= a.C) continue;
+            const T e[4] = {tile[i][4 * q], tile[i][4 * q + 1], tile[i][4 * q + 2], tile[i][4 * q + 3]};
+            *reinterpret_cast<V *>(obase + static_cast<int64_t>(i) * P_pad + p0 + 4 * q) = pack4<T>(e);
+        }
+        __syncthreads();
+    }
+}
+
+// db[o] = sum of colsum[o][0 .. n_pb), one warp per channel, fixed order.
+__global__ void __launch_bounds__(256)
+bias_grad_kernel(const float *__restrict__ colsum, int n_pb, int C_out, float *__restrict__ db)
+{
+    const int o = blockIdx.x * 8 + (threadIdx.x >> 5), lane = threadIdx.x & 31;
+    if (o >= C_out) return;
+    const float *row = colsum + static_cast<int64_t>(o) * n_pb;
+    float s = 0.f;
+    for (int i = lane; i < n_pb; i += 32) s += row[i];
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) s += __shfl_xor_sync(0xffffffffu, s, off);
+    if (lane == 0) db[o] = s;
+}
+
+// dD[z][n] = sum over the S slices of the GEMM partial at row I[z] (the
+// GEMM computes dW^T: rows k, columns o) and column g*N + n, for every kept
+// block z of col-group g (found by binary search in P).  Partial slot
+// i = slice * tiles + tile holds [BN/4][128] float4 (column quad, row).
 __global__ void __launch_bounds__(256)
 wgrad_gather_kernel(const float *__restrict__ partials, const int32_t *__restrict__ P, const int32_t *__restrict__ I,
-                    int N, int64_t t, int bn, int tiles, int n_tn, int S, float *__restrict__ dD)
+                    int G, int N, int64_t t, int bn, int tiles, int n_tn, int S, float *__restrict__ dD)
 {
-    const int g = blockIdx.x;
-    const int64_t z0 = min(static_cast<int64_t>(__ldg(P + g)), t);
-    const int64_t z1 = min(max(static_cast<int64_t>(__ldg(P + g + 1)), z0), t);
     const int64_t slot_f = static_cast<int64_t>(128) * bn;
-    for (int64_t e = z0 * N + threadIdx.x; e < z1 * N; e += blockDim.x) {
+    for (int64_t e = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; e < t * N;
+         e += static_cast<int64_t>(gridDim.x) * blockDim.x) {
         const int64_t z = e / N;
         const int n = static_cast<int>(e - z * N);
-        const int m = g * N + n, k = __ldg(I + z);
-        const int tile = (m / 128) * n_tn + k / bn;
-        const int col = k % bn, row = m % 128;
+        int lo = 0, hi = G;                       // the g with P[g] <= z < P[g + 1]
+        while (hi - lo > 1) {
+            const int mid = (lo + hi) >> 1;
+            if (__ldg(P + mid) <= z) lo = mid; else hi = mid;
+        }
+        const int o = lo * N + n, k = __ldg(I + z);
+        const int tile = (k / 128) * n_tn + o / bn;
+        const int col = o % bn, row = k % 128;
         const int64_t off = (static_cast<int64_t>(col / 4) * 128 + row) * 4 + (col & 3);
         float s = 0.f;
         for (int sl = 0; sl < S; ++sl) s += __ldg(partials + (static_cast<int64_t>(sl) * tiles + tile) * slot_f + off);
         dD[e] = s;
     }
-}
-
-// db[o] = sum_p dYt[o][p], one warp per row, fixed order.
-template <typename T>
-__global__ void __launch_bounds__(256)
-bias_grad_kernel(const T *__restrict__ dyt, int64_t P, int64_t P_pad, int C_out, float *__restrict__ db)
-{
-    const int o = blockIdx.x * 8 + (threadIdx.x >> 5), lane = threadIdx.x & 31;
-    if (o >= C_out) return;
-    const T *row = dyt + static_cast<int64_t>(o) * P_pad;
-    float s = 0.f;
-    for (int64_t p = lane; p < P; p += 32) s += to_f(row[p]);
-#pragma unroll
-    for (int off = 16; off > 0; off >>= 1) s += __shfl_xor_sync(0xffffffffu, s, off);
-    if (lane == 0) db[o] = s;
 }
 
 __global__ void zero_f32_kernel(float *p, int64_t n)
@@ -288,8 +362,9 @@ DgradWs dgrad_ws(const ConvArgs &a, int dtype)
 
 struct WgradWs {
     int64_t P_pad;
+    int n_pb;
     onexn::TcSplitPlan plan;
-    size_t dyt, xhi, xlo, part, total;
+    size_t xcol, dy_hi, dy_lo, colsum, part, total;
 };
 
 WgradWs wgrad_ws(const ConvArgs &a, int dtype)
@@ -298,11 +373,13 @@ WgradWs wgrad_ws(const ConvArgs &a, int dtype)
     const size_t es = dtype == ONEXN_F32 ? 4 : 2;
     const int64_t K = static_cast<int64_t>(a.KH) * a.KW * a.C;
     l.P_pad = (static_cast<int64_t>(a.P_pix) + kPixPad - 1) / kPixPad * kPixPad;
-    l.plan = onexn::tc_split_plan(a.C_out, static_cast<int>(K), l.P_pad, dtype);
-    l.dyt = 0;
-    l.xhi = round256(static_cast<size_t>(a.C_out) * l.P_pad * es);
-    l.xlo = l.xhi + round256(static_cast<size_t>(K) * l.P_pad * es);
-    l.part = l.xlo + (dtype == ONEXN_F32 ? round256(static_cast<size_t>(K) * l.P_pad * es) : 0);
+    l.n_pb = static_cast<int>(l.P_pad / kTile);
+    l.plan = onexn::tc_split_plan(static_cast<int>(K), a.C_out, l.P_pad, dtype);
+    l.xcol = 0;
+    l.dy_hi = round256(static_cast<size_t>(K) * l.P_pad * es);
+    l.dy_lo = l.dy_hi + round256(static_cast<size_t>(a.C_out) * l.P_pad * es);
+    l.colsum = l.dy_lo + (dtype == ONEXN_F32 ? round256(static_cast<size_t>(a.C_out) * l.P_pad * es) : 0);
+    l.part = l.colsum + round256(static_cast<size_t>(a.C_out) * l.n_pb * 4);
     l.total = l.part + round256(l.plan.partial_bytes);
     return l;
 }
@@ -449,47 +526,43 @@ extern "C" onexn_status onexn_conv_bwd_weight(const onexn_conv_desc *desc, const
     unsigned char *ws = static_cast<unsigned char *>(workspace);
     const dim3 block(kTile, 8);
     const int K = a.KH * a.KW * a.C;
-    const dim3 g_dy(static_cast<unsigned>((L.P_pad + kTile - 1) / kTile), (a.C_out + kTile - 1) / kTile);
-    const dim3 g_x(static_cast<unsigned>((L.P_pad + kTile - 1) / kTile), (a.C + kTile - 1) / kTile, a.KH * a.KW);
+    if (L.P_pad > INT32_MAX / 2) return fail(ONEXN_EINVAL, "conv_bwd_weight: too many pixels");
+    const int P_pad = static_cast<int>(L.P_pad);
+    const dim3 g_dy(static_cast<unsigned>(L.n_pb), (a.C_out + kTile - 1) / kTile);
+    const int n_ptiles = (P_pad / kXT + kXcolTiles - 1) / kXcolTiles;
+    const dim3 g_x(static_cast<unsigned>(n_ptiles), (a.C + kXT - 1) / kXT, a.KH * a.KW);
+    const onexn::FastDiv div_hw(static_cast<uint32_t>(a.Ho * a.Wo)), div_wo(static_cast<uint32_t>(a.Wo));
+    float *colsum = reinterpret_cast<float *>(ws + L.colsum);
     if (dtype == ONEXN_F32) {
         dy_transpose_kernel<float><<<g_dy, block, 0, s>>>(static_cast<const float *>(dy), a.P_pix, L.P_pad, a.C_out,
-                                                           reinterpret_cast<float *>(ws + L.dyt));
-        xcol_transpose_kernel<float><<<g_x, block, 0, s>>>(a, L.P_pad, reinterpret_cast<float *>(ws + L.xhi),
-                                                            reinterpret_cast<float *>(ws + L.xlo));
+                                                           reinterpret_cast<float *>(ws + L.dy_hi),
+                                                           reinterpret_cast<float *>(ws + L.dy_lo), colsum, L.n_pb);
+        xcol_transpose_kernel<float><<<g_x, 256, 0, s>>>(a, P_pad, div_hw, div_wo,
+                                                            reinterpret_cast<float *>(ws + L.xcol));
     } else {
-        dy_transpose_kernel<__nv_bfloat16><<<g_dy, block, 0, s>>>(static_cast<const __nv_bfloat16 *>(dy), a.P_pix,
-                                                                   L.P_pad, a.C_out,
-                                                                   reinterpret_cast<__nv_bfloat16 *>(ws + L.dyt));
-        xcol_transpose_kernel<__nv_bfloat16><<<g_x, block, 0, s>>>(a, L.P_pad,
-                                                                    reinterpret_cast<__nv_bfloat16 *>(ws + L.xhi),
-                                                                    nullptr);
+        dy_transpose_kernel<__nv_bfloat16><<<g_dy, block, 0, s>>>(
+            static_cast<const __nv_bfloat16 *>(dy), a.P_pix, L.P_pad, a.C_out,
+            reinterpret_cast<__nv_bfloat16 *>(ws + L.dy_hi), nullptr, colsum, L.n_pb);
+        xcol_transpose_kernel<__nv_bfloat16><<<g_x, 256, 0, s>>>(a, P_pad, div_hw, div_wo,
+                                                                    reinterpret_cast<__nv_bfloat16 *>(ws + L.xcol));
     }
     e = cudaGetLastError();
     if (e != cudaSuccess) return fail(ONEXN_ECUDA, "conv_bwd_weight: transpose: %s", cudaGetErrorString(e));
-    // the GEMM dW[C_out][K] = dYt[C_out][P_pad] . XcolT[K][P_pad]^T, in pixel slices
+    // the GEMM dW^T[K][C_out] = XcolT[K][P_pad] . dYt[C_out][P_pad]^T, in pixel slices
     ConvArgs g{};
-    g.B = 1; g.H = 1; g.W = a.C_out; g.C = static_cast<int>(L.P_pad); g.C_out = K;
+    g.B = 1; g.H = 1; g.W = K; g.C = P_pad; g.C_out = a.C_out;
     g.KH = 1; g.KW = 1; g.sh = 1; g.sw = 1; g.ph = 0; g.pw = 0; g.dh = 1; g.dw = 1;
-    g.Ho = 1; g.Wo = a.C_out; g.P_pix = a.C_out; g.N = 1; g.t = 0;
-    g.x = ws + L.dyt; g.y = ws + L.dyt;
+    g.Ho = 1; g.Wo = K; g.P_pix = K; g.N = 1; g.t = 0;
+    g.x = ws + L.xcol; g.y = ws + L.xcol;
     e = onexn::device_status_ptr(&g.status);
     if (e != cudaSuccess) return fail(ONEXN_ECUDA, "conv_bwd_weight: status word: %s", cudaGetErrorString(e));
-    if (L.P_pad > INT32_MAX) return fail(ONEXN_EINVAL, "conv_bwd_weight: too many pixels");
     float *part = reinterpret_cast<float *>(ws + L.part);
-    e = onexn::tc_gemm_split(g, dtype, ws + L.xhi, dtype == ONEXN_F32 ? ws + L.xlo : nullptr, part, L.plan, s);
+    e = onexn::tc_gemm_split(g, dtype, ws + L.dy_hi, dtype == ONEXN_F32 ? ws + L.dy_lo : nullptr, part, L.plan, s);
     if (e != cudaSuccess) return fail(ONEXN_ECUDA, "conv_bwd_weight: GEMM: %s", cudaGetErrorString(e));
     if (t > 0)
-        wgrad_gather_kernel<<<a.C_out / a.N, 256, 0, s>>>(part, P, I, a.N, t, L.plan.bn, L.plan.tiles, L.plan.n_tn,
-                                                          L.plan.split_s, dD);
-    if (db) {
-        const int gb = (a.C_out + 7) / 8;
-        if (dtype == ONEXN_F32)
-            bias_grad_kernel<float><<<gb, 256, 0, s>>>(reinterpret_cast<const float *>(ws + L.dyt), a.P_pix, L.P_pad,
-                                                        a.C_out, db);
-        else
-            bias_grad_kernel<__nv_bfloat16><<<gb, 256, 0, s>>>(reinterpret_cast<const __nv_bfloat16 *>(ws + L.dyt),
-                                                                a.P_pix, L.P_pad, a.C_out, db);
-    }
+        wgrad_gather_kernel<<<grid_cap(t * a.N, 256, sms), 256, 0, s>>>(part, P, I, a.C_out / a.N, a.N, t, L.plan.bn,
+                                                                        L.plan.tiles, L.plan.n_tn, L.plan.split_s, dD);
+    if (db) bias_grad_kernel<<<(a.C_out + 7) / 8, 256, 0, s>>>(colsum, L.n_pb, a.C_out, db);
     e = cudaGetLastError();
     if (e != cudaSuccess) return fail(ONEXN_ECUDA, "conv_bwd_weight: launch failed: %s", cudaGetErrorString(e));
     return ONEXN_OK;

@@ -1165,10 +1165,9 @@ cudaError_t tc_gemm_weights(const ConvArgs &a, int dtype, const void *W, const v
 TcSplitPlan tc_split_plan(int M, int Ncols, int64_t K, int dtype)
 {
     TcSplitPlan p{};
-    ConvArgs a{};
-    a.P_pix = M;
-    a.C_out = Ncols;
-    p.bn = tc_bn(a);
+    // the columns in as few tiles as possible: the slices, not narrow tiles,
+    // spread the work over the SMs, and each column tile re-reads A
+    p.bn = Ncols <= 64 ? 64 : Ncols <= 128 ? 128 : 256;
     const int64_t tiles = ((static_cast<int64_t>(M) + kBM - 1) / kBM) * ((Ncols + p.bn - 1) / p.bn);
     const int64_t chunks = (K + (dtype == ONEXN_F32 ? TcF32::kBK : TcBf16::kBK) - 1) /
                            (dtype == ONEXN_F32 ? TcF32::kBK : TcBf16::kBK);
