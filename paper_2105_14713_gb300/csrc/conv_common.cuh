@@ -44,6 +44,14 @@ __device__ __forceinline__ float activate(float v, int kind)
     if (kind == 2) v = fminf(v, 6.f);
     return v;
 }
+// The same with the kind fixed at compile time (no branch per value).
+template <int kKind>
+__device__ __forceinline__ float activate_c(float v)
+{
+    if constexpr (kKind >= 1) v = fmaxf(v, 0.f);
+    if constexpr (kKind == 2) v = fminf(v, 6.f);
+    return v;
+}
 
 // Division of 32-bit unsigned integers by an invariant divisor d >= 1 with
 // one multiply-high, after Granlund and Montgomery, "Division by invariant

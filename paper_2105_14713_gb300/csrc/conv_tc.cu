@@ -55,6 +55,7 @@
 #include <cudaTypedefs.h>
 
 #include <algorithm>
+#include <type_traits>
 #include <cstring>
 #include <mutex>
 
@@ -515,10 +516,16 @@ tc_conv_kernel(const ConvArgs a, const __grid_constant__ CUtensorMap tmap_x,
         // ============================ epilogue ============================
         // Per tile, column atom by column atom (128 bytes of output columns:
         // 64 bf16 / 32 fp32): read the atom's accumulator columns from TMEM
-        // (warp w owns TMEM lanes = pixel rows 32*(w%4)..+31), add the bias,
-        // apply ReLU, convert, write the row into the warp's 128-byte-swizzled
-        // staging buffer (two, alternating) and store the warp's 32 x atom box
-        // with TMA.
+        // (warp w owns TMEM lanes = pixel rows 32*(w%4)..+31), add the bias
+        // (and the residual), apply the activation, convert, write the row
+        // into the warp's 128-byte-swizzled staging buffer (two, alternating)
+        // and store the warp's 32 x atom box with TMA.  The residual and the
+        // activation are compile-time variants chosen once per launch, so the
+        // per-value work has no branches (a per-chunk test for the residual
+        // alone cost a third of the epilogue on epilogue-bound 1x1 layers).
+      auto epilogue = [&](auto res_c, auto act_c) {
+        constexpr bool kRes = decltype(res_c)::value;
+        constexpr int kAct = decltype(act_c)::value;
         using T = typename Tr::T;
         constexpr int kAtomCols = kRowBytes / static_cast<int>(sizeof(T));
         constexpr int kAtoms = BN / kAtomCols;
@@ -531,6 +538,7 @@ tc_conv_kernel(const ConvArgs a, const __grid_constant__ CUtensorMap tmap_x,
         float *sbias = reinterpret_cast<float *>(smem + L::kBias);
         const int64_t W_sk = static_cast<int64_t>(sched.sk_tiles) * sched.n_chunks;
         int n_emit = 0;                              // atoms stored so far (staging buffer parity)
+        int staged_tn = -1;                          // column tile whose bias is in shared memory
         TcSegIter it(sched);
         TcSeg sg;
         for (int si = 0; it.next(sg); ++si) {
@@ -580,7 +588,12 @@ tc_conv_kernel(const ConvArgs a, const __grid_constant__ CUtensorMap tmap_x,
             // for another
             // the tile's bias in shared memory, read as broadcast float4
             const float4 *sb4 = reinterpret_cast<const float4 *>(sbias);
+            // (only when the column tile changes: consecutive tiles of a
+            // CTA often share it, and the global load is a full memory
+            // latency on the epilogue's critical path)
             auto stage_bias = [&]() {
+                if (tn == staged_tn) return;         // uniform across the four warps
+                staged_tn = tn;
                 tc::named_bar(1, 128);               // the previous tile's reads are done
                 for (int c = row; c < BN; c += 128) {
                     const int o = tn * BN + c;
@@ -595,31 +608,43 @@ tc_conv_kernel(const ConvArgs a, const __grid_constant__ CUtensorMap tmap_x,
                 const uint32_t wbuf = sout + (q * 2 + buf) * (32 * kRowBytes);
                 const int col0 = tn * BN + at * kAtomCols;
                 // the residual row of this atom (16-byte chunks inside y only)
-                const int pix = tm * kBM + row;
-                const uint4 *res = (a.residual && pix < a.P_pix)
-                                       ? reinterpret_cast<const uint4 *>(static_cast<const T *>(a.residual) +
-                                                                         static_cast<int64_t>(pix) * a.C_out + col0)
-                                       : nullptr;
+                const uint4 *res = nullptr;
+                if constexpr (kRes) {
+                    const int pix = tm * kBM + row;
+                    if (pix < a.P_pix)
+                        res = reinterpret_cast<const uint4 *>(static_cast<const T *>(a.residual) +
+                                                              static_cast<int64_t>(pix) * a.C_out + col0);
+                }
 #pragma unroll
                 for (int j = 0; j < 8; ++j) {        // 16-byte chunk j of the row
                     uint32_t w[4];
-                    uint4 rv = make_uint4(0, 0, 0, 0);
-                    if (res && col0 + j * (16 / static_cast<int>(sizeof(T))) < a.C_out) rv = __ldg(res + j);
-                    const uint32_t rw[4] = {rv.x, rv.y, rv.z, rv.w};
+                    uint32_t rw[4] = {0u, 0u, 0u, 0u};
+                    if constexpr (kRes) {
+                        if (res && col0 + j * (16 / static_cast<int>(sizeof(T))) < a.C_out) {
+                            const uint4 rv = __ldg(res + j);
+                            rw[0] = rv.x; rw[1] = rv.y; rw[2] = rv.z; rw[3] = rv.w;
+                        }
+                    }
                     if constexpr (sizeof(T) == 4) {
                         const float4 bv = sb4[at * (kAtomCols / 4) + j];
                         const float bb[4] = {bv.x, bv.y, bv.z, bv.w};
 #pragma unroll
-                        for (int e = 0; e < 4; ++e)
-                            w[e] = __float_as_uint(activate(f[4 * j + e] + bb[e] + __uint_as_float(rw[e]), a.relu));
+                        for (int e = 0; e < 4; ++e) {
+                            float v = f[4 * j + e] + bb[e];
+                            if constexpr (kRes) v += __uint_as_float(rw[e]);
+                            w[e] = __float_as_uint(activate_c<kAct>(v));
+                        }
                     } else {
                         const float4 b0 = sb4[at * (kAtomCols / 4) + 2 * j], b1 = sb4[at * (kAtomCols / 4) + 2 * j + 1];
                         const float bb[8] = {b0.x, b0.y, b0.z, b0.w, b1.x, b1.y, b1.z, b1.w};
 #pragma unroll
                         for (int e = 0; e < 4; ++e) {
-                            const float v0 = activate(f[8 * j + 2 * e] + bb[2 * e] + bf16lo(rw[e]), a.relu);
-                            const float v1 = activate(f[8 * j + 2 * e + 1] + bb[2 * e + 1] + bf16hi(rw[e]), a.relu);
-                            w[e] = pack_bf16x2(v0, v1);
+                            float v0 = f[8 * j + 2 * e] + bb[2 * e], v1 = f[8 * j + 2 * e + 1] + bb[2 * e + 1];
+                            if constexpr (kRes) {
+                                v0 += bf16lo(rw[e]);
+                                v1 += bf16hi(rw[e]);
+                            }
+                            w[e] = pack_bf16x2(activate_c<kAct>(v0), activate_c<kAct>(v1));
                         }
                     }
                     asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};\n" ::"r"(
@@ -736,6 +761,16 @@ tc_conv_kernel(const ConvArgs a, const __grid_constant__ CUtensorMap tmap_x,
             });
         }
         if (lane == 0) tc::bulk_wait0();
+      };
+        if (a.residual) {
+            if (a.relu == 2) epilogue(std::true_type{}, std::integral_constant<int, 2>{});
+            else if (a.relu == 1) epilogue(std::true_type{}, std::integral_constant<int, 1>{});
+            else epilogue(std::true_type{}, std::integral_constant<int, 0>{});
+        } else {
+            if (a.relu == 2) epilogue(std::false_type{}, std::integral_constant<int, 2>{});
+            else if (a.relu == 1) epilogue(std::false_type{}, std::integral_constant<int, 1>{});
+            else epilogue(std::false_type{}, std::integral_constant<int, 0>{});
+        }
     }
 
     tc::fence_before_sync();
