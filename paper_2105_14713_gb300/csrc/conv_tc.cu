@@ -602,11 +602,16 @@ tc_conv_kernel(const ConvArgs a, const __grid_constant__ CUtensorMap tmap_x,
                 tc::named_bar(1, 128);
             };
             auto emit_atom = [&](int at, float (&f)[kAtomCols]) {
+                const int col0 = tn * BN + at * kAtomCols;
+                if (col0 >= a.C_out) {               // the whole atom lies past y's columns: no work,
+                    ++n_emit;                        // but an (empty) commit group keeps the count
+                    if (lane == 0) tc::bulk_commit();
+                    return;
+                }
                 const int buf = n_emit++ & 1;        // alternate across atoms and tiles
                 if (lane == 0) tc::bulk_wait_read1();   // this warp's store two atoms back has read buf
                 __syncwarp();
                 const uint32_t wbuf = sout + (q * 2 + buf) * (32 * kRowBytes);
-                const int col0 = tn * BN + at * kAtomCols;
                 // the residual row of this atom (16-byte chunks inside y only)
                 const uint4 *res = nullptr;
                 if constexpr (kRes) {
@@ -654,10 +659,11 @@ tc_conv_kernel(const ConvArgs a, const __grid_constant__ CUtensorMap tmap_x,
                 }
                 tc::fence_proxy_async_smem();
                 __syncwarp();
-                // one commit group per atom, empty for an atom past C_out, so
-                // that "at most one group pending" always means buf is free
+                // one commit group per atom (empty for an atom past C_out,
+                // above), so that "at most one group pending" always means
+                // buf is free
                 if (lane == 0) {
-                    if (col0 < a.C_out) tc::tma_store_2d(&tmap_y, col0, tm * kBM + 32 * q, wbuf);
+                    tc::tma_store_2d(&tmap_y, col0, tm * kBM + 32 * q, wbuf);
                     tc::bulk_commit();
                 }
             };
