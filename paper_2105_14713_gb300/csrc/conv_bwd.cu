@@ -7,8 +7,9 @@
 // with the flipped, transposed weights Wt[c][(T-1-tap)*C_out + o] =
 // W[o][tap*C_in + c] (T = KH*KW taps), so it runs on the forward tcgen05
 // GEMM: decode (P, I, D) into W, transpose it per tap with the tap order
-// reversed, and launch the GEMM on (dy, Wt).  Strided layers (and padding
-// beyond d(K-1)) use a direct kernel over the decoded W.
+// reversed, and launch the GEMM on (dy, Wt).  A strided layer runs the same
+// convolution on dy scattered onto a zero grid dilated by the stride.
+// Padding beyond d(K-1) uses a direct kernel over the decoded W.
 //
 // Kept-weight gradient dW[o][k] = sum_p dy[p][o] * xcol[p][k] (k = tap*C_in
 // + c, xcol the im2col view of x): a GEMM with the pixels as its long
@@ -329,25 +330,34 @@ int grid_cap(int64_t work, int per_block, int sms)
     return static_cast<int>(b < 1 ? 1 : b < cap ? b : cap);
 }
 
-// The transposed convolution that computes dx for a stride-1 layer, or
-// false if the forward kernel cannot run it (then the direct kernel does).
+// The transposed convolution that computes dx, or false if the forward
+// kernel cannot run it (then the direct kernel does).  For stride 1 it reads
+// dy itself; for stride s it reads dy scattered onto a zero grid dilated by
+// s (dy[oh] at row oh*s; Hd = (Ho-1)*s + 1 + r rows, r = the rows of x past
+// the last window), so that the same stride-1 convolution with the flipped
+// weights gives dx (s*s more multiply-adds, on the tensor cores).
 bool dgrad_as_conv(const ConvArgs &a, int dtype, ConvArgs *t)
 {
-    if (a.sh != 1 || a.sw != 1) return false;
     const int ph = a.dh * (a.KH - 1) - a.ph, pw = a.dw * (a.KW - 1) - a.pw;
     if (ph < 0 || pw < 0) return false;
+    const int rh = (a.H + 2 * a.ph - a.dh * (a.KH - 1) - 1) % a.sh;
+    const int rw = (a.W + 2 * a.pw - a.dw * (a.KW - 1) - 1) % a.sw;
+    const int Hd = (a.Ho - 1) * a.sh + 1 + rh, Wd = (a.Wo - 1) * a.sw + 1 + rw;
     ConvArgs c{};
-    c.B = a.B; c.H = a.Ho; c.W = a.Wo; c.C = a.C_out; c.C_out = a.C;
+    c.B = a.B; c.H = Hd; c.W = Wd; c.C = a.C_out; c.C_out = a.C;
     c.KH = a.KH; c.KW = a.KW; c.sh = 1; c.sw = 1; c.ph = ph; c.pw = pw; c.dh = a.dh; c.dw = a.dw;
     c.Ho = a.H; c.Wo = a.W; c.P_pix = a.B * a.H * a.W;
     c.N = 1; c.t = 0;
+    // the transposed convolution's output is x's grid exactly
+    if (Hd + 2 * ph - a.dh * (a.KH - 1) != a.H || Wd + 2 * pw - a.dw * (a.KW - 1) != a.W) return false;
+    if (static_cast<int64_t>(a.B) * Hd * Wd >= (int64_t(1) << 31)) return false;
     if (!onexn::tc_supports(c, dtype)) return false;
     *t = c;
     return true;
 }
 
 struct DgradWs {
-    size_t w, wt, total;
+    size_t w, wt, dyd, total;
 };
 
 DgradWs dgrad_ws(const ConvArgs &a, int dtype)
@@ -356,8 +366,35 @@ DgradWs dgrad_ws(const ConvArgs &a, int dtype)
     const size_t wb = onexn::tc_weights_bytes(a, dtype);
     l.w = 0;
     l.wt = wb;
+    l.dyd = 2 * wb;
     l.total = 2 * wb;
+    ConvArgs tr{};
+    if ((a.sh > 1 || a.sw > 1) && dgrad_as_conv(a, dtype, &tr))
+        l.total += round256(static_cast<size_t>(tr.B) * tr.H * tr.W * tr.C * (dtype == ONEXN_F32 ? 4 : 2));
     return l;
+}
+
+// dyd[b][i][j][:] = dy[b][i/sh][j/sw][:] where sh | i and sw | j (inside dy),
+// else 0; one thread per 16-byte channel vector.
+template <typename T>
+__global__ void __launch_bounds__(256)
+dilate_kernel(const T *__restrict__ dy, int B, int Ho, int Wo, int C, int sh, int sw, int Hd, int Wd,
+              T *__restrict__ dyd)
+{
+    constexpr int kV = 16 / sizeof(T);
+    const int n_vec = C / kV;
+    const int64_t total = static_cast<int64_t>(B) * Hd * Wd * n_vec;
+    for (int64_t i = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; i < total;
+         i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+        const int cv = static_cast<int>(i % n_vec);
+        const int64_t q = i / n_vec;
+        const int j = static_cast<int>(q % Wd), r = static_cast<int>((q / Wd) % Hd);
+        const int64_t b = q / (static_cast<int64_t>(Wd) * Hd);
+        uint4 v = make_uint4(0u, 0u, 0u, 0u);
+        if (r % sh == 0 && j % sw == 0 && r / sh < Ho && j / sw < Wo)
+            v = __ldg(reinterpret_cast<const uint4 *>(dy + ((b * Ho + r / sh) * Wo + j / sw) * C) + cv);
+        reinterpret_cast<uint4 *>(dyd + q * C)[cv] = v;
+    }
 }
 
 struct WgradWs {
@@ -460,7 +497,23 @@ extern "C" onexn_status onexn_conv_bwd_data(const onexn_conv_desc *desc, const i
         }
         e = cudaGetLastError();
         if (e != cudaSuccess) return fail(ONEXN_ECUDA, "conv_bwd_data: transpose: %s", cudaGetErrorString(e));
-        tr.x = dy; tr.y = dx; tr.residual = acc ? dx : nullptr; tr.bias = nullptr; tr.relu = 0;
+        const void *src = dy;
+        if (a.sh > 1 || a.sw > 1) {
+            void *dyd = ws + L.dyd;
+            const int kv = dtype == ONEXN_F32 ? 4 : 8;
+            const int g = grid_cap(static_cast<int64_t>(tr.B) * tr.H * tr.W * (tr.C / kv), 256, sms);
+            if (dtype == ONEXN_F32)
+                dilate_kernel<float><<<g, 256, 0, s>>>(static_cast<const float *>(dy), a.B, a.Ho, a.Wo, a.C_out, a.sh,
+                                                        a.sw, tr.H, tr.W, static_cast<float *>(dyd));
+            else
+                dilate_kernel<__nv_bfloat16><<<g, 256, 0, s>>>(static_cast<const __nv_bfloat16 *>(dy), a.B, a.Ho, a.Wo,
+                                                                a.C_out, a.sh, a.sw, tr.H, tr.W,
+                                                                static_cast<__nv_bfloat16 *>(dyd));
+            e = cudaGetLastError();
+            if (e != cudaSuccess) return fail(ONEXN_ECUDA, "conv_bwd_data: dilate: %s", cudaGetErrorString(e));
+            src = dyd;
+        }
+        tr.x = src; tr.y = dx; tr.residual = acc ? dx : nullptr; tr.bias = nullptr; tr.relu = 0;
         tr.status = a.status;
         const void *wt_lo = dtype == ONEXN_F32 ? static_cast<const void *>(static_cast<float *>(wt) + n_w) : nullptr;
         e = onexn::tc_gemm_weights(tr, dtype, wt, wt_lo, nullptr, s);

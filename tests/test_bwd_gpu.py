@@ -28,8 +28,12 @@ CASES = [
     ("3x3_p0", 2, 12, 10, 16, 32, 3, 3, 1, 0, 1, 4),
     ("3x3_d2", 2, 14, 12, 24, 40, 3, 3, 1, 2, 2, 8),
     ("1x3", 2, 9, 17, 32, 48, 1, 3, 1, 0, 1, 16),
-    ("3x3_s2", 3, 15, 13, 32, 64, 3, 3, 2, 1, 1, 8),       # direct input gradient
-    ("1x1_s2", 2, 14, 14, 64, 128, 1, 1, 2, 0, 1, 4),      # direct input gradient
+    ("3x3_s2", 3, 15, 13, 32, 64, 3, 3, 2, 1, 1, 8),       # dy dilated by the stride, tensor cores
+    ("1x1_s2", 2, 14, 14, 64, 128, 1, 1, 2, 0, 1, 4),      # dilated, ragged last row/column of x
+    ("3x3_s2_d2", 2, 15, 15, 16, 32, 3, 3, 2, 2, 2, 4),    # dilated dy, dilated kernel
+    ("3x3_s3", 2, 16, 14, 16, 32, 3, 3, 3, 1, 1, 4),       # stride 3
+    ("1x1_p1", 2, 9, 9, 32, 64, 1, 1, 1, 1, 1, 8),         # padding beyond d(K-1): direct kernel
+    ("3x3_s2_p3", 2, 13, 11, 32, 64, 3, 3, 2, 3, 1, 8),    # direct kernel, strided
 ]
 
 
@@ -84,7 +88,7 @@ def test_kept_weight_and_bias_gradient(case, dtype):
 
 
 def test_accumulate_adds_into_dx():
-    for case in (CASES[0], CASES[5]):                   # tensor-core and direct paths
+    for case in (CASES[0], CASES[5], CASES[-1]):        # stride 1, dilated and direct paths
         layer, conv, x, dy, mask, W, s, p, d = _setup(case, "f32", seed=2)
         base = torch.randn(x.shape, generator=torch.Generator().manual_seed(4)).cuda()
         dx = base.clone()

@@ -386,3 +386,32 @@ def test_device_prune_and_pack_argument_errors_need_no_gpu():
     assert g(base, base, 64, 32, 3, 3, 8, 7, base, base, base, 10, base, 256, None) == ox.ONEXN_EINVAL
     assert g(base, base, 64, 32, 3, 3, 8, 0, base, None, None, 10, base, 256, None) == ox.ONEXN_EINVAL
     assert g(base, base, 64, 32, 3, 3, 8, 0, base, base, base, 10, base, 4, None) == ox.ONEXN_EINVAL
+
+
+def test_bwd_workspace_sizes_show_the_input_gradient_path():
+    """Input gradient: decoded weights + their flipped transpose; a strided
+    layer runs on the tensor cores over dy dilated by the stride (its
+    buffer is in the workspace), padding beyond d(K-1) on the direct kernel
+    (no extra buffer).  Weight gradient: transposed im2col, transposed dy
+    (fp32: tf32 hi and lo), column sums, GEMM partial tiles."""
+    wb = lambda co, k, es: -(-co * k * es // 256) * 256
+    r256 = lambda v: -(-v // 256) * 256
+    d1 = ox.make_desc(2, 15, 13, 32, 64, 3, 3, 1, 1, 1)
+    assert ox.onexn_conv_bwd_data_workspace_size(d1, 8, 100, ox.ONEXN_F32) == 2 * wb(64, 288, 8)
+    d2 = ox.make_desc(3, 15, 13, 32, 64, 3, 3, 2, 1, 1)            # Ho, Wo = 8, 7: dilated 15 x 13
+    assert ox.onexn_conv_bwd_data_workspace_size(d2, 8, 100, ox.ONEXN_F32) == \
+        2 * wb(64, 288, 8) + r256(3 * 15 * 13 * 64 * 4)
+    assert ox.onexn_conv_bwd_data_workspace_size(d2, 8, 100, ox.ONEXN_BF16) == \
+        2 * wb(64, 288, 2) + r256(3 * 15 * 13 * 64 * 2)
+    d3 = ox.make_desc(2, 14, 14, 64, 128, 1, 1, 2, 0, 1)           # 1x1 s2: 7 x 7 -> dilated 13 x 13 + 1
+    assert ox.onexn_conv_bwd_data_workspace_size(d3, 4, 100, ox.ONEXN_F32) == \
+        2 * wb(128, 64, 8) + r256(2 * 14 * 14 * 128 * 4)
+    d4 = ox.make_desc(2, 13, 11, 32, 64, 3, 3, 2, 3, 1)            # pad 3 > d(K-1): direct kernel
+    assert ox.onexn_conv_bwd_data_workspace_size(d4, 8, 100, ox.ONEXN_F32) == 2 * wb(64, 288, 8)
+    # weight gradient on 2 x 15 x 13 -> P = 390 pixels, padded to 448
+    n = ox.onexn_conv_bwd_weight_workspace_size(d1, 8, ox.ONEXN_F32)
+    K, Pp = 288, 448
+    base = r256(K * Pp * 4) + 2 * r256(64 * Pp * 4) + r256(64 * (Pp // 32) * 4)
+    assert n > base and (n - base) % (128 * 64 * 4) == 0           # whole 128 x 64 fp32 partial tiles
+    with pytest.raises(ox.OnexnError):
+        ox.onexn_conv_bwd_data_workspace_size(ox.make_desc(1, 4, 4, 8, 12), 4, 1, ox.ONEXN_F32)   # C_out % 8
