@@ -359,6 +359,34 @@ onexn_status onexn_conv_bwd_weight(const onexn_conv_desc *desc, const int32_t *P
                                    void *workspace, size_t workspace_bytes, void *stream);
 
 /*
+ * onexn_dwproj_fwd -- MobileNet-V2's depthwise 3x3 + ReLU6 fused into the
+ * 1xN-pruned 1x1 projection that follows it (fp32, tensor-core family):
+ *   y = act(Proj(relu6(dw(h))) + bias + residual)
+ * where dw(h)[b,oh,ow,c] = b_dw[c] + sum_{kh,kw} W_dw[kh*3+kw][c]
+ * * h[b, oh*s - 1 + kh, ow*s - 1 + kw, c] (zero padding) and Proj is Eq. 7
+ * with (P, I, D) on the depthwise's output grid; the depthwise output is
+ * computed inside the GEMM's A operand path and never stored.
+ *   dw_desc  the depthwise geometry: B, H, W, C_in = C_out = C, 3x3,
+ *            stride 1 or 2 (both dims), pad 1, dilation 1.
+ *   W_dw     DEVICE fp32 [9][C], TAP-major (note: onexn_dwconv_fwd takes
+ *            [C][3][3]), 16-byte aligned; b_dw nullable DEVICE fp32 [C].
+ *   P, I, D, N, t  the projection's BSR weights (C_out x C); C_out % 8 == 0.
+ *   h        DEVICE fp32 NHWC [B][H][W][C], 16-byte aligned; y DEVICE fp32
+ *            [B][Ho][Wo][C_out], not overlapping h; bias, residual as for
+ *            onexn_conv_fwd_ex.
+ *   flags    ONEXN_RELU / ONEXN_RELU6 (of the projection), ONEXN_DECODED,
+ *            ONEXN_REUSE_DECODE, ONEXN_ALGO_AUTO or ONEXN_ALGO_TC.
+ *   workspace  as onexn_conv_fwd for the 1x1 projection with ONEXN_ALGO_TC
+ *            (onexn_conv_workspace_size of that layer).
+ * Asynchronous; no allocation.  EUNSUPPORTED for bf16 or a projection the
+ * tensor-core family cannot run; EINVAL otherwise as onexn_conv_fwd_ex.
+ */
+onexn_status onexn_dwproj_fwd(const onexn_conv_desc *dw_desc, const float *W_dw, const float *b_dw,
+                              const int32_t *P, const int32_t *I, const void *D, int N, int64_t t, int C_out,
+                              const void *h, void *y, const float *bias, const void *residual, int dtype,
+                              unsigned flags, void *workspace, size_t workspace_bytes, void *stream);
+
+/*
  * onexn_conv_workspace_size -- bytes of device workspace onexn_conv_fwd
  * needs for these arguments with this flags' ALGO (for AUTO: the largest
  * need among the families AUTO may pick, so that passing this many bytes

@@ -25,6 +25,14 @@ struct ConvArgs {
     int relu;               // activation after bias (+ residual): 0 none, 1 ReLU, 2 ReLU6
     const void *residual;   // nullable, NHWC like y: y = act(acc + bias + residual)
     unsigned int *status;   // library status word (device): bits set by kernels on failure
+    // Fused depthwise producer of the A operand (fp32 tensor-core GEMM of a
+    // 1x1 layer only; x is then unused): A[p][c] = relu6(dw_b[c] +
+    // sum_{kh,kw} dw_w[kh*3+kw][c] * dw_x[b, oh*dw_s - 1 + kh, ow*dw_s - 1 + kw, c])
+    // for output pixel p = (b, oh, ow), zero padding.
+    const float *dw_x;      // nullable: NHWC [B][dw_H][dw_W][C]
+    const float *dw_w;      // [9][C], tap-major
+    const float *dw_b;      // [C] or nullptr
+    int dw_H, dw_W, dw_s;
 };
 
 // Bits of the device status word (read by onexn_device_status).

@@ -297,6 +297,72 @@ extern "C" onexn_status onexn_conv_fwd_ex(const onexn_conv_desc *desc, const int
     return ONEXN_OK;
 }
 
+extern "C" onexn_status onexn_dwproj_fwd(const onexn_conv_desc *dw_desc, const float *W_dw, const float *b_dw,
+                                         const int32_t *P, const int32_t *I, const void *D, int N, int64_t t,
+                                         int C_out, const void *h, void *y, const float *bias, const void *residual,
+                                         int dtype, unsigned flags, void *workspace, size_t workspace_bytes,
+                                         void *stream)
+{
+    onexn::clear_error();
+    if (!dw_desc) return fail(ONEXN_EINVAL, "dwproj: dw_desc is NULL");
+    const onexn_conv_desc &d = *dw_desc;
+    if (d.C_in != d.C_out || d.KH != 3 || d.KW != 3 || d.pad_h != 1 || d.pad_w != 1 || d.dil_h != 1 ||
+        d.dil_w != 1 || d.stride_h != d.stride_w || (d.stride_h != 1 && d.stride_h != 2))
+        return fail(ONEXN_EINVAL, "dwproj: the depthwise must be 3x3, pad 1, stride 1 or 2, C_in == C_out");
+    if (dtype != ONEXN_F32) return fail(ONEXN_EUNSUPPORTED, "dwproj: the fused form runs fp32 only");
+    int Ho = 0, Wo = 0;
+    onexn_status st = onexn_conv_out_shape(dw_desc, &Ho, &Wo);
+    if (st != ONEXN_OK) return st;
+    const unsigned forced = flags & ONEXN_ALGO_MASK;
+    if (forced != ONEXN_ALGO_AUTO && forced != ONEXN_ALGO_TC)
+        return fail(ONEXN_EINVAL, "dwproj: only the tensor-core family runs the fused form");
+    // the projection: a 1x1 layer on the depthwise's output grid
+    onexn_conv_desc pd{};
+    pd.B = d.B; pd.H = Ho; pd.W = Wo; pd.C_in = d.C_in; pd.C_out = C_out;
+    pd.KH = 1; pd.KW = 1; pd.stride_h = 1; pd.stride_w = 1; pd.pad_h = 0; pd.pad_w = 0; pd.dil_h = 1; pd.dil_w = 1;
+    onexn::ConvArgs a{};
+    st = check_shape(&pd, N, t, dtype, (flags & ~ONEXN_ALGO_MASK) | ONEXN_ALGO_TC, &a);
+    if (st != ONEXN_OK) return st;
+    st = check_pointers(P, I, D, h, y, bias, dtype, &a);
+    if (st != ONEXN_OK) return st;
+    if (a.P_pix > 0 && !W_dw) return fail(ONEXN_EINVAL, "dwproj: W_dw is NULL");
+    if ((reinterpret_cast<uintptr_t>(W_dw) & 15u) || (reinterpret_cast<uintptr_t>(b_dw) & 3u))
+        return fail(ONEXN_EINVAL, "dwproj: W_dw must be 16-byte and b_dw 4-byte aligned");
+    if (!supports(ONEXN_ALGO_TC, a, dtype))
+        return fail(ONEXN_EUNSUPPORTED, "dwproj: the tensor-core family cannot run this projection");
+    {
+        const uintptr_t h0 = reinterpret_cast<uintptr_t>(h), y0 = reinterpret_cast<uintptr_t>(y);
+        const size_t hb = static_cast<size_t>(d.B) * d.H * d.W * d.C_in * 4, yb = static_cast<size_t>(a.P_pix) * C_out * 4;
+        if (a.P_pix > 0 && h0 < y0 + yb && y0 < h0 + hb) return fail(ONEXN_EINVAL, "dwproj: h and y overlap");
+    }
+    if (residual) {
+        if (reinterpret_cast<uintptr_t>(residual) & 15u)
+            return fail(ONEXN_EINVAL, "dwproj: residual must be 16-byte aligned");
+        const size_t yb = static_cast<size_t>(a.P_pix) * a.C_out * 4;
+        const uintptr_t r0 = reinterpret_cast<uintptr_t>(residual), y0 = reinterpret_cast<uintptr_t>(y);
+        if (r0 != y0 && r0 < y0 + yb && y0 < r0 + yb)
+            return fail(ONEXN_EINVAL, "dwproj: residual overlaps y without being y");
+        a.residual = residual;
+    }
+    if (!workspace) workspace_bytes = 0;
+    if (reinterpret_cast<uintptr_t>(workspace) & 255u)
+        return fail(ONEXN_EINVAL, "dwproj: workspace must be 256-byte aligned");
+    st = check_algo(ONEXN_ALGO_TC, a, dtype, workspace_bytes);
+    if (st != ONEXN_OK) return st;
+    if (a.P_pix == 0) return ONEXN_OK;
+    a.dw_x = static_cast<const float *>(h);
+    a.dw_w = W_dw;
+    a.dw_b = b_dw;
+    a.dw_H = d.H; a.dw_W = d.W; a.dw_s = d.stride_h;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    cudaError_t e = onexn::device_status_ptr(&a.status);
+    if (e != cudaSuccess) return fail(ONEXN_ECUDA, "dwproj: status word: %s", cudaGetErrorString(e));
+    e = (flags & ONEXN_DECODED) ? onexn::tc_gemm(a, dtype, workspace, workspace_bytes, s)
+                                : onexn::launch_tc(a, dtype, workspace, workspace_bytes, s);
+    if (e != cudaSuccess) return fail(ONEXN_ECUDA, "dwproj: launch failed: %s", cudaGetErrorString(e));
+    return ONEXN_OK;
+}
+
 extern "C" onexn_status onexn_conv_fwd(const onexn_conv_desc *desc, const int32_t *P,
                                        const int32_t *I, const void *D, int N, int64_t t,
                                        const void *x, void *y, const float *bias, int dtype,

@@ -369,6 +369,7 @@ tc_conv_kernel(const ConvArgs a, const __grid_constant__ CUtensorMap tmap_x,
     const int n_cchunk = (a.C + Tr::kBK - 1) / Tr::kBK;
     const int n_tn = sched.n_tn;
     auto abort_now = [&]() { atomicOr(a.status, kStatusTimeout); };
+    const bool dw_mode = Tr::kSplit && a.dw_x != nullptr;   // A from the fused depthwise
 
     if (warp == kProdWarp) {
         // ============================ producer ============================
@@ -397,13 +398,18 @@ tc_conv_kernel(const ConvArgs a, const __grid_constant__ CUtensorMap tmap_x,
                     }
                     const uint32_t sa = base + st * L::kStage;
                     const uint32_t sb = sa + L::kA;
-                    tc::mbar_arrive_expect_tx(bar_full + 8 * st, L::kTx);
-                    if (a_tiled)
-                        tc::tma_load_2d(sa, &tmap_x, cc0, p0, bar_full + 8 * st);
-                    else
-                        tc::tma_load_im2col_4d(sa, &tmap_x, cc0, w0, h0, b0,
-                                               static_cast<uint16_t>(kw * a.dw), static_cast<uint16_t>(kh * a.dh),
-                                               bar_full + 8 * st);
+                    if (dw_mode) {
+                        // A comes from the split warps' depthwise; only B is loaded
+                        tc::mbar_arrive_expect_tx(bar_full + 8 * st, L::kTx - L::kA);
+                    } else {
+                        tc::mbar_arrive_expect_tx(bar_full + 8 * st, L::kTx);
+                        if (a_tiled)
+                            tc::tma_load_2d(sa, &tmap_x, cc0, p0, bar_full + 8 * st);
+                        else
+                            tc::tma_load_im2col_4d(sa, &tmap_x, cc0, w0, h0, b0,
+                                                   static_cast<uint16_t>(kw * a.dw), static_cast<uint16_t>(kh * a.dh),
+                                                   bar_full + 8 * st);
+                    }
                     tc::tma_load_2d(sb, &tmap_w, k0tap + cc0, tn * BN, bar_full + 8 * st);
                     if constexpr (Tr::kSplit)
                         tc::tma_load_2d(sb + L::kB, &tmap_wlo, k0tap + cc0, tn * BN, bar_full + 8 * st);
@@ -480,36 +486,103 @@ tc_conv_kernel(const ConvArgs a, const __grid_constant__ CUtensorMap tmap_x,
             const int q = warp & 3;
             const int row = 32 * q + lane;
             const uint32_t lane_base = tmem + (static_cast<uint32_t>(32 * q) << 16) + L::kAcc * BN;
-            const int64_t n_items = TcSegIter(sched).total();
-            for (int64_t item = 0; item < n_items; ++item) {
-                const int st = static_cast<int>(item % L::kS);
-                if (item >= 2 && !mbar_wait(bar_empty + 8 * static_cast<int>((item - 2) % L::kS),
-                                            static_cast<int>((item - 2) / L::kS) & 1)) {
-                    abort_now(); break;
-                }
-                if (!mbar_wait(bar_full + 8 * st, static_cast<int>(item / L::kS) & 1)) { abort_now(); break; }
-                tc::fence_after_sync();
-                const uint32_t src = base + st * L::kStage + row * kRowBytes;
-                uint32_t hi[32], lo[32];
-#pragma unroll
-                for (int j = 0; j < 8; ++j) {
-                    uint32_t v[4];
-                    asm volatile("ld.shared.v4.b32 {%0, %1, %2, %3}, [%4];\n"
-                                 : "=r"(v[0]), "=r"(v[1]), "=r"(v[2]), "=r"(v[3])
-                                 : "r"(src + ((j ^ (row & 7)) << 4))
-                                 : "memory");
-#pragma unroll
-                    for (int e = 0; e < 4; ++e) {
-                        hi[4 * j + e] = v[e] & 0xffffe000u;
-                        lo[4 * j + e] = __float_as_uint(__uint_as_float(v[e]) - __uint_as_float(hi[4 * j + e]));
+            const int hw = a.Ho * a.Wo;
+            int64_t item = 0;
+            bool failed = false;
+            TcSegIter it(sched);
+            TcSeg sg;
+            while (!failed && it.next(sg)) {
+                // dw mode: this thread's output pixel of the tile
+                int pb = -1, poh = 0, pow_ = 0;
+                if (dw_mode) {
+                    const int tm = static_cast<int>(sched.div_tn.div(sg.tile));
+                    const int p = tm * kBM + row;
+                    if (p < a.P_pix) {
+                        pb = static_cast<int>(sched.div_hw.div(p));
+                        const int r = p - pb * hw;
+                        poh = static_cast<int>(sched.div_wo.div(r));
+                        pow_ = r - poh * a.Wo;
                     }
                 }
-                const uint32_t slot = lane_base + static_cast<uint32_t>(item & 1) * 64;
-                tc::st_32x32b_x32(slot, hi);
-                tc::st_32x32b_x32(slot + 32, lo);
-                tc::st_wait();
-                tc::fence_before_sync();
-                mbar_arrive(bar_split + 8 * st);
+                for (int c = sg.c0; c < sg.c1; ++c, ++item) {
+                    const int st = static_cast<int>(item % L::kS);
+                    if (item >= 2 && !mbar_wait(bar_empty + 8 * static_cast<int>((item - 2) % L::kS),
+                                                static_cast<int>((item - 2) / L::kS) & 1)) {
+                        abort_now(); failed = true; break;
+                    }
+                    uint32_t hi[32], lo[32];
+                    if (dw_mode) {
+                        // the depthwise 3x3 + bias + ReLU6 of channels cb .. cb+31
+                        const int cb = c * Tr::kBK;
+                        float v[32];
+#pragma unroll
+                        for (int j = 0; j < 32; ++j) v[j] = 0.f;
+                        if (pb >= 0) {
+                            const bool full = cb + 32 <= a.C;
+#pragma unroll
+                            for (int j = 0; j < 32; ++j)
+                                if (a.dw_b && (full || cb + j < a.C)) v[j] = __ldg(a.dw_b + cb + j);
+                            for (int kh = 0; kh < 3; ++kh) {
+                                const int ih = poh * a.dw_s - 1 + kh;
+                                if (ih < 0 || ih >= a.dw_H) continue;
+                                for (int kw = 0; kw < 3; ++kw) {
+                                    const int iw = pow_ * a.dw_s - 1 + kw;
+                                    if (iw < 0 || iw >= a.dw_W) continue;
+                                    const float *xs = a.dw_x + ((static_cast<int64_t>(pb) * a.dw_H + ih) * a.dw_W + iw) *
+                                                                   a.C + cb;
+                                    const float *ws = a.dw_w + (kh * 3 + kw) * a.C + cb;
+#pragma unroll
+                                    for (int j4 = 0; j4 < 8; ++j4) {
+                                        if (!full && cb + 4 * j4 >= a.C) break;     // C % 4 == 0
+                                        const float4 xv = __ldg(reinterpret_cast<const float4 *>(xs) + j4);
+                                        const float4 wv = __ldg(reinterpret_cast<const float4 *>(ws) + j4);
+                                        v[4 * j4] = fmaf(wv.x, xv.x, v[4 * j4]);
+                                        v[4 * j4 + 1] = fmaf(wv.y, xv.y, v[4 * j4 + 1]);
+                                        v[4 * j4 + 2] = fmaf(wv.z, xv.z, v[4 * j4 + 2]);
+                                        v[4 * j4 + 3] = fmaf(wv.w, xv.w, v[4 * j4 + 3]);
+                                    }
+                                }
+                            }
+#pragma unroll
+                            for (int j = 0; j < 32; ++j)
+                                v[j] = (full || cb + j < a.C) ? fminf(fmaxf(v[j], 0.f), 6.f) : 0.f;
+                        }
+#pragma unroll
+                        for (int j = 0; j < 32; ++j) {
+                            hi[j] = __float_as_uint(v[j]) & 0xffffe000u;
+                            lo[j] = __float_as_uint(v[j] - __uint_as_float(hi[j]));
+                        }
+                        // B of this chunk must have landed before the MMA is released
+                        if (!mbar_wait(bar_full + 8 * st, static_cast<int>(item / L::kS) & 1)) {
+                            abort_now(); failed = true; break;
+                        }
+                    } else {
+                        if (!mbar_wait(bar_full + 8 * st, static_cast<int>(item / L::kS) & 1)) {
+                            abort_now(); failed = true; break;
+                        }
+                        tc::fence_after_sync();
+                        const uint32_t src = base + st * L::kStage + row * kRowBytes;
+#pragma unroll
+                        for (int j = 0; j < 8; ++j) {
+                            uint32_t vv[4];
+                            asm volatile("ld.shared.v4.b32 {%0, %1, %2, %3}, [%4];\n"
+                                         : "=r"(vv[0]), "=r"(vv[1]), "=r"(vv[2]), "=r"(vv[3])
+                                         : "r"(src + ((j ^ (row & 7)) << 4))
+                                         : "memory");
+#pragma unroll
+                            for (int e = 0; e < 4; ++e) {
+                                hi[4 * j + e] = vv[e] & 0xffffe000u;
+                                lo[4 * j + e] = __float_as_uint(__uint_as_float(vv[e]) - __uint_as_float(hi[4 * j + e]));
+                            }
+                        }
+                    }
+                    const uint32_t slot = lane_base + static_cast<uint32_t>(item & 1) * 64;
+                    tc::st_32x32b_x32(slot, hi);
+                    tc::st_32x32b_x32(slot + 32, lo);
+                    tc::st_wait();
+                    tc::fence_before_sync();
+                    mbar_arrive(bar_split + 8 * st);
+                }
             }
         }
     } else {
@@ -912,7 +985,10 @@ cudaError_t launch_bn(const ConvArgs &a, const typename Tr::T *W, const typename
     // bytes of channels per load).
     const int a_tiled = (a.KH == 1 && a.KW == 1 && a.sh == 1 && a.sw == 1 && a.ph == 0 && a.pw == 0);
     CUtensorMap tmap_x;
-    if (a_tiled) {
+    if (a.dw_x) {
+        // A is computed in the kernel (fused depthwise): x has no tensor map
+        std::memset(&tmap_x, 0, sizeof tmap_x);
+    } else if (a_tiled) {
         if (!tmap_2d(&tmap_x, Tr::kTmap, elem, a.x, static_cast<uint64_t>(a.B) * a.H * a.W, a.C, kBM))
             return cudaErrorInvalidValue;
     } else {

@@ -71,6 +71,8 @@ SIGNATURES = {
     "onexn_conv_fwd_ex": ([ctypes.POINTER(ConvDesc), _P, _P, _P, _I32, _I64, _P, _P, _P, _P, _I32,
                            _U32, _P, ctypes.c_size_t, _P], _I32),
     "onexn_dwconv_fwd": ([ctypes.POINTER(ConvDesc), _P, _P, _P, _P, _I32, _U32, _P], _I32),
+    "onexn_dwproj_fwd": ([ctypes.POINTER(ConvDesc), _P, _P, _P, _P, _P, _I32, _I64, _I32, _P, _P, _P, _P, _I32,
+                          _U32, _P, ctypes.c_size_t, _P], _I32),
     "onexn_prune_device_workspace_size": ([_I32, _I32, _I32, _I32, _I32, _I32, _P], _I32),
     "onexn_prune_device": ([_P, _I32, _I32, _I32, _I32, _I32, _DBL, _I32, _P, _P, _P, ctypes.c_size_t, _P],
                            _I32),

@@ -158,6 +158,28 @@ def test_streams_and_repeat_calls_are_deterministic():
     assert torch.equal(y1, y2)
 
 
+# tile counts around whole rounds of 152 CTAs: one tile past two rounds (a
+# one-tile stream-K round after whole tiles), exactly two rounds (no split),
+# and a bf16 3x3 with 36 chunks per tile and a ragged last round
+SK_CASES = [
+    L("sk153", 1, 139, 140, 512, 64, 1, 1, 1, 0, 1, N=8, rate=0.5, dtype="f32", seed=41),     # 153 tiles
+    L("sk304", 1, 152, 256, 512, 64, 1, 1, 1, 0, 1, N=8, rate=0.5, dtype="f32", seed=42),     # 304 tiles
+    L("sk_b", 2, 60, 60, 256, 128, 3, 3, 1, 1, 1, N=8, rate=0.5, dtype="bf16", seed=43),      # 57 tiles
+    L("sk_b2", 10, 46, 46, 256, 128, 3, 3, 1, 1, 1, N=16, rate=0.7, dtype="bf16", seed=44),   # 166 tiles
+]
+
+
+@pytest.mark.parametrize("layer", SK_CASES, ids=[c.name for c in SK_CASES])
+def test_stream_k_around_whole_rounds(layer):
+    """Sampled parity (the first, last and random pixels of every tile
+    region) where the last round of tiles is split across CTAs."""
+    P = layer.pixels
+    must = [0, P - 1] + [min(P - 1, 128 * k + r) for k in range(0, -(-P // 128), 16) for r in (0, 127)]
+    pix = wl.sample_pixels(P, 1500, layer.seed, must=must)
+    y, yr, a, conv = run_layer(layer, pixels=pix, algo=ox.ONEXN_ALGO_TC)
+    assert norm_err(y, yr, a) <= tol(layer)
+
+
 def test_decoded_weights_reused_across_calls():
     """After one tc call a layer passes ONEXN_DECODED and runs the GEMM
     alone; results stay bitwise equal, including the stream-K split tiles

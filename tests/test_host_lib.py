@@ -415,3 +415,20 @@ def test_bwd_workspace_sizes_show_the_input_gradient_path():
     assert n > base and (n - base) % (128 * 64 * 4) == 0           # whole 128 x 64 fp32 partial tiles
     with pytest.raises(ox.OnexnError):
         ox.onexn_conv_bwd_data_workspace_size(ox.make_desc(1, 4, 4, 8, 12), 4, 1, ox.ONEXN_F32)   # C_out % 8
+
+
+def test_dwproj_argument_errors_need_no_gpu():
+    keep, base = _aligned_host(1 << 16)
+    f = ox.lib.onexn_dwproj_fwd
+    def call(desc, dtype=ox.ONEXN_F32, flags=0, C_out=32, W=base):
+        return f(ctypes.byref(desc), W, None, base, base, base, 4, 10, C_out, base, base + 32768, None, None,
+                 dtype, flags, None, 0, None)
+    assert call(ox.make_desc(1, 8, 8, 64, 64, 3, 3, 3, 1, 1)) == ox.ONEXN_EINVAL           # stride 3
+    assert call(ox.make_desc(1, 8, 8, 64, 64, 5, 5, 1, 2, 1)) == ox.ONEXN_EINVAL           # 5x5
+    assert call(ox.make_desc(1, 8, 8, 64, 32, 3, 3, 1, 1, 1)) == ox.ONEXN_EINVAL           # C_in != C_out
+    assert call(ox.make_desc(1, 8, 8, 64, 64, 3, 3, 1, 1, 1), dtype=ox.ONEXN_BF16) == ox.ONEXN_EUNSUPPORTED
+    assert call(ox.make_desc(1, 8, 8, 64, 64, 3, 3, 1, 1, 1), flags=ox.ONEXN_ALGO_FMA) == ox.ONEXN_EINVAL
+    st = call(ox.make_desc(1, 8, 8, 64, 64, 3, 3, 1, 1, 1), W=base + 4)                    # misaligned W_dw
+    assert st == ox.ONEXN_EINVAL and b"aligned" in ox.lib.onexn_last_error()
+    st = call(ox.make_desc(1, 8, 8, 64, 64, 3, 3, 1, 1, 1))                                # no workspace
+    assert st == ox.ONEXN_EINVAL and b"workspace" in ox.lib.onexn_last_error()

@@ -101,9 +101,10 @@ def test_conv_with_residual_and_relu6(dtype, algo, aliased):
     assert (ref == 6).any() and (ref == 0).any()     # both clamps exercised
 
 
-def _block(blk):
+def _block(blk, fuse_dw="auto"):
     we, be, wd, bd, wp, bp = wl.block_weights(blk)
-    return InvertedResidual(we, be, wd, bd, wp, bp, stride=blk.stride, N=blk.N, rate=blk.rate, dtype=blk.dtype)
+    return InvertedResidual(we, be, wd, bd, wp, bp, stride=blk.stride, N=blk.N, rate=blk.rate, dtype=blk.dtype,
+                            fuse_dw=fuse_dw)
 
 
 BLOCKS = [  # name, hw, c_in, hidden, c_out, stride  (MobileNet-V2 shapes at a smaller image)
@@ -119,7 +120,7 @@ BLOCKS = [  # name, hw, c_in, hidden, c_out, stride  (MobileNet-V2 shapes at a s
 def test_inverted_residual_block_stage_by_stage(dtype, spec):
     name, hw, c_in, hidden, c_out, stride = spec
     blk = wl.MBv2Block(name, 2, hw, c_in, hidden, c_out, stride, N=4, rate=0.5, dtype=dtype, seed=len(name))
-    block = _block(blk)
+    block = _block(blk, fuse_dw=False)          # the depthwise output is read back below
     x = _dev(wl.block_input(blk), dtype)
     out = block(x)
     torch.cuda.synchronize()
@@ -141,6 +142,52 @@ def test_inverted_residual_block_stage_by_stage(dtype, spec):
                                 residual=xs if block.residual else None, want_abs=True)
     assert block.residual == (stride == 1 and c_in == c_out)
     assert _err(_host32(out), ref, a) <= TOL[dtype], "project"
+
+
+FUSED = BLOCKS + [("wide_s2_ragged", 11, 40, 240, 48, 2),      # 240 = 7.5 chunks of 32 channels
+                  ("one_image_row", 1, 24, 72, 24, 1)]
+
+
+@pytest.mark.parametrize("spec", FUSED, ids=[b[0] for b in FUSED])
+def test_depthwise_fused_into_the_projection(spec):
+    """onexn_dwproj_fwd (fp32): the projection's GEMM computes relu6(dw(h))
+    itself; against the oracle's depthwise then projection (+ residual) on
+    the GPU's own expand output, and against the unfused kernels."""
+    name, hw, c_in, hidden, c_out, stride = spec
+    blk = wl.MBv2Block(name, 2, hw, c_in, hidden, c_out, stride, N=4, rate=0.5, dtype="f32", seed=len(name) + 1)
+    fused, plain = _block(blk, fuse_dw=True), _block(blk, fuse_dw=False)
+    x = wl.block_input(blk).cuda()
+    out = fused(x).clone()
+    ref_gpu = plain(x).clone()
+    torch.cuda.synchronize()
+    h = plain.buffers(x.shape, x.dtype, x.device)[0]
+    hs = _host32(h) if fused.expand is not None else _host32(x)
+    d = oracle.dwconv(hs, fused.w_dw, fused.b_dw, stride=(stride, stride), pad=(1, 1), relu="relu6")
+    xs = _host32(x)
+    ref, a = oracle.conv_masked(d.astype(np.float32), fused.w_project,
+                                _mask(fused.project, fused.w_project, 4, 0.5), fused.b_project, 4,
+                                residual=xs if fused.residual else None, want_abs=True)
+    assert _err(_host32(out), ref, a) <= 1e-5
+    assert _err(_host32(out), _host32(ref_gpu).astype(np.float64), a) <= 1e-5
+    # a second call runs on the resident decoded weights
+    out2 = fused(x)
+    torch.cuda.synchronize()
+    assert torch.equal(out2, out)
+
+
+def test_dwproj_rejects_bf16_and_bad_depthwise_geometry():
+    from paper_2105_14713_gb300.layer import PrunedConv2d
+    blk = wl.MBv2Block("rej", 1, 8, 32, 64, 32, 1, N=4, rate=0.5, dtype="bf16", seed=1)
+    b16 = _block(blk)
+    assert not b16.fused((1, 8, 8, 32))
+    W = np.random.default_rng(0).standard_normal((32, 64, 1, 1)).astype(np.float32)
+    conv = PrunedConv2d(W, 4, 0.5)
+    h = torch.zeros((1, 8, 8, 64), device="cuda")
+    wt = torch.zeros((9, 64), device="cuda")
+    with pytest.raises(ox.OnexnError):
+        conv.forward_dwproj(h, wt, None, 3)        # stride 3
+    with pytest.raises((ValueError, ox.OnexnError)):
+        conv.forward_dwproj(h.to(torch.bfloat16), wt, None, 1)
 
 
 def test_block_end_to_end_fp32_and_cuda_graph_replay():
