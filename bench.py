@@ -312,7 +312,7 @@ def cpu_baseline(layers, budget_s: float = 10.0):
     rng = np.random.default_rng(0)
     max_pix = 784 if len(layers) <= 2 else 64
     spent, flops, passes = 0.0, 0.0, 0
-    while spent < budget_s and passes < 64:
+    while spent < budget_s and passes < 1024:
         dt, fl = oracle_pass(layers, packs, max_pix, rng)
         spent += dt
         flops += fl
