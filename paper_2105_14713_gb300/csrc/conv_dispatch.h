@@ -34,7 +34,7 @@ TcSplitPlan tc_split_plan(int M, int Ncols, int64_t K, int dtype);
 cudaError_t tc_gemm_split(const ConvArgs &a, int dtype, const void *W, const void *W_lo, float *partials,
                           const TcSplitPlan &plan, cudaStream_t st);
 size_t tc_weights_bytes(const ConvArgs &a, int dtype);
-size_t tc_sk_bytes(const ConvArgs &a);
+size_t tc_sk_bytes(const ConvArgs &a, int dtype);
 
 namespace detail {
 

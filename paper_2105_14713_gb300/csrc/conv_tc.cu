@@ -1112,7 +1112,13 @@ cudaError_t launch_bn(const ConvArgs &a, const typename Tr::T *W, const typename
 // plus a BN-independent share (A loads, epilogue start), 64 columns' worth.
 // Narrow tiles win when there are few pixel tiles (more CTAs busy); wide
 // tiles re-read the A operand fewer times.  Ties go to the wider tile.
-int tc_bn(const ConvArgs &a)
+// fp32 takes 128 instead of 256 unless that leaves a last column tile less
+// than half full: at 256 the fp32 TMEM holds one accumulator next to the A
+// ring, so a tile's MMAs wait for the previous tile's epilogue (measured on
+// GB300: 3x3 512->512 on 128x14x14 472 -> 402 us, 1x1 96->576 33 -> 25 us;
+// but 1x1 24->144, whose second 128-column tile would hold 16 columns,
+// 83 -> 103 us).
+int tc_bn(const ConvArgs &a, int dtype)
 {
     const int64_t n_m = (static_cast<int64_t>(a.P_pix) + kBM - 1) / kBM;
     int best = 256;
@@ -1126,6 +1132,7 @@ int tc_bn(const ConvArgs &a)
             best_cost = cost;
         }
     }
+    if (dtype == ONEXN_F32 && best == 256 && (a.C_out % 128 == 0 || a.C_out % 128 >= 64)) best = 128;
     return best;
 }
 
@@ -1139,7 +1146,10 @@ size_t weights_bytes(const ConvArgs &a, int dtype)
 }
 
 // stream-K space after the weights: the partial slots, then the flags
-size_t sk_bytes(const ConvArgs &a) { return sk_partial_bytes(tc_bn(a)) + round256(kPlanCTAs * sizeof(int)); }
+size_t sk_bytes(const ConvArgs &a, int dtype)
+{
+    return sk_partial_bytes(tc_bn(a, dtype)) + round256(kPlanCTAs * sizeof(int));
+}
 
 template <typename Tr>
 cudaError_t decode_typed(const ConvArgs &a, void *workspace, size_t ws_bytes, cudaStream_t st)
@@ -1151,8 +1161,10 @@ cudaError_t decode_typed(const ConvArgs &a, void *workspace, size_t ws_bytes, cu
     T *W_lo = Tr::kSplit ? W + n : nullptr;
     const size_t wb = weights_bytes(a, Tr::kSplit ? ONEXN_F32 : ONEXN_BF16);
     int *flags = nullptr;
-    if (ws_bytes >= wb + sk_bytes(a))
-        flags = reinterpret_cast<int *>(static_cast<unsigned char *>(workspace) + wb + sk_partial_bytes(tc_bn(a)));
+    const int dtype = Tr::kSplit ? ONEXN_F32 : ONEXN_BF16;
+    if (ws_bytes >= wb + sk_bytes(a, dtype))
+        flags = reinterpret_cast<int *>(static_cast<unsigned char *>(workspace) + wb +
+                                        sk_partial_bytes(tc_bn(a, dtype)));
     const dim3 grid(static_cast<unsigned>((K + kDecodeCols - 1) / kDecodeCols), a.C_out / a.N,
                     (a.N + kDecodeRows - 1) / kDecodeRows);
     bsr_decode_kernel<T><<<grid, kDecodeCols, 0, st>>>(a.P, a.I, static_cast<const T *>(a.D), a.N, a.t, K, W, W_lo,
@@ -1168,10 +1180,11 @@ cudaError_t gemm_typed(const ConvArgs &a, const void *workspace, size_t ws_bytes
     const T *W = static_cast<const T *>(workspace);
     const T *W_lo = Tr::kSplit ? W + n : nullptr;
     const size_t wb = weights_bytes(a, Tr::kSplit ? ONEXN_F32 : ONEXN_BF16);
-    void *sk = ws_bytes >= wb + sk_bytes(a)
+    const int dtype = Tr::kSplit ? ONEXN_F32 : ONEXN_BF16;
+    void *sk = ws_bytes >= wb + sk_bytes(a, dtype)
                    ? static_cast<void *>(static_cast<unsigned char *>(const_cast<void *>(workspace)) + wb)
                    : nullptr;
-    const int bn = tc_bn(a);
+    const int bn = tc_bn(a, dtype);
     if (bn == 64) return launch_bn<Tr, 64>(a, W, W_lo, sk, st);
     if (bn == 128) return launch_bn<Tr, 128>(a, W, W_lo, sk, st);
     return launch_bn<Tr, 256>(a, W, W_lo, sk, st);
@@ -1192,12 +1205,12 @@ double tc_cost_ns(const ConvArgs &a, int dtype, size_t ws_bytes, bool decoded)
     constexpr double kGemmFixedNs = 1200.0, kSkFixupNs = 7000.0, kDecodeFixedNs = 2000.0,
                      kDecodeBytesPerNs = 2000.0;
     const bool f32 = dtype == ONEXN_F32;
-    const int bn = tc_bn(a);
+    const int bn = tc_bn(a, dtype);
     const int bk = f32 ? TcF32::kBK : TcBf16::kBK;
     const int64_t n_m = (static_cast<int64_t>(a.P_pix) + kBM - 1) / kBM, n_n = (a.C_out + bn - 1) / bn;
     const int64_t tiles = n_m * n_n, chunks = static_cast<int64_t>(a.KH) * a.KW * ((a.C + bk - 1) / bk);
     const size_t wb = weights_bytes(a, dtype);
-    const bool sk = ws_bytes >= wb + sk_bytes(a) && tiles < kPlanCTAs && chunks >= sk_min_chunks(f32);
+    const bool sk = ws_bytes >= wb + sk_bytes(a, dtype) && tiles < kPlanCTAs && chunks >= sk_min_chunks(f32);
     double busy;
     if (tiles >= kPlanCTAs)
         busy = static_cast<double>(tiles) / static_cast<double>((tiles + kPlanCTAs - 1) / kPlanCTAs);
@@ -1216,7 +1229,7 @@ double tc_cost_ns(const ConvArgs &a, int dtype, size_t ws_bytes, bool decoded)
 // The decoded weights; with room for the stream-K partial slots and
 // flags after them the GEMM also balances its last round of tiles.
 size_t tc_workspace_min(const ConvArgs &a, int dtype) { return weights_bytes(a, dtype); }
-size_t tc_workspace_bytes(const ConvArgs &a, int dtype) { return weights_bytes(a, dtype) + sk_bytes(a); }
+size_t tc_workspace_bytes(const ConvArgs &a, int dtype) { return weights_bytes(a, dtype) + sk_bytes(a, dtype); }
 
 // C_in, C_out giving 16-byte rows; the im2col box corners within the TMA's
 // [-128, 127] range; strides <= 8; 16-bit tap offsets.
@@ -1263,7 +1276,7 @@ cudaError_t tc_gemm_weights(const ConvArgs &a, int dtype, const void *W, const v
                             cudaStream_t st)
 {
     if (a.P_pix == 0) return cudaSuccess;
-    const int bn = tc_bn(a);
+    const int bn = tc_bn(a, dtype);
     if (dtype == ONEXN_F32) {
         const float *w = static_cast<const float *>(W), *wl = static_cast<const float *>(W_lo);
         if (bn == 64) return launch_bn<TcF32, 64>(a, w, wl, sk_space, st);
@@ -1317,7 +1330,7 @@ cudaError_t tc_gemm_split(const ConvArgs &a, int dtype, const void *W, const voi
 }
 
 size_t tc_weights_bytes(const ConvArgs &a, int dtype) { return weights_bytes(a, dtype); }
-size_t tc_sk_bytes(const ConvArgs &a) { return sk_bytes(a); }
+size_t tc_sk_bytes(const ConvArgs &a, int dtype) { return sk_bytes(a, dtype); }
 
 // decode, then the GEMM as its programmatic dependent (its launch and
 // prologue overlap the decode)
