@@ -1,5 +1,6 @@
 """Parity of the five synthetic workloads at their full sizes, in the launch
-configuration bench.py times (AUTO kernel selection, caller workspace).
+configuration bench.py times (AUTO kernel selection, caller workspace, and
+the weights decoded by the first call reused by the second).
 
 Small layers are compared in full; large ones on seeded sampled output
 pixels (always including the first and last pixel) across all output
@@ -23,8 +24,12 @@ def _run(layer, W, x_cpu, b, pixels, relu=False, master=False):
     conv = PrunedConv2d(W, layer.N, layer.rate, bias=b, stride=layer.stride, padding=layer.pad,
                         dilation=layer.dil, dtype=layer.dtype)
     xd = (x_cpu if layer.dtype == "f32" else x_cpu.to(torch.bfloat16)).cuda()
-    y = conv(xd, relu=relu)
+    y = conv(xd, relu=relu).clone()
+    # the path bench.py times: the second call runs on the decoded weights
+    # the first left in the workspace, and must match it bit for bit
+    y2 = conv(xd, relu=relu)
     torch.cuda.synchronize()
+    assert torch.equal(y, y2), f"{layer.name}: the decoded-weights call differs"
     yf = y.float().reshape(-1, layer.C_out)
     y_s = (yf if pixels is None else yf[torch.as_tensor(pixels, device="cuda")]).cpu().numpy()
     y_ref, a = oracle_ref(layer, W, x_cpu, b, relu=relu, pixels=pixels, master=master)
