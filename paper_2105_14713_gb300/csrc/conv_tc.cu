@@ -232,6 +232,10 @@ struct TcSched {
     int n_tiles, n_tn, n_chunks;
     int dp_tiles, sk_tiles, sk_ctas;
     int split_s;
+    // one K chunk and one column tile: every tile multiplies the same B, which
+    // is loaded once into stage 0's B region and stays there; the stages
+    // then carry A only
+    int b_resident;
     // divisors of the per-tile / per-segment index arithmetic
     FastDiv div_tn, div_hw, div_wo, div_cchunk, div_kw;
     float *partials;     // slot b: CTA b's part of a split tile, [BN/4][128] float4
@@ -398,11 +402,14 @@ tc_conv_kernel(const ConvArgs a, const __grid_constant__ CUtensorMap tmap_x,
                     }
                     const uint32_t sa = base + st * L::kStage;
                     const uint32_t sb = sa + L::kA;
+                    // B bytes of this chunk: none when B is resident, after item 0
+                    const bool load_b = !sched.b_resident || item == 0;
+                    const uint32_t b_tx = load_b ? static_cast<uint32_t>(L::kTx - L::kA) : 0u;
                     if (dw_mode) {
                         // A comes from the split warps' depthwise; only B is loaded
-                        tc::mbar_arrive_expect_tx(bar_full + 8 * st, L::kTx - L::kA);
+                        tc::mbar_arrive_expect_tx(bar_full + 8 * st, b_tx);
                     } else {
-                        tc::mbar_arrive_expect_tx(bar_full + 8 * st, L::kTx);
+                        tc::mbar_arrive_expect_tx(bar_full + 8 * st, L::kA + b_tx);
                         if (a_tiled)
                             tc::tma_load_2d(sa, &tmap_x, cc0, p0, bar_full + 8 * st);
                         else
@@ -410,9 +417,11 @@ tc_conv_kernel(const ConvArgs a, const __grid_constant__ CUtensorMap tmap_x,
                                                    static_cast<uint16_t>(kw * a.dw), static_cast<uint16_t>(kh * a.dh),
                                                    bar_full + 8 * st);
                     }
-                    tc::tma_load_2d(sb, &tmap_w, k0tap + cc0, tn * BN, bar_full + 8 * st);
-                    if constexpr (Tr::kSplit)
-                        tc::tma_load_2d(sb + L::kB, &tmap_wlo, k0tap + cc0, tn * BN, bar_full + 8 * st);
+                    if (load_b) {
+                        tc::tma_load_2d(sb, &tmap_w, k0tap + cc0, tn * BN, bar_full + 8 * st);
+                        if constexpr (Tr::kSplit)
+                            tc::tma_load_2d(sb + L::kB, &tmap_wlo, k0tap + cc0, tn * BN, bar_full + 8 * st);
+                    }
                     cc0 += Tr::kBK;
                     if (cc0 >= a.C) {
                         cc0 = 0; k0tap += a.C;
@@ -443,11 +452,12 @@ tc_conv_kernel(const ConvArgs a, const __grid_constant__ CUtensorMap tmap_x,
                     }
                     tc::fence_after_sync();
                     const uint32_t sa = base + st * L::kStage;
-                    const uint64_t bd = tc::desc_kmajor_sw128(sa + L::kA);
+                    const uint32_t sbm = (sched.b_resident ? base : sa) + L::kA;   // this chunk's B
+                    const uint64_t bd = tc::desc_kmajor_sw128(sbm);
                     const uint32_t first = (c == sg.c0) ? 1u : 0u;   // the first chunk overwrites D
                     if constexpr (Tr::kSplit) {
                         constexpr uint32_t idesc = tc::idesc_tf32_f32(kBM, BN);
-                        const uint64_t bld = tc::desc_kmajor_sw128(sa + L::kA + L::kB);
+                        const uint64_t bld = tc::desc_kmajor_sw128(sbm + L::kB);
                         // A slot of this chunk: x_hi columns, then x_lo 32 columns on
                         const uint32_t a_hi = tmem + L::kAcc * BN + (item & 1) * 64;
 #pragma unroll
@@ -1091,6 +1101,7 @@ cudaError_t launch_bn(const ConvArgs &a, const typename Tr::T *W, const typename
             sc.flags = reinterpret_cast<int *>(static_cast<unsigned char *>(sk_space) + sk_partial_bytes(BN));
         }
     }
+    sc.b_resident = (sc.n_chunks == 1 && sc.n_tn == 1 && sc.sk_tiles == 0 && sc.split_s == 0) ? 1 : 0;
     cudaLaunchConfig_t cfg{};
     cfg.gridDim = dim3(grid);
     cfg.blockDim = dim3(Tr::kWarps * 32);
