@@ -33,7 +33,7 @@ using onexn::fail;
 
 namespace {
 
-constexpr int kTile = 32;           // transpose tiles: 32 x 32 elements, 32 x 8 threads
+constexpr int kTile = 32;           // weight transpose tiles: 32 x 32 elements, 32 x 8 threads
 constexpr int kPixPad = 64;         // pixels padded to the bf16 K chunk
 
 __device__ __forceinline__ float tf32_rna(float v)
@@ -50,135 +50,179 @@ __device__ __forceinline__ float to_f(T v)
     else return __bfloat162float(v);
 }
 
-// dYt[o][p] = dY[p][o] for p < P, 0 for P <= p < P_pad (fp32: as its tf32
-// rounding `hi` and the rest `lo`, the B operand of the weight-gradient
-// GEMM), and the column sums of each 32-pixel block, colsum[o][blockIdx.x]
-// (the bias gradient's first stage).
-template <typename T>
-__global__ void __launch_bounds__(kTile * 8)
-dy_transpose_kernel(const T *__restrict__ dy, int64_t P, int64_t P_pad, int C_out, T *__restrict__ hi,
-                    T *__restrict__ lo, float *__restrict__ colsum, int n_pb)
-{
-    __shared__ T tile[kTile][kTile + 1];
-    const int64_t p0 = static_cast<int64_t>(blockIdx.x) * kTile;
-    const int o0 = blockIdx.y * kTile;
-    const int tx = threadIdx.x, ty = threadIdx.y;
-    for (int i = ty; i < kTile; i += 8) {
-        const int64_t p = p0 + i;
-        const int o = o0 + tx;
-        tile[i][tx] = (p < P && o < C_out) ? dy[p * C_out + o] : T(0.f);
-    }
-    __syncthreads();
-    if (ty == 0 && o0 + tx < C_out) {
-        float c = 0.f;
-        for (int i = 0; i < kTile; ++i) c += to_f(tile[i][tx]);
-        colsum[static_cast<int64_t>(o0 + tx) * n_pb + blockIdx.x] = c;
-    }
-    for (int i = ty; i < kTile; i += 8) {
-        const int o = o0 + i;
-        const int64_t p = p0 + tx;
-        if (o >= C_out || p >= P_pad) continue;
-        const int64_t dst = static_cast<int64_t>(o) * P_pad + p;
-        const T v = tile[tx][i];
-        if constexpr (sizeof(T) == 4) {
-            const float h = tf32_rna(v);
-            hi[dst] = h;
-            lo[dst] = v - h;
-        } else {
-            hi[dst] = v;
-        }
-    }
-}
-
-// XcolT[tap*C_in + c][p] = x[b, oh*sh - ph + kh*dh, ow*sw - pw + kw*dw, c]
-// (0 outside the image and for p >= P).  A CTA takes 64 channels of one tap
-// and kXcolTiles tiles of 64 pixels: it first finds, once per pixel, the
-// input pixel the tap reads (or none), then moves each tile through shared
-// memory with 4-channel vector reads and 4-pixel vector writes.
-constexpr int kXcolTiles = 4;
+// Pixel-contiguous copies of the two operands of the weight-gradient GEMM
+// (both K-major in the pixel index p, pixels padded to P_pad with zeros).
+// One launch, two roles:
+//   dy role   dYt[o][p] = dY[p][o] (fp32: as its tf32 rounding `hi` and the
+//             rest `lo`), and the sums of each 32-pixel block, colsum[o][p/32]
+//             (the bias gradient's first stage);
+//   xcol role XcolT[tap*C + c][p] = x[b, oh*sh - ph + kh*dh, ow*sw - pw + kw*dw, c]
+//             (0 outside the image).
+// A CTA moves 64-pixel x 64-channel tiles through shared memory: 16-byte
+// loads along channels, 16-byte stores along pixels.  bf16 tiles pair two
+// pixels of one channel in a 32-bit shared word.  Each warp covers a slab of
+// the tile whose rows fall on distinct banks on both sides (fp32: 8 channel
+// quads x 4 pixels in, 4 channels x 8 pixel quads out; bf16: 4 channel
+// octets x 8 pixel pairs in, 4 channels x 8 pixel octets out).  xcol CTAs
+// are numbered tap-fastest, so the taps of one pixel range run back to back
+// and re-read their x rows from L2.
 constexpr int kXT = 64;                          // pixels and channels per tile
+constexpr int kXcolTiles = 4;                    // pixel tiles per xcol CTA
+constexpr int kColBlock = 32;                    // pixels per column-sum block
 
-template <typename T> struct Vec4;
-template <> struct Vec4<float> { using type = float4; };
-template <> struct Vec4<__nv_bfloat16> { using type = uint2; };
+struct TransposeGrid {
+    int n_dy;                                    // dy CTAs (one 64-pixel tile each)
+    int cb_dy;                                   // 64-channel blocks of dy
+    int cb_x;                                    // 64-channel blocks of x
+    int taps;
+    int n_x;                                     // xcol CTAs
+};
 
-template <typename T>
-__device__ __forceinline__ void unpack4(const typename Vec4<T>::type &v, T (&e)[4])
+__device__ __forceinline__ uint32_t bf16_pair(uint32_t a, uint32_t b, int hi)
 {
-    if constexpr (sizeof(T) == 4) {
-        e[0] = v.x; e[1] = v.y; e[2] = v.z; e[3] = v.w;
-    } else {
-        const __nv_bfloat162 a = *reinterpret_cast<const __nv_bfloat162 *>(&v.x);
-        const __nv_bfloat162 b = *reinterpret_cast<const __nv_bfloat162 *>(&v.y);
-        e[0] = a.x; e[1] = a.y; e[2] = b.x; e[3] = b.y;
-    }
-}
-
-template <typename T>
-__device__ __forceinline__ typename Vec4<T>::type pack4(const T (&e)[4])
-{
-    typename Vec4<T>::type v;
-    if constexpr (sizeof(T) == 4) {
-        v = make_float4(e[0], e[1], e[2], e[3]);
-    } else {
-        __nv_bfloat162 a, b;
-        a.x = e[0]; a.y = e[1]; b.x = e[2]; b.y = e[3];
-        v.x = *reinterpret_cast<uint32_t *>(&a);
-        v.y = *reinterpret_cast<uint32_t *>(&b);
-    }
-    return v;
+    // (a.half[hi], b.half[hi]) as (low, high) halves of one word
+    return __byte_perm(a, b, hi ? 0x7632 : 0x5410);
 }
 
 template <typename T>
 __global__ void __launch_bounds__(256)
-xcol_transpose_kernel(const ConvArgs a, int P_pad, const onexn::FastDiv div_hw, const onexn::FastDiv div_wo,
-                      T *__restrict__ out)
+wgrad_transpose_kernel(const ConvArgs a, const T *__restrict__ dy, int P_pad, const TransposeGrid g,
+                       const onexn::FastDiv div_hw, const onexn::FastDiv div_wo, T *__restrict__ xcol,
+                       T *__restrict__ hi, T *__restrict__ lo, float *__restrict__ colsum, int n_pb)
 {
-    using V = typename Vec4<T>::type;
-    __shared__ T tile[kXT][kXT + 1];             // [channel][pixel]
-    __shared__ int src[kXcolTiles * kXT];        // input pixel (b*H + ih)*W + iw, or -1
-    const int c0 = blockIdx.y * kXT, tap = blockIdx.z;
-    const int kh = tap / a.KW, kw = tap - (tap / a.KW) * a.KW;
-    const int tid = threadIdx.x;
-    const int hw = a.Ho * a.Wo;
-    const int pb = blockIdx.x * kXcolTiles * kXT;
-    for (int i = tid; i < kXcolTiles * kXT; i += 256) {
-        const int p = pb + i;
-        int sp = -1;
-        if (p < a.P_pix) {
-            const uint32_t b = div_hw.div(static_cast<uint32_t>(p));
-            const uint32_t r = static_cast<uint32_t>(p) - b * hw;
-            const int oh = static_cast<int>(div_wo.div(r)), ow = static_cast<int>(r) - oh * a.Wo;
-            const int ih = oh * a.sh - a.ph + kh * a.dh, iw = ow * a.sw - a.pw + kw * a.dw;
-            if (ih >= 0 && ih < a.H && iw >= 0 && iw < a.W) sp = (static_cast<int>(b) * a.H + ih) * a.W + iw;
+    constexpr bool kF32 = sizeof(T) == 4;
+    __shared__ uint32_t tile[kXT * (kXT + 1)];   // fp32: [64 ch][65]; bf16: [64 ch][33] pixel pairs
+    __shared__ int src[kXcolTiles * kXT];        // source row of each pixel, or -1
+    constexpr int kLd = kF32 ? kXT + 1 : kXT / 2 + 1;
+    const int tid = threadIdx.x, lane = tid & 31, w = tid >> 5;
+    const bool dy_role = static_cast<int>(blockIdx.x) < g.n_dy;
+    int c0, tap = 0, pb, n_tiles, Cn;
+    const T *base;
+    if (dy_role) {
+        const int b = blockIdx.x;
+        c0 = (b % g.cb_dy) * kXT;
+        pb = (b / g.cb_dy) * kXT;
+        n_tiles = 1;
+        Cn = a.C_out;
+        base = dy;
+        for (int i = tid; i < kXT; i += 256) src[i] = pb + i < a.P_pix ? pb + i : -1;
+    } else {
+        const int b = blockIdx.x - g.n_dy;
+        tap = b % g.taps;
+        const int rest = b / g.taps;
+        c0 = (rest % g.cb_x) * kXT;
+        pb = (rest / g.cb_x) * (kXcolTiles * kXT);
+        n_tiles = min(kXcolTiles, (P_pad - pb) / kXT);
+        Cn = a.C;
+        base = static_cast<const T *>(a.x);
+        const int kh = tap / a.KW, kw = tap - (tap / a.KW) * a.KW;
+        const int hw = a.Ho * a.Wo;
+        for (int i = tid; i < kXcolTiles * kXT; i += 256) {
+            const int p = pb + i;
+            int sp = -1;
+            if (p < a.P_pix) {
+                const uint32_t bb = div_hw.div(static_cast<uint32_t>(p));
+                const uint32_t r = static_cast<uint32_t>(p) - bb * hw;
+                const int oh = static_cast<int>(div_wo.div(r)), ow = static_cast<int>(r) - oh * a.Wo;
+                const int ih = oh * a.sh - a.ph + kh * a.dh, iw = ow * a.sw - a.pw + kw * a.dw;
+                if (ih >= 0 && ih < a.H && iw >= 0 && iw < a.W) sp = (static_cast<int>(bb) * a.H + ih) * a.W + iw;
+            }
+            src[i] = sp;
         }
-        src[i] = sp;
     }
     __syncthreads();
-    // read role: 16 threads per pixel row, each 4 channels; write role: 16
-    // threads per channel row, each 4 pixels
-    const int q = tid & 15, r16 = tid >> 4;
-    const int cq = c0 + 4 * q;                   // this thread's channel quad
-    const bool c_ok = cq < a.C;
-    const T *x = static_cast<const T *>(a.x);
-    T *obase = out + (static_cast<int64_t>(tap) * a.C + c0) * P_pad;
-    for (int tt = 0; tt < kXcolTiles; ++tt) {
+    for (int tt = 0; tt < n_tiles; ++tt) {
         const int p0 = pb + tt * kXT;
-        if (p0 >= P_pad) break;
+        const int *s = src + tt * kXT;
+        if constexpr (kF32) {
+            // in: channel quad q, pixels i + 16k
+            const int q = (lane & 7) + 8 * (w & 1), i = (lane >> 3) + 4 * (w >> 1);
+            const bool c_ok = c0 + 4 * q < Cn;
+            float4 v[4];
 #pragma unroll
-        for (int i = r16; i < kXT; i += 16) {
-            const int sp = src[tt * kXT + i];
-            T e[4] = {T(0.f), T(0.f), T(0.f), T(0.f)};
-            if (sp >= 0 && c_ok) unpack4<T>(__ldg(reinterpret_cast<const V *>(x + static_cast<int64_t>(sp) * a.C + cq)), e);
+            for (int k = 0; k < 4; ++k) {
+                const int sp = s[i + 16 * k];
+                v[k] = make_float4(0.f, 0.f, 0.f, 0.f);
+                if (sp >= 0 && c_ok)
+                    v[k] = __ldg(reinterpret_cast<const float4 *>(base + static_cast<int64_t>(sp) * Cn + c0 + 4 * q));
+            }
 #pragma unroll
-            for (int j = 0; j < 4; ++j) tile[4 * q + j][i] = e[j];
+            for (int k = 0; k < 4; ++k) {
+                uint32_t *t = tile + (4 * q) * kLd + i + 16 * k;
+                t[0] = __float_as_uint(v[k].x);
+                t[kLd] = __float_as_uint(v[k].y);
+                t[2 * kLd] = __float_as_uint(v[k].z);
+                t[3 * kLd] = __float_as_uint(v[k].w);
+            }
+        } else {
+            // in: channel octet q, pixels 2r and 2r + 1
+            const int q = (lane & 3) + 4 * (w & 1), r = (lane >> 2) + 8 * (w >> 1);
+            const bool c_ok = c0 + 8 * q < Cn;
+            const int s0 = s[2 * r], s1 = s[2 * r + 1];
+            uint4 u0 = make_uint4(0u, 0u, 0u, 0u), u1 = u0;
+            if (s0 >= 0 && c_ok)
+                u0 = __ldg(reinterpret_cast<const uint4 *>(base + static_cast<int64_t>(s0) * Cn + c0 + 8 * q));
+            if (s1 >= 0 && c_ok)
+                u1 = __ldg(reinterpret_cast<const uint4 *>(base + static_cast<int64_t>(s1) * Cn + c0 + 8 * q));
+            const uint32_t x0[4] = {u0.x, u0.y, u0.z, u0.w}, x1[4] = {u1.x, u1.y, u1.z, u1.w};
+            uint32_t *t = tile + (8 * q) * kLd + r;
+#pragma unroll
+            for (int j = 0; j < 8; ++j) t[j * kLd] = bf16_pair(x0[j >> 1], x1[j >> 1], j & 1);
         }
         __syncthreads();
+        if constexpr (kF32) {
+            // out: channel rows c + 16k, pixel quad q
+            const int q = (lane & 7) + 8 * (w & 1), c = (lane >> 3) + 4 * (w >> 1);
 #pragma unroll
-        for (int i = r16; i < kXT; i += 16) {
-            if (c0 + i >= a.C) continue;
-            const T e[4] = {tile[i][4 * q], tile[i][4 * q + 1], tile[i][4 * q + 2], tile[i][4 * q + 3]};
-            *reinterpret_cast<V *>(obase + static_cast<int64_t>(i) * P_pad + p0 + 4 * q) = pack4<T>(e);
+            for (int k = 0; k < 4; ++k) {
+                const int row = c + 16 * k;
+                const uint32_t *t = tile + row * kLd + 4 * q;
+                const float4 v = make_float4(__uint_as_float(t[0]), __uint_as_float(t[1]), __uint_as_float(t[2]),
+                                             __uint_as_float(t[3]));
+                const bool ok = c0 + row < Cn;
+                if (dy_role) {
+                    float cs = (v.x + v.y) + (v.z + v.w);
+                    cs += __shfl_xor_sync(0xffffffffu, cs, 1);
+                    cs += __shfl_xor_sync(0xffffffffu, cs, 2);
+                    cs += __shfl_xor_sync(0xffffffffu, cs, 4);
+                    if (!ok) continue;
+                    const int64_t o = static_cast<int64_t>(c0 + row);
+                    if ((lane & 7) == 0) colsum[o * n_pb + p0 / kColBlock + (w & 1)] = cs;
+                    const float4 h = make_float4(tf32_rna(v.x), tf32_rna(v.y), tf32_rna(v.z), tf32_rna(v.w));
+                    const float4 l = make_float4(v.x - h.x, v.y - h.y, v.z - h.z, v.w - h.w);
+                    *reinterpret_cast<float4 *>(hi + o * P_pad + p0 + 4 * q) = h;
+                    *reinterpret_cast<float4 *>(lo + o * P_pad + p0 + 4 * q) = l;
+                } else if (ok) {
+                    const int64_t k_row = static_cast<int64_t>(tap) * Cn + c0 + row;
+                    *reinterpret_cast<float4 *>(xcol + k_row * P_pad + p0 + 4 * q) = v;
+                }
+            }
+        } else {
+            // out: channel rows c + 32k, pixel octet q (pixel pairs 4q .. 4q + 3)
+            const int q = lane & 7, c = (lane >> 3) + 4 * w;
+#pragma unroll
+            for (int k = 0; k < 2; ++k) {
+                const int row = c + 32 * k;
+                const uint32_t *t = tile + row * kLd + 4 * q;
+                const uint4 v = make_uint4(t[0], t[1], t[2], t[3]);
+                const bool ok = c0 + row < Cn;
+                if (dy_role) {
+                    float cs = 0.f;
+                    const uint32_t u[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+                    for (int m = 0; m < 4; ++m)
+                        cs += __uint_as_float(u[m] << 16) + __uint_as_float(u[m] & 0xffff0000u);
+                    cs += __shfl_xor_sync(0xffffffffu, cs, 1);
+                    cs += __shfl_xor_sync(0xffffffffu, cs, 2);
+                    if (!ok) continue;
+                    const int64_t o = static_cast<int64_t>(c0 + row);
+                    if ((lane & 3) == 0) colsum[o * n_pb + p0 / kColBlock + (q >> 2)] = cs;
+                    *reinterpret_cast<uint4 *>(hi + o * P_pad + p0 + 8 * q) = v;
+                } else if (ok) {
+                    const int64_t k_row = static_cast<int64_t>(tap) * Cn + c0 + row;
+                    *reinterpret_cast<uint4 *>(xcol + k_row * P_pad + p0 + 8 * q) = v;
+                }
+            }
         }
         __syncthreads();
     }
@@ -410,7 +454,7 @@ WgradWs wgrad_ws(const ConvArgs &a, int dtype)
     const size_t es = dtype == ONEXN_F32 ? 4 : 2;
     const int64_t K = static_cast<int64_t>(a.KH) * a.KW * a.C;
     l.P_pad = (static_cast<int64_t>(a.P_pix) + kPixPad - 1) / kPixPad * kPixPad;
-    l.n_pb = static_cast<int>(l.P_pad / kTile);
+    l.n_pb = static_cast<int>(l.P_pad / kColBlock);
     l.plan = onexn::tc_split_plan(static_cast<int>(K), a.C_out, l.P_pad, dtype);
     l.xcol = 0;
     l.dy_hi = round256(static_cast<size_t>(K) * l.P_pad * es);
@@ -577,27 +621,30 @@ extern "C" onexn_status onexn_conv_bwd_weight(const onexn_conv_desc *desc, const
     }
     a.x = x;
     unsigned char *ws = static_cast<unsigned char *>(workspace);
-    const dim3 block(kTile, 8);
     const int K = a.KH * a.KW * a.C;
     if (L.P_pad > INT32_MAX / 2) return fail(ONEXN_EINVAL, "conv_bwd_weight: too many pixels");
     const int P_pad = static_cast<int>(L.P_pad);
-    const dim3 g_dy(static_cast<unsigned>(L.n_pb), (a.C_out + kTile - 1) / kTile);
-    const int n_ptiles = (P_pad / kXT + kXcolTiles - 1) / kXcolTiles;
-    const dim3 g_x(static_cast<unsigned>(n_ptiles), (a.C + kXT - 1) / kXT, a.KH * a.KW);
+    TransposeGrid tg{};
+    tg.cb_dy = (a.C_out + kXT - 1) / kXT;
+    tg.cb_x = (a.C + kXT - 1) / kXT;
+    tg.taps = a.KH * a.KW;
+    const int64_t n_dy = static_cast<int64_t>(P_pad / kXT) * tg.cb_dy;
+    const int64_t n_x = static_cast<int64_t>((P_pad / kXT + kXcolTiles - 1) / kXcolTiles) * tg.cb_x * tg.taps;
+    if (n_dy + n_x > INT32_MAX) return fail(ONEXN_EINVAL, "conv_bwd_weight: too many pixels x channels");
+    tg.n_dy = static_cast<int>(n_dy);
+    tg.n_x = static_cast<int>(n_x);
+    const unsigned n_cta = static_cast<unsigned>(n_dy + n_x);
     const onexn::FastDiv div_hw(static_cast<uint32_t>(a.Ho * a.Wo)), div_wo(static_cast<uint32_t>(a.Wo));
     float *colsum = reinterpret_cast<float *>(ws + L.colsum);
     if (dtype == ONEXN_F32) {
-        dy_transpose_kernel<float><<<g_dy, block, 0, s>>>(static_cast<const float *>(dy), a.P_pix, L.P_pad, a.C_out,
-                                                           reinterpret_cast<float *>(ws + L.dy_hi),
-                                                           reinterpret_cast<float *>(ws + L.dy_lo), colsum, L.n_pb);
-        xcol_transpose_kernel<float><<<g_x, 256, 0, s>>>(a, P_pad, div_hw, div_wo,
-                                                            reinterpret_cast<float *>(ws + L.xcol));
+        wgrad_transpose_kernel<float><<<n_cta, 256, 0, s>>>(
+            a, static_cast<const float *>(dy), P_pad, tg, div_hw, div_wo, reinterpret_cast<float *>(ws + L.xcol),
+            reinterpret_cast<float *>(ws + L.dy_hi), reinterpret_cast<float *>(ws + L.dy_lo), colsum, L.n_pb);
     } else {
-        dy_transpose_kernel<__nv_bfloat16><<<g_dy, block, 0, s>>>(
-            static_cast<const __nv_bfloat16 *>(dy), a.P_pix, L.P_pad, a.C_out,
-            reinterpret_cast<__nv_bfloat16 *>(ws + L.dy_hi), nullptr, colsum, L.n_pb);
-        xcol_transpose_kernel<__nv_bfloat16><<<g_x, 256, 0, s>>>(a, P_pad, div_hw, div_wo,
-                                                                    reinterpret_cast<__nv_bfloat16 *>(ws + L.xcol));
+        wgrad_transpose_kernel<__nv_bfloat16><<<n_cta, 256, 0, s>>>(
+            a, static_cast<const __nv_bfloat16 *>(dy), P_pad, tg, div_hw, div_wo,
+            reinterpret_cast<__nv_bfloat16 *>(ws + L.xcol), reinterpret_cast<__nv_bfloat16 *>(ws + L.dy_hi), nullptr,
+            colsum, L.n_pb);
     }
     e = cudaGetLastError();
     if (e != cudaSuccess) return fail(ONEXN_ECUDA, "conv_bwd_weight: transpose: %s", cudaGetErrorString(e));
