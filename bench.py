@@ -393,8 +393,9 @@ def build_legs(layers, dev):
     return legs
 
 
-def time_legs(legs, steps, warmup, flush, stream, sampler=None):
-    """Per-leg CUDA-event times (ms) of `steps` steps, L2 flushed before each."""
+def time_legs(legs, steps, warmup, flush, stream, sampler=None, flush_l2=True):
+    """Per-leg CUDA-event times (ms) of `steps` steps, L2 flushed before each
+    (flush_l2=False: back to back, the inputs left in L2 by the step before)."""
     for _ in range(warmup):
         flush.fill_(1)
         for lg in legs:
@@ -406,7 +407,8 @@ def time_legs(legs, steps, warmup, flush, stream, sampler=None):
     with ctx:
         wall0 = time.perf_counter()
         for k in range(steps):
-            flush.fill_(k & 0xff)
+            if flush_l2:
+                flush.fill_(k & 0xff)
             for i, lg in enumerate(legs):
                 evs[k][i][0].record(stream)
                 lg["conv"](lg["x"], lg["y"])
@@ -496,7 +498,7 @@ def measure(layers, args, dev, stream, flush, ws, pk, sampler=None):
         ms = sum(leg_ms[i]) / len(leg_ms[i])
         rf = leg_roofline(layer, t, lg["algo"], ms, pk)
         info.append({"name": layer.name, "dtype": layer.dtype, "algo": lg["algo"], "N": layer.N,
-                     "rate": layer.rate, "ms": ms, "t_kept_blocks": t,
+                     "rate": layer.rate, "ms": ms, "ms_median": statistics.median(leg_ms[i]), "t_kept_blocks": t,
                      "tflops": kept_flops(layer, t) / (ms * 1e-3) / 1e12,
                      "gbs": alg_bytes(layer, t) / (ms * 1e-3) / 1e9,
                      "roofline_frac": rf["frac"], "bound": rf["bound"]})
@@ -576,6 +578,10 @@ def main():
         lg["conv"].reuse_decoded = True
         lg["conv"]._args.clear()
 
+    # the same step without the L2 flush (the previous step's data warm in L2)
+    warm_ms, _ = time_legs(legs, min(args.steps, 1000), args.warmup, flush, stream, flush_l2=False)
+    warm_step_ms = max_over_ranks(sum(sum(m) for m in warm_ms) / len(warm_ms[0]), ws)
+
     e2e_ms, h2d, d2h = e2e_time(legs, dev, max(3, min(args.steps // 4, 200)), 2, flush, stream)
     e2e_ms = max_over_ranks(e2e_ms, ws)
 
@@ -599,6 +605,9 @@ def main():
             "decode_each_call": {"value": ws * flops_step / (dec_step_ms * 1e-3) / 1e12, "unit": "TFLOP/s",
                                  "ms_per_step": dec_step_ms,
                                  "algos": [lg["conv"].algo(lg["x"].shape) for lg in legs]},
+            "warm_l2": {"value": ws * flops_step / (warm_step_ms * 1e-3) / 1e12, "unit": "TFLOP/s",
+                        "ms_per_step": warm_step_ms,
+                        "legs_ms": [sum(m) / len(m) for m in warm_ms]},
             "e2e": {"value": ws * flops_step / (e2e_ms * 1e-3) / 1e12, "unit": "TFLOP/s",
                     "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "ms_per_step": e2e_ms},
             "gpu_launches": launches_per_step(legs) * args.steps,
