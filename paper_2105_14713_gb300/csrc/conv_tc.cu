@@ -130,11 +130,13 @@ struct TcLayout {
     static constexpr int kAccFit = (512 - kARing) / BN;
     static constexpr int kAcc = kAccFit > kAccMax ? kAccMax : kAccFit;
     static constexpr int kTmemCols = pow2_at_least(kAcc * BN + kARing);
-    // partial tiles (128 x BN fp32) the idle ring holds at a split tile's finish
+    // a stream-K tile has at most kMaxParts parts besides the finisher's (as
+    // many 128 x BN fp32 tiles as the stage ring's bytes), which bounds the
+    // additions in the finisher's epilogue
     static constexpr int kSlotBytes = kBM * BN * 4;
-    static constexpr int kRingSlots = kS * kStage / kSlotBytes;
+    static constexpr int kMaxParts = kS * kStage / kSlotBytes;
     static_assert(kS >= 2, "ring too small");
-    static_assert(kRingSlots >= 1, "ring cannot hold a partial tile");
+    static_assert(kMaxParts >= 1, "stream-K parts");
     static_assert(kAlloc <= kSmemMax, "shared memory");
     static_assert(kTmemCols <= 512, "tensor memory");
 };
@@ -213,15 +215,17 @@ __device__ __forceinline__ bool epi_all(bool ok)
 // Work schedule of one launch, the same in every role of every CTA.  Tiles
 // [0, dp_tiles) are whole tiles taken round-robin (CTA b: b, b+G, ...).  The
 // chunk iterations of the remaining sk_tiles tiles are cut into sk_ctas
-// contiguous ranges, one for each of CTAs 0 .. sk_ctas-1 (stream-K), and a
-// CTA walks its range from the end: first the start of one tile, then whole
-// tiles, last the end of another.  A tile cut between CTAs is finished by
-// the highest of them, which reaches it last: the others (lower CTAs, which
-// reached it first) each write their part to their own partial slot and
-// raise their flag; the finisher waits for those flags, copies the parts
-// into its idle shared-memory ring and adds them to its own accumulator in
-// CTA order, so the result does not depend on timing.  Waiting only on
-// lower CTAs, which were scheduled first, cannot deadlock.
+// contiguous ranges, one for each of CTAs 0 .. sk_ctas-1 (stream-K).  A CTA
+// runs its stream-K range before its whole tiles, walking it from the end:
+// first the start of one tile, then whole tiles, last the end of another.
+// A tile cut between CTAs is finished by the highest of them: the others
+// (lower CTAs, for which that tile's piece is the first segment they run)
+// each write their part to their own partial slot and raise their flag; the
+// finisher waits for those flags and adds the parts, read from L2, to its
+// own accumulator in CTA order, so the result does not depend on timing.
+// The finisher's wait and additions run in its epilogue warps while its MMA
+// warp goes on with the whole tiles.  Waiting only on lower CTAs, which
+// were scheduled first, cannot deadlock.
 //
 // Split mode (split_s > 0; plain GEMMs with a long K, e.g. the weight
 // gradient whose K is the pixels): item i = slice * n_tiles + tile covers
@@ -286,34 +290,25 @@ struct TcSegIter {
             return true;
         }
         sg.slot = -1;
-        if (i_dp < n_dp) {
-            sg.tile = b + i_dp * G;
-            sg.c0 = 0;
-            sg.c1 = C;
-            ++i_dp;
+        // the stream-K pieces first (so that a finisher's fixup overlaps the
+        // whole tiles' MMAs instead of trailing the kernel), from the range's
+        // end down: the piece a CTA contributes to a tile finished by a
+        // higher CTA is always the first segment it runs
+        if (e > s) {
+            const int t = static_cast<int>((e - 1) / C);
+            const int64_t t0 = static_cast<int64_t>(t) * C;
+            sg.tile = dp_tiles + t;
+            sg.c1 = static_cast<int>(e - t0);
+            sg.c0 = s > t0 ? static_cast<int>(s - t0) : 0;
+            e -= sg.c1 - sg.c0;
             return true;
         }
-        if (e <= s) return false;
-        const int t = static_cast<int>((e - 1) / C);
-        const int64_t t0 = static_cast<int64_t>(t) * C;
-        sg.tile = dp_tiles + t;
-        sg.c1 = static_cast<int>(e - t0);
-        sg.c0 = s > t0 ? static_cast<int>(s - t0) : 0;
-        e -= sg.c1 - sg.c0;
+        if (i_dp >= n_dp) return false;
+        sg.tile = b + i_dp * G;
+        sg.c0 = 0;
+        sg.c1 = C;
+        ++i_dp;
         return true;
-    }
-    // chunk iterations of this CTA
-    __device__ int64_t total() const
-    {
-        if (split_s > 0) {
-            int64_t n = 0;
-            for (int j = 0; j < n_dp; ++j) {
-                const int i = b + j * G, slice = i / n_tiles;
-                n += static_cast<int64_t>(slice + 1) * C / split_s - static_cast<int64_t>(slice) * C / split_s;
-            }
-            return n;
-        }
-        return static_cast<int64_t>(n_dp) * C + (e - s);
     }
 };
 
@@ -334,7 +329,6 @@ tc_conv_kernel(const ConvArgs a, const __grid_constant__ CUtensorMap tmap_x,
     const uint32_t bar_tfull = bar_empty + 8 * L::kS;
     const uint32_t bar_tempty = bar_tfull + 8 * kAccMax;
     const uint32_t bar_drain = bar_tempty + 8 * kAccMax;
-    const uint32_t bar_fix = bar_drain + 8;
     uint32_t *holder = reinterpret_cast<uint32_t *>(smem + L::kHolder);
     // the MMA waits on "split" (fp32: x_hi / x_lo in TMEM) or "full" (bf16)
     const uint32_t bar_ready = Tr::kSplit ? bar_split : bar_full;
@@ -351,7 +345,6 @@ tc_conv_kernel(const ConvArgs a, const __grid_constant__ CUtensorMap tmap_x,
             mbar_init(bar_tempty + 8 * b, 128);
         }
         mbar_init(bar_drain, 1);
-        mbar_init(bar_fix, 1);
         fence_mbar_init();
     }
     if (warp == kMmaWarp) {
@@ -808,9 +801,8 @@ tc_conv_kernel(const ConvArgs a, const __grid_constant__ CUtensorMap tmap_x,
                 if (leader) tc::st_release_gpu(sched.flags + blockIdx.x, 1);
                 continue;
             }
-            // The finisher (this split tile is this CTA's last segment, so the
-            // ring is idle): wait for the lower CTAs' flags, bring their parts
-            // into the ring, add them to the accumulator in CTA order.
+            // The finisher: wait for the lower CTAs' flags, then add their
+            // parts, read from L2, to the accumulator in CTA order.
             const int n_contrib = b_last - b_first;
             bool ok = true;
             if (leader) {
@@ -819,35 +811,30 @@ tc_conv_kernel(const ConvArgs a, const __grid_constant__ CUtensorMap tmap_x,
                     while (tc::ld_acquire_gpu(sched.flags + k) == 0)
                         if (clock64() - t0 > (1ll << 31)) { ok = false; break; }
                 }
-                if (ok) {
-                    tc::fence_proxy_async_global();
-                    tc::mbar_arrive_expect_tx(bar_fix, static_cast<uint32_t>(n_contrib) * L::kSlotBytes);
-                    for (int k = 0; k < n_contrib; ++k) {
-                        const unsigned char *src = reinterpret_cast<const unsigned char *>(
-                            sched.partials + static_cast<int64_t>(b_first + k) * kSlotF4 * 4);
-                        for (int off = 0; off < L::kSlotBytes; off += 16384)
-                            tc::bulk_load(base + k * L::kSlotBytes + off, src + off, 16384, bar_fix);
-                        sched.flags[b_first + k] = 0;   // ready for the next launch
-                    }
-                }
             }
             if (!epi_all(ok)) { abort_now(); break; }
-            if (!epi_all(mbar_wait(bar_fix, 0))) { abort_now(); break; }
             stage_bias();
+            const float4 *parts = reinterpret_cast<const float4 *>(sched.partials) +
+                                  static_cast<int64_t>(b_first) * kSlotF4;
             run_atoms([&](int at, uint32_t (&r)[kLd][32]) {
                 float f[kAtomCols];
 #pragma unroll
                 for (int e = 0; e < kAtomCols; ++e) f[e] = __uint_as_float(r[e / 32][e % 32]);
                 for (int k = 0; k < n_contrib; ++k) {
-                    const float4 *part = reinterpret_cast<const float4 *>(smem + k * L::kSlotBytes);
+                    const float4 *part = parts + static_cast<int64_t>(k) * kSlotF4;
+                    float4 v[kAtomCols / 4];
+#pragma unroll
+                    for (int v4 = 0; v4 < kAtomCols / 4; ++v4) v[v4] = __ldcg(part + (at * kAtomCols / 4 + v4) * kBM + row);
 #pragma unroll
                     for (int v4 = 0; v4 < kAtomCols / 4; ++v4) {
-                        const float4 v = part[(at * kAtomCols / 4 + v4) * kBM + row];
-                        f[4 * v4] += v.x; f[4 * v4 + 1] += v.y; f[4 * v4 + 2] += v.z; f[4 * v4 + 3] += v.w;
+                        f[4 * v4] += v[v4].x; f[4 * v4 + 1] += v[v4].y; f[4 * v4 + 2] += v[v4].z; f[4 * v4 + 3] += v[v4].w;
                     }
                 }
                 emit_atom(at, f);
             });
+            tc::named_bar(1, 128);                   // every part has been read
+            if (leader)
+                for (int k = b_first; k < b_last; ++k) sched.flags[k] = 0;   // ready for the next launch
         }
         if (lane == 0) tc::bulk_wait0();
       };
@@ -1075,10 +1062,8 @@ cudaError_t launch_bn(const ConvArgs &a, const typename Tr::T *W, const typename
     // are fewer tiles than SMs), with room for the partial slots: whole
     // rounds first, then the remaining tiles' chunk iterations spread over
     // the CTAs.  Each CTA gets at least kMinSplitIters chunk iterations and
-    // at least C / R of them, R = the partial tiles the finisher's ring
-    // holds, so that a split tile has at most R parts besides the
-    // finisher's.  (On the ResNet-50 3x3 128->128 fp32 layer, 392 tiles on
-    // 152 SMs, the last CTA now ends at 50 us instead of 57.)
+    // at least C / kMaxParts of them, so that a split tile has at most
+    // kMaxParts parts besides the finisher's.
     const int G = sms < kPlanCTAs ? sms : kPlanCTAs;
     if (split_s > 0) {
         if (split_s > sc.n_chunks || !split_partials) return cudaErrorInvalidValue;   // every item non-empty
@@ -1089,7 +1074,7 @@ cudaError_t launch_bn(const ConvArgs &a, const typename Tr::T *W, const typename
     } else if (sk_space && sc.n_tiles % G && sc.n_chunks >= sk_min_chunks(Tr::kSplit)) {
         const int dp = (sc.n_tiles / G) * G, skt = sc.n_tiles - dp;
         const int64_t iters = static_cast<int64_t>(skt) * sc.n_chunks;
-        int need = (sc.n_chunks + L::kRingSlots - 1) / L::kRingSlots;
+        int need = (sc.n_chunks + L::kMaxParts - 1) / L::kMaxParts;
         if (need < kMinSplitIters) need = kMinSplitIters;
         const int gs = static_cast<int>(iters / need < G ? iters / need : G);
         if (gs > skt) {
