@@ -492,6 +492,17 @@ onexn_status onexn_conv_fwd_noalloc(const onexn_conv_desc *desc, const int32_t *
  */
 onexn_status onexn_device_status(int clear, int *status);
 
+/*
+ * onexn_selftest_timeout -- check the timeout path without a faulted GPU:
+ * launches on `stream` a one-thread kernel that waits, with the same bounded
+ * wait the library's kernels use, on an mbarrier that nothing signals.  The
+ * wait runs out after about one second (2^31 SM cycles) and the kernel sets
+ * the status word, so a later onexn_device_status reports ONEXN_ETIMEOUT
+ * (clear it there); the context stays usable.  Asynchronous; returns ECUDA
+ * only if the launch fails.
+ */
+onexn_status onexn_selftest_timeout(void *stream);
+
 #ifdef __cplusplus
 }
 #endif

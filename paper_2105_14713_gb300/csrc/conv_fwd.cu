@@ -373,6 +373,34 @@ extern "C" onexn_status onexn_conv_fwd(const onexn_conv_desc *desc, const int32_
                              stream);
 }
 
+namespace onexn {
+
+// Waits on a fresh mbarrier that nothing signals: the bounded wait every
+// library kernel uses runs out (about 2^31 SM cycles) and the kernel reports
+// it in the status word, as a kernel whose pipeline stalled would.
+__global__ void selftest_wait_kernel(unsigned int *status)
+{
+    __shared__ __align__(8) unsigned long long bar;
+    const uint32_t b = static_cast<uint32_t>(__cvta_generic_to_shared(&bar));
+    mbar_init(b, 1);
+    fence_mbar_init();
+    if (!mbar_wait(b, 0)) atomicOr(status, kStatusTimeout);
+    asm volatile("mbarrier.inval.shared::cta.b64 [%0];\n" ::"r"(b) : "memory");
+}
+
+}  // namespace onexn
+
+extern "C" onexn_status onexn_selftest_timeout(void *stream)
+{
+    onexn::clear_error();
+    unsigned int *p = nullptr;
+    cudaError_t e = onexn::device_status_ptr(&p);
+    if (e != cudaSuccess) return fail(ONEXN_ECUDA, "selftest_timeout: status word: %s", cudaGetErrorString(e));
+    onexn::selftest_wait_kernel<<<1, 1, 0, static_cast<cudaStream_t>(stream)>>>(p);
+    e = cudaGetLastError();
+    return e == cudaSuccess ? ONEXN_OK : fail(ONEXN_ECUDA, "selftest_timeout: %s", cudaGetErrorString(e));
+}
+
 extern "C" onexn_status onexn_device_status(int clear, int *status)
 {
     onexn::clear_error();

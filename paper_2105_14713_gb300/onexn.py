@@ -63,6 +63,7 @@ SIGNATURES = {
     "onexn_conv_algo": ([ctypes.POINTER(ConvDesc), _I32, _I64, _I32, _U32, ctypes.c_size_t, _P],
                         _I32),
     "onexn_device_status": ([_I32, _P], _I32),
+    "onexn_selftest_timeout": ([_P], _I32),
     "onexn_conv_fwd_noalloc": ([ctypes.POINTER(ConvDesc), _P, _P, _P, _I32, _I64, _P, _P, _P, _I32,
                                 _U32, _P], _I32),
     "onexn_conv_fwd_host": ([ctypes.POINTER(ConvDesc), _P, _P, _P, _I32, _I64, _P, _P, _P, _I32,
@@ -293,6 +294,14 @@ def onexn_device_status(clear: bool = True) -> int:
     st = ctypes.c_int(0)
     _check(lib.onexn_device_status(int(bool(clear)), ctypes.byref(st)))
     return st.value
+
+
+def onexn_selftest_timeout(stream=None) -> None:
+    """Launch the bounded-wait self-test kernel (about one second on the
+    GPU); afterwards onexn_device_status() reports ONEXN_ETIMEOUT."""
+    import torch
+    st = torch.cuda.current_stream() if stream is None else stream
+    _check(lib.onexn_selftest_timeout(ctypes.c_void_p(st.cuda_stream)))
 
 
 def _cuda_stream(t, stream):
