@@ -84,7 +84,10 @@ typedef enum { ONEXN_GRAN_TAP = 0, ONEXN_GRAN_KERNEL = 1 } onexn_granularity;
 #define ONEXN_ALGO_MASK (0xFu << ONEXN_ALGO_SHIFT)
 #define ONEXN_ALGO_AUTO (0u << ONEXN_ALGO_SHIFT)
 #define ONEXN_ALGO_FMA (1u << ONEXN_ALGO_SHIFT)   /* CUDA-core FFMA, any N, fp32/bf16 */
-#define ONEXN_ALGO_MMA (2u << ONEXN_ALGO_SHIFT)   /* bf16 gathered tensor-core kernel */
+#define ONEXN_ALGO_MMA (2u << ONEXN_ALGO_SHIFT)   /* bf16 sparse tensor-core kernel: each group's
+                                                     kept activations gathered into tensor memory,
+                                                     one MMA per 16 kept blocks (Eq. 7); N in
+                                                     {16, 32, 64, 128}; workspace: its plan */
 #define ONEXN_ALGO_TC (3u << ONEXN_ALGO_SHIFT)    /* tcgen05 GEMM on the decoded mask: bf16,
                                                      or fp32 as three tf32 products */
 
@@ -251,10 +254,14 @@ onexn_status onexn_conv_out_shape(const onexn_conv_desc *desc, int *Ho, int *Wo)
  *           | ONEXN_REUSE_DECODE (AUTO hint: the decode will be reused).
  *   workspace, workspace_bytes
  *           nullable DEVICE scratch owned by the caller, 256-byte aligned.
- *           Some kernel families need it (onexn_conv_workspace_size); the
- *           call overwrites it, so calls that run concurrently need
- *           separate workspaces.  AUTO only picks a family whose minimum
- *           workspace fits in workspace_bytes.
+ *           Some kernel families need it (onexn_conv_workspace_size): the
+ *           tensor-core GEMM (ALGO_TC) decodes the weights into it; the
+ *           sparse tensor-core kernel (ALGO_MMA) writes its plan there (per
+ *           64-channel chunk and tile of 128/N groups: the groups' kept
+ *           entries, counts and channels, 560 bytes).  The call overwrites
+ *           it, so calls that run concurrently need separate workspaces.
+ *           AUTO only picks a family whose minimum workspace fits in
+ *           workspace_bytes.
  *   stream  cudaStream_t to launch on (NULL = legacy default stream).
  * Asynchronous: returns after the launch; errors of the launch itself are
  * returned as ECUDA.  No allocation, no synchronisation, no host read of

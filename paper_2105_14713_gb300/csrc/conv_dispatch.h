@@ -10,8 +10,11 @@
 namespace onexn {
 
 cudaError_t launch_fma(const ConvArgs &a, int dtype, cudaStream_t st);
-cudaError_t launch_mma(const ConvArgs &a, cudaStream_t st);
+// sparse tensor-core family (bf16): a boundary table of the kept lists in
+// the workspace (mma_workspace_bytes), then the kernel
+cudaError_t launch_mma(const ConvArgs &a, void *workspace, size_t ws_bytes, cudaStream_t st);
 bool mma_supports(const ConvArgs &a);
+size_t mma_workspace_bytes(const ConvArgs &a);
 // tensor-core family: decode of (P, I, D) into the workspace, then the GEMM
 // (which splits its last round of tiles across CTAs when ws_bytes has room
 // for tc_workspace_bytes, else needs tc_workspace_min)

@@ -125,12 +125,16 @@ onexn_status check_pointers(const int32_t *P, const int32_t *I, const void *D, c
 // Workspace a family needs for these arguments.
 size_t workspace_for(unsigned algo, const onexn::ConvArgs &a, int dtype)
 {
-    return algo == ONEXN_ALGO_TC ? onexn::tc_workspace_bytes(a, dtype) : 0;
+    if (algo == ONEXN_ALGO_TC) return onexn::tc_workspace_bytes(a, dtype);
+    if (algo == ONEXN_ALGO_MMA) return onexn::mma_workspace_bytes(a);
+    return 0;
 }
 
 size_t workspace_min_for(unsigned algo, const onexn::ConvArgs &a, int dtype)
 {
-    return algo == ONEXN_ALGO_TC ? onexn::tc_workspace_min(a, dtype) : 0;
+    if (algo == ONEXN_ALGO_TC) return onexn::tc_workspace_min(a, dtype);
+    if (algo == ONEXN_ALGO_MMA) return onexn::mma_workspace_bytes(a);
+    return 0;
 }
 
 // Can the family run this case at all (dtype, shape)?
@@ -212,7 +216,7 @@ cudaError_t launch(unsigned algo, const ConvArgs &a, int dtype, void *workspace,
                    cudaStream_t st)
 {
     if (algo == ONEXN_ALGO_FMA) return launch_fma(a, dtype, st);
-    if (algo == ONEXN_ALGO_MMA) return launch_mma(a, st);
+    if (algo == ONEXN_ALGO_MMA) return launch_mma(a, workspace, ws_bytes, st);
     return launch_tc(a, dtype, workspace, ws_bytes, st);
 }
 

@@ -50,6 +50,7 @@
 #include "conv_dispatch.h"
 #include "onexn_internal.h"
 #include "tc_ptx.cuh"
+#include "tc_maps.h"
 
 #include <cuda.h>
 #include <cudaTypedefs.h>
@@ -967,6 +968,50 @@ bool tmap_2d(CUtensorMap *m, CUtensorMapDataType type, int elem, const void *ptr
     });
 }
 
+}  // namespace
+
+// A 1x1, stride-1, unpadded layer reads x as a [B*H*W][C] matrix; any other
+// layer reads x[B][H][W][C] through an im2col view.
+int tc_x_tiled(const ConvArgs &a)
+{
+    return (a.KH == 1 && a.KW == 1 && a.sh == 1 && a.sw == 1 && a.ph == 0 && a.pw == 0) ? 1 : 0;
+}
+
+// Tensor map of the A operand: boxes of 128 output pixels x bk channels
+// (128 bytes) in the 128-byte-swizzled K-major layout; im2col loads walk the
+// output pixels across rows and images and read zeros in the padding.
+bool tc_x_tmap(const ConvArgs &a, CUtensorMapDataType type, int elem, int bk, CUtensorMap *tmap_x)
+{
+    if (tc_x_tiled(a)) return tmap_2d(tmap_x, type, elem, a.x, static_cast<uint64_t>(a.B) * a.H * a.W, a.C, kBM);
+    auto enc_i = encode_im2col_fn();
+    if (!enc_i) return false;
+    const cuuint64_t dims[4] = {static_cast<cuuint64_t>(a.C), static_cast<cuuint64_t>(a.W),
+                                static_cast<cuuint64_t>(a.H), static_cast<cuuint64_t>(a.B)};
+    const cuuint64_t strides[3] = {static_cast<cuuint64_t>(a.C) * elem,
+                                   static_cast<cuuint64_t>(a.C) * elem * a.W,
+                                   static_cast<cuuint64_t>(a.C) * elem * a.W * a.H};
+    int lower[2], upper[2];
+    im2col_corners(a, lower, upper);
+    const cuuint32_t estr[4] = {1, static_cast<cuuint32_t>(a.sw), static_cast<cuuint32_t>(a.sh), 1};
+    TmapKey k;
+    std::memset(&k, 0, sizeof k);
+    k.kind = 1;
+    k.type = static_cast<uint32_t>(type);
+    k.ptr = reinterpret_cast<uint64_t>(a.x);
+    for (int i = 0; i < 4; ++i) k.dims[i] = dims[i];
+    for (int i = 0; i < 3; ++i) k.strides[i] = strides[i];
+    for (int i = 0; i < 2; ++i) { k.lower[i] = lower[i]; k.upper[i] = upper[i]; }
+    k.box[0] = static_cast<uint32_t>(bk); k.box[1] = kBM;
+    for (int i = 0; i < 4; ++i) k.estr[i] = estr[i];
+    return tmap_cached(k, tmap_x, [&](CUtensorMap *mm) {
+        return enc_i(mm, type, 4, const_cast<void *>(a.x), dims, strides, lower, upper, bk, kBM, estr,
+                     CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                     CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+    });
+}
+
+namespace {
+
 template <typename Tr, int BN>
 cudaError_t launch_bn(const ConvArgs &a, const typename Tr::T *W, const typename Tr::T *W_lo, void *sk_space,
                       cudaStream_t st, int split_s = 0, float *split_partials = nullptr)
@@ -977,42 +1022,14 @@ cudaError_t launch_bn(const ConvArgs &a, const typename Tr::T *W, const typename
     const int K = a.KH * a.KW * a.C;
     auto enc_i = encode_im2col_fn();
     if (!enc_i) return cudaErrorNotSupported;
-    // A: a 1x1, stride-1, unpadded layer reads x as a [B*H*W][C] matrix; any
-    // other layer reads x[B][H][W][C] as an im2col view (128 pixels x 128
-    // bytes of channels per load).
-    const int a_tiled = (a.KH == 1 && a.KW == 1 && a.sh == 1 && a.sw == 1 && a.ph == 0 && a.pw == 0);
+    // A: the activations' tensor map (none for the fused depthwise form,
+    // whose A the split warps compute)
+    const int a_tiled = tc_x_tiled(a);
     CUtensorMap tmap_x;
     if (a.dw_x) {
-        // A is computed in the kernel (fused depthwise): x has no tensor map
         std::memset(&tmap_x, 0, sizeof tmap_x);
-    } else if (a_tiled) {
-        if (!tmap_2d(&tmap_x, Tr::kTmap, elem, a.x, static_cast<uint64_t>(a.B) * a.H * a.W, a.C, kBM))
-            return cudaErrorInvalidValue;
-    } else {
-        const cuuint64_t dims[4] = {static_cast<cuuint64_t>(a.C), static_cast<cuuint64_t>(a.W),
-                                    static_cast<cuuint64_t>(a.H), static_cast<cuuint64_t>(a.B)};
-        const cuuint64_t strides[3] = {static_cast<cuuint64_t>(a.C) * elem,
-                                       static_cast<cuuint64_t>(a.C) * elem * a.W,
-                                       static_cast<cuuint64_t>(a.C) * elem * a.W * a.H};
-        int lower[2], upper[2];
-        im2col_corners(a, lower, upper);
-        const cuuint32_t estr[4] = {1, static_cast<cuuint32_t>(a.sw), static_cast<cuuint32_t>(a.sh), 1};
-        TmapKey k;
-        std::memset(&k, 0, sizeof k);
-        k.kind = 1;
-        k.type = static_cast<uint32_t>(Tr::kTmap);
-        k.ptr = reinterpret_cast<uint64_t>(a.x);
-        for (int i = 0; i < 4; ++i) k.dims[i] = dims[i];
-        for (int i = 0; i < 3; ++i) k.strides[i] = strides[i];
-        for (int i = 0; i < 2; ++i) { k.lower[i] = lower[i]; k.upper[i] = upper[i]; }
-        k.box[0] = Tr::kBK; k.box[1] = kBM;
-        for (int i = 0; i < 4; ++i) k.estr[i] = estr[i];
-        if (!tmap_cached(k, &tmap_x, [&](CUtensorMap *mm) {
-                return enc_i(mm, Tr::kTmap, 4, const_cast<void *>(a.x), dims, strides, lower, upper, Tr::kBK, kBM,
-                             estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
-                             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
-            }))
-            return cudaErrorInvalidValue;
+    } else if (!tc_x_tmap(a, Tr::kTmap, elem, Tr::kBK, &tmap_x)) {
+        return cudaErrorInvalidValue;
     }
     // B: W[C_out][K] (and W_lo), box 128 bytes of K x BN rows.  y:
     // [P_pix][C_out], stored in boxes of 128 bytes of columns x 32 rows, one

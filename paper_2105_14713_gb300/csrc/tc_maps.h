@@ -1,0 +1,17 @@
+// TMA descriptors of the activation operand shared by the tensor-core
+// kernels (conv_tc.cu, conv_mma.cu).
+#pragma once
+
+#include <cuda.h>
+
+#include "conv_common.cuh"
+
+namespace onexn {
+
+// 1 when x is read as a plain [B*H*W][C] matrix (1x1, stride 1, no padding).
+int tc_x_tiled(const ConvArgs &a);
+// Encode (or fetch from the cache) the tensor map of x: boxes of 128 output
+// pixels x bk channels (128 bytes), 128-byte swizzle; false on failure.
+bool tc_x_tmap(const ConvArgs &a, CUtensorMapDataType type, int elem, int bk, CUtensorMap *tmap_x);
+
+}  // namespace onexn
