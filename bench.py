@@ -1,12 +1,12 @@
 """Benchmark of the 1xN-pruned convolution forward pass on GB300.
 
-Workloads (--config, default 2; seeded synthetic inputs resident in HBM; L2
+Workloads (--config, default 4; seeded synthetic inputs resident in HBM; L2
 flushed with a 256 MB write before every step, outside the timed events):
   1  1x1 conv 64 -> 64, 1x28x28, fp32, N=4, 50%
   2  ResNet-50 stage-2 3x3 conv, 64x28x28, 128 -> 128, N=8, 50%: one fp32 leg
-     and one bf16-input / fp32-accumulate leg per step           (default)
+     and one bf16-input / fp32-accumulate leg per step
   3  MobileNet-V2 expand/project 1x1 stack (34 layers), 128x224x224 input, fp32, N=4, 50%
-  4  ResNet-50 bottleneck stack (52 convs), 256x224x224 input, bf16, N=16, 70%
+  4  ResNet-50 bottleneck stack (52 convs), 256x224x224 input, bf16, N=16, 70%   (default)
   5  3x3 512 -> 512 on 128x14x14: sweep N in {1..32} x rate in {0..0.9} x {fp32, bf16}
   6  fully connected 1280 -> 1000 as a 1x1 conv on 256 1x1 inputs, fp32 + bf16, N=4, 50%
   7  MobileNet-V2's 17 inverted-residual blocks at batch 1 (224x224 input), fp32, N=4, 50%:
@@ -14,15 +14,21 @@ flushed with a 256 MB write before every step, outside the timed events):
   8  fine-tuning step of the config-2 layer with the mask fixed: forward, input gradient,
      kept-weight and bias gradients, SGD update of D; fp32 leg + bf16 leg
 
-A "step" is one pass over every layer (leg) of the workload.  Prints one JSON
-line.  Metric: effective TFLOP/s = 2 * pixels * t * N / time summed over the
+A "step" is one pass over every layer (leg) of the workload, or, for
+workloads whose pass is short, several passes back to back so that a step
+lasts about 50 ms (the count is `passes_per_step` in the JSON's config;
+between two calls of a layer the other layers move more data than L2
+holds).  Prints one JSON line.  Metric: effective TFLOP/s = 2 * pixels * t * N / time summed over the
 legs (t = kept blocks), plus the roofline fraction of the dominant kernel and
 the speedup over the library's own dense path (rate 0, N = C_out).
 
   python bench.py [--config C] [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+  python bench.py --peaks
 
 --impl reference times the CPU oracle (fp64, plain C) on the host cores on a
-bounded pixel sample of the same workload.
+bounded pixel sample of the same workload.  --peaks measures the GPU's fp32
+FFMA rate and the tcgen05.mma issue rate by block width, issuing warps and
+A-operand source with the library's measurement kernels.
 """
 from __future__ import annotations
 
@@ -103,7 +109,29 @@ def alg_bytes(layer, t):
     return x + y + t * layer.N * es + t * 4 + (layer.C_out // layer.N + 1) * 4
 
 
-def peaks():
+def measure_ffma_tflops(dev, reps=5):
+    """fp32 FFMA rate of this GPU (TFLOP/s), measured with the library's
+    FFMA-chain kernel (onexn_probe_ffma): 16 flops per thread per iteration,
+    8 blocks of 256 threads per SM; best of `reps` CUDA-event timings."""
+    from paper_2105_14713_gb300 import onexn as ox
+    sms = torch.cuda.get_device_properties(dev).multi_processor_count
+    blocks, iters = 8 * sms, 8192
+    sink = torch.zeros(blocks, dtype=torch.float32, device=dev)
+    ox.onexn_probe_ffma(blocks, 64, sink)
+    torch.cuda.synchronize()
+    best = None
+    for _ in range(reps):
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        ox.onexn_probe_ffma(blocks, iters, sink)
+        e1.record()
+        torch.cuda.synchronize()
+        ms = e0.elapsed_time(e1)
+        best = ms if best is None else min(best, ms)
+    return 16.0 * iters * 256 * blocks / (best * 1e-3) / 1e12
+
+
+def peaks(dev=None):
     path = os.path.join(ROOT, "MEASURED_PEAKS.json")
     src = "measured"
     try:
@@ -114,10 +142,16 @@ def peaks():
         sm_max = float(pk.get("sm_max_mhz", 2070.0))
     except (OSError, KeyError, ValueError):
         hbm, bf16, bf16_s, sm_max, src = 6800.0, 1900.0, 1700.0, 2070.0, "fallback"
-    # FFMA peak: 152 SMs x 128 fp32 lanes x 2 flop x max SM clock.
-    fp32 = SM_COUNT_GB300 * FP32_LANES_PER_SM * 2 * sm_max * 1e6 / 1e12
+    # FFMA peak: measured on this GPU when one is given (the
+    # measured file has no FFMA figure); else 152 SMs x 128 fp32
+    # lanes x 2 flop x max SM clock
+    if dev is not None:
+        fp32, fp32_src = measure_ffma_tflops(dev), "measured (onexn_probe_ffma, FFMA chains on every SM)"
+    else:
+        fp32 = SM_COUNT_GB300 * FP32_LANES_PER_SM * 2 * sm_max * 1e6 / 1e12
+        fp32_src = "derived: 152 SMs x 128 lanes x 2 x max SM clock"
     return {"hbm_gbs": hbm, "bf16_tflops": bf16, "bf16_tflops_sustained": bf16_s,
-            "fp32_ffma_tflops": fp32, "sm_max_mhz": sm_max, "source": src}
+            "fp32_ffma_tflops": fp32, "fp32_ffma_source": fp32_src, "sm_max_mhz": sm_max, "source": src}
 
 
 # tf32 / bf16 dense tensor rates, nominal (1.1 / 2.25 PFLOP/s per GB300)
@@ -133,8 +167,7 @@ def leg_roofline(layer, t, algo, ms, pk):
     fl, by = kept_flops(layer, t), alg_bytes(layer, t)
     issued = None
     if algo == "fma":
-        pipe, pipe_name, pipe_src = pk["fp32_ffma_tflops"], "alu", \
-            "FFMA: 152 SMs x 128 lanes x 2 x %.0f MHz (derived)" % pk["sm_max_mhz"]
+        pipe, pipe_name, pipe_src = pk["fp32_ffma_tflops"], "alu", "FFMA " + pk.get("fp32_ffma_source", "")
     elif layer.dtype == "f32":
         pipe, pipe_name = pk["bf16_tflops"] * TF32_PER_BF16, "tensor"
         pipe_src = f"tf32 = {pk['source']} bf16 tensor (burst) x nominal tf32/bf16 1.1/2.25"
@@ -393,15 +426,17 @@ def build_legs(layers, dev):
     return legs
 
 
-def time_legs(legs, steps, warmup, flush, stream, sampler=None, flush_l2=True):
-    """Per-leg CUDA-event times (ms) of `steps` steps, L2 flushed before each
-    (flush_l2=False: back to back, the inputs left in L2 by the step before)."""
+def time_legs(legs, steps, warmup, flush, stream, sampler=None, flush_l2=True, passes=1):
+    """Per-leg CUDA-event times (ms) of `steps` steps of `passes` passes over
+    the legs each (a leg's time in a step sums its calls), L2 flushed before
+    each step (flush_l2=False: back to back, the inputs left in L2 by the step
+    before)."""
     for _ in range(warmup):
         flush.fill_(1)
         for lg in legs:
             lg["conv"](lg["x"], lg["y"])
     torch.cuda.synchronize()
-    evs = [[[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in legs]
+    evs = [[[[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in range(passes)] for _ in legs]
            for _ in range(steps)]
     ctx = sampler if sampler is not None else _Null()
     with ctx:
@@ -409,14 +444,35 @@ def time_legs(legs, steps, warmup, flush, stream, sampler=None, flush_l2=True):
         for k in range(steps):
             if flush_l2:
                 flush.fill_(k & 0xff)
-            for i, lg in enumerate(legs):
-                evs[k][i][0].record(stream)
-                lg["conv"](lg["x"], lg["y"])
-                evs[k][i][1].record(stream)
+            for r in range(passes):
+                for i, lg in enumerate(legs):
+                    evs[k][i][r][0].record(stream)
+                    lg["conv"](lg["x"], lg["y"])
+                    evs[k][i][r][1].record(stream)
         torch.cuda.synchronize()
         wall = time.perf_counter() - wall0
-    return [[evs[k][i][0].elapsed_time(evs[k][i][1]) for k in range(steps)]
+    return [[sum(evs[k][i][r][0].elapsed_time(evs[k][i][r][1]) for r in range(passes)) for k in range(steps)]
             for i in range(len(legs))], wall
+
+
+STEP_TARGET_MS = 50.0
+
+
+def passes_for(legs, flush, stream):
+    """Passes over the legs per step so that a step lasts about
+    STEP_TARGET_MS (one pass for workloads that are already that long)."""
+    for _ in range(2):
+        flush.fill_(1)
+        for lg in legs:
+            lg["conv"](lg["x"], lg["y"])
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    flush.fill_(2)
+    e0.record(stream)
+    for lg in legs:
+        lg["conv"](lg["x"], lg["y"])
+    e1.record(stream)
+    torch.cuda.synchronize()
+    return max(1, int(STEP_TARGET_MS / max(e0.elapsed_time(e1), 1e-3) + 0.5))
 
 
 class _Null:
@@ -480,42 +536,47 @@ def e2e_time(legs, dev, steps, warmup, flush, stream):
     return sum(ts) / len(ts), h2d, d2h
 
 
-def launches_per_step(legs):
-    # one kernel per leg: fma, or the tc GEMM (its weights were decoded on
-    # the first, warm-up call and stay resident)
-    return len(legs)
+def launches_per_step(legs, passes=1):
+    # one kernel per leg and pass: fma, or the tc GEMM (its weights were
+    # decoded on the first, warm-up call and stay resident)
+    return len(legs) * passes
 
 
-def measure(layers, args, dev, stream, flush, ws, pk, sampler=None):
+def measure(layers, args, dev, stream, flush, ws, pk, sampler=None, passes=None):
     legs = build_legs(layers, dev)
-    leg_ms, wall = time_legs(legs, args.steps, args.warmup, flush, stream, sampler)
+    if passes is None:
+        passes = max_over_ranks(passes_for(legs, flush, stream), ws) if getattr(args, "auto_passes", False) else 1
+    passes = int(passes)
+    leg_ms, wall = time_legs(legs, args.steps, args.warmup, flush, stream, sampler, passes=passes)
     step_ms = sum(sum(m) for m in leg_ms) / args.steps
     step_ms_max = max_over_ranks(step_ms, ws)
-    flops_step = sum(kept_flops(lg["layer"], lg["conv"].t) for lg in legs)
+    flops_step = passes * sum(kept_flops(lg["layer"], lg["conv"].t) for lg in legs)
     info = []
     for i, lg in enumerate(legs):
         layer, t = lg["layer"], lg["conv"].t
-        ms = sum(leg_ms[i]) / len(leg_ms[i])
+        ms = sum(leg_ms[i]) / len(leg_ms[i]) / passes
         rf = leg_roofline(layer, t, lg["algo"], ms, pk)
         info.append({"name": layer.name, "dtype": layer.dtype, "algo": lg["algo"], "N": layer.N,
                      "rate": layer.rate, "ms": ms, "ms_median": statistics.median(leg_ms[i]), "t_kept_blocks": t,
                      "tflops": kept_flops(layer, t) / (ms * 1e-3) / 1e12,
                      "gbs": alg_bytes(layer, t) / (ms * 1e-3) / 1e9,
                      "roofline_frac": rf["frac"], "bound": rf["bound"]})
-    return legs, leg_ms, step_ms_max, flops_step, info, wall
+    return legs, leg_ms, step_ms_max, flops_step, info, wall, passes
 
 
 def main():
     ap = argparse.ArgumentParser()
-    ap.add_argument("--config", type=int, default=2, choices=[1, 2, 3, 4, 5, 6, 7, 8])
+    ap.add_argument("--config", type=int, default=4, choices=[1, 2, 3, 4, 5, 6, 7, 8])
     ap.add_argument("--gpus", type=int, default=1)
-    # default: a timed region of ~1 s on the default workload, so that the
-    # clock samples (every 50 ms) fall inside it
-    ap.add_argument("--steps", type=int, default=5000)
+    # default: 20 steps of ~50 ms (several passes over a short workload), a
+    # timed region of ~1 s in which the clock samples (every 50 ms) fall
+    ap.add_argument("--steps", type=int, default=20)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--peaks", action="store_true")
     args = ap.parse_args()
+    args.auto_passes = True
     args.warmup = max(args.warmup, 3)
     rank, local, ws = dist_setup()
     if args.impl == "reference":
@@ -529,7 +590,10 @@ def main():
     dev = torch.device("cuda", local)
     stream = torch.cuda.current_stream(dev)
     flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=dev)
-    pk = peaks()
+    if args.peaks:
+        run_peaks(dev, rank)
+        return
+    pk = peaks(dev)
 
     if args.config == 5:
         run_sweep(args, dev, stream, flush, ws, rank, pk)
@@ -545,7 +609,7 @@ def main():
     sampler = ClockSampler(local)
     barrier(ws)
     torch.cuda.synchronize()
-    legs, leg_ms, step_ms_max, flops_step, info, wall = measure(
+    legs, leg_ms, step_ms_max, flops_step, info, wall, passes = measure(
         layers, args, dev, stream, flush, ws, pk, sampler)
     barrier(ws)
     value = ws * flops_step / (step_ms_max * 1e-3) / 1e12
@@ -572,18 +636,19 @@ def main():
     for lg in legs:
         lg["conv"].reuse_decoded = False
         lg["conv"]._args.clear()
-    dec_ms, _ = time_legs(legs, min(args.steps, 1000), args.warmup, flush, stream)
+    dec_ms, _ = time_legs(legs, min(args.steps, 1000), args.warmup, flush, stream, passes=passes)
     dec_step_ms = max_over_ranks(sum(sum(m) for m in dec_ms) / len(dec_ms[0]), ws)
     for lg in legs:
         lg["conv"].reuse_decoded = True
         lg["conv"]._args.clear()
 
     # the same step without the L2 flush (the previous step's data warm in L2)
-    warm_ms, _ = time_legs(legs, min(args.steps, 1000), args.warmup, flush, stream, flush_l2=False)
+    warm_ms, _ = time_legs(legs, min(args.steps, 1000), args.warmup, flush, stream, flush_l2=False, passes=passes)
     warm_step_ms = max_over_ranks(sum(sum(m) for m in warm_ms) / len(warm_ms[0]), ws)
 
     e2e_ms, h2d, d2h = e2e_time(legs, dev, max(3, min(args.steps // 4, 200)), 2, flush, stream)
     e2e_ms = max_over_ranks(e2e_ms, ws)
+    flops_pass = flops_step / passes
 
     cpu = None
     if rank == 0 and ws == 1 and not args.no_cpu_baseline:
@@ -596,7 +661,7 @@ def main():
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
             "dtype": "+".join(sorted({l.dtype for l in layers})),
             "data": "synthetic (seeded Kaiming-normal or N(0,0.05) weights, ReLU(N(0,1)) activations)",
-            "config": config_json(args.config, layers),
+            "config": dict(config_json(args.config, layers), passes_per_step=passes),
             "roofline": roof,
             "legs": info,
             "speedup_vs_dense": speedup,
@@ -607,10 +672,11 @@ def main():
                                  "algos": [lg["conv"].algo(lg["x"].shape) for lg in legs]},
             "warm_l2": {"value": ws * flops_step / (warm_step_ms * 1e-3) / 1e12, "unit": "TFLOP/s",
                         "ms_per_step": warm_step_ms,
-                        "legs_ms": [sum(m) / len(m) for m in warm_ms]},
-            "e2e": {"value": ws * flops_step / (e2e_ms * 1e-3) / 1e12, "unit": "TFLOP/s",
-                    "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "ms_per_step": e2e_ms},
-            "gpu_launches": launches_per_step(legs) * args.steps,
+                        "legs_ms": [sum(m) / len(m) / passes for m in warm_ms]},
+            "e2e": {"value": ws * flops_pass / (e2e_ms * 1e-3) / 1e12, "unit": "TFLOP/s",
+                    "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "ms_per_step": e2e_ms,
+                    "step": "one pass over the legs from pinned host inputs to pinned host outputs"},
+            "gpu_launches": launches_per_step(legs, passes) * args.steps,
             "clocks": clocks,
             "wall_s_timed_region": wall,
             "peaks": pk,
@@ -620,6 +686,37 @@ def main():
     if ws > 1:
         import torch.distributed as dist
         dist.destroy_process_group()
+
+
+def run_peaks(dev, rank):
+    """--peaks: the fp32 FFMA rate, and the tcgen05.mma issue rate of one
+    SM's tensor core by block width N, number of issuing warps and A-operand
+    source (tensor memory or shared memory), with the library's measurement
+    kernels (onexn_probe_ffma, onexn_probe_mma_issue), CUDA-event timed."""
+    from paper_2105_14713_gb300 import onexn as ox
+    sms = torch.cuda.get_device_properties(dev).multi_processor_count
+    ffma = measure_ffma_tflops(dev)
+    rows = []
+    iters = 20000
+    for a_tmem in (True, False):
+        for N in (16, 32):
+            for issuers in (1, 2, 4, 6, 8):
+                ox.onexn_probe_mma_issue(N, issuers, a_tmem, 16)
+                torch.cuda.synchronize()
+                e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                e0.record()
+                ox.onexn_probe_mma_issue(N, issuers, a_tmem, iters)
+                e1.record()
+                torch.cuda.synchronize()
+                ms = e0.elapsed_time(e1)
+                flops = 2.0 * 128 * N * 16 * 4 * iters * issuers * sms
+                rows.append({"A": "tmem" if a_tmem else "smem", "N": N, "issuers": issuers,
+                             "tflops": flops / (ms * 1e-3) / 1e12,
+                             "ns_per_mma_per_sm": ms * 1e6 / (4 * iters * issuers)})
+    status = ox.onexn_device_status(clear=True)
+    if rank == 0:
+        print(json.dumps({"fp32_ffma_tflops": ffma, "sms": sms, "mma_issue": rows,
+                          "device_status_ok": status == ox.ONEXN_OK}), flush=True)
 
 
 def run_sweep(args, dev, stream, flush, ws, rank, pk):
@@ -635,8 +732,8 @@ def run_sweep(args, dev, stream, flush, ws, rank, pk):
                 for rate in wl.SWEEP_RATE:
                     layer = wl.config5(N=N, rate=rate, dtype=dtype, seed=0)[0]
                     a2 = argparse.Namespace(steps=steps, warmup=args.warmup)
-                    legs, leg_ms, step_ms, flops, info, _ = measure([layer], a2, dev, stream, flush,
-                                                                    ws, pk)
+                    legs, leg_ms, step_ms, flops, info, _, _ = measure([layer], a2, dev, stream, flush,
+                                                                       ws, pk, passes=1)
                     if dense_ms is None:
                         dense_ms = dense_times(legs, dev, flush, stream)[0]
                     total_flops += flops

@@ -77,6 +77,14 @@ typedef enum { ONEXN_GRAN_TAP = 0, ONEXN_GRAN_KERNEL = 1 } onexn_granularity;
 /* ONEXN_ACCUMULATE (onexn_conv_bwd_data only): dx += the gradient instead of
  * dx = the gradient (a layer whose input also feeds another branch). */
 #define ONEXN_ACCUMULATE 0x40u
+/* ONEXN_CHECK_INPUT (onexn_conv_fwd / _ex): checked mode.  Before the
+ * convolution a validation kernel checks the device BSR lists as Sec. 3.4
+ * defines them (P[0] = 0, P[G] = t, P non-decreasing, I strictly increasing
+ * inside every group and within [0, K)) and, if they are malformed, sets a
+ * bit of the status word that onexn_device_status reports as ONEXN_EDEVICE.
+ * The kernels clamp every P and I they read, so a malformed list faults
+ * nothing; the output is then not meaningful.  Costs one small launch. */
+#define ONEXN_CHECK_INPUT 0x80u
 /* Kernel selection (bits 8..11).  AUTO picks by dtype, N and density:
  * the tensor-core GEMM when its workspace fits and its dense work is
  * estimated to take less time than the FFMA kernel's kept work. */
@@ -492,8 +500,11 @@ onexn_status onexn_conv_fwd_noalloc(const onexn_conv_desc *desc, const int32_t *
  * word that the kernels of this library keep on the current device (a
  * 4-byte __device__ variable of the library).  A kernel whose bounded
  * internal wait (about one second) runs out sets it and returns early, so
- * its output is not valid.  Synchronises the device first.
- *   *status = ONEXN_OK (nothing reported since the last clear) or
+ * its output is not valid; the checked mode's validation kernel
+ * (ONEXN_CHECK_INPUT) sets it when the BSR lists are malformed.
+ * Synchronises the device first.
+ *   *status = ONEXN_OK (nothing reported since the last clear),
+ *             ONEXN_EDEVICE (malformed P / I seen in checked mode) or
  *             ONEXN_ETIMEOUT.
  * ECUDA if a runtime call fails (for instance an earlier kernel fault).
  */
@@ -509,6 +520,29 @@ onexn_status onexn_device_status(int clear, int *status);
  * only if the launch fails.
  */
 onexn_status onexn_selftest_timeout(void *stream);
+
+/*
+ * Measurement kernels behind the library's rooflines (no paper counterpart;
+ * they compute nothing of the method).  Launch only, on `stream`; the caller
+ * times them with CUDA events and derives the rates.
+ *
+ * onexn_probe_ffma -- `blocks` blocks of 256 threads; every thread runs 8
+ * independent fp32 fused multiply-add chains of `iters` steps, i.e.
+ * 16 * iters flops per thread.  `sink` (DEVICE, >= blocks floats) is only
+ * written if the chains reach an impossible value.  EINVAL on blocks or
+ * iters < 1 or a NULL sink.
+ */
+onexn_status onexn_probe_ffma(int blocks, int iters, float *sink, void *stream);
+
+/*
+ * onexn_probe_mma_issue -- one CTA per SM; lane 0 of each of `issuers`
+ * (1..8) warps issues 4 * iters back-to-back tcgen05.mma (kind::f16, bf16
+ * operands of zero, fp32 accumulate, M = 128, K = 16, width N in {16, 32})
+ * into its own accumulator, the A operand read from tensor memory
+ * (a_tmem != 0) or from shared memory.  2 * 128 * N * 16 * 4 * iters flops
+ * per issuer per SM.  EINVAL on other N / issuers or iters < 1.
+ */
+onexn_status onexn_probe_mma_issue(int N, int issuers, int a_tmem, int iters, void *stream);
 
 #ifdef __cplusplus
 }

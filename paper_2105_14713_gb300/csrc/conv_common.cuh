@@ -37,9 +37,13 @@ struct ConvArgs {
 
 // Bits of the device status word (read by onexn_device_status).
 constexpr unsigned int kStatusTimeout = 1u;
+constexpr unsigned int kStatusBadInput = 2u;   // the validation kernel found a malformed (P, I)
 
 // Host: SM count of the current device (cached per device).
 cudaError_t device_sm_count(int *sms);
+// Host: the same, or 152 (GB300) if it cannot be queried; for cost models
+// and tile planning, which only need an estimate.
+int device_sms_or_default();
 // Host: device address of the status word of the current device.
 cudaError_t device_status_ptr(unsigned int **p);
 

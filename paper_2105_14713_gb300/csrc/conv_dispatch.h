@@ -58,6 +58,8 @@ onexn_status check_algo(unsigned algo, const ConvArgs &a, int dtype, size_t ws_b
 // Launch one family (decode included for the tensor-core family).
 cudaError_t launch(unsigned algo, const ConvArgs &a, int dtype, void *workspace, size_t ws_bytes,
                    cudaStream_t st);
+// Checked mode: the device-side validation of (P, I) (status bit on failure).
+cudaError_t launch_validate(const ConvArgs &a, cudaStream_t st);
 
 }  // namespace detail
 }  // namespace onexn

@@ -38,6 +38,12 @@ cudaError_t device_sm_count(int *sms)
     return cudaSuccess;
 }
 
+int device_sms_or_default()
+{
+    int sms = 0;
+    return (device_sm_count(&sms) == cudaSuccess && sms > 0) ? sms : 152;
+}
+
 cudaError_t device_status_ptr(unsigned int **p)
 {
     int dev = 0;
@@ -87,7 +93,8 @@ onexn_status check_shape(const onexn_conv_desc *d, int N, int64_t t, int dtype, 
     if (d->C_in % cv)
         return fail(ONEXN_EINVAL, "conv: C_in=%d must be a multiple of %d for %s", d->C_in, cv,
                     dtype == ONEXN_F32 ? "fp32" : "bf16");
-    if (flags & ~(ONEXN_RELU | ONEXN_RELU6 | ONEXN_DECODED | ONEXN_REUSE_DECODE | ONEXN_ALGO_MASK))
+    if (flags & ~(ONEXN_RELU | ONEXN_RELU6 | ONEXN_DECODED | ONEXN_REUSE_DECODE | ONEXN_CHECK_INPUT |
+                  ONEXN_ALGO_MASK))
         return fail(ONEXN_EINVAL, "conv: unknown flags");
     a->B = d->B; a->H = d->H; a->W = d->W; a->C = d->C_in;
     a->C_out = d->C_out; a->KH = d->KH; a->KW = d->KW;
@@ -156,15 +163,16 @@ bool supports(unsigned algo, const onexn::ConvArgs &a, int dtype)
 // for small N) and then does only the kept work (t*N weights per pixel),
 // faster for wider blocks that share each staged activation.  A unit runs
 // on one SM, so a launch with fewer units than SMs (batch-1 layers: a 7x7
-// output is one unit of pixels) takes 152 / units times the machine-rate
-// time, on pixels and columns padded to whole units.  The tensor-core
+// output is one unit of pixels) takes SMs / units times the machine-rate
+// time, on pixels and columns padded to whole units (SMs queried from the
+// device).  The tensor-core
 // family's estimate is tc_cost_ns (conv_tc.cu).  Measured on GB300 at batch
 // 1, the FFMA kernel loses to the decoded GEMM on every MobileNet-V2 1x1
 // layer from 14x14 down (e.g. 76 vs 17 us on the 7x7 960->160 projection).
 namespace {
 double fma_floor(int N) { return N >= 4 ? 1.33e-5 : N >= 2 ? 1.66e-5 : 2.67e-5; }
 double fma_per_kept(int N) { return N >= 8 ? 3.0e-5 : N >= 4 ? 4.3e-5 : N >= 2 ? 7.2e-5 : 1.44e-4; }
-constexpr int kFmaUnitPix = 256, kFmaUnitCols = 64, kSms = 152;
+constexpr int kFmaUnitPix = 256, kFmaUnitCols = 64;
 constexpr double kFmaFixedNs = 700.0;     // pipeline fill beyond a bare launch
 
 double fma_cost_ns(const onexn::ConvArgs &a)
@@ -177,8 +185,9 @@ double fma_cost_ns(const onexn::ConvArgs &a)
     const double K = static_cast<double>(a.KH) * a.KW * a.C;
     const double floor_ns = pix * a.C_out * col_pad * K * fma_floor(a.N);
     const double kept_ns = pix * static_cast<double>(a.t) * a.N * fma_per_kept(a.N);
-    const double waves = static_cast<double>((units + kSms - 1) / kSms);
-    return (floor_ns + kept_ns) * kSms * waves / static_cast<double>(units) + kFmaFixedNs;
+    const int sms = onexn::device_sms_or_default();
+    const double waves = static_cast<double>((units + sms - 1) / sms);
+    return (floor_ns + kept_ns) * sms * waves / static_cast<double>(units) + kFmaFixedNs;
 }
 }  // namespace
 
@@ -220,6 +229,43 @@ cudaError_t launch(unsigned algo, const ConvArgs &a, int dtype, void *workspace,
     return launch_tc(a, dtype, workspace, ws_bytes, st);
 }
 
+}  // namespace detail
+}  // namespace onexn
+
+namespace onexn {
+
+// Checked mode: the BSR lists of Sec. 3.4 as the kernels assume them --
+// P[0] = 0, P[G] = t, P non-decreasing; within every group I strictly
+// increasing and inside [0, K).  One thread per group; every read is
+// clamped to P[0..G] and I[0..t), so a malformed list is reported through
+// the status word instead of being read out of bounds.
+__global__ void validate_bsr_kernel(const int32_t *__restrict__ P, const int32_t *__restrict__ I, int G, int t,
+                                    int K, unsigned int *status)
+{
+    const int g = blockIdx.x * blockDim.x + threadIdx.x;
+    if (g >= G) return;
+    const int p0 = __ldg(P + g), p1 = __ldg(P + g + 1);
+    bool ok = p0 >= 0 && p1 <= t && p0 <= p1;
+    if (g == 0 && p0 != 0) ok = false;
+    if (g == G - 1 && p1 != t) ok = false;
+    const int z0 = clampi(p0, 0, t), z1 = clampi(p1, z0, t);
+    int prev = -1;
+    for (int z = z0; z < z1 && ok; ++z) {
+        const int k = __ldg(I + z);
+        if (k <= prev || k >= K) ok = false;
+        prev = k;
+    }
+    if (!ok) atomicOr(status, kStatusBadInput);
+}
+
+namespace detail {
+cudaError_t launch_validate(const ConvArgs &a, cudaStream_t st)
+{
+    const int G = a.C_out / a.N;
+    if (G == 0) return cudaSuccess;
+    validate_bsr_kernel<<<(G + 127) / 128, 128, 0, st>>>(a.P, a.I, G, a.t, a.KH * a.KW * a.C, a.status);
+    return cudaGetLastError();
+}
 }  // namespace detail
 }  // namespace onexn
 
@@ -296,6 +342,8 @@ extern "C" onexn_status onexn_conv_fwd_ex(const onexn_conv_desc *desc, const int
     cudaStream_t s = static_cast<cudaStream_t>(stream);
     cudaError_t e = onexn::device_status_ptr(&a.status);
     if (e != cudaSuccess) return fail(ONEXN_ECUDA, "conv: status word: %s", cudaGetErrorString(e));
+    if ((flags & ONEXN_CHECK_INPUT) && (e = launch_validate(a, s)) != cudaSuccess)
+        return fail(ONEXN_ECUDA, "conv: validation launch failed: %s", cudaGetErrorString(e));
     e = decoded ? tc_gemm(a, dtype, workspace, workspace_bytes, s) : launch(algo, a, dtype, workspace, workspace_bytes, s);
     if (e != cudaSuccess) return fail(ONEXN_ECUDA, "conv: launch failed: %s", cudaGetErrorString(e));
     return ONEXN_OK;
@@ -416,6 +464,6 @@ extern "C" onexn_status onexn_device_status(int clear, int *status)
     if (e == cudaSuccess) e = cudaMemcpy(&w, p, sizeof(w), cudaMemcpyDeviceToHost);
     if (e == cudaSuccess && clear) e = cudaMemset(p, 0, sizeof(w));
     if (e != cudaSuccess) return fail(ONEXN_ECUDA, "device_status: %s", cudaGetErrorString(e));
-    *status = (w & onexn::kStatusTimeout) ? ONEXN_ETIMEOUT : ONEXN_OK;
+    *status = (w & onexn::kStatusBadInput) ? ONEXN_EDEVICE : (w & onexn::kStatusTimeout) ? ONEXN_ETIMEOUT : ONEXN_OK;
     return ONEXN_OK;
 }

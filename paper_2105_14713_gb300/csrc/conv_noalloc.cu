@@ -21,9 +21,11 @@
 //    different streams, or from different host threads) race on it and may
 //    produce wrong results; serialise them.
 //  * Nothing in the array has to start at zero: the decode step of each
-//    call writes every element of the region the call uses (a kept weight
-//    or zero) before the GEMM reads it; contents left by the previous call
-//    are never read.
+//    call writes every element of the weight region the call uses (a kept
+//    weight or zero) and lowers the stream-K flags before the GEMM reads
+//    them; the GEMM reads a stream-K partial slot only after its writer
+//    raised that slot's flag in the same call.  Contents left by the
+//    previous call are never read.
 //  * The device address of the array is looked up once per device, on the
 //    first call made with that device current (cudaGetSymbolAddress).  Make
 //    that first call before any stream capture begins.
@@ -84,8 +86,11 @@ extern "C" onexn_status onexn_conv_fwd_noalloc(const onexn_conv_desc *desc, cons
     if (st != ONEXN_OK) return st;
     if (!onexn::detail::supports(ONEXN_ALGO_TC, a, dtype))
         return onexn::fail(ONEXN_EUNSUPPORTED, "conv_noalloc: the tensor-core family cannot run this case");
-    // the decoded weights must fit (the stream-K balancing space is not
-    // needed and does not fit in the fixed scratch)
+    // the decoded weights must fit.  The whole scratch is passed on as the
+    // workspace: when the decoded weights plus the stream-K partial slots
+    // and flags also fit in it, the GEMM balances its last round of tiles
+    // there too (each call's decode lowers the flags before the GEMM reads
+    // them, so nothing a previous call left behind is trusted)
     const size_t need = onexn::detail::workspace_min_for(ONEXN_ALGO_TC, a, dtype);
     if (need > kNoAllocScratchBytes)
         return onexn::fail(ONEXN_EINVAL,

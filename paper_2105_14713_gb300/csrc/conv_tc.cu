@@ -90,7 +90,8 @@ struct TcF32 {
 
 constexpr int kSmemMax = 232448;      // dynamic shared memory per CTA (opt-in maximum)
 constexpr int kAccMax = 4;            // accumulator buffers in TMEM at most
-constexpr int kPlanCTAs = 152;        // stream-K: at most this many CTAs (GB300's SM count)
+constexpr int kPlanCTAs = 152;        // stream-K: partial slots / flags for at most this many CTAs
+                                      // (GB300's SM count; a larger GPU splits over 152 of its SMs)
 constexpr int kMinSplitIters = 4;     // stream-K: at least this many chunk iterations per CTA
 
 // Stream-K moves partial tiles through global memory and makes a finisher
@@ -1121,7 +1122,7 @@ cudaError_t launch_bn(const ConvArgs &a, const typename Tr::T *W, const typename
 }
 
 // Column-tile width: the BN in {64, 128, 256} with the least estimated time,
-// rounds of kPlanCTAs tiles x a per-tile cost linear in BN (the MMA's N)
+// rounds of (SM count) tiles x a per-tile cost linear in BN (the MMA's N)
 // plus a BN-independent share (A loads, epilogue start), 64 columns' worth.
 // Narrow tiles win when there are few pixel tiles (more CTAs busy); wide
 // tiles re-read the A operand fewer times.  Ties go to the wider tile.
@@ -1134,12 +1135,13 @@ cudaError_t launch_bn(const ConvArgs &a, const typename Tr::T *W, const typename
 int tc_bn(const ConvArgs &a, int dtype)
 {
     const int64_t n_m = (static_cast<int64_t>(a.P_pix) + kBM - 1) / kBM;
+    const int sms = device_sms_or_default();
     int best = 256;
     int64_t best_cost = -1;
     for (int bn : {256, 128, 64}) {
         if (bn > 64 && a.C_out <= bn / 2) continue;      // half the tile or more would be empty
         const int64_t tiles = n_m * ((a.C_out + bn - 1) / bn);
-        const int64_t cost = ((tiles + kPlanCTAs - 1) / kPlanCTAs) * (bn + 64);
+        const int64_t cost = ((tiles + sms - 1) / sms) * (bn + 64);
         if (best_cost < 0 || cost < best_cost) {
             best = bn;
             best_cost = cost;
@@ -1208,7 +1210,7 @@ cudaError_t gemm_typed(const ConvArgs &a, const void *workspace, size_t ws_bytes
 // Estimated time of the family (ns), for AUTO: the dense GEMM on the
 // decoded weights (padded to whole tiles) at the machine rate measured on
 // full-GPU layers (per multiply-add: fp32 as three tf32 products 7.9e-6 ns,
-// bf16 2.3e-6 ns), scaled by 152 / the CTAs busy on average (fewer tiles,
+// bf16 2.3e-6 ns), scaled by SMs / the CTAs busy on average (fewer tiles,
 // or stream-K pieces, than SMs; a ragged last round), plus fixed costs
 // measured on GB300 against batch-1 layers: the GEMM's prologue, the
 // stream-K fixup (partial tiles out, the finisher's wait and reads), and
@@ -1223,17 +1225,19 @@ double tc_cost_ns(const ConvArgs &a, int dtype, size_t ws_bytes, bool decoded)
     const int64_t n_m = (static_cast<int64_t>(a.P_pix) + kBM - 1) / kBM, n_n = (a.C_out + bn - 1) / bn;
     const int64_t tiles = n_m * n_n, chunks = static_cast<int64_t>(a.KH) * a.KW * ((a.C + bk - 1) / bk);
     const size_t wb = weights_bytes(a, dtype);
-    const bool sk = ws_bytes >= wb + sk_bytes(a, dtype) && tiles < kPlanCTAs && chunks >= sk_min_chunks(f32);
+    const int sms = device_sms_or_default();
+    const int ctas = sms < kPlanCTAs ? sms : kPlanCTAs;
+    const bool sk = ws_bytes >= wb + sk_bytes(a, dtype) && tiles < ctas && chunks >= sk_min_chunks(f32);
     double busy;
-    if (tiles >= kPlanCTAs)
-        busy = static_cast<double>(tiles) / static_cast<double>((tiles + kPlanCTAs - 1) / kPlanCTAs);
+    if (tiles >= sms)
+        busy = static_cast<double>(tiles) / static_cast<double>((tiles + sms - 1) / sms);
     else if (sk)
-        busy = std::min<double>(kPlanCTAs, static_cast<double>(tiles * chunks) / kMinSplitIters);
+        busy = std::min<double>(ctas, static_cast<double>(tiles * chunks) / kMinSplitIters);
     else
         busy = static_cast<double>(tiles);
     const double dense = static_cast<double>(n_m * kBM) * static_cast<double>(n_n * bn) *
                          static_cast<double>(a.KH * a.KW * a.C);
-    double ns = dense * (f32 ? 7.9e-6 : 2.3e-6) * kPlanCTAs / busy + kGemmFixedNs;
+    double ns = dense * (f32 ? 7.9e-6 : 2.3e-6) * sms / busy + kGemmFixedNs;
     if (sk) ns += kSkFixupNs;
     if (!decoded) ns += kDecodeFixedNs + static_cast<double>(wb) / kDecodeBytesPerNs;
     return ns;
@@ -1314,7 +1318,7 @@ TcSplitPlan tc_split_plan(int M, int Ncols, int64_t K, int dtype)
     const int64_t tiles = ((static_cast<int64_t>(M) + kBM - 1) / kBM) * ((Ncols + p.bn - 1) / p.bn);
     const int64_t chunks = (K + (dtype == ONEXN_F32 ? TcF32::kBK : TcBf16::kBK) - 1) /
                            (dtype == ONEXN_F32 ? TcF32::kBK : TcBf16::kBK);
-    int64_t S = kPlanCTAs / (tiles > 0 ? tiles : 1);
+    int64_t S = device_sms_or_default() / (tiles > 0 ? tiles : 1);
     if (S < 1) S = 1;
     if (S > chunks) S = chunks > 0 ? chunks : 1;
     p.tiles = static_cast<int>(tiles);

@@ -21,6 +21,7 @@ ONEXN_RELU6 = 0x2
 ONEXN_DECODED = 0x10
 ONEXN_REUSE_DECODE = 0x20
 ONEXN_ACCUMULATE = 0x40
+ONEXN_CHECK_INPUT = 0x80
 ONEXN_ALGO_SHIFT = 8
 ONEXN_ALGO_MASK = 0xF << ONEXN_ALGO_SHIFT
 ONEXN_ALGO_AUTO = 0 << ONEXN_ALGO_SHIFT
@@ -64,6 +65,8 @@ SIGNATURES = {
                         _I32),
     "onexn_device_status": ([_I32, _P], _I32),
     "onexn_selftest_timeout": ([_P], _I32),
+    "onexn_probe_ffma": ([_I32, _I32, _P, _P], _I32),
+    "onexn_probe_mma_issue": ([_I32, _I32, _I32, _I32, _P], _I32),
     "onexn_conv_fwd_noalloc": ([ctypes.POINTER(ConvDesc), _P, _P, _P, _I32, _I64, _P, _P, _P, _I32,
                                 _U32, _P], _I32),
     "onexn_conv_fwd_host": ([ctypes.POINTER(ConvDesc), _P, _P, _P, _I32, _I64, _P, _P, _P, _I32,
@@ -290,7 +293,8 @@ def onexn_conv_fwd_host(desc: ConvDesc, P, I, D, N: int, t: int, x_host, y_host,
 
 
 def onexn_device_status(clear: bool = True) -> int:
-    """ONEXN_OK or ONEXN_ETIMEOUT (a bounded in-kernel wait ran out)."""
+    """ONEXN_OK, ONEXN_EDEVICE (checked mode found malformed P / I) or
+    ONEXN_ETIMEOUT (a bounded in-kernel wait ran out)."""
     st = ctypes.c_int(0)
     _check(lib.onexn_device_status(int(bool(clear)), ctypes.byref(st)))
     return st.value
@@ -302,6 +306,24 @@ def onexn_selftest_timeout(stream=None) -> None:
     import torch
     st = torch.cuda.current_stream() if stream is None else stream
     _check(lib.onexn_selftest_timeout(ctypes.c_void_p(st.cuda_stream)))
+
+
+def onexn_probe_ffma(blocks: int, iters: int, sink, stream=None) -> None:
+    """Launch the FFMA-chain measurement kernel (16 * iters flops per thread,
+    256 threads per block); sink a CUDA float tensor of >= blocks elements."""
+    import torch
+    st = torch.cuda.current_stream() if stream is None else stream
+    _check(lib.onexn_probe_ffma(int(blocks), int(iters), ctypes.c_void_p(sink.data_ptr()),
+                                ctypes.c_void_p(st.cuda_stream)))
+
+
+def onexn_probe_mma_issue(N: int, issuers: int, a_tmem: bool, iters: int, stream=None) -> None:
+    """Launch the tcgen05.mma issue-rate measurement kernel (one CTA per SM,
+    4 * iters MMAs of M=128 x N x K=16 per issuing warp)."""
+    import torch
+    st = torch.cuda.current_stream() if stream is None else stream
+    _check(lib.onexn_probe_mma_issue(int(N), int(issuers), int(bool(a_tmem)), int(iters),
+                                     ctypes.c_void_p(st.cuda_stream)))
 
 
 def _cuda_stream(t, stream):
