@@ -407,7 +407,7 @@ def config_json(cfg, layers, l2="flushed before every step (256 MB write)"):
 # GPU arm
 # --------------------------------------------------------------------------
 
-def build_legs(layers, dev):
+def build_legs(layers, dev, algo_flag=0):
     from paper_2105_14713_gb300 import workloads as wl
     from paper_2105_14713_gb300.layer import PrunedConv2d
     legs = []
@@ -420,9 +420,9 @@ def build_legs(layers, dev):
         x_cpu = x_cpu if layer.dtype == "f32" else x_cpu.to(torch.bfloat16)
         x = x_cpu.to(dev)
         y = torch.empty(conv.out_shape(x.shape), dtype=x.dtype, device=dev)
-        conv.workspace(x.shape)
-        legs.append({"layer": layer, "conv": conv, "x": x, "y": y, "x_cpu": x_cpu,
-                     "algo": conv.algo(x.shape)})
+        conv.workspace(x.shape, algo_flag)
+        legs.append({"layer": layer, "conv": conv, "x": x, "y": y, "x_cpu": x_cpu, "flag": algo_flag,
+                     "algo": conv.algo(x.shape, algo_flag)})
     return legs
 
 
@@ -434,7 +434,7 @@ def time_legs(legs, steps, warmup, flush, stream, sampler=None, flush_l2=True, p
     for _ in range(warmup):
         flush.fill_(1)
         for lg in legs:
-            lg["conv"](lg["x"], lg["y"])
+            lg["conv"](lg["x"], lg["y"], algo=lg["flag"])
     torch.cuda.synchronize()
     evs = [[[[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in range(passes)] for _ in legs]
            for _ in range(steps)]
@@ -447,7 +447,7 @@ def time_legs(legs, steps, warmup, flush, stream, sampler=None, flush_l2=True, p
             for r in range(passes):
                 for i, lg in enumerate(legs):
                     evs[k][i][r][0].record(stream)
-                    lg["conv"](lg["x"], lg["y"])
+                    lg["conv"](lg["x"], lg["y"], algo=lg["flag"])
                     evs[k][i][r][1].record(stream)
         torch.cuda.synchronize()
         wall = time.perf_counter() - wall0
@@ -464,12 +464,12 @@ def passes_for(legs, flush, stream):
     for _ in range(2):
         flush.fill_(1)
         for lg in legs:
-            lg["conv"](lg["x"], lg["y"])
+            lg["conv"](lg["x"], lg["y"], algo=lg["flag"])
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     flush.fill_(2)
     e0.record(stream)
     for lg in legs:
-        lg["conv"](lg["x"], lg["y"])
+        lg["conv"](lg["x"], lg["y"], algo=lg["flag"])
     e1.record(stream)
     torch.cuda.synchronize()
     return max(1, int(STEP_TARGET_MS / max(e0.elapsed_time(e1), 1e-3) + 0.5))
@@ -543,7 +543,10 @@ def launches_per_step(legs, passes=1):
 
 
 def measure(layers, args, dev, stream, flush, ws, pk, sampler=None, passes=None):
-    legs = build_legs(layers, dev)
+    from paper_2105_14713_gb300 import onexn as ox
+    legs = build_legs(layers, dev, ox.ALGO_BY_NAME.get(getattr(args, "algo", "auto"), 0))
+    if passes is None and getattr(args, "passes", 0) > 0:
+        passes = args.passes
     if passes is None:
         passes = max_over_ranks(passes_for(legs, flush, stream), ws) if getattr(args, "auto_passes", False) else 1
     passes = int(passes)
@@ -575,8 +578,12 @@ def main():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--peaks", action="store_true")
+    # profiling aids: one layer of the workload only, a fixed number of passes
+    ap.add_argument("--layer", default=None)
+    ap.add_argument("--passes", type=int, default=0)
+    ap.add_argument("--algo", default="auto", choices=["auto", "fma", "mma", "tc"])
     args = ap.parse_args()
-    args.auto_passes = True
+    args.auto_passes = args.passes <= 0
     args.warmup = max(args.warmup, 3)
     rank, local, ws = dist_setup()
     if args.impl == "reference":
@@ -606,6 +613,10 @@ def main():
         return
 
     layers = workload(args.config)
+    if args.layer:
+        layers = [l for l in layers if l.name == args.layer]
+        if not layers:
+            raise SystemExit(f"no layer {args.layer} in workload {args.config}")
     sampler = ClockSampler(local)
     barrier(ws)
     torch.cuda.synchronize()

@@ -35,12 +35,12 @@ constexpr int kProbeWarps = 8;
 
 // Back-to-back tcgen05.mma (kind::f16, M = 128, K = 16, zero operands) issued
 // by lane 0 of each of `issuers` warps into its own accumulator: 4 * iters
-// MMAs per issuer.  A is read from tensor memory (a_tmem != 0) or from
-// shared memory; B from shared memory.  One CTA per SM (the shared-memory
+// MMAs per issuer.  A is read from tensor memory (kATmem) or from shared
+// memory; B from shared memory.  The A source is a template parameter: a
+// run-time branch between the issues slows the issue itself.  One CTA per SM (the shared-memory
 // request exceeds half an SM).
-template <int N>
-__global__ void __launch_bounds__(kProbeWarps * 32, 1) mma_issue_kernel(int iters, int issuers, int a_tmem,
-                                                                         unsigned int *status)
+template <int N, bool kATmem>
+__global__ void __launch_bounds__(kProbeWarps * 32, 1) mma_issue_kernel(int iters, int issuers, unsigned int *status)
 {
     extern __shared__ unsigned char smem_raw[];
     const uint32_t raw = smem_u32(smem_raw);
@@ -82,7 +82,7 @@ __global__ void __launch_bounds__(kProbeWarps * 32, 1) mma_issue_kernel(int iter
         for (int it = 0; it < iters; ++it) {
 #pragma unroll
             for (int kk = 0; kk < 4; ++kk) {
-                if (a_tmem)
+                if constexpr (kATmem)
                     tc::mma_bf16_ta(d, tmem + 256 + 8 * kk, bd + 2 * kk, idesc, (it | kk) != 0);
                 else
                     tc::mma_bf16(d, ad + 2 * kk, bd + 2 * kk, idesc, (it | kk) != 0);
@@ -126,11 +126,12 @@ extern "C" onexn_status onexn_probe_mma_issue(int N, int issuers, int a_tmem, in
     int sms = 0;
     e = onexn::device_sm_count(&sms);
     if (e != cudaSuccess) return fail(ONEXN_ECUDA, "probe_mma_issue: %s", cudaGetErrorString(e));
-    auto kern = N == 16 ? onexn::mma_issue_kernel<16> : onexn::mma_issue_kernel<32>;
+    auto kern = N == 16 ? (a_tmem ? onexn::mma_issue_kernel<16, true> : onexn::mma_issue_kernel<16, false>)
+                        : (a_tmem ? onexn::mma_issue_kernel<32, true> : onexn::mma_issue_kernel<32, false>);
     e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, onexn::kMmaProbeSmem);
     if (e == cudaSuccess) {
         kern<<<sms, onexn::kProbeWarps * 32, onexn::kMmaProbeSmem, static_cast<cudaStream_t>(stream)>>>(
-            iters, issuers, a_tmem, st);
+            iters, issuers, st);
         e = cudaGetLastError();
     }
     return e == cudaSuccess ? ONEXN_OK : fail(ONEXN_ECUDA, "probe_mma_issue: %s", cudaGetErrorString(e));
