@@ -730,8 +730,25 @@ def run_peaks(dev, rank):
                           "device_status_ok": status == ox.ONEXN_OK}), flush=True)
 
 
+def time_call(fn, flush, stream, reps=5):
+    """Mean CUDA-event time (ms) of fn() over `reps` calls after two
+    warm-ups, L2 flushed before each."""
+    ts = []
+    for r in range(2 + reps):
+        flush.fill_(r & 0xff)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        fn()
+        e1.record(stream)
+        torch.cuda.synchronize()
+        if r >= 2:
+            ts.append(e0.elapsed_time(e1))
+    return sum(ts) / len(ts)
+
+
 def run_sweep(args, dev, stream, flush, ws, rank, pk):
     from paper_2105_14713_gb300 import workloads as wl
+    from paper_2105_14713_gb300 import onexn as ox
     points = []
     total_flops, total_ms = 0.0, 0.0
     sampler = ClockSampler(0 if dev.index is None else dev.index)
@@ -752,6 +769,22 @@ def run_sweep(args, dev, stream, flush, ws, rank, pk):
                     p = dict(info[0])
                     p["speedup_vs_dense"] = dense_ms[0] / p["ms"]
                     p["dense_algo"] = dense_ms[1]
+                    p["kept_frac"] = 1.0 - rate
+                    # every family that can run the point, forced, for AUTO's check
+                    fam = {}
+                    for name in ("fma", "tc", "mma"):
+                        lg = legs[0]
+                        flag = ox.ALGO_BY_NAME[name]
+                        try:
+                            ox.onexn_conv_algo(lg["conv"].desc(*lg["x"].shape[:3]), lg["conv"].N, lg["conv"].t,
+                                               lg["conv"].cdtype, flag, 1 << 40)
+                        except ox.OnexnError:
+                            continue
+                        fam[name] = time_call(lambda: lg["conv"](lg["x"], lg["y"], algo=flag), flush, stream)
+                    best = min(fam, key=fam.get)
+                    p["family_ms"] = fam
+                    p["fastest"] = best
+                    p["auto_is_fastest"] = fam.get(p["algo"], float("inf")) <= 1.05 * fam[best]
                     points.append(p)
                     del legs
     value = ws * total_flops / (total_ms * 1e-3) / 1e12
@@ -769,6 +802,7 @@ def run_sweep(args, dev, stream, flush, ws, rank, pk):
             "config": {"workload": DESCRIPTIONS[5], "config_id": 5, "points": len(points),
                        "parallelism": "replicas", "l2": "flushed before every step (256 MB write)"},
             "roofline": rf, "points": points, "clocks": sampler.summary(),
+            "auto_fastest_points": sum(1 for p in points if p["auto_is_fastest"]),
             "gpu_launches": len(points) * steps,
             "peaks": pk, "cpu_baseline": None}), flush=True)
 

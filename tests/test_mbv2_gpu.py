@@ -195,15 +195,28 @@ def test_block_end_to_end_fp32_and_cuda_graph_replay():
     block = _block(blk)
     x = wl.block_input(blk).cuda()
     y_eager = block(x).clone()
-    # oracle composition in fp64 from the same input, no intermediate rounding
+    torch.cuda.synchronize()
+    # each stage against the oracle fed the GPU's own input to that stage, at
+    # the fp32 tolerance (an fp64 chain from x alone would add each stage's
+    # rounding, propagated through the later stages, to the comparison)
+    h, d, _ = block.buffers(x.shape, x.dtype, x.device)
     xs = x.cpu().numpy()
-    h = oracle.conv_masked(xs, block.w_expand, _mask(block.expand, block.w_expand, 4, 0.5), block.b_expand, 4,
-                           relu="relu6")
-    dd = oracle.dwconv(h.astype(np.float32), block.w_dw, block.b_dw, pad=(1, 1), relu="relu6")
-    ref, a = oracle.conv_masked(dd.astype(np.float32), block.w_project,
-                                _mask(block.project, block.w_project, 4, 0.5), block.b_project, 4,
-                                residual=xs, want_abs=True)
-    assert _err(y_eager.cpu().numpy(), ref, a) <= 1e-4
+    ref, a = oracle.conv_masked(xs, block.w_expand, _mask(block.expand, block.w_expand, 4, 0.5), block.b_expand, 4,
+                                relu="relu6", want_abs=True)
+    assert _err(_host32(h), ref, a) <= 1e-5, "expand"
+    hs = _host32(h)
+    ref = oracle.dwconv(hs, block.w_dw, block.b_dw, pad=(1, 1), relu="relu6")
+    if block.fused(x.shape):
+        # the projection computed the depthwise itself (fp32): its input is
+        # the oracle's depthwise of the GPU's expand output
+        ds = ref.astype(np.float32)
+    else:
+        a = oracle.dwconv(np.abs(hs), np.abs(block.w_dw), np.abs(block.b_dw), pad=(1, 1))
+        assert _err(_host32(d), ref, a) <= 1e-5, "depthwise"
+        ds = _host32(d)
+    ref, a = oracle.conv_masked(ds, block.w_project, _mask(block.project, block.w_project, 4, 0.5),
+                                block.b_project, 4, residual=xs, want_abs=True)
+    assert _err(y_eager.cpu().numpy(), ref, a) <= 1e-5, "project + residual"
     # the same block captured into a CUDA graph (no allocation after the first call)
     s = torch.cuda.Stream()
     torch.cuda.synchronize()
