@@ -37,6 +37,11 @@ TcSplitPlan tc_split_plan(int M, int Ncols, int64_t K, int dtype);
 cudaError_t tc_gemm_split(const ConvArgs &a, int dtype, const void *W, const void *W_lo, float *partials,
                           const TcSplitPlan &plan, cudaStream_t st);
 size_t tc_weights_bytes(const ConvArgs &a, int dtype);
+// Halo-tile form of the bf16 GEMM for stride-1 spatial layers (conv_halo.cu):
+// whether it takes the layer (against the im2col GEMM's column tile), and
+// the launch on the decoded weights W[C_out][K].
+bool halo_applies(const ConvArgs &a, int im2col_bn);
+cudaError_t halo_gemm(const ConvArgs &a, const void *W, cudaStream_t st);
 size_t tc_sk_bytes(const ConvArgs &a, int dtype);
 
 namespace detail {

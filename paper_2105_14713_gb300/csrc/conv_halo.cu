@@ -1,0 +1,535 @@
+// Tensor-core GEMM of stride-1 spatial convolutions (bf16) on halo tiles.
+//
+// The im2col form of the tcgen05 GEMM (conv_tc.cu) loads a fresh A tile of
+// 128 output pixels for every tap and the B tile of that tap for every
+// pixel tile, so a 3x3 layer moves each activation nine times and its
+// weights once per tile from L2 into shared memory.  Here:
+//  * a tile is R whole output rows of one image, laid out along M with the
+//    padded row width Wp = Wo + (KW-1)*dw: M row m is output pixel
+//    (h0 + m / Wp, m % Wp); rows with m % Wp >= Wo or past the tile's rows
+//    are computed and dropped;
+//  * per 64-channel chunk one TMA im2col load brings the Wp x Rh input
+//    positions of rows h0 - ph .. h0 - ph + R + (KH-1)*dh - 1, columns
+//    -pw .. -pw + Wp - 1 (zeros outside the image), one 128-byte swizzled
+//    row per position, and the A operand of tap (kh, kw) is that buffer
+//    viewed from row kh*dh*Wp + kw*dw on: output pixel (r, w) of the tile
+//    reads input position (r + kh*dh, w + kw*dw) of the halo.  The swizzle
+//    is a function of the shared-memory address, so a view may start at any
+//    128-byte row;
+//  * each CTA serves one column tile of BN output channels, whose decoded
+//    weights (all taps and chunks) it loads once and keeps in shared memory.
+// The sum over taps and chunks is the one of Eq. 6 / Eq. 7 on the decoded
+// weights, as in the im2col GEMM; only the order of the fp32 additions
+// differs.
+//
+// One tcgen05.mma issuing thread sustains about one MMA per 27 ns, and
+// every mbarrier wait placed between its issues costs it about 130 ns more
+// (measured on GB300), while the tensor core needs ~25 ns for a
+// 128 x 64 x 16 MMA.  So a tile's MMAs (taps x chunks x 4) run between
+// waits on whole halo chunks, with slots and phases as running counters and
+// the 3x3 taps unrolled, and two MMA warps take alternate tiles, each with
+// its own halo ring and accumulators, so one warp's waits overlap the
+// other's issues.
+//
+// Warp roles (one persistent CTA per SM): warp 0 issues the TMA loads, warps
+// 1-2 the MMAs (M=128, N=BN, K=16, A and B from shared memory; warp 1 also
+// allocates the TMEM), warps 3-6 read the accumulators, add bias /
+// residual, apply the activation, convert to bf16 and write the valid rows
+// into a staging tile laid out as the output rows, stored with one TMA box
+// per output row.  Every wait is bounded.
+#include "conv_common.cuh"
+#include "conv_dispatch.h"
+#include "tc_maps.h"
+#include "tc_ptx.cuh"
+
+#include <cuda.h>
+
+#include <algorithm>
+#include <mutex>
+#include <type_traits>
+
+namespace onexn {
+
+namespace {
+
+constexpr int kBM = 128;           // M rows per tile
+constexpr int kRow = 128;          // bytes of K per shared-memory row (64 bf16)
+constexpr int kBK = 64;            // channels per chunk
+constexpr int kSmemMax = 232448;   // dynamic shared memory per CTA (opt-in maximum)
+constexpr int kAccMax = 4;
+constexpr int kMmaWarps = 2;
+constexpr int kEpiWarp0 = 1 + kMmaWarps;
+constexpr int kWarps = kEpiWarp0 + 4;
+constexpr int kMaxHalo = 6;        // halo slots at most (all rings)
+constexpr int kBarBytes = (2 * kMaxHalo + 1 + 2 * kAccMax + kMmaWarps) * 8;
+constexpr double kMinRowFill = 0.85;   // valid share of the M rows below which the im2col form is kept
+
+struct HaloPlan {
+    int Wp, R, Rh, n_rb;           // padded width, output rows per tile, halo rows, row blocks per image
+    int n_cc, n_taps, n_tn, n_m;   // chunks, taps, column tiles, pixel tiles (images x row blocks)
+    int S_r, n_mma;                // halo slots per MMA warp, MMA warps
+    int grid;                      // CTAs: a multiple of n_tn, CTA b serves column tile b % n_tn
+    uint32_t halo_tx, slot_bytes, out_row_bytes, b_bytes;
+    uint32_t off_halo, off_out, off_bias, off_bar, bytes;
+    FastDiv div_rb;
+};
+
+constexpr int pow2_cols(int v, int p = 32) { return p >= v ? p : pow2_cols(v, 2 * p); }
+
+template <int BN>
+struct HaloTmem {
+    static constexpr int kAccFit = 512 / BN;
+    static constexpr int kAcc = kAccFit > kAccMax ? kAccMax : kAccFit;   // a multiple of kMmaWarps
+    static constexpr int kCols = pow2_cols(kAcc * BN);
+    static_assert(kAcc % kMmaWarps == 0, "accumulators per MMA warp");
+};
+
+__device__ __forceinline__ bool epi_all4(bool ok)
+{
+    uint32_t r;
+    asm volatile(
+        "{\n\t.reg .pred p, q;\n\tsetp.ne.u32 p, %1, 0;\n\t"
+        "bar.red.and.pred q, 1, 128, p;\n\tselp.u32 %0, 1, 0, q;\n\t}\n"
+        : "=r"(r)
+        : "r"(ok ? 1u : 0u)
+        : "memory");
+    return r != 0;
+}
+
+// KS = 3: 3x3 kernel, taps unrolled; KS = 0: any kernel shape.
+template <int BN, int KS>
+__global__ void __launch_bounds__(kWarps * 32, 1)
+halo_conv_kernel(const ConvArgs a, const __grid_constant__ CUtensorMap tmap_x,
+                 const __grid_constant__ CUtensorMap tmap_w, const __grid_constant__ CUtensorMap tmap_y,
+                 const HaloPlan hp)
+{
+    using TM = HaloTmem<BN>;
+    constexpr int kAcc = TM::kAcc;
+    constexpr uint32_t kBTile = BN * kRow;
+    extern __shared__ unsigned char smem_raw[];
+    const uint32_t raw = smem_u32(smem_raw);
+    const uint32_t base = (raw + 1023u) & ~1023u;
+    unsigned char *smem = smem_raw + (base - raw);
+    const uint32_t sB = base;                       // the column tile's weights: (tap, chunk) B tiles
+    const uint32_t sH = base + hp.off_halo;         // halo slots: ring j = slots j*S_r .. j*S_r + S_r - 1
+    const uint32_t bar_hfull = base + hp.off_bar;
+    const uint32_t bar_hempty = bar_hfull + 8 * kMaxHalo;
+    const uint32_t bar_bfull = bar_hempty + 8 * kMaxHalo;
+    const uint32_t bar_tfull = bar_bfull + 8;
+    const uint32_t bar_tempty = bar_tfull + 8 * kAccMax;
+    const uint32_t bar_drain = bar_tempty + 8 * kAccMax;   // one per MMA warp
+    uint32_t *holder = reinterpret_cast<uint32_t *>(smem + hp.off_bar + kBarBytes);
+
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    if (tid == 0) {
+        for (int s = 0; s < kMaxHalo; ++s) {
+            mbar_init(bar_hfull + 8 * s, 1);
+            mbar_init(bar_hempty + 8 * s, 1);
+        }
+        mbar_init(bar_bfull, 1);
+        for (int b = 0; b < kAccMax; ++b) {
+            mbar_init(bar_tfull + 8 * b, 1);
+            mbar_init(bar_tempty + 8 * b, 128);
+        }
+        for (int j = 0; j < kMmaWarps; ++j) mbar_init(bar_drain + 8 * j, 1);
+        fence_mbar_init();
+    }
+    if (warp == 1) {
+        tc::tmem_alloc(smem_u32(holder), TM::kCols);
+        tc::tmem_relinquish();
+    }
+    tc::fence_before_sync();
+    __syncthreads();
+    tc::fence_after_sync();
+    const uint32_t tmem = *holder;
+    // a programmatic dependent of the previous kernel on the stream: global
+    // memory is touched only after it has completed
+    asm volatile("griddepcontrol.wait;\n" ::: "memory");
+    asm volatile("griddepcontrol.launch_dependents;\n" ::: "memory");
+    auto abort_now = [&]() { atomicOr(a.status, kStatusTimeout); };
+    // this CTA's column tile and pixel tiles: tm = m0, m0 + m_step, ...
+    const int tn = static_cast<int>(blockIdx.x) % hp.n_tn;
+    const int m0 = static_cast<int>(blockIdx.x) / hp.n_tn, m_step = hp.grid / hp.n_tn;
+
+    if (warp == 0) {
+        // ============================ producer ============================
+        if (lane == 0) {
+            bool failed = false;
+            tc::mbar_arrive_expect_tx(bar_bfull, hp.b_bytes);
+            for (int tap = 0, q = 0; tap < hp.n_taps; ++tap)
+                for (int cc = 0; cc < hp.n_cc; ++cc, ++q)
+                    tc::tma_load_2d(sB + q * kBTile, &tmap_w, tap * a.C + cc * kBK, tn * BN, bar_bfull);
+            // per ring: loads issued so far (slot = count % S_r, phase = (count / S_r) & 1)
+            int issued0 = 0, issued1 = 0;
+            int si = 0;
+            for (int tm = m0; tm < hp.n_m && !failed; tm += m_step, ++si) {
+                const int j = hp.n_mma > 1 ? (si & 1) : 0;
+                const int n = static_cast<int>(hp.div_rb.div(tm)), rb = tm - n * hp.n_rb;
+                const int h0 = rb * hp.R;
+                int cnt = j ? issued1 : issued0;
+                for (int cc = 0; cc < hp.n_cc; ++cc, ++cnt) {
+                    const int round = cnt / hp.S_r;
+                    const int slot = j * hp.S_r + (cnt - round * hp.S_r);
+                    if (round >= 1 && !mbar_wait(bar_hempty + 8 * slot, (round - 1) & 1)) {
+                        abort_now(); failed = true; break;
+                    }
+                    tc::mbar_arrive_expect_tx(bar_hfull + 8 * slot, hp.halo_tx);
+                    tc::tma_load_im2col_4d(sH + slot * hp.slot_bytes, &tmap_x, cc * kBK, -a.pw, h0 - a.ph, n, 0, 0,
+                                           bar_hfull + 8 * slot);
+                }
+                if (j) issued1 = cnt; else issued0 = cnt;
+            }
+        }
+        __syncwarp();
+    } else if (warp < kEpiWarp0) {
+        // ============================== MMA ==============================
+        const int j = warp - 1;
+        if (lane == 0 && j < hp.n_mma) {
+            constexpr uint32_t idesc = tc::idesc_bf16_f32(kBM, BN);
+            constexpr uint32_t kBDesc = BN * kRow / 16;          // descriptor units between B tiles
+            bool failed = !mbar_wait(bar_bfull, 0);
+            if (failed) abort_now();
+            const uint64_t b_desc0 = tc::desc_kmajor_sw128(sB);
+            const uint32_t row_step = static_cast<uint32_t>(a.dh * hp.Wp) * (kRow / 16);   // per kh, descriptor units
+            const uint32_t col_step = static_cast<uint32_t>(a.dw) * (kRow / 16);           // per kw
+            const uint32_t b_tap = static_cast<uint32_t>(hp.n_cc) * kBDesc;                 // per tap
+            const int per = kAcc / hp.n_mma;        // accumulators of this warp: j, j + n_mma, ...
+            int hs = 0, hph = 0, si = 0, k = 0;     // k: this warp's tile count
+            for (int tm = m0; tm < hp.n_m && !failed; tm += m_step, ++si) {
+                if (hp.n_mma > 1 && (si & 1) != j) continue;
+                const int acc = j + hp.n_mma * (k % per), use = k / per;
+                ++k;
+                if (use >= 1 && !mbar_wait(bar_tempty + 8 * acc, (use - 1) & 1)) {
+                    abort_now(); failed = true; break;
+                }
+                tc::fence_after_sync();
+                const uint32_t d_tmem = tmem + static_cast<uint32_t>(acc) * BN;
+                for (int cc = 0; cc < hp.n_cc; ++cc) {
+                    const int slot = j * hp.S_r + hs;
+                    if (!mbar_wait(bar_hfull + 8 * slot, hph)) { abort_now(); failed = true; break; }
+                    tc::fence_after_sync();
+                    const uint64_t hd = tc::desc_kmajor_sw128(sH + static_cast<uint32_t>(slot) * hp.slot_bytes);
+                    const uint64_t bd_cc = b_desc0 + static_cast<uint32_t>(cc) * kBDesc;
+                    const uint32_t acc0 = cc != 0 ? 1u : 0u;
+                    auto tap_mmas = [&](uint64_t ad, uint64_t bd, uint32_t first_acc) {
+                        tc::mma_bf16(d_tmem, ad, bd, idesc, first_acc);
+#pragma unroll
+                        for (int kk = 1; kk < kBK / 16; ++kk) tc::mma_bf16(d_tmem, ad + 2 * kk, bd + 2 * kk, idesc, 1u);
+                    };
+                    if constexpr (KS > 0) {
+#pragma unroll
+                        for (int tap = 0; tap < KS * KS; ++tap)
+                            tap_mmas(hd + (tap / KS) * row_step + (tap % KS) * col_step, bd_cc + tap * b_tap,
+                                     tap == 0 ? acc0 : 1u);
+                    } else {
+                        int kw = 0, kh = 0;
+                        for (int tap = 0; tap < hp.n_taps; ++tap) {
+                            tap_mmas(hd + kh * row_step + kw * col_step, bd_cc + static_cast<uint32_t>(tap) * b_tap,
+                                     tap == 0 ? acc0 : 1u);
+                            if (++kw == a.KW) { kw = 0; ++kh; }
+                        }
+                    }
+                    tc::commit(bar_hempty + 8 * slot);
+                    if (++hs == hp.S_r) { hs = 0; hph ^= 1; }
+                }
+                if (failed) break;
+                tc::commit(bar_tfull + 8 * acc);
+            }
+            tc::commit(bar_drain + 8 * j);
+            if (!mbar_wait(bar_drain + 8 * j, 0)) abort_now();
+        }
+        __syncwarp();
+    } else {
+        // ============================ epilogue ============================
+        // Thread (warp w, lane i) owns TMEM lane m = 32*(w%4) + i, output
+        // pixel (h0 + m / Wp, m % Wp) of the tile.  Per 64-column atom: read
+        // the accumulator, add bias (and residual), activate, convert, write
+        // the 128-byte row into the staging tile of its output row (double
+        // buffered across atoms), then one thread stores each output row.
+        auto epilogue = [&](auto res_c, auto act_c) {
+            constexpr bool kRes = decltype(res_c)::value;
+            constexpr int kAct = decltype(act_c)::value;
+            constexpr int kAtoms = BN / 64;
+            const int q = warp & 3;
+            const int m = 32 * q + lane;
+            const int mr = m / hp.Wp, mw = m - mr * hp.Wp;
+            const bool leader = (warp == kEpiWarp0) && lane == 0;
+            const uint32_t sout = base + hp.off_out;
+            const uint32_t buf_bytes = static_cast<uint32_t>(hp.R) * hp.out_row_bytes;
+            float *sbias = reinterpret_cast<float *>(smem + hp.off_bias);
+            const float4 *sb4 = reinterpret_cast<const float4 *>(sbias);
+            for (int c = m; c < BN; c += 128) {      // the column tile's bias, once
+                const int o = tn * BN + c;
+                sbias[c] = (a.bias && o < a.C_out) ? __ldg(a.bias + o) : 0.f;
+            }
+            tc::named_bar(1, 128);
+            // accumulator of the CTA's tile si: MMA warp j = si % n_mma uses
+            // j, j + n_mma, ... in turn
+            const int per = kAcc / hp.n_mma;
+            int n_emit = 0, si = 0;
+            for (int tm = m0; tm < hp.n_m; tm += m_step, ++si) {
+                const int j = hp.n_mma > 1 ? (si & 1) : 0;
+                const int kj = hp.n_mma > 1 ? (si >> 1) : si;          // MMA warp j's tile count before this one
+                const int acc = j + hp.n_mma * (kj % per), use = kj / per;
+                if (!epi_all4(mbar_wait(bar_tfull + 8 * acc, use & 1))) { abort_now(); break; }
+                tc::fence_after_sync();
+                const int n = static_cast<int>(hp.div_rb.div(tm)), rb = tm - n * hp.n_rb;
+                const int h0 = rb * hp.R;
+                const int R_t = min(hp.R, a.Ho - h0);
+                const bool valid = mr < R_t && mw < a.Wo;
+                const int64_t pix = (static_cast<int64_t>(n) * a.Ho + h0 + mr) * a.Wo + mw;
+                const uint32_t t_acc = tmem + (static_cast<uint32_t>(32 * q) << 16) + acc * BN;
+#pragma unroll 1
+                for (int at = 0; at < kAtoms; ++at) {
+                    const int col0 = tn * BN + at * 64;
+                    uint32_t r0[32], r1[32];
+                    tc::ld_32x32b_x32(t_acc + at * 64, r0);
+                    tc::ld_32x32b_x32(t_acc + at * 64 + 32, r1);
+                    tc::ld_wait();
+                    if (at == kAtoms - 1) {
+                        tc::fence_before_sync();
+                        mbar_arrive(bar_tempty + 8 * acc);
+                    }
+                    if (col0 >= a.C_out) continue;   // uniform: the atom lies past y's columns
+                    const uint32_t buf = sout + static_cast<uint32_t>(n_emit & 1) * buf_bytes;
+                    ++n_emit;
+                    // the stores of two atoms back have read this buffer
+                    if (leader) tc::bulk_wait_read1();
+                    tc::named_bar(1, 128);
+                    if (valid) {
+                        const uint4 *res = nullptr;
+                        if constexpr (kRes)
+                            res = reinterpret_cast<const uint4 *>(static_cast<const __nv_bfloat16 *>(a.residual) +
+                                                                  pix * a.C_out + col0);
+                        const uint32_t dst = buf + static_cast<uint32_t>(mr) * hp.out_row_bytes +
+                                             static_cast<uint32_t>(mw) * kRow;
+#pragma unroll
+                        for (int jj = 0; jj < 8; ++jj) {          // 16-byte chunk jj: columns 8jj .. 8jj+7
+                            uint32_t rw[4] = {0u, 0u, 0u, 0u};
+                            if constexpr (kRes) {
+                                if (col0 + 8 * jj < a.C_out) {
+                                    const uint4 rv = __ldg(res + jj);
+                                    rw[0] = rv.x; rw[1] = rv.y; rw[2] = rv.z; rw[3] = rv.w;
+                                }
+                            }
+                            const float4 b0 = sb4[at * 16 + 2 * jj], b1 = sb4[at * 16 + 2 * jj + 1];
+                            const float bb[8] = {b0.x, b0.y, b0.z, b0.w, b1.x, b1.y, b1.z, b1.w};
+                            uint32_t w[4];
+#pragma unroll
+                            for (int e = 0; e < 4; ++e) {
+                                const int c = 8 * jj + 2 * e;
+                                const uint32_t u0 = c < 32 ? r0[c] : r1[c - 32];
+                                const uint32_t u1 = c + 1 < 32 ? r0[c + 1] : r1[c + 1 - 32];
+                                float v0 = __uint_as_float(u0) + bb[2 * e], v1 = __uint_as_float(u1) + bb[2 * e + 1];
+                                if constexpr (kRes) {
+                                    v0 += bf16lo(rw[e]);
+                                    v1 += bf16hi(rw[e]);
+                                }
+                                w[e] = pack_bf16x2(activate_c<kAct>(v0), activate_c<kAct>(v1));
+                            }
+                            asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};\n" ::"r"(
+                                             dst + ((jj ^ (mw & 7)) << 4)),
+                                         "r"(w[0]), "r"(w[1]), "r"(w[2]), "r"(w[3])
+                                         : "memory");
+                        }
+                    }
+                    tc::fence_proxy_async_smem();
+                    tc::named_bar(1, 128);
+                    if (leader) {
+                        for (int r = 0; r < R_t; ++r)
+                            tc::tma_store_3d(&tmap_y, col0, 0, n * a.Ho + h0 + r,
+                                             buf + static_cast<uint32_t>(r) * hp.out_row_bytes);
+                        tc::bulk_commit();
+                    }
+                }
+            }
+            if (leader) tc::bulk_wait0();
+        };
+        if (a.residual) {
+            if (a.relu == 2) epilogue(std::true_type{}, std::integral_constant<int, 2>{});
+            else if (a.relu == 1) epilogue(std::true_type{}, std::integral_constant<int, 1>{});
+            else epilogue(std::true_type{}, std::integral_constant<int, 0>{});
+        } else {
+            if (a.relu == 2) epilogue(std::false_type{}, std::integral_constant<int, 2>{});
+            else if (a.relu == 1) epilogue(std::false_type{}, std::integral_constant<int, 1>{});
+            else epilogue(std::false_type{}, std::integral_constant<int, 0>{});
+        }
+    }
+
+    tc::fence_before_sync();
+    __syncthreads();
+    if (warp == 1) {
+        tc::fence_after_sync();
+        tc::tmem_dealloc(tmem, TM::kCols);
+    }
+}
+
+uint32_t round1024(uint64_t v) { return static_cast<uint32_t>((v + 1023) & ~static_cast<uint64_t>(1023)); }
+
+// The halo plan of a bf16 layer, or false when the layer keeps the im2col
+// form: strided or 1x1 layers, rows too wide for one M tile, too many
+// dropped M rows, or a column tile whose weights do not fit in shared
+// memory next to two halo slots.  The column tile is the widest of 256 /
+// 128 / 64 that fits (no wider than the output channels need).
+bool halo_plan(const ConvArgs &a, int sms, HaloPlan *out, int *bn_out)
+{
+    if (a.sh != 1 || a.sw != 1 || a.KH * a.KW == 1 || a.Ho <= 0 || a.Wo <= 0 || a.B <= 0) return false;
+    HaloPlan p{};
+    p.Wp = a.Wo + (a.KW - 1) * a.dw;
+    if (p.Wp > kBM) return false;
+    p.R = std::min(kBM / p.Wp, a.Ho);
+    p.n_rb = (a.Ho + p.R - 1) / p.R;
+    const double fill = static_cast<double>(a.Ho) * a.Wo / (static_cast<double>(p.n_rb) * kBM);
+    if (fill < kMinRowFill) return false;
+    p.Rh = p.R + (a.KH - 1) * a.dh;
+    if (p.Wp * p.Rh > 1024) return false;                 // positions per im2col load
+    const int reach = (a.KH - 1) * a.dh * p.Wp + (a.KW - 1) * a.dw + kBM;   // rows an MMA view can read
+    p.slot_bytes = round1024(static_cast<uint64_t>(std::max(p.Rh * p.Wp, reach)) * kRow);
+    p.halo_tx = static_cast<uint32_t>(p.Wp * p.Rh * kRow);
+    p.out_row_bytes = round1024(static_cast<uint64_t>(a.Wo) * kRow);
+    p.n_cc = (a.C + kBK - 1) / kBK;
+    p.n_taps = a.KH * a.KW;
+    p.n_m = a.B * p.n_rb;
+    const uint32_t staging = 2u * static_cast<uint32_t>(p.R) * p.out_row_bytes;
+    int bn = 0;
+    for (int cand : {256, 128, 64}) {
+        if (cand > 64 && a.C_out <= cand / 2) continue;
+        const uint64_t b_bytes = static_cast<uint64_t>(p.n_taps) * p.n_cc * cand * kRow;
+        const uint64_t fixed = staging + round1024(static_cast<uint64_t>(cand) * 4 + kBarBytes + 16) + 1024;
+        if (round1024(b_bytes) + 2ull * p.slot_bytes + fixed <= static_cast<uint64_t>(kSmemMax)) {
+            bn = cand;
+            p.b_bytes = static_cast<uint32_t>(b_bytes);
+            const uint64_t left = kSmemMax - fixed - round1024(b_bytes);
+            const int slots = static_cast<int>(std::min<uint64_t>(kMaxHalo, left / p.slot_bytes));
+            // two MMA warps when each can keep two halo slots in flight
+            p.n_mma = slots >= 2 * kMmaWarps ? kMmaWarps : 1;
+            p.S_r = slots / p.n_mma;
+            break;
+        }
+    }
+    if (bn == 0) return false;
+    p.n_tn = (a.C_out + bn - 1) / bn;
+    if (p.n_tn > sms) return false;
+    const int64_t tiles = static_cast<int64_t>(p.n_m) * p.n_tn;
+    p.grid = static_cast<int>(std::min<int64_t>(tiles, sms) / p.n_tn * p.n_tn);
+    p.off_halo = round1024(p.b_bytes);
+    p.off_out = p.off_halo + static_cast<uint32_t>(p.S_r * p.n_mma) * p.slot_bytes;
+    p.off_bias = p.off_out + staging;
+    p.off_bar = p.off_bias + static_cast<uint32_t>(bn) * 4;
+    p.bytes = p.off_bar + kBarBytes + 16;
+    if (p.bytes + 1024 > static_cast<uint32_t>(kSmemMax)) return false;
+    p.div_rb = FastDiv(static_cast<uint32_t>(p.n_rb));
+    *out = p;
+    *bn_out = bn;
+    return true;
+}
+
+// im2col tensor map of the halo: the traversal's bounding box is the padded
+// image, columns -pw .. W - 1 + pw and rows -ph .. H - 1 + ph (corners
+// innermost first: W, H), so a load of Wp x Rh positions from (-pw, h0 - ph)
+// walks whole padded rows.  A last row block that runs past the padded
+// image continues into the next image's rows (or zeros after the last
+// image); those rows feed only the dropped M rows of the tile.
+bool halo_x_tmap(const ConvArgs &a, const HaloPlan &hp, CUtensorMap *m)
+{
+    auto enc = encode_im2col_fn_public();
+    if (!enc) return false;
+    const cuuint64_t dims[4] = {static_cast<cuuint64_t>(a.C), static_cast<cuuint64_t>(a.W),
+                                static_cast<cuuint64_t>(a.H), static_cast<cuuint64_t>(a.B)};
+    const cuuint64_t strides[3] = {static_cast<cuuint64_t>(a.C) * 2, static_cast<cuuint64_t>(a.C) * 2 * a.W,
+                                   static_cast<cuuint64_t>(a.C) * 2 * a.W * a.H};
+    const int lower[2] = {-a.pw, -a.ph};
+    const int upper[2] = {hp.Wp - a.pw - a.W, a.Ho + (a.KH - 1) * a.dh - a.ph - a.H};
+    for (int i = 0; i < 2; ++i)
+        if (lower[i] < -128 || lower[i] > 127 || upper[i] < -128 || upper[i] > 127) return false;
+    const cuuint32_t estr[4] = {1, 1, 1, 1};
+    return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void *>(a.x), dims, strides, lower, upper, kBK,
+               static_cast<cuuint32_t>(hp.Wp * hp.Rh), estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+               CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+template <int BN, int KS>
+cudaError_t halo_launch_bn(const ConvArgs &a, const HaloPlan &hp, const __nv_bfloat16 *W, cudaStream_t st)
+{
+    auto kern = halo_conv_kernel<BN, KS>;
+    const CUtensorMapDataType bf = CU_TENSOR_MAP_DATA_TYPE_BFLOAT16;
+    const uint64_t K = static_cast<uint64_t>(a.KH) * a.KW * a.C;
+    CUtensorMap tmap_x, tmap_w, tmap_y;
+    // x [B][H][W][C]: one im2col load per 64-channel chunk walks the Wp x Rh
+    // halo positions of the tile (columns -pw .. W - 1 + pw of each row,
+    // the padding read as zeros)
+    if (!halo_x_tmap(a, hp, &tmap_x)) return cudaErrorInvalidValue;
+    {   // W [C_out][K]: boxes of 64 K x BN rows
+        const uint64_t dims[2] = {K, static_cast<uint64_t>(a.C_out)};
+        const uint64_t strides[1] = {K * 2};
+        const uint32_t box[2] = {kBK, BN};
+        if (!tc_tmap_tiled(&tmap_w, bf, 2, W, dims, strides, box)) return cudaErrorInvalidValue;
+    }
+    {   // y [B*Ho][Wo][C_out]: one output row of a 64-column atom per box
+        const uint64_t dims[3] = {static_cast<uint64_t>(a.C_out), static_cast<uint64_t>(a.Wo),
+                                  static_cast<uint64_t>(a.B) * a.Ho};
+        const uint64_t strides[2] = {static_cast<uint64_t>(a.C_out) * 2, static_cast<uint64_t>(a.C_out) * 2 * a.Wo};
+        const uint32_t box[3] = {64, static_cast<uint32_t>(a.Wo), 1};
+        if (!tc_tmap_tiled(&tmap_y, bf, 3, a.y, dims, strides, box)) return cudaErrorInvalidValue;
+    }
+    static std::mutex attr_mu;
+    static bool attr_done[64];
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
+    {
+        std::lock_guard<std::mutex> lk(attr_mu);
+        if (!attr_done[dev]) {
+            e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemMax);
+            if (e != cudaSuccess) return e;
+            attr_done[dev] = true;
+        }
+    }
+    cudaLaunchConfig_t cfg{};
+    cfg.gridDim = dim3(static_cast<unsigned>(hp.grid));
+    cfg.blockDim = dim3(kWarps * 32);
+    cfg.dynamicSmemBytes = static_cast<size_t>(hp.bytes) + 1024;
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kern, a, tmap_x, tmap_w, tmap_y, hp);
+}
+
+}  // namespace
+
+// Taken only when the halo plan's column tile is at least as wide as the
+// im2col GEMM's: a narrower one multiplies the MMAs (each reads its A
+// operand again) and loads every halo once per column tile, which measured
+// slower on ResNet-50's stage-2 3x3 layer (BN 64 halo 76.8 us against BN 128
+// im2col 61 us at batch 256).
+bool halo_applies(const ConvArgs &a, int im2col_bn)
+{
+    HaloPlan p;
+    int bn;
+    return halo_plan(a, device_sms_or_default(), &p, &bn) && bn >= im2col_bn;
+}
+
+// The halo GEMM of a bf16 layer on its decoded weights W[C_out][K] (the
+// caller has checked halo_applies).
+cudaError_t halo_gemm(const ConvArgs &a, const void *W, cudaStream_t st)
+{
+    int sms = 0;
+    cudaError_t e = device_sm_count(&sms);
+    if (e != cudaSuccess) return e;
+    HaloPlan hp;
+    int bn = 0;
+    if (!halo_plan(a, sms, &hp, &bn)) return cudaErrorInvalidValue;
+    const __nv_bfloat16 *w = static_cast<const __nv_bfloat16 *>(W);
+    // 3x3 kernels (the ResNet shapes) get the unrolled tap loop
+    const bool k3 = a.KH == 3 && a.KW == 3;
+    if (bn == 64) return k3 ? halo_launch_bn<64, 3>(a, hp, w, st) : halo_launch_bn<64, 0>(a, hp, w, st);
+    if (bn == 128) return k3 ? halo_launch_bn<128, 3>(a, hp, w, st) : halo_launch_bn<128, 0>(a, hp, w, st);
+    return k3 ? halo_launch_bn<256, 3>(a, hp, w, st) : halo_launch_bn<256, 0>(a, hp, w, st);
+}
+
+}  // namespace onexn

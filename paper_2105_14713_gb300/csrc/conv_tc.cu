@@ -908,7 +908,7 @@ struct TmapKey {
     uint64_t ptr;
     uint64_t dims[4], strides[3];
     int32_t lower[2], upper[2];
-    uint32_t box[2], estr[4];
+    uint32_t box[4], estr[4];
 };
 
 struct TmapEntry {
@@ -970,6 +970,40 @@ bool tmap_2d(CUtensorMap *m, CUtensorMapDataType type, int elem, const void *ptr
 }
 
 }  // namespace
+
+PFN_cuTensorMapEncodeIm2col_v12000 encode_im2col_fn_public() { return encode_im2col_fn(); }
+
+// Tiled tensor map of rank 2..4 with the 128-byte swizzle and zero fill
+// outside the tensor, cached like the others.  dims / box innermost first;
+// strides[i] is the byte stride of dimension i + 1.
+bool tc_tmap_tiled(CUtensorMap *m, CUtensorMapDataType type, int rank, const void *ptr, const uint64_t *dims,
+                   const uint64_t *strides, const uint32_t *box)
+{
+    auto enc_t = encode_tiled_fn();
+    if (!enc_t || rank < 2 || rank > 4) return false;
+    cuuint64_t d[4], s[3];
+    cuuint32_t b[4], estr[4] = {1, 1, 1, 1};
+    TmapKey k;
+    std::memset(&k, 0, sizeof k);
+    k.kind = 2 + static_cast<uint32_t>(rank);
+    k.type = static_cast<uint32_t>(type);
+    k.ptr = reinterpret_cast<uint64_t>(ptr);
+    for (int i = 0; i < rank; ++i) {
+        d[i] = dims[i];
+        b[i] = box[i];
+        k.dims[i] = dims[i];
+        k.box[i] = box[i];
+        if (i + 1 < rank) {
+            s[i] = strides[i];
+            k.strides[i] = strides[i];
+        }
+    }
+    return tmap_cached(k, m, [&](CUtensorMap *mm) {
+        return enc_t(mm, type, static_cast<cuuint32_t>(rank), const_cast<void *>(ptr), d, s, b, estr,
+                     CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                     CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+    });
+}
 
 // A 1x1, stride-1, unpadded layer reads x as a [B*H*W][C] matrix; any other
 // layer reads x[B][H][W][C] through an im2col view.
@@ -1200,6 +1234,10 @@ cudaError_t gemm_typed(const ConvArgs &a, const void *workspace, size_t ws_bytes
                    ? static_cast<void *>(static_cast<unsigned char *>(const_cast<void *>(workspace)) + wb)
                    : nullptr;
     const int bn = tc_bn(a, dtype);
+    // stride-1 spatial bf16 layers whose output rows fill the M tile: the
+    // halo form loads each activation once per tile instead of once per tap
+    if constexpr (!Tr::kSplit)
+        if (halo_applies(a, bn)) return halo_gemm(a, W, st);
     if (bn == 64) return launch_bn<Tr, 64>(a, W, W_lo, sk, st);
     if (bn == 128) return launch_bn<Tr, 128>(a, W, W_lo, sk, st);
     return launch_bn<Tr, 256>(a, W, W_lo, sk, st);

@@ -66,6 +66,14 @@ __device__ __forceinline__ void tma_load_im2col_4d(uint32_t dst_smem, const void
         "h"(off_h)
         : "memory");
 }
+// TMA 3-D tiled store shared -> global (bulk async group of this thread).
+__device__ __forceinline__ void tma_store_3d(const void *tmap, int c0, int c1, int c2, uint32_t src_smem)
+{
+    asm volatile("cp.async.bulk.tensor.3d.global.shared::cta.bulk_group [%0, {%1, %2, %3}], [%4];\n" ::"l"(
+                     reinterpret_cast<uint64_t>(tmap)),
+                 "r"(c0), "r"(c1), "r"(c2), "r"(src_smem)
+                 : "memory");
+}
 // TMA tiled store shared -> global (bulk async group of this thread).
 __device__ __forceinline__ void tma_store_2d(const void *tmap, int c0, int c1, uint32_t src_smem)
 {
