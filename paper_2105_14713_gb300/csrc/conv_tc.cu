@@ -78,6 +78,13 @@ struct TcBf16 {
     static constexpr int kKStep = 16;              // K per MMA
     static constexpr CUtensorMapDataType kTmap = CU_TENSOR_MAP_DATA_TYPE_BFLOAT16;
     static constexpr int kWarps = 6;
+    static constexpr int kMT = 1;                  // 128-row halves per tile
+};
+// bf16 with 256-row tiles: the two 128-row halves have their own
+// accumulators and A tiles and share every B tile, so a K chunk moves
+// 2 x 16 KB of A and one B tile for twice the multiply-adds
+struct TcBf16W : TcBf16 {
+    static constexpr int kMT = 2;
 };
 struct TcF32 {
     using T = float;
@@ -86,6 +93,7 @@ struct TcF32 {
     static constexpr int kKStep = 8;
     static constexpr CUtensorMapDataType kTmap = CU_TENSOR_MAP_DATA_TYPE_FLOAT32;
     static constexpr int kWarps = 10;
+    static constexpr int kMT = 1;
 };
 
 constexpr int kSmemMax = 232448;      // dynamic shared memory per CTA (opt-in maximum)
@@ -97,17 +105,18 @@ constexpr int kMinSplitIters = 4;     // stream-K: at least this many chunk iter
 // Stream-K moves partial tiles through global memory and makes a finisher
 // wait for them; on GB300 that pays only when a tile's own K loop is long:
 // from 16 chunks per tile for fp32 (three tf32 MMAs per chunk) and 32 for
-// bf16, measured on batch-1 MobileNet-V2 and ResNet-50 layers.
-constexpr int sk_min_chunks(bool split) { return split ? 16 : 32; }
+// bf16, measured on batch-1 MobileNet-V2 and ResNet-50 layers; 256-row bf16
+// tiles do twice the work per chunk and are fewer, from 8 chunks.
+constexpr int sk_min_chunks(bool split, int MT = 1) { return split ? 16 : (MT > 1 ? 8 : 32); }
 
-// one partial slot (128 x BN fp32) per CTA
-constexpr size_t sk_partial_bytes(int BN) { return static_cast<size_t>(kPlanCTAs) * kBM * BN * 4; }
+// one partial slot (128 MT x BN fp32) per CTA
+constexpr size_t sk_partial_bytes(int BN, int MT = 1) { return static_cast<size_t>(kPlanCTAs) * kBM * MT * BN * 4; }
 
 constexpr int pow2_at_least(int v, int p = 32) { return p >= v ? p : pow2_at_least(v, 2 * p); }
 
 template <typename Tr, int BN>
 struct TcLayout {
-    static constexpr int kA = kBM * kRowBytes;                       // 16 KB
+    static constexpr int kA = Tr::kMT * kBM * kRowBytes;             // 16 KB per 128-row half
     static constexpr int kB = BN * kRowBytes;                        // 8/16/32 KB
     static constexpr int kStage = kA + (Tr::kSplit ? 2 * kB : kB);   // [A | B_hi | B_lo]
     static constexpr int kTx = kStage;                               // bytes the TMA brings
@@ -129,14 +138,17 @@ struct TcLayout {
     // as many accumulator buffers as fit next to the A ring (up to 4): the
     // MMA of tile i + kAcc waits for the epilogue of tile i, so layers with
     // few chunks per tile need several to keep the tensor core busy
-    static constexpr int kAccFit = (512 - kARing) / BN;
+    static constexpr int kAccCols = Tr::kMT * BN;                   // one accumulator: both halves
+    static constexpr int kAccFit = (512 - kARing) / kAccCols;
     static constexpr int kAcc = kAccFit > kAccMax ? kAccMax : kAccFit;
-    static constexpr int kTmemCols = pow2_at_least(kAcc * BN + kARing);
+    static constexpr int kTmemCols = pow2_at_least(kAcc * kAccCols + kARing);
     // a stream-K tile has at most kMaxParts parts besides the finisher's (as
     // many 128 x BN fp32 tiles as the stage ring's bytes), which bounds the
     // additions in the finisher's epilogue
-    static constexpr int kSlotBytes = kBM * BN * 4;
-    static constexpr int kMaxParts = kS * kStage / kSlotBytes;
+    static constexpr int kSlotBytes = Tr::kMT * kBM * BN * 4;
+    // 256-row tiles: the finisher reads its parts from L2 atom by atom, so
+    // their number is not bound by the stage ring; four keep the split fine
+    static constexpr int kMaxParts = Tr::kMT > 1 ? 4 : kS * kStage / kSlotBytes;
     static_assert(kS >= 2, "ring too small");
     static_assert(kMaxParts >= 1, "stream-K parts");
     static_assert(kAlloc <= kSmemMax, "shared memory");
@@ -380,11 +392,18 @@ tc_conv_kernel(const ConvArgs a, const __grid_constant__ CUtensorMap tmap_x,
             TcSeg sg;
             while (!failed && it.next(sg)) {
                 const int tm = static_cast<int>(sched.div_tn.div(sg.tile)), tn = sg.tile - tm * n_tn;
-                // first output pixel of the tile -> its traversal start (w, h, n)
-                const int p0 = tm * kBM;
-                const int b0 = static_cast<int>(sched.div_hw.div(p0)), r0 = p0 - b0 * hw;
-                const int oh0 = static_cast<int>(sched.div_wo.div(r0)), ow0 = r0 - oh0 * a.Wo;
-                const int w0 = ow0 * a.sw - a.pw, h0 = oh0 * a.sh - a.ph;
+                // first output pixel of each 128-row half -> its traversal start (w, h, n)
+                const int p0 = tm * (kBM * Tr::kMT);
+                int hw0[Tr::kMT], hh0[Tr::kMT], hb0[Tr::kMT];
+#pragma unroll
+                for (int hf = 0; hf < Tr::kMT; ++hf) {
+                    const int ph = p0 + hf * kBM;
+                    const int b0 = static_cast<int>(sched.div_hw.div(ph)), r0 = ph - b0 * hw;
+                    const int oh0 = static_cast<int>(sched.div_wo.div(r0)), ow0 = r0 - oh0 * a.Wo;
+                    hw0[hf] = ow0 * a.sw - a.pw;
+                    hh0[hf] = oh0 * a.sh - a.ph;
+                    hb0[hf] = b0;
+                }
                 // chunk c0 -> tap (kh, kw) and channel offset
                 const int tap = static_cast<int>(sched.div_cchunk.div(sg.c0));
                 int cc0 = (sg.c0 - tap * n_cchunk) * Tr::kBK, k0tap = tap * a.C;
@@ -405,12 +424,16 @@ tc_conv_kernel(const ConvArgs a, const __grid_constant__ CUtensorMap tmap_x,
                         tc::mbar_arrive_expect_tx(bar_full + 8 * st, b_tx);
                     } else {
                         tc::mbar_arrive_expect_tx(bar_full + 8 * st, L::kA + b_tx);
-                        if (a_tiled)
-                            tc::tma_load_2d(sa, &tmap_x, cc0, p0, bar_full + 8 * st);
-                        else
-                            tc::tma_load_im2col_4d(sa, &tmap_x, cc0, w0, h0, b0,
-                                                   static_cast<uint16_t>(kw * a.dw), static_cast<uint16_t>(kh * a.dh),
-                                                   bar_full + 8 * st);
+#pragma unroll
+                        for (int hf = 0; hf < Tr::kMT; ++hf) {
+                            const uint32_t dst = sa + hf * (kBM * kRowBytes);
+                            if (a_tiled)
+                                tc::tma_load_2d(dst, &tmap_x, cc0, p0 + hf * kBM, bar_full + 8 * st);
+                            else
+                                tc::tma_load_im2col_4d(dst, &tmap_x, cc0, hw0[hf], hh0[hf], hb0[hf],
+                                                       static_cast<uint16_t>(kw * a.dw),
+                                                       static_cast<uint16_t>(kh * a.dh), bar_full + 8 * st);
+                        }
                     }
                     if (load_b) {
                         tc::tma_load_2d(sb, &tmap_w, k0tap + cc0, tn * BN, bar_full + 8 * st);
@@ -439,7 +462,7 @@ tc_conv_kernel(const ConvArgs a, const __grid_constant__ CUtensorMap tmap_x,
                     abort_now(); failed = true; break;
                 }
                 tc::fence_after_sync();
-                const uint32_t d_tmem = tmem + acc * BN;
+                const uint32_t d_tmem = tmem + acc * L::kAccCols;   // half hf at d_tmem + hf * BN
                 for (int c = sg.c0; c < sg.c1; ++c, ++item) {
                     const int st = item % L::kS;
                     if (!mbar_wait(bar_ready + 8 * st, (item / L::kS) & 1)) {
@@ -454,7 +477,7 @@ tc_conv_kernel(const ConvArgs a, const __grid_constant__ CUtensorMap tmap_x,
                         constexpr uint32_t idesc = tc::idesc_tf32_f32(kBM, BN);
                         const uint64_t bld = tc::desc_kmajor_sw128(sbm + L::kB);
                         // A slot of this chunk: x_hi columns, then x_lo 32 columns on
-                        const uint32_t a_hi = tmem + L::kAcc * BN + (item & 1) * 64;
+                        const uint32_t a_hi = tmem + L::kAcc * L::kAccCols + (item & 1) * 64;
 #pragma unroll
                         for (int kk = 0; kk < Tr::kBK / Tr::kKStep; ++kk) {
                             tc::mma_tf32_ta(d_tmem, a_hi + 8 * kk, bd + 2 * kk, idesc, !(first && kk == 0));
@@ -464,9 +487,13 @@ tc_conv_kernel(const ConvArgs a, const __grid_constant__ CUtensorMap tmap_x,
                     } else {
                         constexpr uint32_t idesc = tc::idesc_bf16_f32(kBM, BN);
                         const uint64_t ad = tc::desc_kmajor_sw128(sa);
+                        constexpr uint32_t kHalfDesc = kBM * kRowBytes / 16;   // next half's A tile
 #pragma unroll
                         for (int kk = 0; kk < Tr::kBK / Tr::kKStep; ++kk)
-                            tc::mma_bf16(d_tmem, ad + 2 * kk, bd + 2 * kk, idesc, !(first && kk == 0));
+#pragma unroll
+                            for (int hf = 0; hf < Tr::kMT; ++hf)
+                                tc::mma_bf16(d_tmem + hf * BN, ad + hf * kHalfDesc + 2 * kk, bd + 2 * kk, idesc,
+                                             !(first && kk == 0));
                     }
                     tc::commit(bar_empty + 8 * st);
                 }
@@ -490,7 +517,7 @@ tc_conv_kernel(const ConvArgs a, const __grid_constant__ CUtensorMap tmap_x,
         if constexpr (Tr::kSplit) {
             const int q = warp & 3;
             const int row = 32 * q + lane;
-            const uint32_t lane_base = tmem + (static_cast<uint32_t>(32 * q) << 16) + L::kAcc * BN;
+            const uint32_t lane_base = tmem + (static_cast<uint32_t>(32 * q) << 16) + L::kAcc * L::kAccCols;
             const int hw = a.Ho * a.Wo;
             int64_t item = 0;
             bool failed = false;
@@ -501,7 +528,7 @@ tc_conv_kernel(const ConvArgs a, const __grid_constant__ CUtensorMap tmap_x,
                 int pb = -1, poh = 0, pow_ = 0;
                 if (dw_mode) {
                     const int tm = static_cast<int>(sched.div_tn.div(sg.tile));
-                    const int p = tm * kBM + row;
+                    const int p = tm * kBM * Tr::kMT + row;
                     if (p < a.P_pix) {
                         pb = static_cast<int>(sched.div_hw.div(p));
                         const int r = p - pb * hw;
@@ -607,8 +634,12 @@ tc_conv_kernel(const ConvArgs a, const __grid_constant__ CUtensorMap tmap_x,
         using T = typename Tr::T;
         constexpr int kAtomCols = kRowBytes / static_cast<int>(sizeof(T));
         constexpr int kAtoms = BN / kAtomCols;
+        // atoms of the whole accumulator: half hf's atoms follow half hf-1's
+        // in the TMEM columns (half hf at column hf * BN), so atom `at` of
+        // the accumulator is columns at * kAtomCols .. + kAtomCols - 1
+        constexpr int kGA = kAtoms * Tr::kMT;
         constexpr int kLd = kAtomCols / 32;               // tcgen05.ld x32 per atom
-        constexpr int kSlotF4 = BN / 4 * kBM;            // float4 per partial slot
+        constexpr int kSlotF4 = BN / 4 * kBM * Tr::kMT;  // float4 per partial slot
         const int q = warp & 3;                      // TMEM lanes 32q .. 32q+31
         const int row = 32 * q + lane;               // pixel row of the tile
         const bool leader = (warp == kEpiWarp0) && lane == 0;
@@ -626,7 +657,7 @@ tc_conv_kernel(const ConvArgs a, const __grid_constant__ CUtensorMap tmap_x,
             if (!epi_all(mbar_wait(bar_tfull + 8 * acc, (si / L::kAcc) & 1))) { abort_now(); break; }
             tc::fence_after_sync();
             const int tm = static_cast<int>(sched.div_tn.div(sg.tile)), tn = sg.tile - tm * n_tn;
-            const uint32_t t_acc = tmem + (static_cast<uint32_t>(32 * q) << 16) + acc * BN;
+            const uint32_t t_acc = tmem + (static_cast<uint32_t>(32 * q) << 16) + acc * L::kAccCols;
             // read the accumulator columns of atom `at`; release the TMEM after the last
             auto issue_atom = [&](int at, uint32_t (&r)[kLd][32]) {
 #pragma unroll
@@ -643,14 +674,14 @@ tc_conv_kernel(const ConvArgs a, const __grid_constant__ CUtensorMap tmap_x,
                 uint32_t r[2][kLd][32];
                 issue_atom(0, r[0]);
                 tc::ld_wait();
-                if (kAtoms == 1) release_acc();
+                if (kGA == 1) release_acc();
 #pragma unroll
-                for (int at = 0; at < kAtoms; ++at) {
-                    if (at + 1 < kAtoms) issue_atom(at + 1, r[(at + 1) & 1]);
+                for (int at = 0; at < kGA; ++at) {
+                    if (at + 1 < kGA) issue_atom(at + 1, r[(at + 1) & 1]);
                     body(at, r[at & 1]);
-                    if (at + 1 < kAtoms) {
+                    if (at + 1 < kGA) {
                         tc::ld_wait();
-                        if (at + 2 == kAtoms) release_acc();
+                        if (at + 2 == kGA) release_acc();
                     }
                 }
             };
@@ -658,7 +689,7 @@ tc_conv_kernel(const ConvArgs a, const __grid_constant__ CUtensorMap tmap_x,
             auto load_atom = [&](int at, uint32_t (&r)[kLd][32]) {
                 issue_atom(at, r);
                 tc::ld_wait();
-                if (at == kAtoms - 1) release_acc();
+                if (at == kGA - 1) release_acc();
             };
             // bias / ReLU / convert the row's atom values f and store the
             // warp's 32 rows of the atom: each warp has its own two staging
@@ -679,7 +710,9 @@ tc_conv_kernel(const ConvArgs a, const __grid_constant__ CUtensorMap tmap_x,
                 }
                 tc::named_bar(1, 128);
             };
-            auto emit_atom = [&](int at, float (&f)[kAtomCols]) {
+            auto emit_atom = [&](int ga, float (&f)[kAtomCols]) {
+                const int at = ga % kAtoms;                           // atom within the half
+                const int row0 = (tm * Tr::kMT + ga / kAtoms) * kBM;  // first pixel row of the half
                 const int col0 = tn * BN + at * kAtomCols;
                 if (col0 >= a.C_out) {               // the whole atom lies past y's columns: no work,
                     ++n_emit;                        // but an (empty) commit group keeps the count
@@ -693,7 +726,7 @@ tc_conv_kernel(const ConvArgs a, const __grid_constant__ CUtensorMap tmap_x,
                 // the residual row of this atom (16-byte chunks inside y only)
                 const uint4 *res = nullptr;
                 if constexpr (kRes) {
-                    const int pix = tm * kBM + row;
+                    const int pix = row0 + row;
                     if (pix < a.P_pix)
                         res = reinterpret_cast<const uint4 *>(static_cast<const T *>(a.residual) +
                                                               static_cast<int64_t>(pix) * a.C_out + col0);
@@ -741,7 +774,7 @@ tc_conv_kernel(const ConvArgs a, const __grid_constant__ CUtensorMap tmap_x,
                 // above), so that "at most one group pending" always means
                 // buf is free
                 if (lane == 0) {
-                    tc::tma_store_2d(&tmap_y, col0, tm * kBM + 32 * q, wbuf);
+                    tc::tma_store_2d(&tmap_y, col0, row0 + 32 * q, wbuf);
                     tc::bulk_commit();
                 }
             };
@@ -750,7 +783,7 @@ tc_conv_kernel(const ConvArgs a, const __grid_constant__ CUtensorMap tmap_x,
                 // ---- split mode: the item's accumulator -> its partial slot ----
                 float4 *mine = reinterpret_cast<float4 *>(sched.partials) + static_cast<int64_t>(sg.slot) * kSlotF4;
 #pragma unroll 1
-                for (int at = 0; at < kAtoms; ++at) {
+                for (int at = 0; at < kGA; ++at) {
                     uint32_t r[kLd][32];
                     load_atom(at, r);
 #pragma unroll
@@ -785,7 +818,7 @@ tc_conv_kernel(const ConvArgs a, const __grid_constant__ CUtensorMap tmap_x,
                 // a lower CTA: accumulator -> own partial slot, then the flag
                 float4 *mine = reinterpret_cast<float4 *>(sched.partials) + static_cast<int64_t>(blockIdx.x) * kSlotF4;
 #pragma unroll 1
-                for (int at = 0; at < kAtoms; ++at) {
+                for (int at = 0; at < kGA; ++at) {
                     uint32_t r[kLd][32];
                     load_atom(at, r);
 #pragma unroll
@@ -1100,7 +1133,8 @@ cudaError_t launch_bn(const ConvArgs &a, const typename Tr::T *W, const typename
     if (e != cudaSuccess) return e;
     TcSched sc{};
     sc.n_tn = (a.C_out + BN - 1) / BN;
-    sc.n_tiles = ((a.P_pix + kBM - 1) / kBM) * sc.n_tn;
+    constexpr int kTileM = kBM * Tr::kMT;
+    sc.n_tiles = ((a.P_pix + kTileM - 1) / kTileM) * sc.n_tn;
     const int n_cchunk = (a.C + Tr::kBK - 1) / Tr::kBK;
     sc.n_chunks = a.KH * a.KW * n_cchunk;
     sc.div_tn = FastDiv(static_cast<uint32_t>(sc.n_tn));
@@ -1123,7 +1157,7 @@ cudaError_t launch_bn(const ConvArgs &a, const typename Tr::T *W, const typename
         sc.partials = split_partials;
         const int items = sc.n_tiles * split_s;
         grid = items < sms ? items : sms;
-    } else if (sk_space && sc.n_tiles % G && sc.n_chunks >= sk_min_chunks(Tr::kSplit)) {
+    } else if (sk_space && sc.n_tiles % G && sc.n_chunks >= sk_min_chunks(Tr::kSplit, Tr::kMT)) {
         const int dp = (sc.n_tiles / G) * G, skt = sc.n_tiles - dp;
         const int64_t iters = static_cast<int64_t>(skt) * sc.n_chunks;
         int need = (sc.n_chunks + L::kMaxParts - 1) / L::kMaxParts;
@@ -1135,7 +1169,7 @@ cudaError_t launch_bn(const ConvArgs &a, const typename Tr::T *W, const typename
             sc.sk_tiles = skt;
             sc.sk_ctas = gs;
             sc.partials = static_cast<float *>(sk_space);
-            sc.flags = reinterpret_cast<int *>(static_cast<unsigned char *>(sk_space) + sk_partial_bytes(BN));
+            sc.flags = reinterpret_cast<int *>(static_cast<unsigned char *>(sk_space) + sk_partial_bytes(BN, Tr::kMT));
         }
     }
     sc.b_resident = (sc.n_chunks == 1 && sc.n_tn == 1 && sc.sk_tiles == 0 && sc.split_s == 0) ? 1 : 0;
@@ -1185,6 +1219,31 @@ int tc_bn(const ConvArgs &a, int dtype)
     return best;
 }
 
+// The im2col GEMM's tile.  Where the L2 -> SM stream of A and B tiles binds
+// (stride-1 spatial bf16 layers with a long K loop: ~54 B per SM cycle on
+// ResNet-50's stage-2 to -4 3x3 layers) and the 128-row plan takes 128
+// columns, tiles of 256 rows (two 128-row halves sharing each B tile) move
+// a quarter fewer bytes per multiply-add (measured in the ResNet-50 stack:
+// stage-4 3x3 55.5 -> 48.6 us, stage-2 3x3 60.7 -> 58.2 us).  Not for 1x1 or
+// strided layers, nor short K loops (stage-2 1x1 512 -> 128 over 8 chunks
+// 51.5 -> 65.3 us, stage-2 stride-2 3x3 69.4 -> 79.3 us: the larger
+// epilogue per tile and the stream-K fixup outweigh the bytes), nor at 256
+// columns: one 2 x 256-column accumulator fills the tensor memory, so every
+// tile's (and stream-K piece's) epilogue stalls the next tile's MMAs
+// (stage-3 3x3 46.8 -> 62.5 us).
+struct TcPlanTile {
+    int bn, mt;
+};
+constexpr int kWideMinChunks = 16;
+TcPlanTile tc_plan_tile(const ConvArgs &a, int dtype)
+{
+    const int bn = tc_bn(a, dtype);
+    const int n_chunks = a.KH * a.KW * ((a.C + TcBf16::kBK - 1) / TcBf16::kBK);
+    const bool spatial_s1 = a.KH * a.KW > 1 && a.sh == 1 && a.sw == 1;
+    if (dtype == ONEXN_BF16 && bn == 128 && spatial_s1 && n_chunks >= kWideMinChunks) return {128, 2};
+    return {bn, 1};
+}
+
 size_t round256(size_t v) { return (v + 255) & ~static_cast<size_t>(255); }
 
 // decoded weights: bf16 C_out * K values; fp32 C_out * K values twice (hi, lo)
@@ -1197,7 +1256,8 @@ size_t weights_bytes(const ConvArgs &a, int dtype)
 // stream-K space after the weights: the partial slots, then the flags
 size_t sk_bytes(const ConvArgs &a, int dtype)
 {
-    return sk_partial_bytes(tc_bn(a, dtype)) + round256(kPlanCTAs * sizeof(int));
+    const TcPlanTile pt = tc_plan_tile(a, dtype);
+    return sk_partial_bytes(pt.bn, pt.mt) + round256(kPlanCTAs * sizeof(int));
 }
 
 template <typename Tr>
@@ -1211,9 +1271,11 @@ cudaError_t decode_typed(const ConvArgs &a, void *workspace, size_t ws_bytes, cu
     const size_t wb = weights_bytes(a, Tr::kSplit ? ONEXN_F32 : ONEXN_BF16);
     int *flags = nullptr;
     const int dtype = Tr::kSplit ? ONEXN_F32 : ONEXN_BF16;
-    if (ws_bytes >= wb + sk_bytes(a, dtype))
+    if (ws_bytes >= wb + sk_bytes(a, dtype)) {
+        const TcPlanTile pt = tc_plan_tile(a, dtype);
         flags = reinterpret_cast<int *>(static_cast<unsigned char *>(workspace) + wb +
-                                        sk_partial_bytes(tc_bn(a, dtype)));
+                                        sk_partial_bytes(pt.bn, pt.mt));
+    }
     const dim3 grid(static_cast<unsigned>((K + kDecodeCols - 1) / kDecodeCols), a.C_out / a.N,
                     (a.N + kDecodeRows - 1) / kDecodeRows);
     bsr_decode_kernel<T><<<grid, kDecodeCols, 0, st>>>(a.P, a.I, static_cast<const T *>(a.D), a.N, a.t, K, W, W_lo,
@@ -1233,11 +1295,14 @@ cudaError_t gemm_typed(const ConvArgs &a, const void *workspace, size_t ws_bytes
     void *sk = ws_bytes >= wb + sk_bytes(a, dtype)
                    ? static_cast<void *>(static_cast<unsigned char *>(const_cast<void *>(workspace)) + wb)
                    : nullptr;
-    const int bn = tc_bn(a, dtype);
+    const TcPlanTile pt = tc_plan_tile(a, dtype);
+    const int bn = pt.bn;
     // stride-1 spatial bf16 layers whose output rows fill the M tile: the
     // halo form loads each activation once per tile instead of once per tap
-    if constexpr (!Tr::kSplit)
+    if constexpr (!Tr::kSplit) {
         if (halo_applies(a, bn)) return halo_gemm(a, W, st);
+        if (pt.mt == 2) return launch_bn<TcBf16W, 128>(a, W, W_lo, sk, st);
+    }
     if (bn == 64) return launch_bn<Tr, 64>(a, W, W_lo, sk, st);
     if (bn == 128) return launch_bn<Tr, 128>(a, W, W_lo, sk, st);
     return launch_bn<Tr, 256>(a, W, W_lo, sk, st);

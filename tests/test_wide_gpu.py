@@ -1,0 +1,81 @@
+"""GPU parity of the im2col GEMM on 256-row tiles against the fp64 oracle
+(Eq. 6 / Eq. 7).
+
+Stride-1 spatial bf16 layers with a K loop of 16 or more 64-channel
+chunks, for which the 128-row plan takes 128-column tiles (more than 76
+pixel tiles, so at least ~10k output pixels), run the tensor-core GEMM on
+tiles of 256 output pixels: two 128-row halves with their own accumulators
+and A tiles share every B tile.  The cases cover a last tile whose second
+half is partly or wholly past the output, fewer output channels than the
+column tile, several rounds with a ragged last one split across CTAs
+(stream-K), and the residual + ReLU6 epilogue; a strided and a 1x1 layer of
+the same size check the boundary of the choice (128-row tiles).  Checked on 2000 seeded output pixels spread over every image,
+plus every pixel of the last tile.  Tolerance: 4e-3 = 2^-8 output rounding
+on bf16-rounded inputs, normalised by sum |w x| + |b|."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2105_14713_gb300 import onexn as ox
+from paper_2105_14713_gb300 import workloads as wl
+from paper_2105_14713_gb300.layer import PrunedConv2d
+from tests.gpu_util import TOL_BF16_ROUNDED, norm_err, run_layer
+
+pytestmark = pytest.mark.gpu
+
+L = wl.ConvLayer
+
+WIDE_GEOMS = [
+    # name, B, H, W, C_in, C_out, KH, KW, stride, pad, N
+    ("3x3_c128", 16, 28, 28, 128, 128, 3, 3, 1, 1, 16),      # 12544 pixels = 49 tiles of 256
+    ("3x3_half_partly", 13, 28, 28, 128, 128, 3, 3, 1, 1, 16),  # last tile: second half 80 of 128 rows
+    ("3x3_half_empty", 17, 24, 24, 128, 128, 3, 3, 1, 1, 16),   # last tile: second half wholly past y
+    ("3x3_cout96", 16, 28, 28, 128, 96, 3, 3, 1, 1, 8),      # 96 of 128 columns
+    ("3x3_cout512_rounds", 200, 7, 7, 128, 512, 3, 3, 1, 1, 16),  # 156 tiles: a ragged second round
+    ("3x3_s2_128rows", 16, 56, 56, 128, 128, 3, 3, 2, 1, 16),   # strided: 128-row tiles
+    ("1x1_k1024_128rows", 64, 14, 14, 1024, 128, 1, 1, 1, 0, 8),  # 1x1: 128-row tiles
+]
+
+
+def _pixels(layer, seed):
+    """2000 seeded pixels plus the whole last 256-row tile."""
+    rng = np.random.default_rng(seed)
+    last = np.arange((layer.pixels - 1) // 256 * 256, layer.pixels)
+    return np.unique(np.concatenate([rng.choice(layer.pixels, 2000, replace=False), last]))
+
+
+@pytest.mark.parametrize("geom", WIDE_GEOMS, ids=[g[0] for g in WIDE_GEOMS])
+@pytest.mark.parametrize("rate", [0.0, 0.7])
+def test_wide_tiles_match_oracle(geom, rate):
+    name, B, H, W, Ci, Co, KH, KW, s, p, N = geom
+    layer = L(name, B, H, W, Ci, Co, KH, KW, s, p, 1, N=N, rate=rate, dtype="bf16", seed=Ci + Co + B)
+    pix = _pixels(layer, B)
+    y, yr, a, conv = run_layer(layer, relu=True, algo=ox.ONEXN_ALGO_TC, pixels=pix)
+    assert conv.algo((B, H, W, Ci), ox.ONEXN_ALGO_TC) == "tc"
+    assert norm_err(y, yr, a) <= TOL_BF16_ROUNDED
+    # again with the decoded weights resident: bitwise the same
+    x = wl.activations(layer).to(torch.bfloat16).cuda()
+    y1 = conv(x, relu=True, algo=ox.ONEXN_ALGO_TC)
+    y2 = conv(x, relu=True, algo=ox.ONEXN_ALGO_TC)
+    torch.cuda.synchronize()
+    assert torch.equal(y1, y2)
+
+
+def test_wide_tiles_residual_relu6():
+    layer = L("wide_res", 16, 28, 28, 128, 128, 3, 3, 1, 1, 1, N=16, rate=0.5, dtype="bf16", seed=13)
+    W, b = wl.weights(layer).numpy(), wl.bias(layer).numpy()
+    conv = PrunedConv2d(W, 16, 0.5, bias=b, padding=1, dtype="bf16")
+    x = wl.activations(layer).to(torch.bfloat16).cuda()
+    rng = np.random.default_rng(9)
+    r = torch.from_numpy((3 * rng.standard_normal((16, 28, 28, 128))).astype(np.float32)).to(torch.bfloat16).cuda()
+    y = conv(x, relu="relu6", algo=ox.ONEXN_ALGO_TC, residual=r)
+    torch.cuda.synchronize()
+    pix = _pixels(layer, 9)
+    mask, _ = oracle.prune(W, 16, 0.5, ox.ONEXN_GRAN_TAP)
+    r_pix = r.float().cpu().numpy().reshape(-1, 128)[pix]
+    ref, absacc = oracle.conv_masked(x.float().cpu().numpy(), oracle.round_bf16(W), mask, b, 16, (1, 1), (1, 1),
+                                     relu="relu6", pixels=pix, residual=r_pix, want_abs=True)
+    got = y.float().cpu().numpy().reshape(-1, 128)[pix].astype(np.float64)
+    assert norm_err(got, ref, absacc) <= TOL_BF16_ROUNDED
+    assert (ref == 6).any() and (ref == 0).any()
