@@ -66,7 +66,7 @@ namespace {
 
 constexpr int kProdWarp = 0;
 constexpr int kMmaWarp = 1;
-constexpr int kEpiWarp0 = 2;          // warps 2..5
+constexpr int kEpiWarp0 = 2;          // warps 2..5 (fp32), 2..9 (bf16)
 constexpr int kSplitWarp0 = 6;        // warps 6..9 (fp32 only)
 constexpr int kBM = 128;              // pixels per tile (UMMA M)
 constexpr int kRowBytes = 128;        // bytes of K per tile row: one 128-byte swizzle row
@@ -77,7 +77,12 @@ struct TcBf16 {
     static constexpr int kBK = 64;                 // channels per chunk
     static constexpr int kKStep = 16;              // K per MMA
     static constexpr CUtensorMapDataType kTmap = CU_TENSOR_MAP_DATA_TYPE_BFLOAT16;
-    static constexpr int kWarps = 6;
+    // warps: producer, MMA, and eight epilogue warps, two per TMEM lane
+    // quarter taking every other 64-column atom: an epilogue warp is bound
+    // by its own latencies (~0.5 us per 128 x 64 atom), so a second warp per
+    // quarter doubles the output rate of tiles with short K loops
+    static constexpr int kWarps = 10;
+    static constexpr int kEpiWarps = 8;
     static constexpr int kMT = 1;                  // 128-row halves per tile
 };
 // bf16 with 256-row tiles: the two 128-row halves have their own
@@ -92,7 +97,8 @@ struct TcF32 {
     static constexpr int kBK = 32;
     static constexpr int kKStep = 8;
     static constexpr CUtensorMapDataType kTmap = CU_TENSOR_MAP_DATA_TYPE_FLOAT32;
-    static constexpr int kWarps = 10;
+    static constexpr int kWarps = 10;              // warps 6-9 split x into tf32 parts
+    static constexpr int kEpiWarps = 4;
     static constexpr int kMT = 1;
 };
 
@@ -120,8 +126,10 @@ struct TcLayout {
     static constexpr int kB = BN * kRowBytes;                        // 8/16/32 KB
     static constexpr int kStage = kA + (Tr::kSplit ? 2 * kB : kB);   // [A | B_hi | B_lo]
     static constexpr int kTx = kStage;                               // bytes the TMA brings
-    // output staging: per epilogue warp two buffers of 32 rows x one 128-byte column atom
-    static constexpr int kOutBytes = 4 * 2 * 32 * kRowBytes;
+    // output staging: per epilogue warp buffers of 32 rows x one 128-byte
+    // column atom, two per warp with four epilogue warps, one with eight
+    static constexpr int kOutBufs = Tr::kEpiWarps == 4 ? 2 : 1;
+    static constexpr int kOutBytes = Tr::kEpiWarps * kOutBufs * 32 * kRowBytes;
     static constexpr int kFixed = 1024 + kOutBytes + BN * 4 + (3 * 6 + 2 * 4 + 2) * 8 + 16;
     static constexpr int kS = ((kSmemMax - kFixed) / kStage) > 6 ? 6 : ((kSmemMax - kFixed) / kStage);
     static constexpr int kOut = kS * kStage;
@@ -213,15 +221,15 @@ bsr_decode_kernel(const int32_t *__restrict__ P, const int32_t *__restrict__ I, 
     }
 }
 
-// barrier over the 4 epilogue warps that also returns the AND of `ok`
-__device__ __forceinline__ bool epi_all(bool ok)
+// barrier over the epilogue warps (n threads) that also returns the AND of `ok`
+__device__ __forceinline__ bool epi_all(bool ok, int n)
 {
     uint32_t r;
     asm volatile(
         "{\n\t.reg .pred p, q;\n\tsetp.ne.u32 p, %1, 0;\n\t"
-        "bar.red.and.pred q, 1, 128, p;\n\tselp.u32 %0, 1, 0, q;\n\t}\n"
+        "bar.red.and.pred q, 1, %2, p;\n\tselp.u32 %0, 1, 0, q;\n\t}\n"
         : "=r"(r)
-        : "r"(ok ? 1u : 0u)
+        : "r"(ok ? 1u : 0u), "r"(n)
         : "memory");
     return r != 0;
 }
@@ -356,7 +364,7 @@ tc_conv_kernel(const ConvArgs a, const __grid_constant__ CUtensorMap tmap_x,
         }
         for (int b = 0; b < kAccMax; ++b) {
             mbar_init(bar_tfull + 8 * b, 1);
-            mbar_init(bar_tempty + 8 * b, 128);
+            mbar_init(bar_tempty + 8 * b, 32 * Tr::kEpiWarps);
         }
         mbar_init(bar_drain, 1);
         fence_mbar_init();
@@ -504,7 +512,7 @@ tc_conv_kernel(const ConvArgs a, const __grid_constant__ CUtensorMap tmap_x,
             if (!mbar_wait(bar_drain, 0)) abort_now();
         }
         __syncwarp();
-    } else if (warp >= kSplitWarp0) {
+    } else if (Tr::kSplit && warp >= kSplitWarp0) {
         // ============================ split (fp32) ========================
         // Thread i of warp w owns pixel row 32*(w%4) + i of the tile: it reads
         // the row's 32 fp32 values from the swizzled A tile (logical 16-byte
@@ -643,6 +651,12 @@ tc_conv_kernel(const ConvArgs a, const __grid_constant__ CUtensorMap tmap_x,
         const int q = warp & 3;                      // TMEM lanes 32q .. 32q+31
         const int row = 32 * q + lane;               // pixel row of the tile
         const bool leader = (warp == kEpiWarp0) && lane == 0;
+        // eight epilogue warps: warp group eg (of nG) takes atoms eg, eg + nG, ...
+        constexpr int kEpiThreads = 32 * Tr::kEpiWarps;
+        constexpr int nG = Tr::kEpiWarps / 4;
+        const int ew = warp - kEpiWarp0;             // this warp among the epilogue warps
+        const int eg = ew / 4;
+        const int et = 32 * ew + lane;               // this thread among the epilogue threads
         const uint32_t sout = base + L::kOut;
         float *sbias = reinterpret_cast<float *>(smem + L::kBias);
         const int64_t W_sk = static_cast<int64_t>(sched.sk_tiles) * sched.n_chunks;
@@ -652,9 +666,9 @@ tc_conv_kernel(const ConvArgs a, const __grid_constant__ CUtensorMap tmap_x,
         TcSeg sg;
         for (int si = 0; it.next(sg); ++si) {
             const int acc = si % L::kAcc;
-            // all four warps take the same decision (tcgen05.ld and the named
-            // barriers below need all of them)
-            if (!epi_all(mbar_wait(bar_tfull + 8 * acc, (si / L::kAcc) & 1))) { abort_now(); break; }
+            // all epilogue warps take the same decision (tcgen05.ld and the
+            // named barriers below need all of them)
+            if (!epi_all(mbar_wait(bar_tfull + 8 * acc, (si / L::kAcc) & 1), kEpiThreads)) { abort_now(); break; }
             tc::fence_after_sync();
             const int tm = static_cast<int>(sched.div_tn.div(sg.tile)), tn = sg.tile - tm * n_tn;
             const uint32_t t_acc = tmem + (static_cast<uint32_t>(32 * q) << 16) + acc * L::kAccCols;
@@ -667,21 +681,39 @@ tc_conv_kernel(const ConvArgs a, const __grid_constant__ CUtensorMap tmap_x,
                 tc::fence_before_sync();
                 mbar_arrive(bar_tempty + 8 * acc);       // accumulator free for segment si + kAcc
             };
-            // the atoms in order, the TMEM loads of atom at+1 in flight while
-            // atom at is processed; the accumulator is released as soon as
-            // its last columns are in registers
+            // four epilogue warps: the atoms in order, the TMEM loads of atom
+            // at+1 in flight while atom at is processed; eight: each warp its
+            // own atoms (every nG-th), the other warp of its lane quarter
+            // covering its latencies.  A warp releases the accumulator as
+            // soon as its last columns are in registers (at once if it has
+            // none).
             auto run_atoms = [&](auto &&body) {
-                uint32_t r[2][kLd][32];
-                issue_atom(0, r[0]);
-                tc::ld_wait();
-                if (kGA == 1) release_acc();
+                if constexpr (nG == 1) {
+                    uint32_t r[2][kLd][32];
+                    issue_atom(0, r[0]);
+                    tc::ld_wait();
+                    if (kGA == 1) release_acc();
 #pragma unroll
-                for (int at = 0; at < kGA; ++at) {
-                    if (at + 1 < kGA) issue_atom(at + 1, r[(at + 1) & 1]);
-                    body(at, r[at & 1]);
-                    if (at + 1 < kGA) {
-                        tc::ld_wait();
-                        if (at + 2 == kGA) release_acc();
+                    for (int at = 0; at < kGA; ++at) {
+                        if (at + 1 < kGA) issue_atom(at + 1, r[(at + 1) & 1]);
+                        body(at, r[at & 1]);
+                        if (at + 1 < kGA) {
+                            tc::ld_wait();
+                            if (at + 2 == kGA) release_acc();
+                        }
+                    }
+                } else {
+                    if (eg >= kGA) release_acc();
+#pragma unroll
+                    for (int i = 0; i < (kGA + nG - 1) / nG; ++i) {
+                        const int at = i * nG + eg;
+                        if (at < kGA) {
+                            uint32_t r[kLd][32];
+                            issue_atom(at, r);
+                            tc::ld_wait();
+                            if (at + nG >= kGA) release_acc();
+                            body(at, r);
+                        }
                     }
                 }
             };
@@ -689,7 +721,7 @@ tc_conv_kernel(const ConvArgs a, const __grid_constant__ CUtensorMap tmap_x,
             auto load_atom = [&](int at, uint32_t (&r)[kLd][32]) {
                 issue_atom(at, r);
                 tc::ld_wait();
-                if (at == kGA - 1) release_acc();
+                if (at + nG >= kGA) release_acc();
             };
             // bias / ReLU / convert the row's atom values f and store the
             // warp's 32 rows of the atom: each warp has its own two staging
@@ -701,14 +733,14 @@ tc_conv_kernel(const ConvArgs a, const __grid_constant__ CUtensorMap tmap_x,
             // CTA often share it, and the global load is a full memory
             // latency on the epilogue's critical path)
             auto stage_bias = [&]() {
-                if (tn == staged_tn) return;         // uniform across the four warps
+                if (tn == staged_tn) return;         // uniform across the epilogue warps
                 staged_tn = tn;
-                tc::named_bar(1, 128);               // the previous tile's reads are done
-                for (int c = row; c < BN; c += 128) {
+                tc::named_bar(1, kEpiThreads);       // the previous tile's reads are done
+                for (int c = et; c < BN; c += kEpiThreads) {
                     const int o = tn * BN + c;
                     sbias[c] = (a.bias && o < a.C_out) ? __ldg(a.bias + o) : 0.f;
                 }
-                tc::named_bar(1, 128);
+                tc::named_bar(1, kEpiThreads);
             };
             auto emit_atom = [&](int ga, float (&f)[kAtomCols]) {
                 const int at = ga % kAtoms;                           // atom within the half
@@ -719,10 +751,17 @@ tc_conv_kernel(const ConvArgs a, const __grid_constant__ CUtensorMap tmap_x,
                     if (lane == 0) tc::bulk_commit();
                     return;
                 }
-                const int buf = n_emit++ & 1;        // alternate across atoms and tiles
-                if (lane == 0) tc::bulk_wait_read1();   // this warp's store two atoms back has read buf
+                // this warp's staging buffers alternate across its atoms and
+                // tiles (two with four epilogue warps); the store that last
+                // used the buffer has read it
+                const int buf = L::kOutBufs == 2 ? (n_emit & 1) : 0;
+                ++n_emit;
+                if (lane == 0) {
+                    if constexpr (L::kOutBufs == 2) tc::bulk_wait_read1();
+                    else tc::bulk_wait_read0();
+                }
                 __syncwarp();
-                const uint32_t wbuf = sout + (q * 2 + buf) * (32 * kRowBytes);
+                const uint32_t wbuf = sout + (ew * L::kOutBufs + buf) * (32 * kRowBytes);
                 // the residual row of this atom (16-byte chunks inside y only)
                 const uint4 *res = nullptr;
                 if constexpr (kRes) {
@@ -782,8 +821,9 @@ tc_conv_kernel(const ConvArgs a, const __grid_constant__ CUtensorMap tmap_x,
             if (sched.split_s > 0) {
                 // ---- split mode: the item's accumulator -> its partial slot ----
                 float4 *mine = reinterpret_cast<float4 *>(sched.partials) + static_cast<int64_t>(sg.slot) * kSlotF4;
+                if (eg >= kGA) release_acc();
 #pragma unroll 1
-                for (int at = 0; at < kGA; ++at) {
+                for (int at = eg; at < kGA; at += nG) {
                     uint32_t r[kLd][32];
                     load_atom(at, r);
 #pragma unroll
@@ -817,8 +857,9 @@ tc_conv_kernel(const ConvArgs a, const __grid_constant__ CUtensorMap tmap_x,
             if (static_cast<int>(blockIdx.x) != b_last) {
                 // a lower CTA: accumulator -> own partial slot, then the flag
                 float4 *mine = reinterpret_cast<float4 *>(sched.partials) + static_cast<int64_t>(blockIdx.x) * kSlotF4;
+                if (eg >= kGA) release_acc();
 #pragma unroll 1
-                for (int at = 0; at < kGA; ++at) {
+                for (int at = eg; at < kGA; at += nG) {
                     uint32_t r[kLd][32];
                     load_atom(at, r);
 #pragma unroll
@@ -832,7 +873,7 @@ tc_conv_kernel(const ConvArgs a, const __grid_constant__ CUtensorMap tmap_x,
                 }
                 __threadfence();
                 tc::fence_proxy_async_global();      // the finisher reads the slot with TMA
-                tc::named_bar(1, 128);
+                tc::named_bar(1, kEpiThreads);
                 if (leader) tc::st_release_gpu(sched.flags + blockIdx.x, 1);
                 continue;
             }
@@ -847,7 +888,7 @@ tc_conv_kernel(const ConvArgs a, const __grid_constant__ CUtensorMap tmap_x,
                         if (clock64() - t0 > (1ll << 31)) { ok = false; break; }
                 }
             }
-            if (!epi_all(ok)) { abort_now(); break; }
+            if (!epi_all(ok, kEpiThreads)) { abort_now(); break; }
             stage_bias();
             const float4 *parts = reinterpret_cast<const float4 *>(sched.partials) +
                                   static_cast<int64_t>(b_first) * kSlotF4;
@@ -867,7 +908,7 @@ tc_conv_kernel(const ConvArgs a, const __grid_constant__ CUtensorMap tmap_x,
                 }
                 emit_atom(at, f);
             });
-            tc::named_bar(1, 128);                   // every part has been read
+            tc::named_bar(1, kEpiThreads);           // every part has been read
             if (leader)
                 for (int k = b_first; k < b_last; ++k) sched.flags[k] = 0;   // ready for the next launch
         }
