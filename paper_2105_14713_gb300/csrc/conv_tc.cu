@@ -258,9 +258,10 @@ struct TcSched {
     int n_tiles, n_tn, n_chunks;
     int dp_tiles, sk_tiles, sk_ctas;
     int split_s;
-    // one K chunk and one column tile: every tile multiplies the same B, which
-    // is loaded once into stage 0's B region and stays there; the stages
-    // then carry A only
+    // every tile of a CTA multiplies the same B (one column tile, or a grid
+    // that is a multiple of their number) and its K loop fits in the stage
+    // ring: chunk c's B is loaded once into stage c's B region and stays
+    // there; the stages then carry A only
     int b_resident;
     // divisors of the per-tile / per-segment index arithmetic
     FastDiv div_tn, div_hw, div_wo, div_cchunk, div_kw;
@@ -424,8 +425,9 @@ tc_conv_kernel(const ConvArgs a, const __grid_constant__ CUtensorMap tmap_x,
                     }
                     const uint32_t sa = base + st * L::kStage;
                     const uint32_t sb = sa + L::kA;
-                    // B bytes of this chunk: none when B is resident, after item 0
-                    const bool load_b = !sched.b_resident || item == 0;
+                    // B bytes of this chunk: when B is resident only the CTA's
+                    // first tile loads it, chunk c into stage c's B region
+                    const bool load_b = !sched.b_resident || item < sched.n_chunks;
                     const uint32_t b_tx = load_b ? static_cast<uint32_t>(L::kTx - L::kA) : 0u;
                     if (dw_mode) {
                         // A comes from the split warps' depthwise; only B is loaded
@@ -478,7 +480,8 @@ tc_conv_kernel(const ConvArgs a, const __grid_constant__ CUtensorMap tmap_x,
                     }
                     tc::fence_after_sync();
                     const uint32_t sa = base + st * L::kStage;
-                    const uint32_t sbm = (sched.b_resident ? base : sa) + L::kA;   // this chunk's B
+                    // this chunk's B: the stage's, or resident in stage c's B region
+                    const uint32_t sbm = (sched.b_resident ? base + c * L::kStage : sa) + L::kA;
                     const uint64_t bd = tc::desc_kmajor_sw128(sbm);
                     const uint32_t first = (c == sg.c0) ? 1u : 0u;   // the first chunk overwrites D
                     if constexpr (Tr::kSplit) {
@@ -1213,7 +1216,16 @@ cudaError_t launch_bn(const ConvArgs &a, const typename Tr::T *W, const typename
             sc.flags = reinterpret_cast<int *>(static_cast<unsigned char *>(sk_space) + sk_partial_bytes(BN, Tr::kMT));
         }
     }
-    sc.b_resident = (sc.n_chunks == 1 && sc.n_tn == 1 && sc.sk_tiles == 0 && sc.split_s == 0) ? 1 : 0;
+    // Resident B: when the K loop fits in the stage ring, the column tile
+    // of every tile of a CTA is the same (one column tile, or a grid that is
+    // a multiple of their number, tiles dealt round-robin) and no tile is
+    // split, each CTA loads its column tile's B chunks once, chunk c into
+    // stage c's B region, and the stages then carry A only (ResNet-50's
+    // 1x1 expansions re-read 2-4 B chunks of 32 KB per 128-row tile else).
+    sc.b_resident = (sc.n_chunks <= L::kS && (sc.n_tn == 1 || grid % sc.n_tn == 0) && sc.sk_tiles == 0 &&
+                     sc.split_s == 0)
+                        ? 1
+                        : 0;
     cudaLaunchConfig_t cfg{};
     cfg.gridDim = dim3(grid);
     cfg.blockDim = dim3(Tr::kWarps * 32);

@@ -79,3 +79,32 @@ def test_wide_tiles_residual_relu6():
     got = y.float().cpu().numpy().reshape(-1, 128)[pix].astype(np.float64)
     assert norm_err(got, ref, absacc) <= TOL_BF16_ROUNDED
     assert (ref == 6).any() and (ref == 0).any()
+
+
+RESIDENT_GEOMS = [
+    # name, B, H, W, C_in, C_out, dtype: 1x1 layers whose K loop fits in the stage ring
+    ("bf16_k128_cout512", 64, 28, 28, 128, 512, "bf16"),    # 2 chunks, 2 column tiles of 256 on 152 CTAs
+    ("bf16_k256_cout1024", 128, 14, 14, 256, 1024, "bf16"),  # 4 chunks, 4 column tiles
+    ("bf16_k256_cout768", 128, 14, 14, 256, 768, "bf16"),   # 3 column tiles: 152 CTAs do not divide, B streamed
+    ("f32_k96_cout512", 32, 28, 28, 96, 512, "f32"),        # 3 chunks of 32 channels, hi and lo B parts
+]
+
+
+@pytest.mark.parametrize("geom", RESIDENT_GEOMS, ids=[g[0] for g in RESIDENT_GEOMS])
+def test_resident_weights_multi_chunk(geom):
+    """1x1 layers with a short K loop: each CTA keeps its column tile's B
+    chunks in the stage ring (loaded by its first tile) when every tile it
+    takes has the same column tile; checked on sampled pixels of every
+    image, and bitwise equal on a second call with the weights resident."""
+    name, B, H, W, Ci, Co, dt = geom
+    layer = L(name, B, H, W, Ci, Co, 1, 1, 1, 0, 1, N=16, rate=0.7, dtype=dt, seed=Co)
+    pix = _pixels(layer, Co)
+    y, yr, a, conv = run_layer(layer, relu=True, algo=ox.ONEXN_ALGO_TC, pixels=pix)
+    tol = TOL_BF16_ROUNDED if dt == "bf16" else 1e-5
+    assert norm_err(y, yr, a) <= tol
+    x = wl.activations(layer)
+    x = (x if dt == "f32" else x.to(torch.bfloat16)).cuda()
+    y1 = conv(x, relu=True, algo=ox.ONEXN_ALGO_TC)
+    y2 = conv(x, relu=True, algo=ox.ONEXN_ALGO_TC)
+    torch.cuda.synchronize()
+    assert torch.equal(y1, y2)
