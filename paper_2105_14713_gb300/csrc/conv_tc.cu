@@ -1284,16 +1284,22 @@ int tc_bn(const ConvArgs &a, int dtype)
 // columns: one 2 x 256-column accumulator fills the tensor memory, so every
 // tile's (and stream-K piece's) epilogue stalls the next tile's MMAs
 // (stage-3 3x3 46.8 -> 62.5 us).
+// Fewer than two rounds of 256-row tiles leave a ragged round that stream-K
+// has to split, which pays only on long K loops (cfg2's 3x3 128 -> 128 at
+// batch 64, 196 tiles of 18 chunks: 24.3 -> 27.9 us on 256-row tiles).
 struct TcPlanTile {
     int bn, mt;
 };
-constexpr int kWideMinChunks = 16;
+constexpr int kWideMinChunks = 16, kWideFewTilesMinChunks = 32;
 TcPlanTile tc_plan_tile(const ConvArgs &a, int dtype)
 {
     const int bn = tc_bn(a, dtype);
     const int n_chunks = a.KH * a.KW * ((a.C + TcBf16::kBK - 1) / TcBf16::kBK);
     const bool spatial_s1 = a.KH * a.KW > 1 && a.sh == 1 && a.sw == 1;
-    if (dtype == ONEXN_BF16 && bn == 128 && spatial_s1 && n_chunks >= kWideMinChunks) return {128, 2};
+    const int64_t wide_tiles = ((static_cast<int64_t>(a.P_pix) + 2 * kBM - 1) / (2 * kBM)) * ((a.C_out + 127) / 128);
+    const bool enough = wide_tiles >= 2 * static_cast<int64_t>(device_sms_or_default()) ||
+                        n_chunks >= kWideFewTilesMinChunks;
+    if (dtype == ONEXN_BF16 && bn == 128 && spatial_s1 && n_chunks >= kWideMinChunks && enough) return {128, 2};
     return {bn, 1};
 }
 

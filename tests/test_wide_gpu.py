@@ -1,17 +1,19 @@
 """GPU parity of the im2col GEMM on 256-row tiles against the fp64 oracle
 (Eq. 6 / Eq. 7).
 
-Stride-1 spatial bf16 layers with a K loop of 16 or more 64-channel
-chunks, for which the 128-row plan takes 128-column tiles (more than 76
-pixel tiles, so at least ~10k output pixels), run the tensor-core GEMM on
-tiles of 256 output pixels: two 128-row halves with their own accumulators
-and A tiles share every B tile.  The cases cover a last tile whose second
-half is partly or wholly past the output, fewer output channels than the
-column tile, several rounds with a ragged last one split across CTAs
-(stream-K), and the residual + ReLU6 epilogue; a strided and a 1x1 layer of
-the same size check the boundary of the choice (128-row tiles).  Checked on 2000 seeded output pixels spread over every image,
-plus every pixel of the last tile.  Tolerance: 4e-3 = 2^-8 output rounding
-on bf16-rounded inputs, normalised by sum |w x| + |b|."""
+Stride-1 spatial bf16 layers with a K loop of 16 or more 64-channel chunks,
+for which the 128-row plan takes 128-column tiles (more than 76 pixel
+tiles, so at least ~10k output pixels), and with either two full rounds of
+256-row tiles or 32 or more chunks, run the tensor-core GEMM on tiles of
+256 output pixels: two 128-row halves with their own accumulators and A
+tiles share every B tile.  The cases (3x3 over 256 channels: 36 chunks)
+cover a last tile whose second half is partly or wholly past the output,
+fewer output channels than the column tile, a ragged round split across
+CTAs (stream-K), and the residual + ReLU6 epilogue; a strided and a 1x1
+layer of the same size check the boundary of the choice (128-row tiles).
+Checked on 2000 seeded output pixels spread over every image, plus every
+pixel of the last tile.  Tolerance: 4e-3 = 2^-8 output rounding on
+bf16-rounded inputs, normalised by sum |w x| + |b|."""
 import numpy as np
 import pytest
 import torch
@@ -28,11 +30,11 @@ L = wl.ConvLayer
 
 WIDE_GEOMS = [
     # name, B, H, W, C_in, C_out, KH, KW, stride, pad, N
-    ("3x3_c128", 16, 28, 28, 128, 128, 3, 3, 1, 1, 16),      # 12544 pixels = 49 tiles of 256
-    ("3x3_half_partly", 13, 28, 28, 128, 128, 3, 3, 1, 1, 16),  # last tile: second half 80 of 128 rows
-    ("3x3_half_empty", 17, 24, 24, 128, 128, 3, 3, 1, 1, 16),   # last tile: second half wholly past y
-    ("3x3_cout96", 16, 28, 28, 128, 96, 3, 3, 1, 1, 8),      # 96 of 128 columns
-    ("3x3_cout512_rounds", 200, 7, 7, 128, 512, 3, 3, 1, 1, 16),  # 156 tiles: a ragged second round
+    ("3x3_c256", 16, 28, 28, 256, 128, 3, 3, 1, 1, 16),      # 12544 pixels = 49 tiles of 256
+    ("3x3_half_partly", 13, 28, 28, 256, 128, 3, 3, 1, 1, 16),  # last tile: second half 80 of 128 rows
+    ("3x3_half_empty", 17, 24, 24, 256, 128, 3, 3, 1, 1, 16),   # last tile: second half wholly past y
+    ("3x3_cout96", 16, 28, 28, 256, 96, 3, 3, 1, 1, 8),      # 96 of 128 columns
+    ("3x3_cout512_rounds", 200, 7, 7, 256, 512, 3, 3, 1, 1, 16),  # 156 tiles: a ragged second round
     ("3x3_s2_128rows", 16, 56, 56, 128, 128, 3, 3, 2, 1, 16),   # strided: 128-row tiles
     ("1x1_k1024_128rows", 64, 14, 14, 1024, 128, 1, 1, 1, 0, 8),  # 1x1: 128-row tiles
 ]
@@ -63,7 +65,7 @@ def test_wide_tiles_match_oracle(geom, rate):
 
 
 def test_wide_tiles_residual_relu6():
-    layer = L("wide_res", 16, 28, 28, 128, 128, 3, 3, 1, 1, 1, N=16, rate=0.5, dtype="bf16", seed=13)
+    layer = L("wide_res", 16, 28, 28, 256, 128, 3, 3, 1, 1, 1, N=16, rate=0.5, dtype="bf16", seed=13)
     W, b = wl.weights(layer).numpy(), wl.bias(layer).numpy()
     conv = PrunedConv2d(W, 16, 0.5, bias=b, padding=1, dtype="bf16")
     x = wl.activations(layer).to(torch.bfloat16).cuda()
