@@ -1273,20 +1273,19 @@ int tc_bn(const ConvArgs &a, int dtype)
 }
 
 // The im2col GEMM's tile.  Where the L2 -> SM stream of A and B tiles binds
-// (stride-1 spatial bf16 layers with a long K loop: ~54 B per SM cycle on
-// ResNet-50's stage-2 to -4 3x3 layers) and the 128-row plan takes 128
-// columns, tiles of 256 rows (two 128-row halves sharing each B tile) move
-// a quarter fewer bytes per multiply-add (measured in the ResNet-50 stack:
-// stage-4 3x3 55.5 -> 48.6 us, stage-2 3x3 60.7 -> 58.2 us).  Not for 1x1 or
-// strided layers, nor short K loops (stage-2 1x1 512 -> 128 over 8 chunks
-// 51.5 -> 65.3 us, stage-2 stride-2 3x3 69.4 -> 79.3 us: the larger
-// epilogue per tile and the stream-K fixup outweigh the bytes), nor at 256
-// columns: one 2 x 256-column accumulator fills the tensor memory, so every
-// tile's (and stream-K piece's) epilogue stalls the next tile's MMAs
-// (stage-3 3x3 46.8 -> 62.5 us).
-// Fewer than two rounds of 256-row tiles leave a ragged round that stream-K
-// has to split, which pays only on long K loops (cfg2's 3x3 128 -> 128 at
-// batch 64, 196 tiles of 18 chunks: 24.3 -> 27.9 us on 256-row tiles).
+// (bf16 layers with a long K loop: ~50-54 B per SM cycle on ResNet-50's
+// stage-2 to -4 3x3 layers) and the 128-row plan takes 128 columns, tiles of
+// 256 rows (two 128-row halves sharing each B tile) move a quarter fewer
+// bytes per multiply-add (measured in the ResNet-50 stack: stage-4 3x3
+// 55.5 -> 48.6 us, its stride-2 3x3 56.7 -> 49.3 us, stage-2 3x3 60.7 ->
+// 58.2 us).  Taken for K loops of 32 or more chunks, and for stride-1
+// spatial layers from 16 chunks; not for shorter K loops of 1x1 or strided
+// layers (stage-2 1x1 512 -> 128 over 8 chunks 51.5 -> 65.3 us, stage-2
+// stride-2 3x3 over 18 chunks 69.4 -> 79.3 us: the larger epilogue per tile
+// and the stream-K fixup outweigh the bytes), nor at 256 columns: one
+// 2 x 256-column accumulator fills the tensor memory, so every tile's (and
+// stream-K piece's) epilogue stalls the next tile's MMAs (stage-3 3x3 46.8
+// -> 62.5 us).
 struct TcPlanTile {
     int bn, mt;
 };
@@ -1299,7 +1298,8 @@ TcPlanTile tc_plan_tile(const ConvArgs &a, int dtype)
     const int64_t wide_tiles = ((static_cast<int64_t>(a.P_pix) + 2 * kBM - 1) / (2 * kBM)) * ((a.C_out + 127) / 128);
     const bool enough = wide_tiles >= 2 * static_cast<int64_t>(device_sms_or_default()) ||
                         n_chunks >= kWideFewTilesMinChunks;
-    if (dtype == ONEXN_BF16 && bn == 128 && spatial_s1 && n_chunks >= kWideMinChunks && enough) return {128, 2};
+    const bool wide = (spatial_s1 && n_chunks >= kWideMinChunks && enough) || n_chunks >= kWideFewTilesMinChunks;
+    if (dtype == ONEXN_BF16 && bn == 128 && wide) return {128, 2};
     return {bn, 1};
 }
 

@@ -1,16 +1,18 @@
 """GPU parity of the im2col GEMM on 256-row tiles against the fp64 oracle
 (Eq. 6 / Eq. 7).
 
-Stride-1 spatial bf16 layers with a K loop of 16 or more 64-channel chunks,
-for which the 128-row plan takes 128-column tiles (more than 76 pixel
-tiles, so at least ~10k output pixels), and with either two full rounds of
-256-row tiles or 32 or more chunks, run the tensor-core GEMM on tiles of
-256 output pixels: two 128-row halves with their own accumulators and A
-tiles share every B tile.  The cases (3x3 over 256 channels: 36 chunks)
-cover a last tile whose second half is partly or wholly past the output,
-fewer output channels than the column tile, a ragged round split across
-CTAs (stream-K), and the residual + ReLU6 epilogue; a strided and a 1x1
-layer of the same size check the boundary of the choice (128-row tiles).
+bf16 layers for which the 128-row plan takes 128-column tiles (more than 76
+pixel tiles, so at least ~10k output pixels) run the tensor-core GEMM on
+tiles of 256 output pixels (two 128-row halves with their own accumulators
+and A tiles sharing every B tile) when their K loop has 32 or more
+64-channel chunks, or, for stride-1 spatial layers, 16 or more chunks and
+two full rounds of 256-row tiles.  The cases (3x3 over 256 channels: 36
+chunks) cover a last tile whose second half is partly or wholly past the
+output, fewer output channels than the column tile, a ragged round split
+across CTAs (stream-K), a stride-2 layer and a 1x1 layer over 2048
+channels, and the residual + ReLU6 epilogue; a strided 18-chunk and a 1x1
+16-chunk layer of the same size check the boundary of the choice (128-row
+tiles).
 Checked on 2000 seeded output pixels spread over every image, plus every
 pixel of the last tile.  Tolerance: 4e-3 = 2^-8 output rounding on
 bf16-rounded inputs, normalised by sum |w x| + |b|."""
@@ -35,7 +37,9 @@ WIDE_GEOMS = [
     ("3x3_half_empty", 17, 24, 24, 256, 128, 3, 3, 1, 1, 16),   # last tile: second half wholly past y
     ("3x3_cout96", 16, 28, 28, 256, 96, 3, 3, 1, 1, 8),      # 96 of 128 columns
     ("3x3_cout512_rounds", 200, 7, 7, 256, 512, 3, 3, 1, 1, 16),  # 156 tiles: a ragged second round
-    ("3x3_s2_128rows", 16, 56, 56, 128, 128, 3, 3, 2, 1, 16),   # strided: 128-row tiles
+    ("3x3_s2_c256", 16, 56, 56, 256, 128, 3, 3, 2, 1, 16),   # strided traversal of each half, 36 chunks
+    ("1x1_k2048", 64, 14, 14, 2048, 128, 1, 1, 1, 0, 16),    # plain-matrix A, 32 chunks
+    ("3x3_s2_128rows", 16, 56, 56, 128, 128, 3, 3, 2, 1, 16),   # strided, 18 chunks: 128-row tiles
     ("1x1_k1024_128rows", 64, 14, 14, 1024, 128, 1, 1, 1, 0, 8),  # 1x1: 128-row tiles
 ]
 
