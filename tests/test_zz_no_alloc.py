@@ -6,8 +6,9 @@ that forbid allocation after start-up so that latency stays predictable, or
 a plug-in that only receives pointers from a framework that owns the memory.
 For them the library keeps the tensor-core family's scratch in a fixed 8 MiB
 device array instead of a caller workspace.  These tests call it through the
-C ABI on two layers in a row and then on the first layer again (so it runs
-over what the second left in the shared array), and check each output
+C ABI on three layers in a row (the third a stride-1 3x3 layer that the
+GEMM runs on halo tiles) and then on the first layer again (so it runs over
+what the others left in the shared array), and check each output
 against the fp64 oracle and bit for bit against the regular onexn_conv_fwd
 with a workspace (the same kernels on the same decoded weights and the same
 tile plan).  The file name sorts last so that a run that stops at the first
@@ -50,11 +51,12 @@ def _noalloc(conv, x, relu):
 LAYERS = [
     wl.ConvLayer("na_3x3", 4, 14, 14, 128, 128, 3, 3, 1, 1, 1, N=8, rate=0.5, dtype="bf16", seed=1),
     wl.ConvLayer("na_1x1_s2", 3, 15, 15, 64, 256, 1, 1, 2, 0, 1, N=16, rate=0.7, dtype="bf16", seed=2),
+    wl.ConvLayer("na_3x3_halo", 2, 28, 28, 64, 64, 3, 3, 1, 1, 1, N=16, rate=0.7, dtype="bf16", seed=3),
 ]
 
 
-def test_noalloc_two_layers_then_the_first_again():
-    runs = [(LAYERS[0], True), (LAYERS[1], False), (LAYERS[0], True)]
+def test_noalloc_three_layers_then_the_first_again():
+    runs = [(LAYERS[0], True), (LAYERS[1], False), (LAYERS[2], True), (LAYERS[0], True)]
     for layer, relu in runs:
         conv, x_cpu, x, W, b = _layer_and_input(layer)
         y_na = _noalloc(conv, x, relu)
