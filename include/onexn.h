@@ -426,6 +426,29 @@ onexn_status onexn_conv_algo(const onexn_conv_desc *desc, int N, int64_t t, int 
                              unsigned flags, size_t workspace_bytes, unsigned *algo);
 
 /*
+ * onexn_conv_tc_form -- which form the tensor-core family's GEMM takes for
+ * these arguments (Eq. 6 / Eq. 7 on the decoded weights in every form; they
+ * differ in how the activations reach the tensor cores), without launching:
+ *   ONEXN_GEMM_IM2COL        one TMA im2col tile of 128 output pixels per
+ *                            (tap, 64-channel chunk)
+ *   ONEXN_GEMM_IM2COL_WIDE   the same on tiles of 256 output pixels (two
+ *                            halves sharing each weight tile; bf16)
+ *   ONEXN_GEMM_HALO_RESIDENT stride-1 spatial bf16 layers: tiles of whole
+ *                            output rows, one load of the tile's input rows
+ *                            per channel chunk read by every tap, the column
+ *                            tile's weights kept in shared memory
+ *   ONEXN_GEMM_HALO_STREAMED the same input loads on tiles of 256 positions
+ *                            of the padded output, weights streamed
+ * Reads the current device's SM count (152 when there is no device).
+ * EINVAL as onexn_conv_fwd's shape checks.
+ */
+#define ONEXN_GEMM_IM2COL 0
+#define ONEXN_GEMM_IM2COL_WIDE 1
+#define ONEXN_GEMM_HALO_RESIDENT 2
+#define ONEXN_GEMM_HALO_STREAMED 3
+onexn_status onexn_conv_tc_form(const onexn_conv_desc *desc, int N, int64_t t, int dtype, int *form);
+
+/*
  * onexn_conv_fwd_host -- onexn_conv_fwd on activations in HOST memory:
  * y_host = conv(x_host), with the copies to and from the GPU inside the
  * call.  The batch is cut into chunks of whole images; each chunk is copied

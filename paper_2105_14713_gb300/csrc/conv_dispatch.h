@@ -37,11 +37,15 @@ TcSplitPlan tc_split_plan(int M, int Ncols, int64_t K, int dtype);
 cudaError_t tc_gemm_split(const ConvArgs &a, int dtype, const void *W, const void *W_lo, float *partials,
                           const TcSplitPlan &plan, cudaStream_t st);
 size_t tc_weights_bytes(const ConvArgs &a, int dtype);
-// Halo-tile form of the bf16 GEMM for stride-1 spatial layers (conv_halo.cu):
-// whether it takes the layer (against the im2col GEMM's column tile), and
-// the launch on the decoded weights W[C_out][K].
-bool halo_applies(const ConvArgs &a, int im2col_bn);
-cudaError_t halo_gemm(const ConvArgs &a, const void *W, cudaStream_t st);
+// Forms of the tensor-core GEMM (values of onexn_conv_tc_form).
+enum : int { kGemmIm2col = 0, kGemmIm2colWide = 1, kGemmHaloResident = 2, kGemmHaloStreamed = 3 };
+// Halo-tile forms of the bf16 GEMM for stride-1 spatial layers (conv_halo.cu):
+// which one takes the layer (against the im2col GEMM's column tile;
+// kGemmIm2col for none), and the launch on the decoded weights W[C_out][K].
+int halo_form(const ConvArgs &a, int im2col_bn);
+cudaError_t halo_gemm(const ConvArgs &a, const void *W, int im2col_bn, cudaStream_t st);
+// The form the tensor-core GEMM takes for this layer and dtype (conv_tc.cu).
+int tc_gemm_form(const ConvArgs &a, int dtype);
 size_t tc_sk_bytes(const ConvArgs &a, int dtype);
 
 namespace detail {

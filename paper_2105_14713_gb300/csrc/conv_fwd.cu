@@ -288,6 +288,17 @@ extern "C" onexn_status onexn_conv_algo(const onexn_conv_desc *desc, int N, int6
     return ONEXN_OK;
 }
 
+extern "C" onexn_status onexn_conv_tc_form(const onexn_conv_desc *desc, int N, int64_t t, int dtype, int *form)
+{
+    onexn::clear_error();
+    if (!form) return fail(ONEXN_EINVAL, "conv_tc_form: form is NULL");
+    onexn::ConvArgs a{};
+    onexn_status st = check_shape(desc, N, t, dtype, 0, &a);
+    if (st != ONEXN_OK) return st;
+    *form = onexn::tc_gemm_form(a, dtype);
+    return ONEXN_OK;
+}
+
 extern "C" onexn_status onexn_conv_workspace_size(const onexn_conv_desc *desc, int N, int64_t t,
                                                   int dtype, unsigned flags, size_t *bytes)
 {

@@ -364,6 +364,300 @@ halo_conv_kernel(const ConvArgs a, const __grid_constant__ CUtensorMap tmap_x,
     }
 }
 
+// ---------------------------------------------------------------------------
+// Streamed-weights form (layers whose column tile of weights does not fit in
+// shared memory next to the halo slots).  The output of an image is laid
+// out in the padded space of Hp = Ho + (KH-1)*dh rows of Wp positions
+// (position (n*Hp + r)*Wp + w is output pixel (n, r, w) when r < Ho and
+// w < Wo, else a dropped row), and the input in the same space (row r,
+// column w = input pixel (r - ph, w - pw)); output position P of tap
+// (kh, kw) reads input position P + kh*dh*Wp + kw*dw.  A tile is 256
+// consecutive positions, two M = 128 halves; it may run across rows and
+// images, so only the padding columns and rows are wasted.  Per 64-channel
+// chunk one TMA im2col load brings its 256 + (KH-1)*dh*Wp + (KW-1)*dw input
+// positions (the traversal continues into the next image, zeros after the
+// last one), and the A operand of (half h, tap) is that buffer viewed from
+// row 128*h + kh*dh*Wp + kw*dw on.  The weights are streamed: one B stage
+// holds one kernel row of taps (3x3) or one tap, 128-byte swizzled, shared
+// by both halves.  MMA warp h issues the MMAs of half h (its own
+// accumulators), so each issuing thread meets one stage wait per kernel row
+// of taps; the epilogue warps (two per TMEM lane quarter, one per half)
+// store their valid rows straight to global memory.
+constexpr int kWRows = 2 * kBM;            // positions per tile
+constexpr int kWEpiWarp0 = 3;
+constexpr int kWWarps = kWEpiWarp0 + 8;    // producer, two MMA warps, eight epilogue warps
+constexpr int kWMaxHalo = 2;
+constexpr int kWMaxStages = 12;
+constexpr int kWAccMax = 4;
+constexpr int kWBarBytes = (2 * kWMaxHalo + 2 * kWMaxStages + 4 * kWAccMax + 2) * 8;
+
+struct WidePlan {
+    int Wp, Hp;                    // padded output width and rows per image
+    int n_cc, n_taps, tps, n_st;   // chunks, taps, taps per B stage, B stages per chunk
+    int n_tn, n_m, grid;           // column tiles, position tiles, CTAs (a multiple of n_tn)
+    int S_h, S_b;                  // halo slots, B stages
+    uint32_t halo_pix, halo_tx, slot_bytes, stage_bytes;
+    uint32_t off_b, off_bias, off_bar, bytes;
+    FastDiv div_img, div_wp;       // Hp*Wp, Wp
+};
+
+template <int BN>
+struct WideTmem {
+    static constexpr int kAccFit = 512 / (2 * BN);
+    static constexpr int kAcc = kAccFit > kWAccMax ? kWAccMax : kAccFit;   // buffers of two halves
+    static constexpr int kCols = pow2_cols(kAcc * 2 * BN);
+};
+
+// KS = 3: 3x3 kernel (a B stage is one kernel row of three taps, unrolled);
+// KS = 0: any kernel shape (one tap per stage).
+template <int BN, int KS>
+__global__ void __launch_bounds__(kWWarps * 32, 1)
+halo_wide_kernel(const ConvArgs a, const __grid_constant__ CUtensorMap tmap_x,
+                 const __grid_constant__ CUtensorMap tmap_w, const WidePlan wp)
+{
+    using TM = WideTmem<BN>;
+    constexpr int kAcc = TM::kAcc;
+    constexpr uint32_t kBTile = BN * kRow;
+    extern __shared__ unsigned char smem_raw[];
+    const uint32_t raw = smem_u32(smem_raw);
+    const uint32_t base = (raw + 1023u) & ~1023u;
+    unsigned char *smem = smem_raw + (base - raw);
+    const uint32_t sH = base;                      // halo slots
+    const uint32_t sB = base + wp.off_b;           // B stages
+    const uint32_t bar_hfull = base + wp.off_bar;
+    const uint32_t bar_hempty = bar_hfull + 8 * kWMaxHalo;
+    const uint32_t bar_bfull = bar_hempty + 8 * kWMaxHalo;
+    const uint32_t bar_bempty = bar_bfull + 8 * kWMaxStages;
+    const uint32_t bar_tfull = bar_bempty + 8 * kWMaxStages;   // [acc][half]
+    const uint32_t bar_tempty = bar_tfull + 16 * kWAccMax;     // [acc][half]
+    const uint32_t bar_drain = bar_tempty + 16 * kWAccMax;     // one per MMA warp
+    uint32_t *holder = reinterpret_cast<uint32_t *>(smem + wp.off_bar + kWBarBytes);
+
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    if (tid == 0) {
+        for (int s = 0; s < kWMaxHalo; ++s) {
+            mbar_init(bar_hfull + 8 * s, 1);
+            mbar_init(bar_hempty + 8 * s, 2);       // both MMA warps commit
+        }
+        for (int s = 0; s < kWMaxStages; ++s) {
+            mbar_init(bar_bfull + 8 * s, 1);
+            mbar_init(bar_bempty + 8 * s, 2);
+        }
+        for (int b = 0; b < 2 * kWAccMax; ++b) {
+            mbar_init(bar_tfull + 8 * b, 1);
+            mbar_init(bar_tempty + 8 * b, 128);     // the four epilogue warps of the half
+        }
+        for (int j = 0; j < 2; ++j) mbar_init(bar_drain + 8 * j, 1);
+        fence_mbar_init();
+    }
+    if (warp == 1) {
+        tc::tmem_alloc(smem_u32(holder), TM::kCols);
+        tc::tmem_relinquish();
+    }
+    tc::fence_before_sync();
+    __syncthreads();
+    tc::fence_after_sync();
+    const uint32_t tmem = *holder;
+    // a programmatic dependent of the previous kernel on the stream: global
+    // memory is touched only after it has completed
+    asm volatile("griddepcontrol.wait;\n" ::: "memory");
+    asm volatile("griddepcontrol.launch_dependents;\n" ::: "memory");
+    auto abort_now = [&]() { atomicOr(a.status, kStatusTimeout); };
+    const int tn = static_cast<int>(blockIdx.x) % wp.n_tn;
+    const int m0 = static_cast<int>(blockIdx.x) / wp.n_tn, m_step = wp.grid / wp.n_tn;
+    const uint32_t img = static_cast<uint32_t>(wp.Hp) * static_cast<uint32_t>(wp.Wp);
+
+    if (warp == 0) {
+        // ============================ producer ============================
+        if (lane == 0) {
+            bool failed = false;
+            int hs = 0, hround = 0, bs = 0, bround = 0;
+            for (int tm = m0; tm < wp.n_m && !failed; tm += m_step) {
+                const uint32_t P0 = static_cast<uint32_t>(tm) * kWRows;
+                const uint32_t n0 = wp.div_img.div(P0), rem = P0 - n0 * img;
+                const uint32_t r0 = wp.div_wp.div(rem), w0 = rem - r0 * static_cast<uint32_t>(wp.Wp);
+                for (int cc = 0; cc < wp.n_cc && !failed; ++cc) {
+                    if (hround >= 1 && !mbar_wait(bar_hempty + 8 * hs, (hround - 1) & 1)) {
+                        failed = true;
+                        break;
+                    }
+                    tc::mbar_arrive_expect_tx(bar_hfull + 8 * hs, wp.halo_tx);
+                    tc::tma_load_im2col_4d(sH + static_cast<uint32_t>(hs) * wp.slot_bytes, &tmap_x, cc * kBK,
+                                           static_cast<int>(w0) - a.pw, static_cast<int>(r0) - a.ph,
+                                           static_cast<int>(n0), 0, 0, bar_hfull + 8 * hs);
+                    if (++hs == wp.S_h) { hs = 0; ++hround; }
+                    for (int st = 0; st < wp.n_st; ++st) {
+                        if (bround >= 1 && !mbar_wait(bar_bempty + 8 * bs, (bround - 1) & 1)) {
+                            failed = true;
+                            break;
+                        }
+                        tc::mbar_arrive_expect_tx(bar_bfull + 8 * bs, wp.stage_bytes);
+                        const uint32_t dst = sB + static_cast<uint32_t>(bs) * wp.stage_bytes;
+                        for (int i = 0; i < wp.tps; ++i)
+                            tc::tma_load_2d(dst + static_cast<uint32_t>(i) * kBTile, &tmap_w,
+                                            (st * wp.tps + i) * a.C + cc * kBK, tn * BN, bar_bfull + 8 * bs);
+                        if (++bs == wp.S_b) { bs = 0; ++bround; }
+                    }
+                }
+            }
+            if (failed) abort_now();
+        }
+        __syncwarp();
+    } else if (warp < kWEpiWarp0) {
+        // ============================== MMA ==============================
+        const int h = warp - 1;                    // the half this warp multiplies
+        if (lane == 0) {
+            constexpr uint32_t idesc = tc::idesc_bf16_f32(kBM, BN);
+            constexpr uint32_t kBDesc = kBTile / 16;                  // descriptor units between B tiles
+            const uint32_t row_step = static_cast<uint32_t>(a.dh * wp.Wp) * (kRow / 16);   // per kh
+            const uint32_t col_step = static_cast<uint32_t>(a.dw) * (kRow / 16);           // per kw
+            const uint32_t half_off = static_cast<uint32_t>(h * kBM) * (kRow / 16);
+            bool failed = false;
+            int hs = 0, hph = 0, bs = 0, bph = 0, k = 0;
+            for (int tm = m0; tm < wp.n_m && !failed; tm += m_step, ++k) {
+                const int acc = k % kAcc, use = k / kAcc;
+                if (use >= 1 && !mbar_wait(bar_tempty + 8 * (2 * acc + h), (use - 1) & 1)) {
+                    failed = true;
+                    break;
+                }
+                tc::fence_after_sync();
+                const uint32_t d_tmem = tmem + static_cast<uint32_t>(2 * acc + h) * BN;
+                for (int cc = 0; cc < wp.n_cc && !failed; ++cc) {
+                    if (!mbar_wait(bar_hfull + 8 * hs, hph)) { failed = true; break; }
+                    tc::fence_after_sync();
+                    const uint64_t hd = tc::desc_kmajor_sw128(sH + static_cast<uint32_t>(hs) * wp.slot_bytes) + half_off;
+                    int kh = 0, kw = 0;                  // tap of the generic path
+                    for (int st = 0; st < wp.n_st; ++st) {
+                        if (!mbar_wait(bar_bfull + 8 * bs, bph)) { failed = true; break; }
+                        tc::fence_after_sync();
+                        const uint64_t bd = tc::desc_kmajor_sw128(sB + static_cast<uint32_t>(bs) * wp.stage_bytes);
+                        const uint32_t first = (cc == 0 && st == 0) ? 0u : 1u;
+                        auto tap_mmas = [&](uint64_t ad, uint64_t b, uint32_t first_acc) {
+                            tc::mma_bf16(d_tmem, ad, b, idesc, first_acc);
+#pragma unroll
+                            for (int kk = 1; kk < kBK / 16; ++kk) tc::mma_bf16(d_tmem, ad + 2 * kk, b + 2 * kk, idesc, 1u);
+                        };
+                        if constexpr (KS > 0) {
+                            const uint64_t ad_row = hd + static_cast<uint32_t>(st) * row_step;
+#pragma unroll
+                            for (int t = 0; t < KS; ++t)
+                                tap_mmas(ad_row + t * col_step, bd + t * kBDesc, t == 0 ? first : 1u);
+                        } else {
+                            tap_mmas(hd + kh * row_step + kw * col_step, bd, first);
+                            if (++kw == a.KW) { kw = 0; ++kh; }
+                        }
+                        tc::commit(bar_bempty + 8 * bs);
+                        if (++bs == wp.S_b) { bs = 0; bph ^= 1; }
+                    }
+                    if (failed) break;
+                    tc::commit(bar_hempty + 8 * hs);
+                    if (++hs == wp.S_h) { hs = 0; hph ^= 1; }
+                }
+                if (failed) break;
+                tc::commit(bar_tfull + 8 * (2 * acc + h));
+            }
+            if (failed) abort_now();
+            // everything this thread issued completes before the TMEM is freed
+            tc::commit(bar_drain + 8 * h);
+            if (!mbar_wait(bar_drain + 8 * h, 0)) abort_now();
+        }
+        __syncwarp();
+    } else {
+        // ============================ epilogue ============================
+        // Warp w (3..10) reads TMEM lane quarter w % 4 of half (w - 3) / 4:
+        // thread (w, i) owns position 128*half + 32*(w % 4) + i of each tile.
+        // Per 64-column atom: read the accumulator, add bias (and
+        // residual), activate, convert to bf16 and store the pixel's 128
+        // bytes when the position is an output pixel.
+        auto epilogue = [&](auto res_c, auto act_c) {
+            constexpr bool kRes = decltype(res_c)::value;
+            constexpr int kAct = decltype(act_c)::value;
+            constexpr int kAtoms = BN / 64;
+            const int h = (warp - kWEpiWarp0) >> 2, q = warp & 3;
+            const int m = h * kBM + 32 * q + lane;
+            float *sbias = reinterpret_cast<float *>(smem + wp.off_bias);
+            const float4 *sb4 = reinterpret_cast<const float4 *>(sbias);
+            for (int c = tid - kWEpiWarp0 * 32; c < BN; c += 256) {     // the column tile's bias, once
+                const int o = tn * BN + c;
+                sbias[c] = (a.bias && o < a.C_out) ? __ldg(a.bias + o) : 0.f;
+            }
+            tc::named_bar(1, 256);
+            __nv_bfloat16 *y = static_cast<__nv_bfloat16 *>(a.y);
+            int k = 0;
+            for (int tm = m0; tm < wp.n_m; tm += m_step, ++k) {
+                const int acc = k % kAcc, use = k / kAcc;
+                if (!mbar_wait(bar_tfull + 8 * (2 * acc + h), use & 1)) { abort_now(); break; }
+                tc::fence_after_sync();
+                const uint32_t P = static_cast<uint32_t>(tm) * kWRows + static_cast<uint32_t>(m);
+                const uint32_t n = wp.div_img.div(P), rem = P - n * img;
+                const uint32_t r = wp.div_wp.div(rem), w = rem - r * static_cast<uint32_t>(wp.Wp);
+                const bool valid = static_cast<int>(n) < a.B && static_cast<int>(r) < a.Ho && static_cast<int>(w) < a.Wo;
+                const int64_t pix = (static_cast<int64_t>(n) * a.Ho + r) * a.Wo + w;
+                const uint32_t t_acc = tmem + (static_cast<uint32_t>(32 * q) << 16) + static_cast<uint32_t>(2 * acc + h) * BN;
+#pragma unroll 1
+                for (int at = 0; at < kAtoms; ++at) {
+                    const int col0 = tn * BN + at * 64;
+                    uint32_t r0[32], r1[32];
+                    tc::ld_32x32b_x32(t_acc + at * 64, r0);
+                    tc::ld_32x32b_x32(t_acc + at * 64 + 32, r1);
+                    tc::ld_wait();
+                    if (at == kAtoms - 1) {
+                        tc::fence_before_sync();
+                        mbar_arrive(bar_tempty + 8 * (2 * acc + h));
+                    }
+                    if (!valid || col0 >= a.C_out) continue;
+                    __nv_bfloat16 *yp = y + pix * a.C_out + col0;
+                    const uint4 *res = nullptr;
+                    if constexpr (kRes)
+                        res = reinterpret_cast<const uint4 *>(static_cast<const __nv_bfloat16 *>(a.residual) +
+                                                              pix * a.C_out + col0);
+#pragma unroll
+                    for (int jj = 0; jj < 8; ++jj) {          // 16-byte chunk jj: columns 8jj .. 8jj+7
+                        if (col0 + 8 * jj >= a.C_out) break;
+                        uint32_t rw[4] = {0u, 0u, 0u, 0u};
+                        if constexpr (kRes) {
+                            const uint4 rv = __ldg(res + jj);
+                            rw[0] = rv.x; rw[1] = rv.y; rw[2] = rv.z; rw[3] = rv.w;
+                        }
+                        const float4 b0 = sb4[at * 16 + 2 * jj], b1 = sb4[at * 16 + 2 * jj + 1];
+                        const float bb[8] = {b0.x, b0.y, b0.z, b0.w, b1.x, b1.y, b1.z, b1.w};
+                        uint32_t wv[4];
+#pragma unroll
+                        for (int e = 0; e < 4; ++e) {
+                            const int c = 8 * jj + 2 * e;
+                            const uint32_t u0 = c < 32 ? r0[c] : r1[c - 32];
+                            const uint32_t u1 = c + 1 < 32 ? r0[c + 1] : r1[c + 1 - 32];
+                            float v0 = __uint_as_float(u0) + bb[2 * e], v1 = __uint_as_float(u1) + bb[2 * e + 1];
+                            if constexpr (kRes) {
+                                v0 += bf16lo(rw[e]);
+                                v1 += bf16hi(rw[e]);
+                            }
+                            wv[e] = pack_bf16x2(activate_c<kAct>(v0), activate_c<kAct>(v1));
+                        }
+                        *reinterpret_cast<uint4 *>(yp + 8 * jj) = make_uint4(wv[0], wv[1], wv[2], wv[3]);
+                    }
+                }
+            }
+        };
+        if (a.residual) {
+            if (a.relu == 2) epilogue(std::true_type{}, std::integral_constant<int, 2>{});
+            else if (a.relu == 1) epilogue(std::true_type{}, std::integral_constant<int, 1>{});
+            else epilogue(std::true_type{}, std::integral_constant<int, 0>{});
+        } else {
+            if (a.relu == 2) epilogue(std::false_type{}, std::integral_constant<int, 2>{});
+            else if (a.relu == 1) epilogue(std::false_type{}, std::integral_constant<int, 1>{});
+            else epilogue(std::false_type{}, std::integral_constant<int, 0>{});
+        }
+    }
+
+    tc::fence_before_sync();
+    __syncthreads();
+    if (warp == 1) {
+        tc::fence_after_sync();
+        tc::tmem_dealloc(tmem, TM::kCols);
+    }
+}
+
 uint32_t round1024(uint64_t v) { return static_cast<uint32_t>((v + 1023) & ~static_cast<uint64_t>(1023)); }
 
 // The halo plan of a bf16 layer, or false when the layer keeps the im2col
@@ -426,11 +720,12 @@ bool halo_plan(const ConvArgs &a, int sms, HaloPlan *out, int *bn_out)
 
 // im2col tensor map of the halo: the traversal's bounding box is the padded
 // image, columns -pw .. W - 1 + pw and rows -ph .. H - 1 + ph (corners
-// innermost first: W, H), so a load of Wp x Rh positions from (-pw, h0 - ph)
-// walks whole padded rows.  A last row block that runs past the padded
-// image continues into the next image's rows (or zeros after the last
-// image); those rows feed only the dropped M rows of the tile.
-bool halo_x_tmap(const ConvArgs &a, const HaloPlan &hp, CUtensorMap *m)
+// innermost first: W, H), so a load of `pixels` positions walks whole
+// padded rows from its start (Wp x Rh positions from (-pw, h0 - ph) for a
+// row block; any position for the streamed form).  A load that runs past
+// the padded image continues into the next image's rows (or zeros after
+// the last image); those rows feed only dropped M rows.
+bool halo_x_tmap(const ConvArgs &a, int Wp, int pixels, CUtensorMap *m)
 {
     auto enc = encode_im2col_fn_public();
     if (!enc) return false;
@@ -439,14 +734,105 @@ bool halo_x_tmap(const ConvArgs &a, const HaloPlan &hp, CUtensorMap *m)
     const cuuint64_t strides[3] = {static_cast<cuuint64_t>(a.C) * 2, static_cast<cuuint64_t>(a.C) * 2 * a.W,
                                    static_cast<cuuint64_t>(a.C) * 2 * a.W * a.H};
     const int lower[2] = {-a.pw, -a.ph};
-    const int upper[2] = {hp.Wp - a.pw - a.W, a.Ho + (a.KH - 1) * a.dh - a.ph - a.H};
+    const int upper[2] = {Wp - a.pw - a.W, a.Ho + (a.KH - 1) * a.dh - a.ph - a.H};
     for (int i = 0; i < 2; ++i)
         if (lower[i] < -128 || lower[i] > 127 || upper[i] < -128 || upper[i] > 127) return false;
     const cuuint32_t estr[4] = {1, 1, 1, 1};
     return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void *>(a.x), dims, strides, lower, upper, kBK,
-               static_cast<cuuint32_t>(hp.Wp * hp.Rh), estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+               static_cast<cuuint32_t>(pixels), estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
                CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+// The streamed-weights plan, or false: strided or 1x1 layers, too many
+// dropped positions (Ho*Wo below 85% of Hp*Wp), more positions per load
+// than one im2col load can walk, or shared memory for fewer than two B
+// stages.  The column tile is 128 (64 when the output channels fit in
+// 64), so that two accumulator buffers of two halves fit in the TMEM.
+bool wide_plan(const ConvArgs &a, int sms, WidePlan *out, int *bn_out)
+{
+    if (a.sh != 1 || a.sw != 1 || a.KH * a.KW == 1 || a.Ho <= 0 || a.Wo <= 0 || a.B <= 0) return false;
+    WidePlan p{};
+    p.Wp = a.Wo + (a.KW - 1) * a.dw;
+    p.Hp = a.Ho + (a.KH - 1) * a.dh;
+    const double fill = static_cast<double>(a.Ho) * a.Wo / (static_cast<double>(p.Hp) * p.Wp);
+    if (fill < kMinRowFill) return false;
+    const int64_t positions = static_cast<int64_t>(a.B) * p.Hp * p.Wp;
+    if (positions + kWRows > INT32_MAX) return false;
+    const int64_t halo = kWRows + static_cast<int64_t>(a.KH - 1) * a.dh * p.Wp + static_cast<int64_t>(a.KW - 1) * a.dw;
+    if (halo > 1024) return false;                        // positions per im2col load
+    p.halo_pix = static_cast<uint32_t>(halo);
+    p.halo_tx = p.halo_pix * kRow;
+    p.slot_bytes = round1024(static_cast<uint64_t>(p.halo_pix) * kRow);
+    p.n_cc = (a.C + kBK - 1) / kBK;
+    p.n_taps = a.KH * a.KW;
+    p.tps = (a.KH == 3 && a.KW == 3) ? 3 : 1;
+    p.n_st = p.n_taps / p.tps;
+    const int bn = a.C_out <= 64 ? 64 : 128;
+    p.stage_bytes = static_cast<uint32_t>(p.tps * bn * kRow);
+    p.S_h = kWMaxHalo;
+    const uint64_t fixed = round1024(static_cast<uint64_t>(bn) * 4) + kWBarBytes + 16 + 1024;
+    const uint64_t halo_bytes = static_cast<uint64_t>(p.S_h) * p.slot_bytes;
+    if (halo_bytes + fixed + 2ull * p.stage_bytes > static_cast<uint64_t>(kSmemMax)) return false;
+    p.S_b = static_cast<int>(std::min<uint64_t>(kWMaxStages, (kSmemMax - fixed - halo_bytes) / p.stage_bytes));
+    p.n_tn = (a.C_out + bn - 1) / bn;
+    if (p.n_tn > sms) return false;
+    p.n_m = static_cast<int>((positions + kWRows - 1) / kWRows);
+    const int64_t tiles = static_cast<int64_t>(p.n_m) * p.n_tn;
+    p.grid = static_cast<int>(std::min<int64_t>(tiles, sms) / p.n_tn * p.n_tn);
+    p.off_b = static_cast<uint32_t>(halo_bytes);
+    p.off_bias = p.off_b + static_cast<uint32_t>(p.S_b) * p.stage_bytes;
+    p.off_bar = p.off_bias + round1024(static_cast<uint64_t>(bn) * 4);
+    p.bytes = p.off_bar + kWBarBytes + 16;
+    if (p.bytes + 1024 > static_cast<uint32_t>(kSmemMax)) return false;
+    p.div_img = FastDiv(static_cast<uint32_t>(p.Hp) * static_cast<uint32_t>(p.Wp));
+    p.div_wp = FastDiv(static_cast<uint32_t>(p.Wp));
+    *out = p;
+    *bn_out = bn;
+    return true;
+}
+
+template <int BN, int KS>
+cudaError_t wide_launch_bn(const ConvArgs &a, const WidePlan &wp, const __nv_bfloat16 *W, cudaStream_t st)
+{
+    auto kern = halo_wide_kernel<BN, KS>;
+    const CUtensorMapDataType bf = CU_TENSOR_MAP_DATA_TYPE_BFLOAT16;
+    const uint64_t K = static_cast<uint64_t>(a.KH) * a.KW * a.C;
+    CUtensorMap tmap_x, tmap_w;
+    // x [B][H][W][C]: one im2col load per 64-channel chunk walks the tile's
+    // halo_pix positions of the padded space from the tile's first one
+    if (!halo_x_tmap(a, wp.Wp, static_cast<int>(wp.halo_pix), &tmap_x)) return cudaErrorInvalidValue;
+    {   // W [C_out][K]: boxes of 64 K x BN rows
+        const uint64_t dims[2] = {K, static_cast<uint64_t>(a.C_out)};
+        const uint64_t strides[1] = {K * 2};
+        const uint32_t box[2] = {kBK, BN};
+        if (!tc_tmap_tiled(&tmap_w, bf, 2, W, dims, strides, box)) return cudaErrorInvalidValue;
+    }
+    static std::mutex attr_mu;
+    static bool attr_done[64];
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
+    {
+        std::lock_guard<std::mutex> lk(attr_mu);
+        if (!attr_done[dev]) {
+            e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemMax);
+            if (e != cudaSuccess) return e;
+            attr_done[dev] = true;
+        }
+    }
+    cudaLaunchConfig_t cfg{};
+    cfg.gridDim = dim3(static_cast<unsigned>(wp.grid));
+    cfg.blockDim = dim3(kWWarps * 32);
+    cfg.dynamicSmemBytes = static_cast<size_t>(wp.bytes) + 1024;
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kern, a, tmap_x, tmap_w, wp);
 }
 
 template <int BN, int KS>
@@ -459,7 +845,7 @@ cudaError_t halo_launch_bn(const ConvArgs &a, const HaloPlan &hp, const __nv_bfl
     // x [B][H][W][C]: one im2col load per 64-channel chunk walks the Wp x Rh
     // halo positions of the tile (columns -pw .. W - 1 + pw of each row,
     // the padding read as zeros)
-    if (!halo_x_tmap(a, hp, &tmap_x)) return cudaErrorInvalidValue;
+    if (!halo_x_tmap(a, hp.Wp, hp.Wp * hp.Rh, &tmap_x)) return cudaErrorInvalidValue;
     {   // W [C_out][K]: boxes of 64 K x BN rows
         const uint64_t dims[2] = {K, static_cast<uint64_t>(a.C_out)};
         const uint64_t strides[1] = {K * 2};
@@ -502,34 +888,45 @@ cudaError_t halo_launch_bn(const ConvArgs &a, const HaloPlan &hp, const __nv_bfl
 
 }  // namespace
 
-// Taken only when the halo plan's column tile is at least as wide as the
-// im2col GEMM's: a narrower one multiplies the MMAs (each reads its A
-// operand again) and loads every halo once per column tile, which measured
-// slower on ResNet-50's stage-2 3x3 layer (BN 64 halo 76.8 us against BN 128
-// im2col 61 us at batch 256).
-bool halo_applies(const ConvArgs &a, int im2col_bn)
+// The halo form of this layer's bf16 GEMM, against the im2col GEMM's
+// column tile: the resident-weights form only when its column tile is at
+// least as wide (a narrower one multiplies the MMAs, each reading its A
+// operand again, and loads every halo once per column tile: measured slower
+// on ResNet-50's stage-2 3x3 layer, BN 64 halo 76.8 us against BN 128
+// im2col 61 us at batch 256); else the streamed-weights form when its plan
+// exists; else none (the im2col GEMM).
+int halo_form(const ConvArgs &a, int im2col_bn)
 {
-    HaloPlan p;
-    int bn;
-    return halo_plan(a, device_sms_or_default(), &p, &bn) && bn >= im2col_bn;
+    const int sms = device_sms_or_default();
+    HaloPlan hp;
+    WidePlan wp;
+    int bn = 0;
+    if (halo_plan(a, sms, &hp, &bn) && bn >= im2col_bn) return kGemmHaloResident;
+    if (wide_plan(a, sms, &wp, &bn)) return kGemmHaloStreamed;
+    return kGemmIm2col;
 }
 
 // The halo GEMM of a bf16 layer on its decoded weights W[C_out][K] (the
-// caller has checked halo_applies).
-cudaError_t halo_gemm(const ConvArgs &a, const void *W, cudaStream_t st)
+// caller has checked that halo_form is not the im2col GEMM).
+cudaError_t halo_gemm(const ConvArgs &a, const void *W, int im2col_bn, cudaStream_t st)
 {
     int sms = 0;
     cudaError_t e = device_sm_count(&sms);
     if (e != cudaSuccess) return e;
-    HaloPlan hp;
-    int bn = 0;
-    if (!halo_plan(a, sms, &hp, &bn)) return cudaErrorInvalidValue;
     const __nv_bfloat16 *w = static_cast<const __nv_bfloat16 *>(W);
     // 3x3 kernels (the ResNet shapes) get the unrolled tap loop
     const bool k3 = a.KH == 3 && a.KW == 3;
-    if (bn == 64) return k3 ? halo_launch_bn<64, 3>(a, hp, w, st) : halo_launch_bn<64, 0>(a, hp, w, st);
-    if (bn == 128) return k3 ? halo_launch_bn<128, 3>(a, hp, w, st) : halo_launch_bn<128, 0>(a, hp, w, st);
-    return k3 ? halo_launch_bn<256, 3>(a, hp, w, st) : halo_launch_bn<256, 0>(a, hp, w, st);
+    HaloPlan hp;
+    int bn = 0;
+    if (halo_plan(a, sms, &hp, &bn) && bn >= im2col_bn) {
+        if (bn == 64) return k3 ? halo_launch_bn<64, 3>(a, hp, w, st) : halo_launch_bn<64, 0>(a, hp, w, st);
+        if (bn == 128) return k3 ? halo_launch_bn<128, 3>(a, hp, w, st) : halo_launch_bn<128, 0>(a, hp, w, st);
+        return k3 ? halo_launch_bn<256, 3>(a, hp, w, st) : halo_launch_bn<256, 0>(a, hp, w, st);
+    }
+    WidePlan wp;
+    if (!wide_plan(a, sms, &wp, &bn)) return cudaErrorInvalidValue;
+    if (bn == 64) return k3 ? wide_launch_bn<64, 3>(a, wp, w, st) : wide_launch_bn<64, 0>(a, wp, w, st);
+    return k3 ? wide_launch_bn<128, 3>(a, wp, w, st) : wide_launch_bn<128, 0>(a, wp, w, st);
 }
 
 }  // namespace onexn

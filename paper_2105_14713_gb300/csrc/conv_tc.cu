@@ -1359,7 +1359,7 @@ cudaError_t gemm_typed(const ConvArgs &a, const void *workspace, size_t ws_bytes
     // stride-1 spatial bf16 layers whose output rows fill the M tile: the
     // halo form loads each activation once per tile instead of once per tap
     if constexpr (!Tr::kSplit) {
-        if (halo_applies(a, bn)) return halo_gemm(a, W, st);
+        if (halo_form(a, bn) != kGemmIm2col) return halo_gemm(a, W, bn, st);
         if (pt.mt == 2) return launch_bn<TcBf16W, 128>(a, W, W_lo, sk, st);
     }
     if (bn == 64) return launch_bn<Tr, 64>(a, W, W_lo, sk, st);
@@ -1412,6 +1412,16 @@ size_t tc_workspace_bytes(const ConvArgs &a, int dtype) { return weights_bytes(a
 
 // C_in, C_out giving 16-byte rows; the im2col box corners within the TMA's
 // [-128, 127] range; strides <= 8; 16-bit tap offsets.
+int tc_gemm_form(const ConvArgs &a, int dtype)
+{
+    const TcPlanTile pt = tc_plan_tile(a, dtype);
+    if (dtype == ONEXN_BF16) {
+        const int h = halo_form(a, pt.bn);
+        if (h != kGemmIm2col) return h;
+    }
+    return pt.mt == 2 ? kGemmIm2colWide : kGemmIm2col;
+}
+
 bool tc_supports(const ConvArgs &a, int dtype)
 {
     const int v = dtype == ONEXN_F32 ? 4 : 8;

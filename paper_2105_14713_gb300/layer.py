@@ -102,6 +102,12 @@ class PrunedConv2d:
                                0 if ws is None else ws.numel())
         return _c.ALGO_NAMES[a]
 
+    def tc_form(self, x_shape) -> str:
+        """The form the tensor-core family's GEMM takes for this input shape:
+        "im2col", "im2col_wide", "halo_resident" or "halo_streamed"."""
+        B, H, W, _ = x_shape
+        return _c.onexn_conv_tc_form(self.desc(B, H, W), self.N, self.t, self.cdtype)
+
     def forward(self, x: torch.Tensor, y: torch.Tensor = None, relu=False,
                 algo: int = _c.ONEXN_ALGO_AUTO, stream=None, residual: torch.Tensor = None) -> torch.Tensor:
         """x: NHWC CUDA tensor of this layer's dtype.  Returns y (NHWC):

@@ -63,6 +63,7 @@ SIGNATURES = {
     "onexn_conv_workspace_size": ([ctypes.POINTER(ConvDesc), _I32, _I64, _I32, _U32, _P], _I32),
     "onexn_conv_algo": ([ctypes.POINTER(ConvDesc), _I32, _I64, _I32, _U32, ctypes.c_size_t, _P],
                         _I32),
+    "onexn_conv_tc_form": ([ctypes.POINTER(ConvDesc), _I32, _I64, _I32, _P], _I32),
     "onexn_device_status": ([_I32, _P], _I32),
     "onexn_selftest_timeout": ([_P], _I32),
     "onexn_probe_ffma": ([_I32, _I32, _P, _P], _I32),
@@ -207,6 +208,20 @@ def onexn_conv_algo(desc: ConvDesc, N: int, t: int, dtype: int, flags: int = 0,
     _check(lib.onexn_conv_algo(ctypes.byref(desc), int(N), int(t), int(dtype), int(flags),
                                int(workspace_bytes), ctypes.byref(out)))
     return out.value
+
+
+ONEXN_GEMM_IM2COL = 0
+ONEXN_GEMM_IM2COL_WIDE = 1
+ONEXN_GEMM_HALO_RESIDENT = 2
+ONEXN_GEMM_HALO_STREAMED = 3
+GEMM_FORMS = {ONEXN_GEMM_IM2COL: "im2col", ONEXN_GEMM_IM2COL_WIDE: "im2col_wide",
+              ONEXN_GEMM_HALO_RESIDENT: "halo_resident", ONEXN_GEMM_HALO_STREAMED: "halo_streamed"}
+
+
+def onexn_conv_tc_form(desc: ConvDesc, N: int, t: int, dtype: int) -> str:
+    out = ctypes.c_int(0)
+    _check(lib.onexn_conv_tc_form(ctypes.byref(desc), int(N), int(t), int(dtype), ctypes.byref(out)))
+    return GEMM_FORMS[out.value]
 
 
 def onexn_conv_workspace_size(desc: ConvDesc, N: int, t: int, dtype: int, flags: int = 0) -> int:

@@ -211,6 +211,32 @@ def test_auto_cost_model():
     assert ox.onexn_conv_algo(tiny, 8, 1, ox.ONEXN_F32, ox.ONEXN_REUSE_DECODE, 1 << 20) == ox.ONEXN_ALGO_TC
 
 
+def test_tc_form_of_the_resnet50_stack_needs_no_gpu():
+    """The GEMM form per layer of the ResNet-50 bottleneck stack (batch 256,
+    bf16, 152 SMs): resident-weights halo tiles on the stage-1 3x3 layers
+    (64 channels: the 3x3 x 64 x 64 weights fit in shared memory),
+    streamed-weights halo tiles on the stride-1 stage-2 3x3 layers, the
+    im2col GEMM (128- or 256-row tiles) everywhere else: strided and 1x1
+    layers, and 14x14 / 7x7 layers whose padding would waste over 15% of
+    the rows.  The fp32 GEMM has one form."""
+    forms = {}
+    for l in wl.config4():
+        d = ox.make_desc(l.B, l.H, l.W, l.C_in, l.C_out, l.KH, l.KW, l.stride, l.pad, l.dil)
+        forms[l.name] = ox.onexn_conv_tc_form(d, 16, 10, ox.ONEXN_BF16)
+        assert ox.onexn_conv_tc_form(d, 16, 10, ox.ONEXN_F32) == "im2col"
+    for name, f in forms.items():
+        stage, kind = name.split(".")[0], name.split("_")[-1]
+        if kind == "3x3" and stage == "r50_s1":
+            assert f == "halo_resident", name
+        elif kind == "3x3" and stage == "r50_s2" and ".b1_" not in name:
+            assert f == "halo_streamed", name
+        else:
+            assert f in ("im2col", "im2col_wide"), name
+    assert forms["r50_s4.b2_3x3"] == "im2col_wide" and forms["r50_s3.b2_3x3"] == "im2col"
+    assert _status(ox.onexn_conv_tc_form, ox.make_desc(1, 8, 8, 6, 8, 3, 3, 1, 1, 1), 8, 10, ox.ONEXN_BF16) == \
+        ox.ONEXN_EINVAL                                                      # C_in % 8 for bf16
+
+
 def test_auto_batch1_mobilenet_v2_layers_pick_the_gemm():
     """Batch-1 MobileNet-V2 1x1 layers (N=4, 50%): with its workspace and the
     decode amortised (ONEXN_REUSE_DECODE, as the layer object passes), the
