@@ -455,6 +455,47 @@ def time_legs(legs, steps, warmup, flush, stream, sampler=None, flush_l2=True, p
             for i in range(len(legs))], wall
 
 
+def time_steps(legs, steps, warmup, flush, stream, sampler=None, flush_l2=True, passes=1, watch=None):
+    """Step times (ms) of `steps` steps of `passes` passes over the legs, with
+    CUDA events only at the step boundaries, so that consecutive layers run
+    back to back as a model runs them: each launched as a programmatic
+    dependent of the kernel before it, its launch and set-up overlapping that
+    kernel's tail (an event recorded between two kernels serialises them).
+    With `watch` = i, events also bracket every call of leg i, whose mean
+    per-call time is returned as well.  L2 flushed before each step, outside
+    the events (flush_l2=False: back to back)."""
+    for _ in range(warmup):
+        flush.fill_(1)
+        for lg in legs:
+            lg["conv"](lg["x"], lg["y"], algo=lg["flag"])
+    torch.cuda.synchronize()
+    ev = lambda: torch.cuda.Event(enable_timing=True)
+    evs = [(ev(), ev()) for _ in range(steps)]
+    wev = [[(ev(), ev()) for _ in range(passes)] for _ in range(steps)] if watch is not None else None
+    ctx = sampler if sampler is not None else _Null()
+    with ctx:
+        wall0 = time.perf_counter()
+        for k in range(steps):
+            if flush_l2:
+                flush.fill_(k & 0xff)
+            evs[k][0].record(stream)
+            for r in range(passes):
+                for i, lg in enumerate(legs):
+                    if i == watch:
+                        wev[k][r][0].record(stream)
+                    lg["conv"](lg["x"], lg["y"], algo=lg["flag"])
+                    if i == watch:
+                        wev[k][r][1].record(stream)
+            evs[k][1].record(stream)
+        torch.cuda.synchronize()
+        wall = time.perf_counter() - wall0
+    step_ms = [a.elapsed_time(b) for a, b in evs]
+    watch_ms = None
+    if watch is not None:
+        watch_ms = sum(a.elapsed_time(b) for row in wev for a, b in row) / (steps * passes)
+    return step_ms, watch_ms, wall
+
+
 STEP_TARGET_MS = 50.0
 
 
@@ -550,8 +591,14 @@ def measure(layers, args, dev, stream, flush, ws, pk, sampler=None, passes=None)
     if passes is None:
         passes = max_over_ranks(passes_for(legs, flush, stream), ws) if getattr(args, "auto_passes", False) else 1
     passes = int(passes)
-    leg_ms, wall = time_legs(legs, args.steps, args.warmup, flush, stream, sampler, passes=passes)
-    step_ms = sum(sum(m) for m in leg_ms) / args.steps
+    # per-leg breakdown (events around every call): the legs table and the
+    # dominant leg; then the timed region (events at the step boundaries and
+    # around the dominant leg's calls only)
+    leg_ms, _ = time_legs(legs, args.steps, args.warmup, flush, stream, None, passes=passes)
+    dom = max(range(len(legs)), key=lambda i: sum(leg_ms[i]))
+    steps_ms, dom_ms, wall = time_steps(legs, args.steps, args.warmup, flush, stream, sampler, passes=passes,
+                                        watch=dom)
+    step_ms = sum(steps_ms) / len(steps_ms)
     step_ms_max = max_over_ranks(step_ms, ws)
     flops_step = passes * sum(kept_flops(lg["layer"], lg["conv"].t) for lg in legs)
     info = []
@@ -564,6 +611,9 @@ def measure(layers, args, dev, stream, flush, ws, pk, sampler=None, passes=None)
                      "tflops": kept_flops(layer, t) / (ms * 1e-3) / 1e12,
                      "gbs": alg_bytes(layer, t) / (ms * 1e-3) / 1e9,
                      "roofline_frac": rf["frac"], "bound": rf["bound"]})
+    info[dom]["dominant"] = True
+    info[dom]["ms_timed_region"] = dom_ms
+    info[dom]["legs_sum_ms_per_step"] = sum(sum(m) for m in leg_ms) / args.steps
     return legs, leg_ms, step_ms_max, flops_step, info, wall, passes
 
 
@@ -626,10 +676,11 @@ def main():
     value = ws * flops_step / (step_ms_max * 1e-3) / 1e12
     clocks = sampler.summary()
 
-    # dominant kernel: the leg with the largest time
-    dom = max(range(len(legs)), key=lambda i: info[i]["ms"])
+    # dominant kernel: the leg with the largest time, its roofline from its
+    # calls' CUDA-event times inside the timed region
+    dom = next(i for i in range(len(legs)) if info[i].get("dominant"))
     dl, dlay = info[dom], legs[dom]["layer"]
-    rf = leg_roofline(dlay, legs[dom]["conv"].t, dl["algo"], dl["ms"], pk)
+    rf = leg_roofline(dlay, legs[dom]["conv"].t, dl["algo"], dl["ms_timed_region"], pk)
     roof = dict(rf)
     roof["traffic"] = traffic_for(f"{dl['algo']}_{dlay.name}")
     roof["kernel"] = f"{dl['algo']} ({dlay.name})"
@@ -647,15 +698,17 @@ def main():
     for lg in legs:
         lg["conv"].reuse_decoded = False
         lg["conv"]._args.clear()
-    dec_ms, _ = time_legs(legs, min(args.steps, 1000), args.warmup, flush, stream, passes=passes)
-    dec_step_ms = max_over_ranks(sum(sum(m) for m in dec_ms) / len(dec_ms[0]), ws)
+    dec_ms, _, _ = time_steps(legs, min(args.steps, 1000), args.warmup, flush, stream, passes=passes)
+    dec_step_ms = max_over_ranks(sum(dec_ms) / len(dec_ms), ws)
     for lg in legs:
         lg["conv"].reuse_decoded = True
         lg["conv"]._args.clear()
 
     # the same step without the L2 flush (the previous step's data warm in L2)
+    warm_steps, _, _ = time_steps(legs, min(args.steps, 1000), args.warmup, flush, stream, flush_l2=False,
+                                  passes=passes)
+    warm_step_ms = max_over_ranks(sum(warm_steps) / len(warm_steps), ws)
     warm_ms, _ = time_legs(legs, min(args.steps, 1000), args.warmup, flush, stream, flush_l2=False, passes=passes)
-    warm_step_ms = max_over_ranks(sum(sum(m) for m in warm_ms) / len(warm_ms[0]), ws)
 
     e2e_ms, h2d, d2h = e2e_time(legs, dev, max(3, min(args.steps // 4, 200)), 2, flush, stream)
     e2e_ms = max_over_ranks(e2e_ms, ws)
@@ -670,6 +723,10 @@ def main():
             "metric": METRIC, "value": value, "unit": "TFLOP/s", "n_gpus": ws,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": step_ms_max,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+            "timing": "CUDA events at the step boundaries (layers back to back, each launched as a programmatic "
+                      "dependent of the one before) and around the dominant leg's calls; legs[] from a separate "
+                      "run with events around every call (their sum: legs_sum_ms_per_step)",
+            "legs_sum_ms_per_step": dl["legs_sum_ms_per_step"],
             "dtype": "+".join(sorted({l.dtype for l in layers})),
             "data": "synthetic (seeded Kaiming-normal or N(0,0.05) weights, ReLU(N(0,1)) activations)",
             "config": dict(config_json(args.config, layers), passes_per_step=passes),
