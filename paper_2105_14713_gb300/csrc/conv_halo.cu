@@ -366,28 +366,36 @@ halo_conv_kernel(const ConvArgs a, const __grid_constant__ CUtensorMap tmap_x,
 
 // ---------------------------------------------------------------------------
 // Streamed-weights form (layers whose column tile of weights does not fit in
-// shared memory next to the halo slots).  The output of an image is laid
-// out in the padded space of Hp = Ho + (KH-1)*dh rows of Wp positions
+// shared memory next to the halo slots, and strided layers).  The output of
+// an image is laid out in the padded space of Hp rows of Wp positions
 // (position (n*Hp + r)*Wp + w is output pixel (n, r, w) when r < Ho and
-// w < Wo, else a dropped row), and the input in the same space (row r,
-// column w = input pixel (r - ph, w - pw)); output position P of tap
-// (kh, kw) reads input position P + kh*dh*Wp + kw*dw.  A tile is 256
+// w < Wo, else a dropped row).  For stride 1 the input is in the same
+// space (row r, column w = input pixel (r - ph, w - pw)), Hp = Ho + (KH-1)*dh,
+// Wp = Wo + (KW-1)*dw, and output position P of tap (kh, kw) reads input
+// position P + kh*dh*Wp + kw*dw.  A strided layer is split into the phases
+// of its input (the pixels s*i + phase, per dimension): tap k reads phase
+// (k*d - p) mod s at an index shifted by floor((k*d - p) / s), so each phase
+// is a stride-1 problem on its own padded space of the same Hp x Wp, and
+// each tap a shift within one phase (phase_dim below).  A tile is 256
 // consecutive positions, two M = 128 halves; it may run across rows and
-// images, so only the padding columns and rows are wasted.  Per 64-channel
-// chunk one TMA im2col load brings its 256 + (KH-1)*dh*Wp + (KW-1)*dw input
-// positions (the traversal continues into the next image, zeros after the
-// last one), and the A operand of (half h, tap) is that buffer viewed from
-// row 128*h + kh*dh*Wp + kw*dw on.  The weights are streamed: one B stage
-// holds one kernel row of taps (3x3) or one tap, 128-byte swizzled, shared
-// by both halves.  MMA warp h issues the MMAs of half h (its own
-// accumulators), so each issuing thread meets one stage wait per kernel row
-// of taps; the epilogue warps (two per TMEM lane quarter, one per half)
-// store their valid rows straight to global memory.
+// images, so only the padding positions are wasted.  Per (64-channel chunk,
+// phase) one TMA im2col load, stepping by the layer's strides and offset by
+// the phase, brings the tile's positions plus the largest shift (the
+// traversal continues into the next image, zeros after the last one), and
+// the A operand of (half h, tap) is that buffer viewed from row 128*h +
+// the tap's shift.  The weights are streamed: one B stage holds one kernel
+// row of taps (stride-1 3x3) or one tap, 128-byte swizzled, shared by both
+// halves.  MMA warp h issues the MMAs of half h (its own accumulators), so
+// each issuing thread meets one stage wait per stage; the epilogue warps
+// (two per TMEM lane quarter, one per half) store their valid rows straight
+// to global memory.
 constexpr int kWRows = 2 * kBM;            // positions per tile
 constexpr int kWEpiWarp0 = 3;
 constexpr int kWWarps = kWEpiWarp0 + 8;    // producer, two MMA warps, eight epilogue warps
-constexpr int kWMaxHalo = 2;
+constexpr int kWMaxHalo = 4;
 constexpr int kWMaxStages = 12;
+constexpr int kWMaxTaps = 49;              // taps of the tap table (7x7 at most)
+constexpr int kWMaxPhases = 4;
 constexpr int kWAccMax = 4;
 constexpr int kWBarBytes = (2 * kWMaxHalo + 2 * kWMaxStages + 4 * kWAccMax + 2) * 8;
 
@@ -396,9 +404,15 @@ struct WidePlan {
     int n_cc, n_taps, tps, n_st;   // chunks, taps, taps per B stage, B stages per chunk
     int n_tn, n_m, grid;           // column tiles, position tiles, CTAs (a multiple of n_tn)
     int S_h, S_b;                  // halo slots, B stages
+    int n_ph;                      // input phases (1 for stride 1)
+    int lower_w, lower_h;          // TMA start of padded position (r, c): (lower_w + sw*c, lower_h + sh*r)
     uint32_t halo_pix, halo_tx, slot_bytes, stage_bytes;
-    uint32_t off_b, off_bias, off_bar, bytes;
+    uint32_t off_b, off_bias, off_bar, off_tab, bytes;
     FastDiv div_img, div_wp;       // Hp*Wp, Wp
+    // tap table (grouped by phase): K tap index << 16 | A view shift in rows;
+    // phase table: first tap | end tap << 8 | im2col w offset << 16 | h offset << 24
+    uint32_t tap[kWMaxTaps];
+    uint32_t ph[kWMaxPhases];
 };
 
 template <int BN>
@@ -408,8 +422,9 @@ struct WideTmem {
     static constexpr int kCols = pow2_cols(kAcc * 2 * BN);
 };
 
-// KS = 3: 3x3 kernel (a B stage is one kernel row of three taps, unrolled);
-// KS = 0: any kernel shape (one tap per stage).
+// KS = 3: stride-1 3x3 kernel (a B stage is one kernel row of three taps,
+// unrolled); KS = 0: any kernel shape and stride, one halo per (chunk,
+// phase) and one tap per stage, from the plan's tap table.
 template <int BN, int KS>
 __global__ void __launch_bounds__(kWWarps * 32, 1)
 halo_wide_kernel(const ConvArgs a, const __grid_constant__ CUtensorMap tmap_x,
@@ -449,6 +464,9 @@ halo_wide_kernel(const ConvArgs a, const __grid_constant__ CUtensorMap tmap_x,
         }
         for (int j = 0; j < 2; ++j) mbar_init(bar_drain + 8 * j, 1);
         fence_mbar_init();
+        uint32_t *tab = reinterpret_cast<uint32_t *>(smem + wp.off_tab);
+        for (int i = 0; i < kWMaxTaps; ++i) tab[i] = wp.tap[i];
+        for (int i = 0; i < kWMaxPhases; ++i) tab[kWMaxTaps + i] = wp.ph[i];
     }
     if (warp == 1) {
         tc::tmem_alloc(smem_u32(holder), TM::kCols);
@@ -466,6 +484,20 @@ halo_wide_kernel(const ConvArgs a, const __grid_constant__ CUtensorMap tmap_x,
     const int tn = static_cast<int>(blockIdx.x) % wp.n_tn;
     const int m0 = static_cast<int>(blockIdx.x) / wp.n_tn, m_step = wp.grid / wp.n_tn;
     const uint32_t img = static_cast<uint32_t>(wp.Hp) * static_cast<uint32_t>(wp.Wp);
+    const uint32_t *s_tap = reinterpret_cast<const uint32_t *>(smem + wp.off_tab);
+    const uint32_t *s_ph = s_tap + kWMaxTaps;
+    // phases and their B stages: the stride-1 3x3 form has one phase of
+    // n_st stages (kernel rows); the general one takes both from the tables
+    const int n_ph = KS > 0 ? 1 : wp.n_ph;
+    auto ph_stages = [&](int ph, int &st0, int &st1) {
+        if constexpr (KS > 0) {
+            st0 = 0;
+            st1 = wp.n_st;
+        } else {
+            st0 = static_cast<int>(s_ph[ph] & 0xffu);
+            st1 = static_cast<int>((s_ph[ph] >> 8) & 0xffu);
+        }
+    };
 
     if (warp == 0) {
         // ============================ producer ============================
@@ -476,26 +508,35 @@ halo_wide_kernel(const ConvArgs a, const __grid_constant__ CUtensorMap tmap_x,
                 const uint32_t P0 = static_cast<uint32_t>(tm) * kWRows;
                 const uint32_t n0 = wp.div_img.div(P0), rem = P0 - n0 * img;
                 const uint32_t r0 = wp.div_wp.div(rem), w0 = rem - r0 * static_cast<uint32_t>(wp.Wp);
-                for (int cc = 0; cc < wp.n_cc && !failed; ++cc) {
+                const int w_start = wp.lower_w + a.sw * static_cast<int>(w0);
+                const int h_start = wp.lower_h + a.sh * static_cast<int>(r0);
+                for (int u = 0; u < wp.n_cc * n_ph && !failed; ++u) {
+                    const int cc = u / n_ph, ph = u - cc * n_ph;
                     if (hround >= 1 && !mbar_wait(bar_hempty + 8 * hs, (hround - 1) & 1)) {
                         failed = true;
                         break;
                     }
+                    const uint32_t phv = KS > 0 ? 0u : s_ph[ph];
                     tc::mbar_arrive_expect_tx(bar_hfull + 8 * hs, wp.halo_tx);
                     tc::tma_load_im2col_4d(sH + static_cast<uint32_t>(hs) * wp.slot_bytes, &tmap_x, cc * kBK,
-                                           static_cast<int>(w0) - a.pw, static_cast<int>(r0) - a.ph,
-                                           static_cast<int>(n0), 0, 0, bar_hfull + 8 * hs);
+                                           w_start, h_start, static_cast<int>(n0),
+                                           static_cast<uint16_t>((phv >> 16) & 0xffu),
+                                           static_cast<uint16_t>(phv >> 24), bar_hfull + 8 * hs);
                     if (++hs == wp.S_h) { hs = 0; ++hround; }
-                    for (int st = 0; st < wp.n_st; ++st) {
+                    int st0, st1;
+                    ph_stages(ph, st0, st1);
+                    for (int st = st0; st < st1; ++st) {
                         if (bround >= 1 && !mbar_wait(bar_bempty + 8 * bs, (bround - 1) & 1)) {
                             failed = true;
                             break;
                         }
                         tc::mbar_arrive_expect_tx(bar_bfull + 8 * bs, wp.stage_bytes);
                         const uint32_t dst = sB + static_cast<uint32_t>(bs) * wp.stage_bytes;
-                        for (int i = 0; i < wp.tps; ++i)
+                        for (int i = 0; i < wp.tps; ++i) {
+                            const int ktap = KS > 0 ? st * wp.tps + i : static_cast<int>(s_tap[st] >> 16);
                             tc::tma_load_2d(dst + static_cast<uint32_t>(i) * kBTile, &tmap_w,
-                                            (st * wp.tps + i) * a.C + cc * kBK, tn * BN, bar_bfull + 8 * bs);
+                                            ktap * a.C + cc * kBK, tn * BN, bar_bfull + 8 * bs);
+                        }
                         if (++bs == wp.S_b) { bs = 0; ++bround; }
                     }
                 }
@@ -522,12 +563,14 @@ halo_wide_kernel(const ConvArgs a, const __grid_constant__ CUtensorMap tmap_x,
                 }
                 tc::fence_after_sync();
                 const uint32_t d_tmem = tmem + static_cast<uint32_t>(2 * acc + h) * BN;
-                for (int cc = 0; cc < wp.n_cc && !failed; ++cc) {
+                for (int u = 0; u < wp.n_cc * n_ph && !failed; ++u) {
+                    const int cc = u / n_ph, ph = u - cc * n_ph;
                     if (!mbar_wait(bar_hfull + 8 * hs, hph)) { failed = true; break; }
                     tc::fence_after_sync();
                     const uint64_t hd = tc::desc_kmajor_sw128(sH + static_cast<uint32_t>(hs) * wp.slot_bytes) + half_off;
-                    int kh = 0, kw = 0;                  // tap of the generic path
-                    for (int st = 0; st < wp.n_st; ++st) {
+                    int st0, st1;
+                    ph_stages(ph, st0, st1);
+                    for (int st = st0; st < st1; ++st) {
                         if (!mbar_wait(bar_bfull + 8 * bs, bph)) { failed = true; break; }
                         tc::fence_after_sync();
                         const uint64_t bd = tc::desc_kmajor_sw128(sB + static_cast<uint32_t>(bs) * wp.stage_bytes);
@@ -543,8 +586,7 @@ halo_wide_kernel(const ConvArgs a, const __grid_constant__ CUtensorMap tmap_x,
                             for (int t = 0; t < KS; ++t)
                                 tap_mmas(ad_row + t * col_step, bd + t * kBDesc, t == 0 ? first : 1u);
                         } else {
-                            tap_mmas(hd + kh * row_step + kw * col_step, bd, first);
-                            if (++kw == a.KW) { kw = 0; ++kh; }
+                            tap_mmas(hd + (s_tap[st] & 0xffffu) * (kRow / 16), bd, first);
                         }
                         tc::commit(bar_bempty + 8 * bs);
                         if (++bs == wp.S_b) { bs = 0; bph ^= 1; }
@@ -718,14 +760,23 @@ bool halo_plan(const ConvArgs &a, int sms, HaloPlan *out, int *bn_out)
     return true;
 }
 
-// im2col tensor map of the halo: the traversal's bounding box is the padded
-// image, columns -pw .. W - 1 + pw and rows -ph .. H - 1 + ph (corners
-// innermost first: W, H), so a load of `pixels` positions walks whole
-// padded rows from its start (Wp x Rh positions from (-pw, h0 - ph) for a
-// row block; any position for the streamed form).  A load that runs past
-// the padded image continues into the next image's rows (or zeros after
-// the last image); those rows feed only dropped M rows.
-bool halo_x_tmap(const ConvArgs &a, int Wp, int pixels, CUtensorMap *m)
+// im2col tensor map of the halo.  The traversal's bounding box is the
+// padded image (corners innermost first: W, H): base positions lower ..
+// W - 1 + upper, stepped by the traversal strides (the layer's strides for
+// the streamed form, 1 for the resident one), each loading x at base + the
+// load's im2col offsets (a phase of a strided layer, else 0).  So a load of
+// `pixels` positions walks whole padded rows from its start, and one that
+// runs past the padded image continues into the next image's rows (or zeros
+// after the last image); those rows feed only dropped M rows.
+bool box_ok(const int lower[2], const int upper[2])
+{
+    for (int i = 0; i < 2; ++i)
+        if (lower[i] < -128 || lower[i] > 127 || upper[i] < -128 || upper[i] > 127) return false;
+    return true;
+}
+
+bool halo_x_tmap(const ConvArgs &a, const int lower[2], const int upper[2], int estr_w, int estr_h, int pixels,
+                 CUtensorMap *m)
 {
     auto enc = encode_im2col_fn_public();
     if (!enc) return false;
@@ -733,45 +784,118 @@ bool halo_x_tmap(const ConvArgs &a, int Wp, int pixels, CUtensorMap *m)
                                 static_cast<cuuint64_t>(a.H), static_cast<cuuint64_t>(a.B)};
     const cuuint64_t strides[3] = {static_cast<cuuint64_t>(a.C) * 2, static_cast<cuuint64_t>(a.C) * 2 * a.W,
                                    static_cast<cuuint64_t>(a.C) * 2 * a.W * a.H};
-    const int lower[2] = {-a.pw, -a.ph};
-    const int upper[2] = {Wp - a.pw - a.W, a.Ho + (a.KH - 1) * a.dh - a.ph - a.H};
-    for (int i = 0; i < 2; ++i)
-        if (lower[i] < -128 || lower[i] > 127 || upper[i] < -128 || upper[i] > 127) return false;
-    const cuuint32_t estr[4] = {1, 1, 1, 1};
+    if (!box_ok(lower, upper)) return false;
+    const cuuint32_t estr[4] = {1, static_cast<cuuint32_t>(estr_w), static_cast<cuuint32_t>(estr_h), 1};
     return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void *>(a.x), dims, strides, lower, upper, kBK,
                static_cast<cuuint32_t>(pixels), estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
                CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-// The streamed-weights plan, or false: strided or 1x1 layers, too many
-// dropped positions (Ho*Wo below 85% of Hp*Wp), more positions per load
-// than one im2col load can walk, or shared memory for fewer than two B
-// stages.  The column tile is 128 (64 when the output channels fit in
-// 64), so that two accumulator buffers of two halves fit in the TMEM.
+// One spatial dimension of a (possibly strided) layer in the streamed form.
+// Output o of tap k reads input s*o + q, q = k*d - p, which is phase
+// q mod s of the input (the inputs s*i + phase) at phase index
+// o + floor(q / s).  In the padded space, position c of a row holds phase
+// index c + lo (lo = the smallest floor(q / s)), so tap k is a shift of
+// floor(q / s) - lo positions, and the row is P = Out + (largest - smallest
+// floor) long; the TMA traversal's base positions are s*(c + lo), i.e.
+// lower = s*lo, and lower + s*(P - 1) is the last one (upper corner).
+struct PhaseDim {
+    int lo, P, lower;
+    int phase[kWMaxTaps], shift[kWMaxTaps];
+};
+
+bool phase_dim(int K, int s, int p, int d, int Out, PhaseDim *g)
+{
+    if (K > kWMaxTaps || s < 1) return false;
+    int lo = INT32_MAX, hi = INT32_MIN;
+    for (int k = 0; k < K; ++k) {
+        const int q = k * d - p;
+        const int ph = ((q % s) + s) % s;
+        g->phase[k] = ph;
+        g->shift[k] = (q - ph) / s;
+        lo = std::min(lo, g->shift[k]);
+        hi = std::max(hi, g->shift[k]);
+    }
+    for (int k = 0; k < K; ++k) g->shift[k] -= lo;
+    g->lo = lo;
+    g->P = Out + (hi - lo);
+    g->lower = s * lo;
+    return true;
+}
+
+// The streamed-weights plan, or false: 1x1 layers, too many dropped
+// positions (Ho*Wo below 85% of Hp*Wp), more than four input phases
+// (strides above 2 in both dimensions) or 49 taps, more positions per load
+// than one im2col load can walk, a traversal box out of the TMA's range, or
+// shared memory for fewer than two B stages.  The column tile is 128 (64
+// when the output channels fit in 64), so that two accumulator buffers of
+// two halves fit in the TMEM.
 bool wide_plan(const ConvArgs &a, int sms, WidePlan *out, int *bn_out)
 {
-    if (a.sh != 1 || a.sw != 1 || a.KH * a.KW == 1 || a.Ho <= 0 || a.Wo <= 0 || a.B <= 0) return false;
+    if (a.KH * a.KW == 1 || a.Ho <= 0 || a.Wo <= 0 || a.B <= 0 || a.KH * a.KW > kWMaxTaps) return false;
     WidePlan p{};
-    p.Wp = a.Wo + (a.KW - 1) * a.dw;
-    p.Hp = a.Ho + (a.KH - 1) * a.dh;
+    PhaseDim gw, gh;
+    if (!phase_dim(a.KW, a.sw, a.pw, a.dw, a.Wo, &gw) || !phase_dim(a.KH, a.sh, a.ph, a.dh, a.Ho, &gh)) return false;
+    p.Wp = gw.P;
+    p.Hp = gh.P;
+    p.lower_w = gw.lower;
+    p.lower_h = gh.lower;
+    const int lower[2] = {p.lower_w, p.lower_h};
+    const int upper[2] = {p.lower_w + a.sw * (p.Wp - 1) - (a.W - 1), p.lower_h + a.sh * (p.Hp - 1) - (a.H - 1)};
+    if (!box_ok(lower, upper)) return false;
     const double fill = static_cast<double>(a.Ho) * a.Wo / (static_cast<double>(p.Hp) * p.Wp);
     if (fill < kMinRowFill) return false;
     const int64_t positions = static_cast<int64_t>(a.B) * p.Hp * p.Wp;
     if (positions + kWRows > INT32_MAX) return false;
-    const int64_t halo = kWRows + static_cast<int64_t>(a.KH - 1) * a.dh * p.Wp + static_cast<int64_t>(a.KW - 1) * a.dw;
+    // the tap table grouped by input phase (phases in order of first use)
+    int ph_key[kWMaxPhases], n_ph = 0, t = 0, max_shift = 0;
+    for (int kh = 0; kh < a.KH; ++kh)
+        for (int kw = 0; kw < a.KW; ++kw) {
+            const int key = gh.phase[kh] * 256 + gw.phase[kw];
+            int i = 0;
+            while (i < n_ph && ph_key[i] != key) ++i;
+            if (i == n_ph) {
+                if (n_ph == kWMaxPhases) return false;
+                ph_key[n_ph++] = key;
+            }
+        }
+    for (int i = 0; i < n_ph; ++i) {
+        const int t0 = t;
+        for (int kh = 0; kh < a.KH; ++kh)
+            for (int kw = 0; kw < a.KW; ++kw) {
+                if (gh.phase[kh] * 256 + gw.phase[kw] != ph_key[i]) continue;
+                const int shift = gh.shift[kh] * p.Wp + gw.shift[kw];
+                max_shift = std::max(max_shift, shift);
+                if (shift > 0xffff) return false;
+                p.tap[t++] = (static_cast<uint32_t>(kh * a.KW + kw) << 16) | static_cast<uint32_t>(shift);
+            }
+        p.ph[i] = static_cast<uint32_t>(t0) | (static_cast<uint32_t>(t) << 8) |
+                  (static_cast<uint32_t>(ph_key[i] & 0xff) << 16) | (static_cast<uint32_t>(ph_key[i] >> 8) << 24);
+    }
+    p.n_ph = n_ph;
+    const int64_t halo = kWRows + max_shift;
     if (halo > 1024) return false;                        // positions per im2col load
     p.halo_pix = static_cast<uint32_t>(halo);
     p.halo_tx = p.halo_pix * kRow;
     p.slot_bytes = round1024(static_cast<uint64_t>(p.halo_pix) * kRow);
     p.n_cc = (a.C + kBK - 1) / kBK;
     p.n_taps = a.KH * a.KW;
-    p.tps = (a.KH == 3 && a.KW == 3) ? 3 : 1;
+    // stride-1 3x3: one phase, B stages of one kernel row (the unrolled form)
+    const bool k3 = a.KH == 3 && a.KW == 3 && a.sh == 1 && a.sw == 1;
+    p.tps = k3 ? 3 : 1;
     p.n_st = p.n_taps / p.tps;
     const int bn = a.C_out <= 64 ? 64 : 128;
     p.stage_bytes = static_cast<uint32_t>(p.tps * bn * kRow);
-    p.S_h = kWMaxHalo;
-    const uint64_t fixed = round1024(static_cast<uint64_t>(bn) * 4) + kWBarBytes + 16 + 1024;
+    const uint64_t tab = (kWMaxTaps + kWMaxPhases) * 4;
+    const uint64_t fixed = static_cast<uint64_t>(bn) * 4 + kWBarBytes + 16 + tab + 1024;   // + base alignment
+    // halo slots: two for one phase; with several phases (each read by
+    // fewer taps) up to four, keeping at least four B stages
+    int S_h = n_ph > 1 ? kWMaxHalo : 2;
+    while (S_h > 2 && static_cast<uint64_t>(S_h) * p.slot_bytes + fixed + 4ull * p.stage_bytes >
+                          static_cast<uint64_t>(kSmemMax))
+        --S_h;
+    p.S_h = S_h;
     const uint64_t halo_bytes = static_cast<uint64_t>(p.S_h) * p.slot_bytes;
     if (halo_bytes + fixed + 2ull * p.stage_bytes > static_cast<uint64_t>(kSmemMax)) return false;
     p.S_b = static_cast<int>(std::min<uint64_t>(kWMaxStages, (kSmemMax - fixed - halo_bytes) / p.stage_bytes));
@@ -782,8 +906,9 @@ bool wide_plan(const ConvArgs &a, int sms, WidePlan *out, int *bn_out)
     p.grid = static_cast<int>(std::min<int64_t>(tiles, sms) / p.n_tn * p.n_tn);
     p.off_b = static_cast<uint32_t>(halo_bytes);
     p.off_bias = p.off_b + static_cast<uint32_t>(p.S_b) * p.stage_bytes;
-    p.off_bar = p.off_bias + round1024(static_cast<uint64_t>(bn) * 4);
-    p.bytes = p.off_bar + kWBarBytes + 16;
+    p.off_bar = p.off_bias + static_cast<uint32_t>(bn) * 4;
+    p.off_tab = p.off_bar + kWBarBytes + 16;
+    p.bytes = p.off_tab + static_cast<uint32_t>(tab);
     if (p.bytes + 1024 > static_cast<uint32_t>(kSmemMax)) return false;
     p.div_img = FastDiv(static_cast<uint32_t>(p.Hp) * static_cast<uint32_t>(p.Wp));
     p.div_wp = FastDiv(static_cast<uint32_t>(p.Wp));
@@ -801,7 +926,9 @@ cudaError_t wide_launch_bn(const ConvArgs &a, const WidePlan &wp, const __nv_bfl
     CUtensorMap tmap_x, tmap_w;
     // x [B][H][W][C]: one im2col load per 64-channel chunk walks the tile's
     // halo_pix positions of the padded space from the tile's first one
-    if (!halo_x_tmap(a, wp.Wp, static_cast<int>(wp.halo_pix), &tmap_x)) return cudaErrorInvalidValue;
+    const int lower[2] = {wp.lower_w, wp.lower_h};
+    const int upper[2] = {wp.lower_w + a.sw * (wp.Wp - 1) - (a.W - 1), wp.lower_h + a.sh * (wp.Hp - 1) - (a.H - 1)};
+    if (!halo_x_tmap(a, lower, upper, a.sw, a.sh, static_cast<int>(wp.halo_pix), &tmap_x)) return cudaErrorInvalidValue;
     {   // W [C_out][K]: boxes of 64 K x BN rows
         const uint64_t dims[2] = {K, static_cast<uint64_t>(a.C_out)};
         const uint64_t strides[1] = {K * 2};
@@ -845,7 +972,9 @@ cudaError_t halo_launch_bn(const ConvArgs &a, const HaloPlan &hp, const __nv_bfl
     // x [B][H][W][C]: one im2col load per 64-channel chunk walks the Wp x Rh
     // halo positions of the tile (columns -pw .. W - 1 + pw of each row,
     // the padding read as zeros)
-    if (!halo_x_tmap(a, hp.Wp, hp.Wp * hp.Rh, &tmap_x)) return cudaErrorInvalidValue;
+    const int lower[2] = {-a.pw, -a.ph};
+    const int upper[2] = {hp.Wp - a.pw - a.W, a.Ho + (a.KH - 1) * a.dh - a.ph - a.H};
+    if (!halo_x_tmap(a, lower, upper, 1, 1, hp.Wp * hp.Rh, &tmap_x)) return cudaErrorInvalidValue;
     {   // W [C_out][K]: boxes of 64 K x BN rows
         const uint64_t dims[2] = {K, static_cast<uint64_t>(a.C_out)};
         const uint64_t strides[1] = {K * 2};
@@ -889,12 +1018,13 @@ cudaError_t halo_launch_bn(const ConvArgs &a, const HaloPlan &hp, const __nv_bfl
 }  // namespace
 
 // The halo form of this layer's bf16 GEMM, against the im2col GEMM's
-// column tile: the resident-weights form only when its column tile is at
-// least as wide (a narrower one multiplies the MMAs, each reading its A
-// operand again, and loads every halo once per column tile: measured slower
-// on ResNet-50's stage-2 3x3 layer, BN 64 halo 76.8 us against BN 128
-// im2col 61 us at batch 256); else the streamed-weights form when its plan
-// exists; else none (the im2col GEMM).
+// column tile: either form only when its column tile is at least as wide,
+// since a narrower one loads every halo once per column tile where the
+// im2col GEMM shares each A tile over all its columns (resident weights:
+// ResNet-50's stage-2 3x3 layer at BN 64 76.8 us against BN 128 im2col
+// 61 us at batch 256; streamed weights: the stride-2 stage-3 3x3 layer at
+// BN 128 53.6 us against BN 256 im2col 48.7 us).  The resident form first;
+// else none (the im2col GEMM).
 int halo_form(const ConvArgs &a, int im2col_bn)
 {
     const int sms = device_sms_or_default();
@@ -902,7 +1032,7 @@ int halo_form(const ConvArgs &a, int im2col_bn)
     WidePlan wp;
     int bn = 0;
     if (halo_plan(a, sms, &hp, &bn) && bn >= im2col_bn) return kGemmHaloResident;
-    if (wide_plan(a, sms, &wp, &bn)) return kGemmHaloStreamed;
+    if (wide_plan(a, sms, &wp, &bn) && bn >= im2col_bn) return kGemmHaloStreamed;
     return kGemmIm2col;
 }
 
@@ -925,8 +1055,9 @@ cudaError_t halo_gemm(const ConvArgs &a, const void *W, int im2col_bn, cudaStrea
     }
     WidePlan wp;
     if (!wide_plan(a, sms, &wp, &bn)) return cudaErrorInvalidValue;
-    if (bn == 64) return k3 ? wide_launch_bn<64, 3>(a, wp, w, st) : wide_launch_bn<64, 0>(a, wp, w, st);
-    return k3 ? wide_launch_bn<128, 3>(a, wp, w, st) : wide_launch_bn<128, 0>(a, wp, w, st);
+    const bool w3 = wp.tps == 3;           // stride-1 3x3: kernel rows as B stages, unrolled
+    if (bn == 64) return w3 ? wide_launch_bn<64, 3>(a, wp, w, st) : wide_launch_bn<64, 0>(a, wp, w, st);
+    return w3 ? wide_launch_bn<128, 3>(a, wp, w, st) : wide_launch_bn<128, 0>(a, wp, w, st);
 }
 
 }  // namespace onexn

@@ -16,6 +16,11 @@ chunk, each tap's A operand a row-shifted view of it.
    and 128-column tiles, two and four column tiles, a partial channel chunk
    and a partial column tile, 1 to 8 chunks, padding 0 / 1 / 2, dilation 2,
    5x5, 3x1 and 1x3 kernels, and a last tile past the last image.
+ * Strided layers on the streamed form, split into the phases of their
+   input (one strided load per chunk and phase, each tap a shift within
+   its phase): stride 2 with 3x3 (four phases of 4, 2, 2 and 1 taps), 5x5
+   (25 taps), padding 0 and 1, an odd input size, dilation 2 (one phase),
+   a partial channel chunk and a partial column tile.
 A layer of each form with the residual + ReLU6 epilogue, and every case's
 form checked.  The 5x5 28-wide case wastes too many rows and runs the
 im2col form, checked here all the same.  Tolerance: 4e-3 = 2^-8 output
@@ -74,19 +79,48 @@ def test_halo_layers_match_oracle(geom, rate):
     assert torch.equal(y1, y2)
 
 
-@pytest.mark.parametrize("C_in,form", [(64, "halo_resident"), (256, "halo_streamed")])
-def test_halo_residual_relu6(C_in, form):
-    layer = L("halo_res", 2, 28, 28, C_in, 64, 3, 3, 1, 1, 1, N=16, rate=0.5, dtype="bf16", seed=11)
+STRIDED_GEOMS = [
+    # name, B, H, W, C_in, C_out, KH, KW, stride, pad, dil, N
+    ("s2_3x3_c128", 2, 56, 56, 128, 128, 3, 3, 2, 1, 1, 16),    # ResNet-50 stage-2 b1 shape: 29x29 phase space
+    ("s2_3x3_c256", 2, 28, 28, 256, 256, 3, 3, 2, 1, 1, 16),    # stage-3 b1 shape: 15x15, two column tiles
+    ("s2_3x3_odd", 2, 29, 29, 64, 128, 3, 3, 2, 1, 1, 8),       # odd input: 15x15 output, 16x16 phase space
+    ("s2_5x5", 1, 56, 56, 128, 128, 5, 5, 2, 2, 1, 16),         # 25 taps in four phases
+    ("s2_3x3_p0", 2, 57, 57, 128, 128, 3, 3, 2, 0, 1, 16),
+    ("s2_3x3_d2", 1, 56, 56, 128, 128, 3, 3, 2, 2, 2, 16),      # every tap in one phase
+    ("s2_c72_co96", 1, 56, 56, 72, 96, 3, 3, 2, 1, 1, 8),       # partial chunk and column tile
+    ("s2_co64", 2, 56, 56, 128, 64, 3, 3, 2, 1, 1, 16),         # 64-column tiles
+]
+
+
+@pytest.mark.parametrize("geom", STRIDED_GEOMS, ids=[g[0] for g in STRIDED_GEOMS])
+@pytest.mark.parametrize("rate", [0.0, 0.7])
+def test_halo_strided_layers_match_oracle(geom, rate):
+    name, B, H, W, Ci, Co, KH, KW, s, p, d, N = geom
+    layer = L(name, B, H, W, Ci, Co, KH, KW, s, p, d, N=N, rate=rate, dtype="bf16", seed=Ci + Co + s)
+    y, yr, a, conv = run_layer(layer, relu=True, algo=ox.ONEXN_ALGO_TC)
+    assert conv.tc_form((B, H, W, Ci)) == "halo_streamed"
+    assert norm_err(y, yr, a) <= TOL_BF16_ROUNDED
+    x = wl.activations(layer).to(torch.bfloat16).cuda()
+    y1 = conv(x, relu=True, algo=ox.ONEXN_ALGO_TC)
+    y2 = conv(x, relu=True, algo=ox.ONEXN_ALGO_TC)
+    torch.cuda.synchronize()
+    assert torch.equal(y1, y2)
+
+
+@pytest.mark.parametrize("C_in,H,s,form", [(64, 28, 1, "halo_resident"), (256, 28, 1, "halo_streamed"),
+                                           (128, 56, 2, "halo_streamed")])
+def test_halo_residual_relu6(C_in, H, s, form):
+    layer = L("halo_res", 2, H, H, C_in, 64, 3, 3, s, 1, 1, N=16, rate=0.5, dtype="bf16", seed=11)
     W, b = wl.weights(layer).numpy(), wl.bias(layer).numpy()
-    conv = PrunedConv2d(W, 16, 0.5, bias=b, padding=1, dtype="bf16")
-    assert conv.tc_form((2, 28, 28, C_in)) == form
+    conv = PrunedConv2d(W, 16, 0.5, bias=b, stride=s, padding=1, dtype="bf16")
+    assert conv.tc_form((2, H, H, C_in)) == form
     x = wl.activations(layer).to(torch.bfloat16).cuda()
     rng = np.random.default_rng(7)
     r = torch.from_numpy((3 * rng.standard_normal((2, 28, 28, 64))).astype(np.float32)).to(torch.bfloat16).cuda()
     y = conv(x, relu="relu6", algo=ox.ONEXN_ALGO_TC, residual=r)
     torch.cuda.synchronize()
     mask, _ = oracle.prune(W, 16, 0.5, ox.ONEXN_GRAN_TAP)
-    ref, absacc = oracle.conv_masked(x.float().cpu().numpy(), oracle.round_bf16(W), mask, b, 16, (1, 1), (1, 1),
+    ref, absacc = oracle.conv_masked(x.float().cpu().numpy(), oracle.round_bf16(W), mask, b, 16, (s, s), (1, 1),
                                      relu="relu6", residual=r.float().cpu().numpy(), want_abs=True)
     e = norm_err(y.float().cpu().numpy().reshape(-1, 64).astype(np.float64), ref.reshape(-1, 64),
                  absacc.reshape(-1, 64))
@@ -114,20 +148,25 @@ def test_halo_empty_batch_and_output_untouched_outside(C_in, form):
     assert not torch.any(torch.isnan(y))           # every output written
 
 
-@pytest.mark.parametrize("B,C_in,C_out", [(32, 128, 128), (64, 64, 256), (256, 128, 128)],
-                         ids=["bn128", "bn256", "r50_s2_3x3"])
-def test_halo_streamed_sampled(B, C_in, C_out):
-    """Enough pixel tiles that the im2col GEMM takes 128- and 256-column
-    tiles, wider than the resident-weights form allows, so the layer runs
-    the streamed-weights form (the last case is ResNet-50's stage-2 3x3
-    layer at batch 256); checked on 3000 seeded output pixels over every
-    image, plus every pixel of the last image."""
-    layer = L("halo_wide", B, 28, 28, C_in, C_out, 3, 3, 1, 1, 1, N=16, rate=0.5, dtype="bf16", seed=B)
+@pytest.mark.parametrize("B,H,C_in,C_out,s,form", [
+    (32, 28, 128, 128, 1, "halo_streamed"), (64, 28, 64, 256, 1, "im2col"), (256, 28, 128, 128, 1, "halo_streamed"),
+    (256, 56, 128, 128, 2, "halo_streamed"), (256, 28, 256, 256, 2, "im2col")],
+    ids=["bn128", "bn256", "r50_s2_3x3", "r50_s2_b1_3x3_s2", "r50_s3_b1_3x3_s2"])
+def test_halo_streamed_sampled(B, H, C_in, C_out, s, form):
+    """Enough pixel tiles that the im2col GEMM takes 128- or 256-column
+    tiles, wider than the resident-weights form allows: at 128 columns the
+    layer runs the streamed-weights form (ResNet-50's stage-2 3x3 layers and
+    the stride-2 one at batch 256 among them), at 256 it keeps the im2col
+    form (the halo would be loaded once per 128-column tile); checked on
+    3000 seeded output pixels over every image, plus every pixel of the last
+    image."""
+    layer = L("halo_wide", B, H, H, C_in, C_out, 3, 3, s, 1, 1, N=16, rate=0.5, dtype="bf16", seed=B + s)
+    ho = (H - 1) // s + 1
     rng = np.random.default_rng(B)
-    last = np.arange(layer.pixels - 28 * 28, layer.pixels)
+    last = np.arange(layer.pixels - ho * ho, layer.pixels)
     pix = np.unique(np.concatenate([rng.choice(layer.pixels, 3000, replace=False), last]))
     y, yr, a, conv = run_layer(layer, relu=True, algo=ox.ONEXN_ALGO_TC, pixels=pix)
-    assert conv.tc_form((B, 28, 28, C_in)) == "halo_streamed"
+    assert conv.tc_form((B, H, H, C_in)) == form
     assert norm_err(y, yr, a) <= TOL_BF16_ROUNDED
     x = wl.activations(layer).to(torch.bfloat16).cuda()
     y1 = conv(x, relu=True, algo=ox.ONEXN_ALGO_TC)
