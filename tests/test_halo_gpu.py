@@ -59,6 +59,8 @@ HALO_GEOMS = [
     ("st_3x1", 2, 28, 28, 512, 128, 3, 1, 1, 1, 16, "halo_streamed"),
     ("st_1x3", 2, 26, 28, 512, 128, 1, 3, 1, 1, 16, "halo_streamed"),
     ("st_p0", 2, 30, 30, 256, 128, 3, 3, 0, 1, 16, "halo_streamed"),
+    ("st_w120", 1, 120, 120, 128, 128, 3, 3, 1, 1, 16, "halo_streamed"),    # 122-wide rows: 502-position loads
+    ("st_b1", 1, 28, 28, 256, 128, 3, 3, 1, 1, 16, "halo_streamed"),        # 4 tiles on 152 SMs
 ]
 
 
@@ -89,6 +91,7 @@ STRIDED_GEOMS = [
     ("s2_3x3_d2", 1, 56, 56, 128, 128, 3, 3, 2, 2, 2, 16),      # every tap in one phase
     ("s2_c72_co96", 1, 56, 56, 72, 96, 3, 3, 2, 1, 1, 8),       # partial chunk and column tile
     ("s2_co64", 2, 56, 56, 128, 64, 3, 3, 2, 1, 1, 16),         # 64-column tiles
+    ("s2_w120", 1, 120, 120, 128, 128, 3, 3, 2, 1, 1, 16),      # 61-wide phase rows
 ]
 
 

@@ -6,9 +6,11 @@ that forbid allocation after start-up so that latency stays predictable, or
 a plug-in that only receives pointers from a framework that owns the memory.
 For them the library keeps the tensor-core family's scratch in a fixed 8 MiB
 device array instead of a caller workspace.  These tests call it through the
-C ABI on three layers in a row (the third a stride-1 3x3 layer that the
-GEMM runs on halo tiles) and then on the first layer again (so it runs over
-what the others left in the shared array), and check each output
+C ABI on five layers in a row (the last three run the GEMM on halo tiles:
+a stride-1 3x3 layer with its weights resident in shared memory, one with
+them streamed, and a stride-2 3x3 layer over its four input phases) and
+then on the first layer again (so it runs over what the others left in the
+shared array), and check each output
 against the fp64 oracle and bit for bit against the regular onexn_conv_fwd
 with a workspace (the same kernels on the same decoded weights and the same
 tile plan).  The file name sorts last so that a run that stops at the first
@@ -52,13 +54,18 @@ LAYERS = [
     wl.ConvLayer("na_3x3", 4, 14, 14, 128, 128, 3, 3, 1, 1, 1, N=8, rate=0.5, dtype="bf16", seed=1),
     wl.ConvLayer("na_1x1_s2", 3, 15, 15, 64, 256, 1, 1, 2, 0, 1, N=16, rate=0.7, dtype="bf16", seed=2),
     wl.ConvLayer("na_3x3_halo", 2, 28, 28, 64, 64, 3, 3, 1, 1, 1, N=16, rate=0.7, dtype="bf16", seed=3),
+    wl.ConvLayer("na_3x3_streamed", 2, 28, 28, 256, 128, 3, 3, 1, 1, 1, N=16, rate=0.7, dtype="bf16", seed=4),
+    wl.ConvLayer("na_3x3_s2_phases", 1, 56, 56, 64, 128, 3, 3, 2, 1, 1, N=16, rate=0.5, dtype="bf16", seed=5),
 ]
+FORMS = ["im2col", "im2col", "halo_resident", "halo_streamed", "halo_streamed"]
 
 
-def test_noalloc_three_layers_then_the_first_again():
-    runs = [(LAYERS[0], True), (LAYERS[1], False), (LAYERS[2], True), (LAYERS[0], True)]
-    for layer, relu in runs:
+def test_noalloc_five_layers_then_the_first_again():
+    runs = [(0, True), (1, False), (2, True), (3, True), (4, False), (0, True)]
+    for i, relu in runs:
+        layer = LAYERS[i]
         conv, x_cpu, x, W, b = _layer_and_input(layer)
+        assert conv.tc_form(x.shape) == FORMS[i], layer.name
         y_na = _noalloc(conv, x, relu)
         y_ws = conv(x, relu=relu, algo=ox.ONEXN_ALGO_TC)
         torch.cuda.synchronize()
