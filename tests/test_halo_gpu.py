@@ -22,8 +22,8 @@ chunk, each tap's A operand a row-shifted view of it.
    (25 taps), padding 0 and 1, an odd input size, dilation 2 (one phase),
    a partial channel chunk and a partial column tile.
 A layer of each form with the residual + ReLU6 epilogue, and every case's
-form checked.  The 5x5 28-wide case wastes too many rows and runs the
-im2col form, checked here all the same.  Tolerance: 4e-3 = 2^-8 output
+form checked.  The 28-wide 5x5 and the 7x7 3x3 cases would waste 23% of a
+halo tile and run the im2col form, checked here all the same.  Tolerance: 4e-3 = 2^-8 output
 rounding on bf16-rounded inputs, normalised by sum |w x| + |b|."""
 import numpy as np
 import pytest
@@ -45,7 +45,8 @@ HALO_GEOMS = [
     ("r50_s2_like", 2, 28, 28, 128, 128, 3, 3, 1, 1, 16, "halo_resident"),   # two column tiles of 64, two chunks
     ("w56_co128", 1, 56, 56, 64, 128, 3, 3, 1, 1, 16, "halo_resident"),      # two rows per tile, two column tiles
     ("w112_c32", 1, 112, 112, 32, 32, 3, 3, 1, 1, 8, "halo_resident"),       # one row per tile, half-empty chunk
-    ("5x5_p2", 1, 28, 28, 32, 64, 5, 5, 2, 1, 16, "im2col"),                 # 23% of the rows dropped
+    ("5x5_p2", 1, 28, 28, 32, 64, 5, 5, 2, 1, 16, "im2col"),                 # 32x32 padded: 23% dropped
+    ("7x7_im2col", 4, 7, 7, 64, 64, 3, 3, 1, 1, 16, "im2col"),               # 8x8 padded: 23% dropped
     ("3x3_d2", 2, 28, 28, 64, 64, 3, 3, 2, 2, 16, "halo_resident"),
     ("3x3_p0", 2, 30, 30, 64, 64, 3, 3, 0, 1, 16, "halo_resident"),
     ("3x1_p1", 2, 28, 28, 64, 64, 3, 1, 1, 1, 16, "halo_resident"),

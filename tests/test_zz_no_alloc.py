@@ -51,7 +51,7 @@ def _noalloc(conv, x, relu):
 
 
 LAYERS = [
-    wl.ConvLayer("na_3x3", 4, 14, 14, 128, 128, 3, 3, 1, 1, 1, N=8, rate=0.5, dtype="bf16", seed=1),
+    wl.ConvLayer("na_3x3", 16, 7, 7, 128, 128, 3, 3, 1, 1, 1, N=8, rate=0.5, dtype="bf16", seed=1),
     wl.ConvLayer("na_1x1_s2", 3, 15, 15, 64, 256, 1, 1, 2, 0, 1, N=16, rate=0.7, dtype="bf16", seed=2),
     wl.ConvLayer("na_3x3_halo", 2, 28, 28, 64, 64, 3, 3, 1, 1, 1, N=16, rate=0.7, dtype="bf16", seed=3),
     wl.ConvLayer("na_3x3_streamed", 2, 28, 28, 256, 128, 3, 3, 1, 1, 1, N=16, rate=0.7, dtype="bf16", seed=4),
