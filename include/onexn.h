@@ -266,7 +266,8 @@ onexn_status onexn_conv_out_shape(const onexn_conv_desc *desc, int *Ho, int *Wo)
  *           tensor-core GEMM (ALGO_TC) decodes the weights into it; the
  *           sparse tensor-core kernel (ALGO_MMA) writes its plan there (per
  *           64-channel chunk and tile of 128/N groups: the groups' kept
- *           entries, counts and channels, 560 bytes).  The call overwrites
+ *           entry counts and channels and those entries' D rows, 16944
+ *           bytes).  The call overwrites
  *           it, so calls that run concurrently need separate workspaces.
  *           AUTO only picks a family whose minimum workspace fits in
  *           workspace_bytes.

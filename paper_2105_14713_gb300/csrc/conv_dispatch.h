@@ -10,8 +10,9 @@
 namespace onexn {
 
 cudaError_t launch_fma(const ConvArgs &a, int dtype, cudaStream_t st);
-// sparse tensor-core family (bf16): a boundary table of the kept lists in
-// the workspace (mma_workspace_bytes), then the kernel
+// sparse tensor-core family (bf16): a plan of the kept lists (per chunk and
+// group tile: entry counts, channels and D rows) in the workspace
+// (mma_workspace_bytes), then the kernel
 cudaError_t launch_mma(const ConvArgs &a, void *workspace, size_t ws_bytes, cudaStream_t st);
 bool mma_supports(const ConvArgs &a);
 size_t mma_workspace_bytes(const ConvArgs &a);

@@ -19,7 +19,10 @@
 //
 // Warp roles (one persistent CTA per SM):
 //  * warp 2, producer: one thread issues the TMA load of each chunk's
-//    activation tile (128 pixels x 64 channels, 128-byte swizzle).
+//    activation tile (128 pixels x 64 channels, 128-byte swizzle) and one
+//    bulk copy of the chunk's plan record, which a plan kernel wrote once
+//    per layer with the kept entries' channels and their D rows, so no load
+//    depends on another.
 //  * warps 4-11, gather: warp w handles pixel rows 32*(w%4) .. +31 of the
 //    tile (its TMEM lanes) and half-chunk (w-4)/4.  Per chunk and group it
 //    reads the entries' input channels from I, copies x[row][c] into the
@@ -52,18 +55,22 @@ constexpr int kMaxGS = 8;                  // groups per tile at most (N = 16)
 constexpr int kBK = 64;                    // channels per chunk (128 bytes of bf16)
 constexpr int kHalf = 32;                  // channels per gathered half-chunk
 constexpr int kStages = 4;
-constexpr int kLookahead = kStages - 1;    // the producer issues a chunk's D rows this many chunks later
 // plan record of one (chunk, group tile), built once per layer:
 //   [0, 16)   uint8 count[h * 8 + gl]   kept entries of group g0+gl in half-chunk h (<= 32)
 //   [16, 48)  int32 zs[gl]              first entry of the chunk in the group's list
 //   [48, 560) uint8 ch[(h*8 + gl)*32 + j]  channel of entry j inside half-chunk h (0..31)
-constexpr int kRecCnt = 0, kRecZs = 16, kRecCh = 48, kRecBytes = 560;
-// stage: activation tile | B of the tile's groups | the groups' raw D rows | record
+//   [560, +kDBytes) the D rows of those entries: group gl's at gl * 64 * N
+//             bf16, half 0's entries then half 1's, N values each
+// so that one copy per chunk brings everything its gathers and MMAs read.
+constexpr int kRecCnt = 0, kRecZs = 16, kRecCh = 48, kRecHdr = 560;
 constexpr int kXBytes = kBM * 128;                   // 128 pixels x 64 channels, 128-byte swizzle
 constexpr int kBBytes = kTileCols * 128;             // per group N rows x 64 entries, K-major, 128-byte swizzle
 constexpr int kDBytes = kTileCols * kBK * 2;         // per group up to 64 rows of N bf16
-constexpr int kXOff = 0, kBOff = kXBytes, kDOff = kBOff + kBBytes, kRecOff = kDOff + kDBytes;
+constexpr int kRecBytes = kRecHdr + kDBytes;         // a multiple of 16 (bulk copy)
+// stage: activation tile | B of the tile's groups | record (its D rows inside)
+constexpr int kXOff = 0, kBOff = kXBytes, kRecOff = kBOff + kBBytes, kDOff = kRecOff + kRecHdr;
 constexpr int kStageBytes = ((kRecOff + kRecBytes + 1023) / 1024) * 1024;
+static_assert(kRecBytes % 16 == 0 && kDOff % 16 == 0, "bulk copy and 16-byte D row loads");
 constexpr int kAccCols = kTileCols;        // one fp32 accumulator buffer; two of them
 constexpr int kACol0 = 2 * kAccCols;       // A blocks after the accumulators: [half][group]
 constexpr int kABlockCols = 16;            // per (half, group): 32 bf16 entries per lane
@@ -78,8 +85,8 @@ constexpr int kWarps = 16;
 constexpr int kXtWarpBytes = 16 * 32 * 4;  // a gather warp's transposed half rows: 16 words x 32 lanes
 constexpr int kXtOff = kStages * kStageBytes;
 constexpr int kBarOff = kXtOff + 8 * kXtWarpBytes;
-// full[S], dfull[S], empty[S], gathered[2], consumed[2], tfull[2], tempty[2], drain[kIssuers]
-constexpr int kNumBars = 3 * kStages + 2 + 2 + 2 + 2 + kIssuers;
+// full[S], empty[S], gathered[2], consumed[2], tfull[2], tempty[2], drain[kIssuers]
+constexpr int kNumBars = 2 * kStages + 2 + 2 + 2 + 2 + kIssuers;
 constexpr int kMaskOff = kBarOff + kNumBars * 8;       // uint32 [2][kIssuers]: groups an issuer touched
 constexpr int kHolderOff = kMaskOff + 2 * kIssuers * 4;
 constexpr int kSmemBytes = kHolderOff + 16;
@@ -113,10 +120,12 @@ __device__ __forceinline__ int lower_bound_k(const int32_t *__restrict__ I, int 
 // half-chunk h, the kept entries z of group g = tg*GS + gl whose index
 // I[z] = tap*C + c has c in the half-chunk's 32 channels (a contiguous
 // range of the group's list, found by binary search), their count and
-// channels; and the chunk's first entry.  P and I are clamped so that a
-// corrupted list cannot index outside I.  One thread per (ci, tg, gl, h).
-__global__ void mma_plan_kernel(const int32_t *__restrict__ P, const int32_t *__restrict__ I, int t, int G, int GS,
-                                int C, int n_cchunk, int n_chunks, int n_g, unsigned char *__restrict__ rec)
+// channels, their D rows (after the chunk's half-0 rows); and the chunk's
+// first entry.  P and I are clamped so that a corrupted list cannot index
+// outside I or D.  One thread per (ci, tg, gl, h).
+__global__ void mma_plan_kernel(const int32_t *__restrict__ P, const int32_t *__restrict__ I,
+                                const __nv_bfloat16 *__restrict__ D, int N, int t, int G, int GS, int C,
+                                int n_cchunk, int n_chunks, int n_g, unsigned char *__restrict__ rec)
 {
     const int64_t idx = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
     if (idx >= static_cast<int64_t>(n_chunks) * n_g * GS * 2) return;
@@ -137,6 +146,12 @@ __global__ void mma_plan_kernel(const int32_t *__restrict__ P, const int32_t *__
         const int z1 = lower_bound_k(I, z0, hi, static_cast<int64_t>(tap) * C + c_hi);
         cnt = min(z1 - z0, kHalf);
         if (h == 0) reinterpret_cast<int32_t *>(r + kRecZs)[gl] = z0;
+        // D rows of this half's entries: after the chunk's half-0 entries
+        const int zc = h ? lower_bound_k(I, lo, z0, static_cast<int64_t>(tap) * C + cc * kBK) : z0;
+        const int off = min(z0 - zc, kHalf);
+        const uint4 *src = reinterpret_cast<const uint4 *>(D + static_cast<int64_t>(z0) * N);
+        uint4 *dst = reinterpret_cast<uint4 *>(r + kRecHdr + gl * (kBK * N * 2) + off * (N * 2));
+        for (int i = 0; i < cnt * (N / 8); ++i) dst[i] = __ldg(src + i);
     } else if (h == 0) {
         reinterpret_cast<int32_t *>(r + kRecZs)[gl] = 0;
     }
@@ -168,8 +183,7 @@ mma_conv_kernel(const ConvArgs a, const __grid_constant__ CUtensorMap tmap_x, co
     const uint32_t base = (raw + 1023u) & ~1023u;
     unsigned char *smem = smem_raw + (base - raw);
     const uint32_t bar_full = base + kBarOff;
-    const uint32_t bar_dfull = bar_full + 8 * kStages;
-    const uint32_t bar_empty = bar_dfull + 8 * kStages;
+    const uint32_t bar_empty = bar_full + 8 * kStages;
     const uint32_t bar_gath = bar_empty + 8 * kStages;
     const uint32_t bar_cons = bar_gath + 16;
     const uint32_t bar_tfull = bar_cons + 16;
@@ -182,7 +196,6 @@ mma_conv_kernel(const ConvArgs a, const __grid_constant__ CUtensorMap tmap_x, co
     if (tid == 0) {
         for (int s = 0; s < kStages; ++s) {
             mbar_init(bar_full + 8 * s, 1);
-            mbar_init(bar_dfull + 8 * s, 1);
             mbar_init(bar_empty + 8 * s, kIssuers);
         }
         for (int b = 0; b < 2; ++b) {
@@ -213,37 +226,11 @@ mma_conv_kernel(const ConvArgs a, const __grid_constant__ CUtensorMap tmap_x, co
 
     if (warp == kProdWarp) {
         // ============================ producer ============================
-        // Per chunk: the activation tile (TMA) and the chunk's plan record
-        // (bulk copy) on "full"; kLookahead chunks later, once that record
-        // has landed, the D rows of the chunk's kept entries of each group
-        // (one bulk copy per group) on "dfull".
+        // Per chunk: the activation tile (TMA) and the chunk's plan record,
+        // its D rows inside (one bulk copy), both on "full".
         if (lane == 0) {
             const int hw = a.Ho * a.Wo;
-            const __nv_bfloat16 *D = static_cast<const __nv_bfloat16 *>(a.D);
-            int pend_g0[kStages] = {};
             bool failed = false;
-            auto issue_d = [&](int i) {
-                const int s = i % kStages;
-                if (!mbar_wait(bar_full + 8 * s, (i / kStages) & 1)) return false;
-                const unsigned char *r = smem + s * kStageBytes + kRecOff;
-                const int g0 = pend_g0[s];
-                uint32_t bytes = 0;
-                // (entries clamped to D's t rows, whatever the record says)
-                auto rows = [&](int gl, int &zs) {
-                    zs = clampi(reinterpret_cast<const int32_t *>(r + kRecZs)[gl], 0, a.t);
-                    return min(r[kRecCnt + gl] + r[kRecCnt + kMaxGS + gl], a.t - zs);
-                };
-                int zs = 0;
-                for (int gl = 0; gl < GS && g0 + gl < G; ++gl) bytes += rows(gl, zs) * (N * 2);
-                tc::mbar_arrive_expect_tx(bar_dfull + 8 * s, bytes);
-                for (int gl = 0; gl < GS && g0 + gl < G; ++gl) {
-                    const int n = rows(gl, zs);
-                    if (n == 0) continue;
-                    tc::bulk_load(base + s * kStageBytes + kDOff + gl * (kBK * N * 2), D + static_cast<int64_t>(zs) * N,
-                                  static_cast<uint32_t>(n * N * 2), bar_dfull + 8 * s);
-                }
-                return true;
-            };
             int item = 0;
             for (int T = blockIdx.x; T < sc.tiles && !failed; T += gridDim.x) {
                 const int tm = static_cast<int>(sc.div_g.div(T)), tg = T - tm * sc.n_g;
@@ -269,16 +256,8 @@ mma_conv_kernel(const ConvArgs a, const __grid_constant__ CUtensorMap tmap_x, co
                     tc::bulk_load(base + s * kStageBytes + kRecOff,
                                   sc.rec + (static_cast<int64_t>(ci) * sc.n_g + tg) * kRecBytes, kRecBytes,
                                   bar_full + 8 * s);
-                    pend_g0[s] = tg * GS;
-                    if (item >= kLookahead && !issue_d(item - kLookahead)) {
-                        failed = true;
-                        break;
-                    }
                 }
             }
-            // the D rows of the last chunks
-            for (int i = item - kLookahead < 0 ? 0 : item - kLookahead; i < item && !failed; ++i)
-                if (!issue_d(i)) failed = true;
             if (failed) abort_now();
         }
         __syncwarp();
@@ -355,14 +334,9 @@ mma_conv_kernel(const ConvArgs a, const __grid_constant__ CUtensorMap tmap_x, co
                     }
                 }
                 // the staged groups' B: entry j of the half -> K position
-                // 32h + j of rows n = 0..N-1 (from the group's raw D rows in
-                // this stage, after the half-0 entries for h = 1); the rest of
-                // each used 16-entry step is zeroed
-                if (!mbar_wait(bar_dfull + 8 * s, (item / kStages) & 1)) {
-                    abort_now();
-                    failed = true;
-                    break;
-                }
+                // 32h + j of rows n = 0..N-1 (from the group's D rows in this
+                // stage's copy of the record, after the half-0 entries for
+                // h = 1); the rest of each used 16-entry step is zeroed
                 for (int g = q; g < GS; g += 4) {
                     if (g0 + g >= G) break;
                     const int cnt = r[kRecCnt + h * kMaxGS + g], nb = (cnt + 15) >> 4;
@@ -581,7 +555,8 @@ cudaError_t mma_plan(const ConvArgs &a, void *workspace, size_t ws_bytes, cudaSt
     const int64_t n = static_cast<int64_t>(n_chunks) * n_g * GS * 2;
     const int threads = 256;
     mma_plan_kernel<<<static_cast<unsigned>((n + threads - 1) / threads), threads, 0, st>>>(
-        a.P, a.I, a.t, G, GS, a.C, n_cchunk_of(a), n_chunks, n_g, static_cast<unsigned char *>(workspace));
+        a.P, a.I, static_cast<const __nv_bfloat16 *>(a.D), a.N, a.t, G, GS, a.C, n_cchunk_of(a), n_chunks, n_g,
+        static_cast<unsigned char *>(workspace));
     return cudaGetLastError();
 }
 
