@@ -450,6 +450,30 @@ onexn_status onexn_conv_algo(const onexn_conv_desc *desc, int N, int64_t t, int 
 onexn_status onexn_conv_tc_form(const onexn_conv_desc *desc, int N, int64_t t, int dtype, int *form);
 
 /*
+ * onexn_conv_halo_geometry -- the plan of the streamed halo form
+ * (ONEXN_GEMM_HALO_STREAMED) for a bf16 layer, for inspection and tests;
+ * no device work.  The output is laid out in a padded space of Hp rows of
+ * Wp positions per image (position (n*Hp + r)*Wp + c is output pixel
+ * (n, r, c) when r < Ho and c < Wo).  A strided layer is split into the
+ * phases of its input (Eq. 6's taps regrouped by which input pixels they
+ * read).  The halo load at padded position (r, c) starts at input base
+ * (lower_w + stride_w*c, lower_h + stride_h*r), steps by the strides, and
+ * reads x at base + the phase's offsets, zeros outside x.  Tap k of a phase
+ * reads the load from row shift(k) on.
+ *   geom    HOST int[8]: Wp, Hp, lower_w, lower_h, positions per halo load,
+ *           phases, taps, column tile.
+ *   taps    HOST uint32[49]: per tap in phase order, (kh*KW + kw) << 16 | shift.
+ *   phases  HOST uint32[4]: first tap | end tap << 8 | w offset << 16 |
+ *           h offset << 24.
+ * Reads the current device's SM count (152 when there is no device).
+ * EINVAL as onexn_conv_fwd's shape checks or a NULL output; EUNSUPPORTED
+ * when the layer has no streamed plan (1x1, too much padding, ...).  The
+ * GEMM may still run another form (onexn_conv_tc_form decides).
+ */
+onexn_status onexn_conv_halo_geometry(const onexn_conv_desc *desc, int N, int64_t t, int *geom,
+                                      uint32_t *taps, uint32_t *phases);
+
+/*
  * onexn_conv_fwd_host -- onexn_conv_fwd on activations in HOST memory:
  * y_host = conv(x_host), with the copies to and from the GPU inside the
  * call.  The batch is cut into chunks of whole images; each chunk is copied

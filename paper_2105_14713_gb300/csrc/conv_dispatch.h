@@ -47,6 +47,9 @@ int halo_form(const ConvArgs &a, int im2col_bn);
 cudaError_t halo_gemm(const ConvArgs &a, const void *W, int im2col_bn, cudaStream_t st);
 // The form the tensor-core GEMM takes for this layer and dtype (conv_tc.cu).
 int tc_gemm_form(const ConvArgs &a, int dtype);
+// The streamed halo form's plan geometry (conv_halo.cu): geom[8], taps[49],
+// phases[4]; false when the layer has no streamed plan.
+bool halo_streamed_geometry(const ConvArgs &a, int geom[8], uint32_t *taps, uint32_t *phases);
 size_t tc_sk_bytes(const ConvArgs &a, int dtype);
 
 namespace detail {

@@ -299,6 +299,19 @@ extern "C" onexn_status onexn_conv_tc_form(const onexn_conv_desc *desc, int N, i
     return ONEXN_OK;
 }
 
+extern "C" onexn_status onexn_conv_halo_geometry(const onexn_conv_desc *desc, int N, int64_t t, int *geom,
+                                                 uint32_t *taps, uint32_t *phases)
+{
+    onexn::clear_error();
+    if (!geom || !taps || !phases) return fail(ONEXN_EINVAL, "conv_halo_geometry: NULL output");
+    onexn::ConvArgs a{};
+    onexn_status st = check_shape(desc, N, t, ONEXN_BF16, 0, &a);
+    if (st != ONEXN_OK) return st;
+    if (!onexn::halo_streamed_geometry(a, geom, taps, phases))
+        return fail(ONEXN_EUNSUPPORTED, "conv_halo_geometry: no streamed halo plan for this layer");
+    return ONEXN_OK;
+}
+
 extern "C" onexn_status onexn_conv_workspace_size(const onexn_conv_desc *desc, int N, int64_t t,
                                                   int dtype, unsigned flags, size_t *bytes)
 {

@@ -1036,6 +1036,22 @@ int halo_form(const ConvArgs &a, int im2col_bn)
     return kGemmIm2col;
 }
 
+// The streamed form's plan geometry, for inspection: geom = {Wp, Hp, TMA
+// lower corner w, h, positions per halo load, phases, taps, column tile},
+// taps[kWMaxTaps] and phases[kWMaxPhases] as in WidePlan.  False when the
+// layer has no streamed plan.
+bool halo_streamed_geometry(const ConvArgs &a, int geom[8], uint32_t *taps, uint32_t *phases)
+{
+    WidePlan p;
+    int bn = 0;
+    if (!wide_plan(a, device_sms_or_default(), &p, &bn)) return false;
+    const int g[8] = {p.Wp, p.Hp, p.lower_w, p.lower_h, static_cast<int>(p.halo_pix), p.n_ph, p.n_taps, bn};
+    for (int i = 0; i < 8; ++i) geom[i] = g[i];
+    for (int i = 0; i < kWMaxTaps; ++i) taps[i] = p.tap[i];
+    for (int i = 0; i < kWMaxPhases; ++i) phases[i] = p.ph[i];
+    return true;
+}
+
 // The halo GEMM of a bf16 layer on its decoded weights W[C_out][K] (the
 // caller has checked that halo_form is not the im2col GEMM).
 cudaError_t halo_gemm(const ConvArgs &a, const void *W, int im2col_bn, cudaStream_t st)

@@ -64,6 +64,7 @@ SIGNATURES = {
     "onexn_conv_algo": ([ctypes.POINTER(ConvDesc), _I32, _I64, _I32, _U32, ctypes.c_size_t, _P],
                         _I32),
     "onexn_conv_tc_form": ([ctypes.POINTER(ConvDesc), _I32, _I64, _I32, _P], _I32),
+    "onexn_conv_halo_geometry": ([ctypes.POINTER(ConvDesc), _I32, _I64, _P, _P, _P], _I32),
     "onexn_device_status": ([_I32, _P], _I32),
     "onexn_selftest_timeout": ([_P], _I32),
     "onexn_probe_ffma": ([_I32, _I32, _P, _P], _I32),
@@ -222,6 +223,19 @@ def onexn_conv_tc_form(desc: ConvDesc, N: int, t: int, dtype: int) -> str:
     out = ctypes.c_int(0)
     _check(lib.onexn_conv_tc_form(ctypes.byref(desc), int(N), int(t), int(dtype), ctypes.byref(out)))
     return GEMM_FORMS[out.value]
+
+
+def onexn_conv_halo_geometry(desc: ConvDesc, N: int, t: int) -> dict:
+    geom = (ctypes.c_int * 8)()
+    taps = (ctypes.c_uint32 * 49)()
+    phases = (ctypes.c_uint32 * 4)()
+    _check(lib.onexn_conv_halo_geometry(ctypes.byref(desc), int(N), int(t), geom, taps, phases))
+    n_ph, n_taps = geom[5], geom[6]
+    return {"Wp": geom[0], "Hp": geom[1], "lower_w": geom[2], "lower_h": geom[3], "halo_pix": geom[4],
+            "bn": geom[7],
+            "taps": [(taps[i] >> 16, taps[i] & 0xFFFF) for i in range(n_taps)],
+            "phases": [(phases[i] & 0xFF, (phases[i] >> 8) & 0xFF, (phases[i] >> 16) & 0xFF, phases[i] >> 24)
+                       for i in range(n_ph)]}
 
 
 def onexn_conv_workspace_size(desc: ConvDesc, N: int, t: int, dtype: int, flags: int = 0) -> int:
